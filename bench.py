@@ -1,0 +1,384 @@
+#!/usr/bin/env python
+"""Throughput of the DriveCache hot path on one GB300 (or N replicas).
+
+One bench step = one dc_denoise call on the workload's batch of scenes: the
+host planner (motion statistics, support gate, scene tables, exact DP) for
+every scene, the conditioning/modulation kernels, then K Euler steps in
+which each scene either runs the full block stack or reuses its cached
+backbone output after the causal drift check (with refresh + suffix replan
+when the check refuses).  Inputs are seeded synthetic latents, random-init
+weights and synthetic ego trajectories (synth/); anchors, anchor drift
+tables (measured on the device from two full traces) and the budget tau are
+calibrated once before timing.  The same inputs are restored before every
+step, so every step executes the same schedule.
+
+Metric: denoising scene-steps per second with the cache enabled
+(B * K / wall time of one call), summed over ranks.  Also reported:
+videos/s, the all-compute throughput and the speedup, per-kernel device
+times, the roofline of the dominant kernel, an end-to-end number through
+dc_denoise_host (host latents in and out) and the CPU oracle baseline.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c2]
+  python bench.py --impl reference ...   (times the CPU oracle instead)
+"""
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from synth import WORKLOADS, gen  # noqa: E402
+
+METRIC = "denoising steps/s (cache-enabled, fixed schedule)"
+UNIT = "scene-steps/s"
+L2_BYTES = 129 * 2 ** 20
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=5)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--workload", default="c2", choices=sorted(WORKLOADS))
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+def peaks():
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))), "measured"
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                "sm_max_mhz": 2070.0}, "fallback"
+
+
+# ------------------------------------------------------------ clock sampler
+
+class Clocks:
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{index}.csv")
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = float(parts[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": mx,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------ calibration
+
+def calibrate(dc, model, wl, torch, dev):
+    """Anchors (Sec. 3.1), anchor drift tables from two full traces on the
+    device (Eq. 5), synthetic q tables, tau (Sec. 3.2)."""
+    K, H = wl.steps, wl.h_max
+    clips = gen.calibration_trajectories(wl)
+    stats = [dc.motion_stats(c) for c in clips]
+    anc = dc.select_anchors([s[0] for s in stats], [s[1] for s in stats])
+    q0, q1 = gen.synthetic_q_tables(K, H)
+    sig = gen.sigmas(K)
+    noise = torch.tensor(gen.anchor_noise(wl), device=dev)
+    d0 = dc.anchor_drift(model, noise, clips[anc["i0"]], K, sig, H)
+    d1 = dc.anchor_drift(model, noise, clips[anc["i1"]], K, sig, H)
+    tables = dict(q0=q0, q1=q1, d0=d0, d1=d1)
+    A = dc.AnchorArgs(K, H, anc, tables)
+    tau, reached = dc.calibrate_budget(list(clips), A, wl.target(), K)
+    return anc, tables, A, tau, reached
+
+
+# ------------------------------------------------------------ cpu baseline
+
+def oracle_rate(wl, n_compute, n_reuse, blocks=1):
+    """Time the CPU oracle on a bounded sample of the workload and convert to
+    scene-steps/s for the given mix of compute and reuse scene-steps: one
+    compute scene-step is timed on `blocks` blocks and scaled to L blocks
+    (plus the embedding, conditioning and interface, timed in full); one
+    reuse scene-step is timed in full."""
+    from oracle import dit as O
+    w = gen.weights(wl.with_(n_blocks=blocks))
+    m = O.Model(wl.with_(n_blocks=blocks), w)
+    x = gen.latents(wl, batch=1)[0]
+    tr = gen.scene_trajectories(wl, batch=1)[0]
+    t0 = time.perf_counter()
+    blk, fmod = m.mods(0.5, tr)
+    u = O.embed(m.w, x)
+    t1 = time.perf_counter()
+    h = O.backbone(m.w, u, blk, m.heads)
+    t2 = time.perf_counter()
+    O.head(m.w, h, fmod)
+    t3 = time.perf_counter()
+    t_compute = (t1 - t0) + (t2 - t1) * wl.n_blocks / blocks + (t3 - t2)
+    t4 = time.perf_counter()
+    m.reuse_step(x, h - u, 0.5, tr)
+    t_reuse = time.perf_counter() - t4
+    total = n_compute * t_compute + n_reuse * t_reuse
+    return (n_compute + n_reuse) / total, t_compute, t_reuse, (t3 - t0) + t_reuse
+
+
+def cpu_threads():
+    try:
+        import threadpoolctl
+        info = threadpoolctl.threadpool_info()
+        return max([i.get("num_threads", 1) for i in info] + [1])
+    except Exception:
+        return os.cpu_count()
+
+
+def planned_mix(wl):
+    """Compute/reuse scene-step counts of the planned schedules (oracle
+    planner; drift vetoes ignored) for the reference arm."""
+    from oracle import planner as P
+    K, H = wl.steps, wl.h_max
+    clips = gen.calibration_trajectories(wl)
+    st = [P.motion_stats(c) for c in clips]
+    anc = P.select_anchors([s[0] for s in st], [s[1] for s in st])
+    q0, q1 = gen.synthetic_q_tables(K, H)
+    z = [[0.0] * (H + 1) for _ in range(K)]
+    tabs = dict(q0=q0, q1=q1, d0=z, d1=z)
+    tau, _ = P.calibrate_budget(list(clips), anc, tabs, wl.target(), K, H)
+    nr = sum(P.plan_scene(t, anc, tabs, tau, K, H)["n_reuse"] for t in gen.scene_trajectories(wl))
+    return wl.batch * K - nr, nr
+
+
+def run_reference(args, wl, rank, world):
+    if rank != 0:
+        return
+    nc, nr = planned_mix(wl)
+    times, rates = [], []
+    for i in range(args.warmup + args.steps):
+        t0 = time.perf_counter()
+        rate, tc, tr, _ = oracle_rate(wl, nc, nr)
+        if i >= args.warmup:
+            times.append(time.perf_counter() - t0)
+            rates.append(rate)
+    rate = statistics.median(rates)
+    cores = cpu_threads()
+    sample = (f"per step: one block of one compute scene-step scaled to L={wl.n_blocks} blocks "
+              f"plus one reuse scene-step, fp64 NumPy, weighted by the planned mix "
+              f"({nc} compute / {nr} reuse scene-steps per call)")
+    line = {"impl": "reference", "metric": METRIC, "value": rate, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1000.0 * wl.batch * wl.steps / rate, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": wl.name, "batch": wl.batch, "steps": wl.steps,
+                       "tokens": wl.n_tokens},
+            "cpu_baseline": {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": rate, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------ main bench
+
+def main():
+    args = parse()
+    wl = WORKLOADS[args.workload]
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        return run_reference(args, wl, rank, world)
+
+    import torch
+    import torch.distributed as dist
+    from paper_2608_16354_gb300 import binding as dc
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    dc.lib()
+    # replicas: every rank runs the same model on its own scenes (weak scaling)
+    weights = gen.weights(wl)
+    model = dc.Model(wl, gen.flat_blob(wl, weights))
+    del weights
+    anc, tables, A, tau, reached = calibrate(dc, model, wl, torch, dev)
+    K, B = wl.steps, wl.batch
+    sig = gen.sigmas(K)
+    x1 = torch.tensor(gen.latents(wl, seed=wl.seed + 7919 * rank), device=dev)
+    trajs = list(gen.scene_trajectories(wl, seed=wl.seed + 7919 * rank))
+    lat = torch.empty_like(x1)
+    sched = dc.SchedArgs(K, sig, A, tau, veto=True)
+    stream = torch.cuda.current_stream()
+    flush = torch.empty(4 * L2_BYTES // 4, dtype=torch.float32, device=dev)
+
+    def one_call(s=sched, record=None):
+        lat.copy_(x1)
+        flush.fill_(1.0)  # evict L2 between steps
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        st = dc.denoise(model, lat, trajs, s, stream=stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1), st
+
+    for _ in range(args.warmup):
+        one_call()
+    ref_exec = None
+    clocks = Clocks(local)
+    dc.profile(model, True)
+    barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    ms_list, launches, calls = [], 0, 0
+    for _ in range(args.steps):
+        ms, st = one_call()
+        ms_list.append(ms)
+        launches += st["launches"]
+        calls += st["backbone_calls"]
+        if ref_exec is None:
+            ref_exec = st["executed"].copy()
+            stats0 = st
+        assert np.array_equal(ref_exec, st["executed"]), "schedule changed between steps"
+    torch.cuda.synchronize()
+    barrier()
+    clk = clocks.stop()
+    dc.profile(model, False)
+    prof = dc.profile_read(model)
+    total_ms = sum(ms_list)
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = t.item()
+    ms_step = total_ms / args.steps
+    value = world * B * K / (ms_step / 1000.0)
+
+    # all-compute reference (no cache) for the speedup
+    forced = np.full((B, K + 1), dc.COMPUTE, np.uint8)
+    full_s = dc.SchedArgs(K, sig, A, tau, forced=forced)
+    one_call(full_s)
+    full_ms = statistics.median([one_call(full_s)[0] for _ in range(2)])
+
+    # end to end through the C ABI with host buffers (pinned)
+    host = torch.empty(x1.shape, dtype=torch.float32).pin_memory()
+    x1_host = x1.cpu()
+    e2e_ms = []
+    for i in range(max(2, min(args.steps, 3))):
+        host.copy_(x1_host)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        dc.denoise_host(model, host, trajs, sched, stream=stream, stats=False)
+        torch.cuda.synchronize()
+        e2e_ms.append(1000.0 * (time.perf_counter() - t0))
+    e2e_step = statistics.median(e2e_ms)
+
+    pk, pk_src = peaks()
+    # dominant kernel category by device time
+    dom = max((k for k in prof if k != "condition"), key=lambda k: prof[k]["ms"])
+    p = prof[dom]
+    tensor = dom.startswith("gemm") or dom == "attention"
+    n_launch = max(p["launches"], 1)
+    avg_s = p["ms"] / 1000.0 / n_launch
+    if tensor:
+        achieved = p["flops"] / n_launch / avg_s / 1e12
+        peak = pk.get("bf16_tflops_sustained", pk.get("bf16_tflops"))
+        unit = "TFLOP/s"
+    else:
+        achieved = p["bytes"] / n_launch / avg_s / 1e9
+        peak = pk["hbm_gbs"]
+        unit = "GB/s"
+    traffic = None
+    tpath = os.path.join(ROOT, "profiles", "traffic.json")
+    if os.path.exists(tpath):
+        try:
+            tinfo = json.load(open(tpath))
+            if tinfo.get("workload") == wl.name and dom in tinfo.get("per_launch_bytes", {}):
+                traffic = tinfo["per_launch_bytes"][dom]
+        except Exception:
+            traffic = None
+    kernels = {k: {"ms_per_call": v["ms"] / args.steps, "launches_per_call": v["launches"] / args.steps,
+                   "tflops": (v["flops"] / (v["ms"] / 1000.0) / 1e12) if v["ms"] > 0 and v["flops"] else None,
+                   "gbs": (v["bytes"] / (v["ms"] / 1000.0) / 1e9) if v["ms"] > 0 else None}
+               for k, v in prof.items() if v["launches"]}
+    n_reuse = int(np.sum(ref_exec[:, 1:] == dc.REUSE))
+    n_comp = B * K - n_reuse
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32", "data": "synthetic",
+        "config": {"workload": wl.name, "batch": B, "steps": K, "tokens": wl.n_tokens,
+                   "d_model": wl.d_model, "blocks": wl.n_blocks, "heads": wl.n_heads,
+                   "rho_tar": wl.rho_tar, "tau": tau, "parallelism": f"replicas{world}",
+                   "l2": "flushed between steps (512 MB write)"},
+        "videos_per_s": world * B / (ms_step / 1000.0),
+        "full_compute_steps_per_s": world * B * K / (full_ms / 1000.0),
+        "speedup_vs_full_compute": full_ms / ms_step,
+        "schedule": {"compute_scene_steps": n_comp, "reuse_scene_steps": n_reuse,
+                     "vetoes": int(np.sum(stats0["n_veto"])),
+                     "unsupported_scenes": int(B - np.sum(stats0["supported"]))},
+        "gpu_launches": int(launches),
+        "e2e": {"value": world * B * K / (e2e_step / 1000.0), "unit": UNIT,
+                "h2d_bytes_per_step": int(x1.numel() * 4), "d2h_bytes_per_step": int(x1.numel() * 4)},
+        "roofline": {"kernel": dom, "bound": "tensor" if tensor else "hbm", "achieved": achieved,
+                     "peak": peak, "unit": unit, "frac": achieved / peak, "traffic": traffic,
+                     "peak_source": f"{pk_src} ({'bf16 sustained' if tensor else 'HBM copy'})"},
+        "kernels": kernels,
+        "clocks": clk,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        rate, tc, tr, spent = oracle_rate(wl, n_comp, n_reuse)
+        line["cpu_baseline"] = {
+            "value": rate, "unit": UNIT, "cores": cpu_threads(), "kind": "oracle",
+            "sample": (f"one block of one compute scene-step ({tc:.2f} s when scaled to "
+                       f"L={wl.n_blocks}) and one reuse scene-step ({tr:.3f} s), fp64 NumPy, "
+                       f"weighted by this run's executed mix ({n_comp} compute / {n_reuse} reuse)")}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    model.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,273 @@
+/*
+ * drivecache.h -- C ABI of the GB300 DriveCache hot path.
+ *
+ * DriveCache (action-aware caching for driving world-model inference) lets a
+ * diffusion sampler skip the expensive backbone F_k on some denoising steps
+ * by substituting the most recently computed backbone output r_j (Eq. 1).
+ * The host planner places those reuses from the planned ego motion with an
+ * exact DP under a response budget (Eq. 2-11); at run time a causal drift
+ * check (Eq. 12) may refuse a planned reuse, refresh the cache and replan the
+ * remaining steps (Sec. 3.2).  The backbone here is a synthetic adaLN DiT.
+ *
+ * Conventions for every call:
+ *  - Steps are 1-based: k = 1..K.  Arrays "[K+1]" leave index 0 unused.
+ *  - Response / drift tables are row-major [K][H_max+1] doubles indexed
+ *    [j][h]: j = 1..K-1 is the step of the last full evaluation, h = 1..H_max
+ *    the cache age; row 0 and column 0 are ignored.
+ *  - Actions: DC_ACT_COMPUTE (full backbone evaluation) or DC_ACT_REUSE.
+ *  - The caller owns every pointer it passes; the library never keeps one
+ *    after the call returns, except the model's own device memory.
+ *  - Errors: calls return a dc_status and never abort.  Arguments are
+ *    validated before any device work; dc_last_error() gives a thread-local
+ *    message for the last failure on the calling thread.
+ *  - Host planner calls (dc_motion_stats .. dc_calibrate_budget) are pure
+ *    fp64 host code with no device dependency and are thread-safe.
+ */
+#ifndef DRIVECACHE_H
+#define DRIVECACHE_H
+
+#include <stddef.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  DC_OK = 0,
+  DC_ERR_INVALID_ARG = 1,
+  DC_ERR_NOMEM = 2,
+  DC_ERR_CUDA = 3,
+  DC_ERR_DEVICE_TIMEOUT = 4, /* a bounded device wait gave up */
+  DC_ERR_NONFINITE = 5,      /* a latent or drift statistic became NaN/Inf */
+  DC_ERR_UNSUPPORTED = 6     /* shape/dtype this build has no kernel for */
+} dc_status;
+
+enum { DC_ACT_COMPUTE = 1, DC_ACT_REUSE = 2 };
+enum { DC_DTYPE_F32 = 0, DC_DTYPE_BF16 = 1 };
+
+/* One planned ego pose: position in metres, heading in radians. */
+typedef struct { double x, y, psi; } dc_pose;
+
+/* A planned trajectory: n_poses consecutive poses (host memory). */
+typedef struct { const dc_pose* poses; int n_poses; } dc_trajectory;
+
+/* Calibrated anchor responses (Sec. 3.1-3.2).
+ *  (L0,T0), (L1,T1): low-motion and moving-turn anchor statistics (Eq. 2);
+ *  valid = 0 means no moving-turn anchor exists -> every scene runs full
+ *  inference.  q0/q1: joint run responses q^(i)_{j,h} (Eq. 7) of the two
+ *  anchors; d0/d1: anchor input drifts d^(i)_{j,h} (Eq. 5).  All four are
+ *  [K][H_max+1] (see conventions), finite and >= 0.
+ *  legal: optional [K+1][H_max+1] bytes, legal[k][h] != 0 iff reusing at
+ *  step k with cache age h is allowed (the L(k,h) mask of Eq. 10); NULL means
+ *  every age 1..H_max at every step k >= 2.  eps: the epsilon of Eq. 3 and of
+ *  the veto slack (1e-6 by default). */
+typedef struct {
+  int K, H_max;
+  double L0, T0, L1, T1;
+  int valid;
+  const double *q0, *q1, *d0, *d1;
+  const unsigned char* legal;
+  double eps;
+} dc_anchor_responses;
+
+/* A per-scene schedule.  action: caller-owned [T+1] bytes (index 0 unused). */
+typedef struct {
+  int T;
+  unsigned char* action;
+  int n_reuse;      /* number of REUSE steps */
+  double cost;      /* min_h J_T(n_reuse, h) of the plan (Eq. 10-11) */
+  int supported;    /* 1 iff (z^L, z^Theta) in [0,1]^2 and anchors valid */
+  double D;         /* motion intensity (Eq. 4); 0 when unsupported */
+  double L, Theta;  /* motion statistics (Eq. 2) */
+} dc_schedule;
+
+/* Eq. 2: total translation L = sum ||p_t - p_{t-1}|| and accumulated
+ * absolute wrapped yaw Theta = sum |wrap(psi_t - psi_{t-1})|, wrap into
+ * (-pi, pi].  Needs n_poses >= 1 and finite poses. */
+dc_status dc_motion_stats(const dc_trajectory* traj, double* L, double* Theta);
+
+/* Sec. 3.1 anchor selection over n >= 1 calibration clips' (L, Theta):
+ * population z-scores; low-motion anchor = argmin zL + zTheta; moving-turn
+ * anchor = argmax zL * zTheta among clips with Theta > median(Theta),
+ * L > L0 and Theta > Theta0; ties to the lowest index.  Writes
+ * anchors_out = {L0, T0, L1, T1}, *valid (0 = empty candidate set) and,
+ * if index_out != NULL, index_out = {i0, i1} (i1 = -1 when invalid). */
+dc_status dc_select_anchors(const double* L, const double* Theta, int n,
+                            double anchors_out[4], int* valid, int* index_out);
+
+/* Sec. 3.1-3.2: plan one scene.  Eq. 2 -> Eq. 3 support gate -> Eq. 4 ->
+ * Eq. 8/9 scene tables -> Eq. 10 DP from J_1(0,0) = 0 -> Eq. 11 B* under
+ * `budget` (tau) -> backtracking (ties: smallest final age, then smallest
+ * age before each refresh).  T must equal anc->K; out->action must hold T+1
+ * bytes.  An unsupported scene gets an all-COMPUTE schedule. */
+dc_status dc_plan(const dc_trajectory* traj, const dc_anchor_responses* anc, double budget,
+                  int T, dc_schedule* out);
+
+/* Sec. 3.2 suffix replanning after a forced full evaluation at step
+ * k_refresh: DP from J_{k_refresh}(0,0) = 0 over steps k_refresh..T under
+ * `remaining` (= tau - C_k) with the scene tables of intensity D.  Overwrites
+ * inout->action[k_refresh..T] (action[k_refresh] = COMPUTE) and leaves the
+ * prefix untouched; sets inout->n_reuse to the REUSE count of the whole
+ * action array and inout->cost to the suffix plan's cost. */
+dc_status dc_replan(const dc_anchor_responses* anc, double D, int k_refresh, double remaining,
+                    dc_schedule* inout);
+
+/* Sec. 3.2 budget calibration: the smallest table-cost threshold tau whose
+ * median B* over the n calibration clips reaches `target` reuses (callers
+ * pass target = ceil(rho_tar (T-1))).  Candidates are the finite
+ * min_h J_T(n, h) of every supported clip; unsupported clips count as zero
+ * reuses.  *reached = 0 if no candidate reaches the target, in which case
+ * *tau is the largest candidate. */
+dc_status dc_calibrate_budget(const dc_trajectory* clips, int n, const dc_anchor_responses* anc,
+                              int target, int T, double* tau, int* reached);
+
+/* ------------------------------------------------------------------ model */
+
+/* Shape of the synthetic DiT.  n_tokens = views x frames x rows x cols
+ * (patch 1); head_dim = d_model / n_heads must be 16, 64, 72 or 128 for
+ * bf16 and d_model % 4 == 0 for f32.  max_batch / max_steps bound the
+ * per-call workspace allocated by dc_model_create. */
+typedef struct {
+  int dtype;       /* DC_DTYPE_F32 or DC_DTYPE_BF16 */
+  int n_blocks, d_model, n_heads, mlp_ratio, channels, n_tokens, n_poses;
+  int max_batch, max_steps;
+} dc_model_desc;
+
+typedef struct dc_model dc_model;
+
+/* Number of floats dc_model_create expects in host_weights. */
+size_t dc_model_weight_count(const dc_model_desc* desc);
+
+/* Create a model on `device` (the caller's current CUDA device when < 0).
+ * host_weights: fp32, all tensors concatenated in this order, matrices
+ * [out][in] row-major:
+ *   w_embed[d][C] b_embed[d] pos[N][d] w_t1[d][256] b_t1[d] w_t2[d][d] b_t2[d]
+ *   w_traj[d][3P] b_traj[d] w_ada[(6L+2)d][d] b_ada[(6L+2)d]
+ *   per block l: w_qkv[3d][d] b_qkv[3d] w_o[d][d] b_o[d] w_1[md][d] b_1[md]
+ *                w_2[d][md] b_2[d]            (md = mlp_ratio d)
+ *   w_final[C][d] b_final[C]
+ * For bf16 models the values are converted to bf16 (round to nearest even).
+ * The model owns its weights and a workspace for max_batch scenes. */
+dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, size_t n_floats,
+                          int device, dc_model** out);
+void dc_model_destroy(dc_model* m);
+
+/* Per-scene conditioning: planned poses of each of the B scenes (host). */
+typedef struct { int B; const dc_trajectory* traj; } dc_cond;
+
+/* Sampler + controller settings for one dc_denoise call.
+ *  sigmas: [K+1] host doubles, sigma_1 .. sigma_{K+1} stored 0-based.
+ *  anchors: calibrated responses (anchors->K must equal K); tau: budget.
+ *  veto: 1 = check drift and charge before every planned reuse (Eq. 12);
+ *        0 = execute the plan as made.
+ *  forced: NULL, or [B][K+1] actions replayed verbatim (no planning, no
+ *        checks; step 1 is always computed). */
+typedef struct {
+  int K;
+  const double* sigmas;
+  const dc_anchor_responses* anchors;
+  double tau;
+  int veto;
+  const unsigned char* forced;
+} dc_sched;
+
+/* Optional per-call record (every pointer may be NULL; arrays caller-owned).
+ * [B][K+1] arrays are indexed [s*(K+1) + k]. */
+typedef struct {
+  unsigned char* planned;   /* [B][K+1] initial plan */
+  unsigned char* executed;  /* [B][K+1] executed actions */
+  double* d_obs;            /* [B][K+1] observed drift at checked steps, NaN elsewhere */
+  double* d_bar;            /* [B][K+1] threshold d_bar_{j,h} at checked steps */
+  unsigned char* checked;   /* [B][K+1] 0 unchecked, 1 accepted, 2 refused */
+  int* n_compute;           /* [B] */
+  int* n_reuse;             /* [B] */
+  int* n_veto;              /* [B] refused planned reuses */
+  int* n_replan;            /* [B] */
+  double* charge;           /* [B] final accumulated charge C */
+  int* supported;           /* [B] */
+  double* D;                /* [B] */
+  long long backbone_calls; /* out: scene-steps that ran the block stack */
+  long long launches;       /* out: kernels launched by the call */
+} dc_run_stats;
+
+/* Run the K-step Euler sampler on B <= max_batch scenes with the cache
+ * controller (Eq. 1, Sec. 3.2).  latents: DEVICE fp32 [B][N][C], x_1 in,
+ * x_{K+1} out.  stream: a cudaStream_t (NULL = legacy default stream).
+ * Device work is enqueued on `stream`; the call synchronises the stream once
+ * per step that has a planned reuse to read the drift statistics back, and
+ * once at the end.  Returns DC_ERR_NONFINITE if a drift statistic is not
+ * finite and DC_ERR_DEVICE_TIMEOUT if a bounded device wait gave up. */
+dc_status dc_denoise(dc_model* m, float* latents, const dc_cond* cond, const dc_sched* sched,
+                     void* stream, dc_run_stats* stats);
+
+/* dc_denoise on HOST latents: copies [B][N][C] fp32 to the device, runs the
+ * sampler, copies the result back into host_latents, synchronises `stream`.
+ * Page-locked host memory gives asynchronous copies; pageable also works. */
+dc_status dc_denoise_host(dc_model* m, float* host_latents, const dc_cond* cond,
+                          const dc_sched* sched, void* stream, dc_run_stats* stats);
+
+/* Eq. 5 along one full trace: run all K steps as full evaluations from
+ * `noise` (DEVICE fp32 [N][C], not modified) under `traj`, and write
+ * d_out[j*(H_max+1)+h] = ||u_{j+h} - u_j|| / (||u_{j+h}|| + eps) for
+ * j = 1..K-1, h = 1..min(H_max, K-j) (other entries 0).  Host d_out. */
+dc_status dc_anchor_drift(dc_model* m, const float* noise, const dc_trajectory* traj, int K,
+                          const double* sigmas, int H_max, double eps, double* d_out, void* stream);
+
+/* Drift sums for Eq. 12 on B scenes: for each scene s, out[2s] =
+ * sum ||u(x_now_s) - u(x_ref_s)||^2 = sum ||(x_now_s - x_ref_s) W_e^T||^2 and
+ * out[2s+1] = sum ||u(x_now_s)||^2 with u(x) = x W_e^T + b_e + pos, summed
+ * over all tokens and channels in fp32 in a fixed order (deterministic).
+ * x_now, x_ref: DEVICE fp32 [B][N][C]; out: DEVICE fp32 [2B].  The sums use
+ * the model's per-call workspace (B <= max_batch). */
+dc_status dc_drift_sums(dc_model* m, const float* x_now, const float* x_ref, int B, float* out,
+                        void* stream);
+
+/* Copy the cached backbone output r_j (Eq. 1: r = h_L - u of the scene's
+ * last full evaluation) of `scene` (0 <= scene < max_batch) into DEVICE
+ * memory dst.  The cache holds [N][d] elements of the model dtype (fp32 or
+ * bf16); `bytes` must equal N * d * sizeof(element).  Asynchronous on
+ * `stream`.  Intended for inspection and tests. */
+dc_status dc_cache_copy(dc_model* m, int scene, void* dst, size_t bytes, void* stream);
+
+/* The attention kernel of the block stack on caller-provided operands:
+ * o = softmax(q k^T / sqrt(head_dim)) v over all n_tokens of each
+ * (slot, head).  qkv: DEVICE [3][slots][heads][n_tokens][dhp] (q, k, v
+ * planes) with dhp = head_dim rounded up to a multiple of 16 for bf16 (pad
+ * columns must be zero) and dhp = head_dim for fp32; out: DEVICE
+ * [slots][n_tokens][heads * head_dim].  dtype DC_DTYPE_BF16 supports
+ * head_dim 64, 72, 128 (and 16); DC_DTYPE_F32 supports 8, 16, 32, 64. */
+dc_status dc_attention(int dtype, const void* qkv, int slots, int heads, int n_tokens,
+                       int head_dim, void* out, void* stream);
+
+/* Per-kernel timing of dc_denoise: when enabled, every launch is bracketed
+ * by CUDA events on the call's stream and, at the end of each dc_denoise
+ * call, its device time is added to its category together with the
+ * algorithmic work of the launch (flops for the contractions, bytes for the
+ * memory-bound kernels).  dc_profile(m, 1) resets the totals and starts
+ * recording; dc_profile(m, 0) stops.  dc_profile_read fills DC_PROF_N
+ * entries per array (any may be NULL). */
+enum {
+  DC_PROF_CONDITION = 0, /* timestep/trajectory MLPs + adaLN modulation table */
+  DC_PROF_EMBED,         /* u = x W_e^T + b_e + pos */
+  DC_PROF_LN,            /* adaLN LayerNorm + modulation */
+  DC_PROF_GEMM_QKV,      /* tcgen05 GEMM, QKV scatter epilogue */
+  DC_PROF_ATTENTION,     /* full spatiotemporal attention */
+  DC_PROF_GEMM_OUT,      /* out-projection GEMM + gated residual */
+  DC_PROF_GEMM_MLP1,     /* MLP-up GEMM + GELU */
+  DC_PROF_GEMM_MLP2,     /* MLP-down GEMM + gated residual */
+  DC_PROF_FINAL,         /* interface + Euler + cache write (compute steps) */
+  DC_PROF_REUSE,         /* reuse step: cached r + interface + Euler */
+  DC_PROF_DRIFT,         /* drift sums of Eq. 12 */
+  DC_PROF_N
+};
+dc_status dc_profile(dc_model* m, int enable);
+dc_status dc_profile_read(dc_model* m, double* ms, long long* launches, double* flops,
+                          double* bytes);
+
+const char* dc_status_string(dc_status s);
+const char* dc_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* DRIVECACHE_H */

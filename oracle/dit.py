@@ -117,6 +117,17 @@ def embed(w, x):
     return linear(x, w["w_embed"], w["b_embed"]) + f64(w["pos"])
 
 
+def attention_core(q, k, v):
+    """softmax(q k^T / sqrt(dh)) v per head; q, k, v: [heads][n][dh]."""
+    q, k, v = f64(q), f64(k), f64(v)
+    dh = q.shape[-1]
+    o = np.empty_like(q)
+    for hd in range(q.shape[0]):
+        p = softmax(q[hd] @ k[hd].T / math.sqrt(dh))
+        o[hd] = p @ v[hd]
+    return o
+
+
 def attention(a, w_qkv, b_qkv, n_heads):
     n, d = a.shape
     dh = d // n_heads
@@ -124,11 +135,7 @@ def attention(a, w_qkv, b_qkv, n_heads):
     q = qkv[:, :d].reshape(n, n_heads, dh).transpose(1, 0, 2)
     k = qkv[:, d:2 * d].reshape(n, n_heads, dh).transpose(1, 0, 2)
     v = qkv[:, 2 * d:].reshape(n, n_heads, dh).transpose(1, 0, 2)
-    o = np.empty((n_heads, n, dh))
-    for hd in range(n_heads):
-        p = softmax(q[hd] @ k[hd].T / math.sqrt(dh))
-        o[hd] = p @ v[hd]
-    return o.transpose(1, 0, 2).reshape(n, d)
+    return attention_core(q, k, v).transpose(1, 0, 2).reshape(n, d)
 
 
 def block(wb, h, mod, n_heads):

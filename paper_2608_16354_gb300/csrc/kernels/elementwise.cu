@@ -1,0 +1,579 @@
+// HBM-bound kernels of the hot path: conditioning (timestep + trajectory
+// features, small MLPs, adaLN modulation table), patch embedding, adaLN
+// LayerNorm, the interface + Euler update on compute and on reuse steps, and
+// the deterministic drift reduction of Eq. 12.
+//
+// Row-wise kernels use one warp per token row with float4 accesses; each
+// lane holds NV float4 of the row in registers (NV = ceil(d / 128)).
+#include <math.h>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace dc {
+
+namespace {
+
+constexpr double kPiD = 3.141592653589793238462643383279502884;
+
+// ------------------------------------------------------------ conditioning
+
+__global__ void pose_features_kernel(const double* __restrict__ poses, int B, int P,
+                                     float* __restrict__ out) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= B * P) return;
+  const int s = i / P, t = i - s * P;
+  const double* p0 = poses + (size_t)s * P * 3;
+  const double* pt = p0 + (size_t)t * 3;
+  double dpsi = remainder(pt[2] - p0[2], 2.0 * kPiD);
+  if (dpsi == -kPiD) dpsi = kPiD;
+  float* o = out + (size_t)s * 3 * P + 3 * t;
+  o[0] = (float)((pt[0] - p0[0]) / 10.0);
+  o[1] = (float)((pt[1] - p0[1]) / 10.0);
+  o[2] = (float)dpsi;
+}
+
+__global__ void temb_features_kernel(const double* __restrict__ sig, int K, float* __restrict__ out) {
+  const int k = blockIdx.x, i = threadIdx.x;  // 128 threads
+  if (k >= K) return;
+  const double t = 1000.0 * sig[k];
+  const double f = exp(-log(10000.0) * (double)i / 128.0);
+  out[(size_t)k * 256 + i] = (float)cos(t * f);
+  out[(size_t)k * 256 + 128 + i] = (float)sin(t * f);
+}
+
+template <typename TW>
+__global__ void rows_linear_kernel(const float* __restrict__ X, int R, int I,
+                                   const TW* __restrict__ W, const float* __restrict__ b, int O,
+                                   float* __restrict__ Y, int in_silu) {
+  const int o = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (o >= O) return;
+  const TW* w = W + (size_t)o * I;
+  constexpr int RT = 8;
+  for (int r0 = 0; r0 < R; r0 += RT) {
+    float acc[RT];
+#pragma unroll
+    for (int j = 0; j < RT; ++j) acc[j] = 0.f;
+    for (int i = lane; i < I; i += 32) {
+      const float wv = to_f(w[i]);
+#pragma unroll
+      for (int j = 0; j < RT; ++j) {
+        if (r0 + j < R) {
+          float xv = X[(size_t)(r0 + j) * I + i];
+          if (in_silu) xv = silu(xv);
+          acc[j] += xv * wv;
+        }
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < RT; ++j) {
+      const float v = warp_sum(acc[j]);
+      if (lane == 0 && r0 + j < R) Y[(size_t)(r0 + j) * O + o] = v + b[o];
+    }
+  }
+}
+
+__global__ void cond_combine_kernel(const float* __restrict__ temb, const float* __restrict__ traj,
+                                    int K, int B, int d, float* __restrict__ out) {
+  const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const size_t total = (size_t)K * B * d;
+  if (i >= total) return;
+  const int e = (int)(i % d);
+  const int s = (int)((i / d) % B);
+  const int k = (int)(i / ((size_t)d * B));
+  out[i] = silu(temb[(size_t)k * d + e] + traj[(size_t)s * d + e]);
+}
+
+// ------------------------------------------------------------- embedding
+
+template <typename T>
+__global__ void embed_kernel(const float* __restrict__ x, const float* __restrict__ w_e,
+                             const float* __restrict__ b_e, const T* __restrict__ pos, SlotMap map,
+                             int N, int C, int d, float* __restrict__ u, float* __restrict__ h) {
+  // one thread per 4 consecutive outputs of one token of one slot
+  const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int d4 = d >> 2;
+  const size_t total = (size_t)map.n * N * d4;
+  if (i >= total) return;
+  const int e4 = (int)(i % d4);
+  const size_t row = i / d4;  // slot * N + tok
+  const int slot = (int)(row / N), tok = (int)(row - (size_t)slot * N);
+  const float* xr = x + ((size_t)map.scene[slot] * N + tok) * C;
+  float acc[4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const int e = e4 * 4 + j;
+    float a = b_e[e] + to_f(pos[(size_t)tok * d + e]);
+    const float* w = w_e + (size_t)e * C;
+    for (int c = 0; c < C; ++c) a += w[c] * xr[c];
+    acc[j] = a;
+  }
+  const float4 v = make_float4(acc[0], acc[1], acc[2], acc[3]);
+  reinterpret_cast<float4*>(u)[i] = v;
+  reinterpret_cast<float4*>(h)[i] = v;
+}
+
+// --------------------------------------------------------------- LN + mod
+
+template <int NV>
+__device__ __forceinline__ void load_row(const float* __restrict__ src, int d4, int lane,
+                                         float4 (&v)[NV]) {
+#pragma unroll
+  for (int j = 0; j < NV; ++j) {
+    const int i = lane + 32 * j;
+    v[j] = i < d4 ? reinterpret_cast<const float4*>(src)[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+}
+
+// mean and rstd of the row held in registers (two-pass)
+template <int NV>
+__device__ __forceinline__ void row_stats(const float4 (&v)[NV], int d, int d4, int lane,
+                                          float* mean, float* rstd) {
+  float s = 0.f;
+#pragma unroll
+  for (int j = 0; j < NV; ++j) s += (v[j].x + v[j].y) + (v[j].z + v[j].w);
+  const float mu = warp_sum(s) / (float)d;
+  float q = 0.f;
+#pragma unroll
+  for (int j = 0; j < NV; ++j) {
+    if (lane + 32 * j < d4) {
+      const float a = v[j].x - mu, b = v[j].y - mu, c = v[j].z - mu, e = v[j].w - mu;
+      q += (a * a + b * b) + (c * c + e * e);
+    }
+  }
+  const float var = warp_sum(q) / (float)d;
+  *mean = mu;
+  *rstd = rsqrtf(var + 1e-6f);
+}
+
+template <typename T>
+__device__ __forceinline__ void store4(T* dst, float a, float b, float c, float d_);
+template <>
+__device__ __forceinline__ void store4<float>(float* dst, float a, float b, float c, float d_) {
+  *reinterpret_cast<float4*>(dst) = make_float4(a, b, c, d_);
+}
+template <>
+__device__ __forceinline__ void store4<__nv_bfloat16>(__nv_bfloat16* dst, float a, float b, float c,
+                                                      float d_) {
+  __align__(8) __nv_bfloat162 t[2] = {__floats2bfloat162_rn(a, b), __floats2bfloat162_rn(c, d_)};
+  *reinterpret_cast<uint2*>(dst) = *reinterpret_cast<const uint2*>(t);
+}
+
+template <typename T>
+__device__ __forceinline__ float4 load4(const T* src);
+template <>
+__device__ __forceinline__ float4 load4<float>(const float* src) {
+  return *reinterpret_cast<const float4*>(src);
+}
+template <>
+__device__ __forceinline__ float4 load4<__nv_bfloat16>(const __nv_bfloat16* src) {
+  const uint2 raw = *reinterpret_cast<const uint2*>(src);
+  const __nv_bfloat162* p = reinterpret_cast<const __nv_bfloat162*>(&raw);
+  const float2 a = __bfloat1622float2(p[0]), b = __bfloat1622float2(p[1]);
+  return make_float4(a.x, a.y, b.x, b.y);
+}
+
+template <typename T, int NV>
+__global__ void ln_mod_kernel(const float* __restrict__ h, int rows, int N, int d,
+                              const float* __restrict__ mod, int mod_stride, int shift_off,
+                              int scale_off, SlotMap map, T* __restrict__ a) {
+  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const int d4 = d >> 2;
+  float4 v[NV];
+  load_row<NV>(h + (size_t)row * d, d4, lane, v);
+  float mu, rs;
+  row_stats<NV>(v, d, d4, lane, &mu, &rs);
+  const int slot = row / N;
+  const float* mrow = mod + (size_t)map.scene[slot] * mod_stride;
+  const float4* sh = reinterpret_cast<const float4*>(mrow + shift_off);
+  const float4* sc = reinterpret_cast<const float4*>(mrow + scale_off);
+  T* dst = a + (size_t)row * d;
+#pragma unroll
+  for (int j = 0; j < NV; ++j) {
+    const int i = lane + 32 * j;
+    if (i < d4) {
+      const float4 s = sh[i], c = sc[i];
+      store4<T>(dst + 4 * i, (v[j].x - mu) * rs * (1.f + c.x) + s.x,
+                (v[j].y - mu) * rs * (1.f + c.y) + s.y, (v[j].z - mu) * rs * (1.f + c.z) + s.z,
+                (v[j].w - mu) * rs * (1.f + c.w) + s.w);
+    }
+  }
+}
+
+// ---------------------------------------------------- interface + Euler
+
+// v[c] = sum_e a_e w_f[c][e] + b_f[c] for the modulated, normalised row held
+// in registers; returns v[c] on every lane.
+template <int NV, int C>
+__device__ __forceinline__ void head_dot(const float4 (&a)[NV], int d, int d4, int lane,
+                                         const float* __restrict__ w_f,
+                                         const float* __restrict__ b_f, float (&v)[C]) {
+#pragma unroll
+  for (int c = 0; c < C; ++c) {
+    const float4* w = reinterpret_cast<const float4*>(w_f + (size_t)c * d);
+    float s = 0.f;
+#pragma unroll
+    for (int j = 0; j < NV; ++j) {
+      const int i = lane + 32 * j;
+      if (i < d4) {
+        const float4 ww = __ldg(w + i);
+        s += (a[j].x * ww.x + a[j].y * ww.y) + (a[j].z * ww.z + a[j].w * ww.w);
+      }
+    }
+    v[c] = warp_sum(s) + b_f[c];
+  }
+}
+
+template <int NV>
+__device__ __forceinline__ void modulate(float4 (&v)[NV], float mu, float rs, const float* mrow,
+                                         int shift_off, int scale_off, int d4, int lane) {
+  const float4* sh = reinterpret_cast<const float4*>(mrow + shift_off);
+  const float4* sc = reinterpret_cast<const float4*>(mrow + scale_off);
+#pragma unroll
+  for (int j = 0; j < NV; ++j) {
+    const int i = lane + 32 * j;
+    if (i < d4) {
+      const float4 s = sh[i], c = sc[i];
+      v[j].x = (v[j].x - mu) * rs * (1.f + c.x) + s.x;
+      v[j].y = (v[j].y - mu) * rs * (1.f + c.y) + s.y;
+      v[j].z = (v[j].z - mu) * rs * (1.f + c.z) + s.z;
+      v[j].w = (v[j].w - mu) * rs * (1.f + c.w) + s.w;
+    } else {
+      v[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+  }
+}
+
+template <typename T, int NV, int C>
+__global__ void final_compute_kernel(const float* __restrict__ hL, const float* __restrict__ u,
+                                     float* __restrict__ x, float* __restrict__ xj,
+                                     T* __restrict__ r, SlotMap map, int N, int d,
+                                     const float* __restrict__ mod, int mod_stride, int fin_off,
+                                     const float* __restrict__ w_f, const float* __restrict__ b_f,
+                                     float dsig) {
+  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;  // slot * N + tok
+  const int lane = threadIdx.x & 31;
+  if (row >= map.n * N) return;
+  const int slot = row / N, tok = row - slot * N;
+  const int scene = map.scene[slot];
+  const int d4 = d >> 2;
+  float4 hv[NV];
+  load_row<NV>(hL + (size_t)row * d, d4, lane, hv);
+  // cache the reusable backbone output r = h_L - u
+  {
+    const float4* up = reinterpret_cast<const float4*>(u + (size_t)row * d);
+    T* rd = r + ((size_t)scene * N + tok) * d;
+#pragma unroll
+    for (int j = 0; j < NV; ++j) {
+      const int i = lane + 32 * j;
+      if (i < d4) {
+        const float4 uu = up[i];
+        store4<T>(rd + 4 * i, hv[j].x - uu.x, hv[j].y - uu.y, hv[j].z - uu.z, hv[j].w - uu.w);
+      }
+    }
+  }
+  float mu, rs;
+  row_stats<NV>(hv, d, d4, lane, &mu, &rs);
+  modulate<NV>(hv, mu, rs, mod + (size_t)scene * mod_stride, fin_off, fin_off + d, d4, lane);
+  float v[C];
+  head_dot<NV, C>(hv, d, d4, lane, w_f, b_f, v);
+  if (lane < C) {
+    float vc = v[0];
+#pragma unroll
+    for (int c = 1; c < C; ++c)
+      if (lane == c) vc = v[c];
+    const size_t xi = ((size_t)scene * N + tok) * C + lane;
+    const float xo = x[xi];
+    xj[xi] = xo;
+    x[xi] = xo + dsig * vc;
+  }
+}
+
+template <typename T, int NV, int C>
+__global__ void final_reuse_kernel(float* __restrict__ x, const T* __restrict__ r,
+                                   const float* __restrict__ w_e, const float* __restrict__ b_e,
+                                   const T* __restrict__ pos, SlotMap map, int N, int d,
+                                   const float* __restrict__ mod, int mod_stride, int fin_off,
+                                   const float* __restrict__ w_f, const float* __restrict__ b_f,
+                                   float dsig) {
+  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (row >= map.n * N) return;
+  const int slot = row / N, tok = row - slot * N;
+  const int scene = map.scene[slot];
+  const int d4 = d >> 2;
+  const float* xr = x + ((size_t)scene * N + tok) * C;
+  float xv[C];
+#pragma unroll
+  for (int c = 0; c < C; ++c) xv[c] = xr[c];
+  const T* rr = r + ((size_t)scene * N + tok) * d;
+  const T* pr = pos + (size_t)tok * d;
+  float4 hv[NV];
+#pragma unroll
+  for (int j = 0; j < NV; ++j) {
+    const int i = lane + 32 * j;
+    if (i < d4) {
+      const float4 rv = load4<T>(rr + 4 * i);
+      const float4 pv = load4<T>(pr + 4 * i);
+      const float4 bv = reinterpret_cast<const float4*>(b_e)[i];
+      float o[4] = {bv.x + pv.x, bv.y + pv.y, bv.z + pv.z, bv.w + pv.w};
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float* w = w_e + (size_t)(4 * i + q) * C;
+#pragma unroll
+        for (int c = 0; c < C; ++c) o[q] += w[c] * xv[c];
+      }
+      hv[j] = make_float4(o[0] + rv.x, o[1] + rv.y, o[2] + rv.z, o[3] + rv.w);
+    } else {
+      hv[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+  }
+  float mu, rs;
+  row_stats<NV>(hv, d, d4, lane, &mu, &rs);
+  modulate<NV>(hv, mu, rs, mod + (size_t)scene * mod_stride, fin_off, fin_off + d, d4, lane);
+  float v[C];
+  head_dot<NV, C>(hv, d, d4, lane, w_f, b_f, v);
+  __syncwarp();
+  if (lane < C) {
+    float vc = v[0];
+#pragma unroll
+    for (int c = 1; c < C; ++c)
+      if (lane == c) vc = v[c];
+    float xo = xv[0];
+#pragma unroll
+    for (int c = 1; c < C; ++c)
+      if (lane == c) xo = xv[c];
+    x[((size_t)scene * N + tok) * C + lane] = xo + dsig * vc;
+  }
+}
+
+// ------------------------------------------------------------ drift sums
+
+template <typename T, int C>
+__global__ void drift_partial_kernel(DriftItems items, const float* __restrict__ w_e,
+                                     const float* __restrict__ b_e, const T* __restrict__ pos,
+                                     int N, int d, float* __restrict__ partials) {
+  const int part = blockIdx.x, item = blockIdx.y;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nw = blockDim.x >> 5;
+  const int per = (N + kDriftParts - 1) / kDriftParts;
+  const int t0 = part * per, t1 = min(N, t0 + per);
+  const float* xn = items.now[item];
+  const float* xr = items.ref[item];
+  float sd = 0.f, su = 0.f;
+  for (int t = t0 + warp; t < t1; t += nw) {
+    float xv[C], dv[C];
+#pragma unroll
+    for (int c = 0; c < C; ++c) {
+      xv[c] = xn[(size_t)t * C + c];
+      dv[c] = xv[c] - xr[(size_t)t * C + c];
+    }
+    for (int e = lane; e < d; e += 32) {
+      const float* w = w_e + (size_t)e * C;
+      float du = 0.f, uu = b_e[e] + to_f(pos[(size_t)t * d + e]);
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        du += w[c] * dv[c];
+        uu += w[c] * xv[c];
+      }
+      sd += du * du;
+      su += uu * uu;
+    }
+  }
+  __shared__ float red[32][2];
+  sd = warp_sum(sd);
+  su = warp_sum(su);
+  if (lane == 0) { red[warp][0] = sd; red[warp][1] = su; }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float a = 0.f, b = 0.f;
+    for (int w = 0; w < nw; ++w) { a += red[w][0]; b += red[w][1]; }
+    partials[((size_t)item * kDriftParts + part) * 2 + 0] = a;
+    partials[((size_t)item * kDriftParts + part) * 2 + 1] = b;
+  }
+}
+
+__global__ void drift_final_kernel(const float* __restrict__ partials, int n, float* __restrict__ out) {
+  const int item = blockIdx.x * blockDim.x + threadIdx.x;
+  if (item >= n) return;
+  float a = 0.f, b = 0.f;
+  for (int p = 0; p < kDriftParts; ++p) {
+    a += partials[((size_t)item * kDriftParts + p) * 2 + 0];
+    b += partials[((size_t)item * kDriftParts + p) * 2 + 1];
+  }
+  out[2 * item] = a;
+  out[2 * item + 1] = b;
+}
+
+int nv_for(int d) {
+  const int need = (d / 4 + 31) / 32;
+  const int opts[] = {1, 2, 3, 4, 6, 8, 9, 12, 16, 24};
+  for (int o : opts)
+    if (o >= need) return o;
+  return -1;
+}
+
+#define DC_NV_SWITCH(nv, ...)                        \
+  switch (nv) {                                      \
+    case 1: { constexpr int NV = 1; __VA_ARGS__; } break;   \
+    case 2: { constexpr int NV = 2; __VA_ARGS__; } break;   \
+    case 3: { constexpr int NV = 3; __VA_ARGS__; } break;   \
+    case 4: { constexpr int NV = 4; __VA_ARGS__; } break;   \
+    case 6: { constexpr int NV = 6; __VA_ARGS__; } break;   \
+    case 8: { constexpr int NV = 8; __VA_ARGS__; } break;   \
+    case 9: { constexpr int NV = 9; __VA_ARGS__; } break;   \
+    case 12: { constexpr int NV = 12; __VA_ARGS__; } break; \
+    case 16: { constexpr int NV = 16; __VA_ARGS__; } break; \
+    case 24: { constexpr int NV = 24; __VA_ARGS__; } break; \
+    default: return cudaErrorInvalidValue;           \
+  }
+
+}  // namespace
+
+cudaError_t launch_pose_features(const double* poses, int B, int P, float* out, cudaStream_t st) {
+  const int n = B * P;
+  pose_features_kernel<<<(n + 127) / 128, 128, 0, st>>>(poses, B, P, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_temb_features(const double* sigmas, int K, float* out, cudaStream_t st) {
+  temb_features_kernel<<<K, 128, 0, st>>>(sigmas, K, out);
+  return cudaGetLastError();
+}
+
+template <typename TW>
+cudaError_t launch_rows_linear(const float* X, int R, int I, const TW* W, const float* b, int O,
+                               float* Y, int in_silu, cudaStream_t st) {
+  const int threads = 256;
+  const int blocks = (int)(((size_t)O * 32 + threads - 1) / threads);
+  rows_linear_kernel<TW><<<blocks, threads, 0, st>>>(X, R, I, W, b, O, Y, in_silu);
+  return cudaGetLastError();
+}
+template cudaError_t launch_rows_linear<float>(const float*, int, int, const float*, const float*,
+                                               int, float*, int, cudaStream_t);
+template cudaError_t launch_rows_linear<__nv_bfloat16>(const float*, int, int, const __nv_bfloat16*,
+                                                       const float*, int, float*, int, cudaStream_t);
+
+cudaError_t launch_cond_combine(const float* temb, const float* traj, int K, int B, int d,
+                                float* silu_c, cudaStream_t st) {
+  const size_t n = (size_t)K * B * d;
+  cond_combine_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(temb, traj, K, B, d, silu_c);
+  return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t launch_embed(const float* x, const float* w_e, const float* b_e, const T* pos,
+                         const SlotMap& map, int N, int C, int d, float* u, float* h,
+                         cudaStream_t st) {
+  if (map.n <= 0) return cudaSuccess;
+  const size_t n = (size_t)map.n * N * (d / 4);
+  embed_kernel<T><<<(unsigned)((n + 255) / 256), 256, 0, st>>>(x, w_e, b_e, pos, map, N, C, d, u, h);
+  return cudaGetLastError();
+}
+template cudaError_t launch_embed<float>(const float*, const float*, const float*, const float*,
+                                         const SlotMap&, int, int, int, float*, float*, cudaStream_t);
+template cudaError_t launch_embed<__nv_bfloat16>(const float*, const float*, const float*,
+                                                 const __nv_bfloat16*, const SlotMap&, int, int,
+                                                 int, float*, float*, cudaStream_t);
+
+template <typename T>
+cudaError_t launch_ln_mod(const float* h, int rows, int N, int d, const float* mod, int mod_stride,
+                          int shift_off, int scale_off, const SlotMap& map, T* a, cudaStream_t st) {
+  if (rows <= 0) return cudaSuccess;
+  const int threads = 256;
+  const int blocks = (int)(((size_t)rows * 32 + threads - 1) / threads);
+  DC_NV_SWITCH(nv_for(d), (ln_mod_kernel<T, NV><<<blocks, threads, 0, st>>>(
+                              h, rows, N, d, mod, mod_stride, shift_off, scale_off, map, a)));
+  return cudaGetLastError();
+}
+template cudaError_t launch_ln_mod<float>(const float*, int, int, int, const float*, int, int, int,
+                                          const SlotMap&, float*, cudaStream_t);
+template cudaError_t launch_ln_mod<__nv_bfloat16>(const float*, int, int, int, const float*, int,
+                                                  int, int, const SlotMap&, __nv_bfloat16*,
+                                                  cudaStream_t);
+
+template <typename T>
+cudaError_t launch_final_compute(const float* hL, const float* u, float* x, float* xj, T* r,
+                                 const SlotMap& map, int N, int C, int d, const float* mod,
+                                 int mod_stride, int fin_off, const float* w_f, const float* b_f,
+                                 float dsig, cudaStream_t st) {
+  if (map.n <= 0) return cudaSuccess;
+  const int rows = map.n * N;
+  const int threads = 256;
+  const int blocks = (int)(((size_t)rows * 32 + threads - 1) / threads);
+  if (C == 16) {
+    DC_NV_SWITCH(nv_for(d), (final_compute_kernel<T, NV, 16><<<blocks, threads, 0, st>>>(
+                                hL, u, x, xj, r, map, N, d, mod, mod_stride, fin_off, w_f, b_f, dsig)));
+  } else if (C == 4) {
+    DC_NV_SWITCH(nv_for(d), (final_compute_kernel<T, NV, 4><<<blocks, threads, 0, st>>>(
+                                hL, u, x, xj, r, map, N, d, mod, mod_stride, fin_off, w_f, b_f, dsig)));
+  } else {
+    return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+template cudaError_t launch_final_compute<float>(const float*, const float*, float*, float*, float*,
+                                                 const SlotMap&, int, int, int, const float*, int,
+                                                 int, const float*, const float*, float, cudaStream_t);
+template cudaError_t launch_final_compute<__nv_bfloat16>(const float*, const float*, float*, float*,
+                                                         __nv_bfloat16*, const SlotMap&, int, int,
+                                                         int, const float*, int, int, const float*,
+                                                         const float*, float, cudaStream_t);
+
+template <typename T>
+cudaError_t launch_final_reuse(float* x, const T* r, const float* w_e, const float* b_e,
+                               const T* pos, const SlotMap& map, int N, int C, int d,
+                               const float* mod, int mod_stride, int fin_off, const float* w_f,
+                               const float* b_f, float dsig, cudaStream_t st) {
+  if (map.n <= 0) return cudaSuccess;
+  const int rows = map.n * N;
+  const int threads = 256;
+  const int blocks = (int)(((size_t)rows * 32 + threads - 1) / threads);
+  if (C == 16) {
+    DC_NV_SWITCH(nv_for(d), (final_reuse_kernel<T, NV, 16><<<blocks, threads, 0, st>>>(
+                                x, r, w_e, b_e, pos, map, N, d, mod, mod_stride, fin_off, w_f, b_f, dsig)));
+  } else if (C == 4) {
+    DC_NV_SWITCH(nv_for(d), (final_reuse_kernel<T, NV, 4><<<blocks, threads, 0, st>>>(
+                                x, r, w_e, b_e, pos, map, N, d, mod, mod_stride, fin_off, w_f, b_f, dsig)));
+  } else {
+    return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+template cudaError_t launch_final_reuse<float>(float*, const float*, const float*, const float*,
+                                               const float*, const SlotMap&, int, int, int,
+                                               const float*, int, int, const float*, const float*,
+                                               float, cudaStream_t);
+template cudaError_t launch_final_reuse<__nv_bfloat16>(float*, const __nv_bfloat16*, const float*,
+                                                       const float*, const __nv_bfloat16*,
+                                                       const SlotMap&, int, int, int, const float*,
+                                                       int, int, const float*, const float*, float,
+                                                       cudaStream_t);
+
+template <typename T>
+cudaError_t launch_drift(const DriftItems& items, const float* w_e, const float* b_e, const T* pos,
+                         int N, int C, int d, float* partials, float* out, cudaStream_t st) {
+  if (items.n <= 0) return cudaSuccess;
+  dim3 grid(kDriftParts, items.n);
+  if (C == 16) {
+    drift_partial_kernel<T, 16><<<grid, 256, 0, st>>>(items, w_e, b_e, pos, N, d, partials);
+  } else if (C == 4) {
+    drift_partial_kernel<T, 4><<<grid, 256, 0, st>>>(items, w_e, b_e, pos, N, d, partials);
+  } else {
+    return cudaErrorInvalidValue;
+  }
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  drift_final_kernel<<<(items.n + 63) / 64, 64, 0, st>>>(partials, items.n, out);
+  return cudaGetLastError();
+}
+template cudaError_t launch_drift<float>(const DriftItems&, const float*, const float*, const float*,
+                                         int, int, int, float*, float*, cudaStream_t);
+template cudaError_t launch_drift<__nv_bfloat16>(const DriftItems&, const float*, const float*,
+                                                 const __nv_bfloat16*, int, int, int, float*,
+                                                 float*, cudaStream_t);
+
+}  // namespace dc

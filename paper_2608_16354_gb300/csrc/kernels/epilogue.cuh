@@ -1,0 +1,79 @@
+// Fused GEMM epilogues of the DiT block (shared by the tcgen05 bf16 GEMM and
+// the fp32 SIMT GEMM).  Each works on 8 consecutive output columns of one row.
+//
+//  kEpiQKV  : y = acc + b, scattered head-major into q / k / v
+//             [3][slots][heads][tokens][dh_pad]
+//  kEpiGELU : y = gelu_tanh(acc + b)             -> [rows][N]
+//  kEpiResid: h[row][col] += gate[scene][col] * (acc + b)   (fp32 residual)
+#pragma once
+
+#include "common.cuh"
+
+namespace dc {
+
+enum { kEpiQKV = 0, kEpiGELU = 1, kEpiResid = 2 };
+
+struct EpiArgs {
+  int M, N;            // valid rows / cols of the product
+  int n_tok;           // tokens per slot (row -> slot = row / n_tok)
+  const float* bias;   // [N]
+  void* out;           // QKV: q/k/v base; GELU: [M][N]
+  int d, heads, dh, dhp, nslots;  // QKV layout
+  float* h;            // Resid: fp32 residual [M][N]
+  const float* mod;    // Resid: modulation table of this step [B][mod_stride]
+  int mod_stride;      // floats per scene in the table
+  int gate_off;        // offset of this block's gate vector inside a scene's row
+};
+
+template <typename T> struct Pack8;
+template <> struct Pack8<__nv_bfloat16> {
+  static __device__ __forceinline__ void store(__nv_bfloat16* p, const float* v) {
+    __align__(16) __nv_bfloat162 t[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) t[i] = __floats2bfloat162_rn(v[2 * i], v[2 * i + 1]);
+    *reinterpret_cast<uint4*>(p) = *reinterpret_cast<const uint4*>(t);
+  }
+};
+template <> struct Pack8<float> {
+  static __device__ __forceinline__ void store(float* p, const float* v) {
+    reinterpret_cast<float4*>(p)[0] = make_float4(v[0], v[1], v[2], v[3]);
+    reinterpret_cast<float4*>(p)[1] = make_float4(v[4], v[5], v[6], v[7]);
+  }
+};
+
+template <int MODE, typename T>
+__device__ __forceinline__ void epilogue8(const EpiArgs& e, const SlotMap& map, int row, int col,
+                                          float (&v)[8]) {
+  const float4 b0 = *reinterpret_cast<const float4*>(e.bias + col);
+  const float4 b1 = *reinterpret_cast<const float4*>(e.bias + col + 4);
+  v[0] += b0.x; v[1] += b0.y; v[2] += b0.z; v[3] += b0.w;
+  v[4] += b1.x; v[5] += b1.y; v[6] += b1.z; v[7] += b1.w;
+  if constexpr (MODE == kEpiQKV) {
+    const int which = col / e.d;
+    const int within = col - which * e.d;
+    const int head = within / e.dh;
+    const int c = within - head * e.dh;
+    const int slot = row / e.n_tok;
+    const int tok = row - slot * e.n_tok;
+    T* dst = reinterpret_cast<T*>(e.out) +
+             ((((size_t)which * e.nslots + slot) * e.heads + head) * e.n_tok + tok) * e.dhp + c;
+    Pack8<T>::store(dst, v);
+  } else if constexpr (MODE == kEpiGELU) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = gelu_tanh(v[i]);
+    Pack8<T>::store(reinterpret_cast<T*>(e.out) + (size_t)row * e.N + col, v);
+  } else {
+    const int slot = row / e.n_tok;
+    const float* g = e.mod + (size_t)map.scene[slot] * e.mod_stride + e.gate_off + col;
+    const float4 g0 = *reinterpret_cast<const float4*>(g);
+    const float4 g1 = *reinterpret_cast<const float4*>(g + 4);
+    float4* hp = reinterpret_cast<float4*>(e.h + (size_t)row * e.N + col);
+    float4 h0 = hp[0], h1 = hp[1];
+    h0.x += g0.x * v[0]; h0.y += g0.y * v[1]; h0.z += g0.z * v[2]; h0.w += g0.w * v[3];
+    h1.x += g1.x * v[4]; h1.y += g1.y * v[5]; h1.z += g1.z * v[6]; h1.w += g1.w * v[7];
+    hp[0] = h0;
+    hp[1] = h1;
+  }
+}
+
+}  // namespace dc

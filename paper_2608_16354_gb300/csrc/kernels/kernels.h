@@ -1,0 +1,77 @@
+// Launchers of the device kernels (host-callable, all asynchronous on `st`).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+#include "epilogue.cuh"
+
+namespace dc {
+
+// ---- conditioning (once per dc_denoise call) -------------------------
+// pose features (dx/10, dy/10, wrap(dpsi)) of B trajectories [B][P][3] fp64
+cudaError_t launch_pose_features(const double* poses, int B, int P, float* out, cudaStream_t st);
+// sinusoidal features of t = 1000 sigma for K sigmas -> [K][256]
+cudaError_t launch_temb_features(const double* sigmas, int K, float* out, cudaStream_t st);
+// Y[r][o] = sum_i act(X[r][i]) W[o][i] + b[o]  (act = silu if in_silu), W fp32 or bf16
+template <typename TW>
+cudaError_t launch_rows_linear(const float* X, int R, int I, const TW* W, const float* b, int O,
+                               float* Y, int in_silu, cudaStream_t st);
+// c[k][s] = temb[k] + traj[s]; out = silu(c)   ([K][B][d])
+cudaError_t launch_cond_combine(const float* temb, const float* traj, int K, int B, int d,
+                                float* silu_c, cudaStream_t st);
+
+// ---- per-step kernels --------------------------------------------------
+// u = x W_e^T + b_e + pos (fp32) for each compute slot; h = u
+template <typename T>
+cudaError_t launch_embed(const float* x, const float* w_e, const float* b_e, const T* pos,
+                         const SlotMap& map, int N, int C, int d, float* u, float* h,
+                         cudaStream_t st);
+// a = LN(h) * (1 + scale) + shift  (per-slot modulation)  -> T
+template <typename T>
+cudaError_t launch_ln_mod(const float* h, int rows, int N, int d, const float* mod, int mod_stride,
+                          int shift_off, int scale_off, const SlotMap& map, T* a, cudaStream_t st);
+// GEMMs
+cudaError_t launch_gemm_tc(int mode, const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N,
+                           int K, const EpiArgs& ep, const SlotMap& map, int* err, int n_sms,
+                           cudaStream_t st);
+cudaError_t launch_gemm_f32(int mode, const float* A, const float* W, int M, int N, int K,
+                            const EpiArgs& ep, const SlotMap& map, cudaStream_t st);
+size_t gemm_tc_smem_bytes();
+int gemm_tc_tile_n();
+int gemm_tc_tile_k();
+int gemm_tc_tile_m();
+// attention: q/k/v [3][slots][heads][N][dhp] -> o [slots][N][heads*dh]
+cudaError_t launch_attention_bf16(const __nv_bfloat16* qkv, int slots, int heads, int N, int dh,
+                                  int dhp, __nv_bfloat16* o, cudaStream_t st);
+cudaError_t launch_attention_f32(const float* qkv, int slots, int heads, int N, int dh, int dhp,
+                                 float* o, cudaStream_t st);
+// compute-step interface + Euler: v = head(h_L); x_j <- x; x += dsig v; r <- h_L - u
+template <typename T>
+cudaError_t launch_final_compute(const float* hL, const float* u, float* x, float* xj, T* r,
+                                 const SlotMap& map, int N, int C, int d, const float* mod,
+                                 int mod_stride, int fin_off, const float* w_f, const float* b_f,
+                                 float dsig, cudaStream_t st);
+// reuse step: u = embed(x); h = u + r_j; v = head(h); x += dsig v
+template <typename T>
+cudaError_t launch_final_reuse(float* x, const T* r, const float* w_e, const float* b_e,
+                               const T* pos, const SlotMap& map, int N, int C, int d,
+                               const float* mod, int mod_stride, int fin_off, const float* w_f,
+                               const float* b_f, float dsig, cudaStream_t st);
+
+// drift sums over items: out[2i] = sum ||(now_i - ref_i) W_e^T||^2,
+// out[2i+1] = sum ||now_i W_e^T + b_e + pos||^2   (deterministic order)
+struct DriftItems {
+  int n;
+  const float* now[kMaxBatch];
+  const float* ref[kMaxBatch];
+};
+constexpr int kDriftParts = 64;
+template <typename T>
+cudaError_t launch_drift(const DriftItems& items, const float* w_e, const float* b_e, const T* pos,
+                         int N, int C, int d, float* partials /* [n][kDriftParts][2] */,
+                         float* out /* [2n] */, cudaStream_t st);
+
+}  // namespace dc

@@ -1,0 +1,955 @@
+// Sampler runtime of the DriveCache hot path: model construction (weights to
+// HBM, TMA descriptors), and the K-step Euler sampler with the causal cache
+// controller (Eq. 1, Eq. 12, Sec. 3.2).
+//
+// Per step: scenes whose plan says REUSE are checked first (drift sums on
+// the device, one readback, fp64 decision on the host); refused reuses turn
+// into full evaluations and the scene's suffix is replanned.  Scenes that
+// compute are packed into slots 0..n-1 of the activation workspace and run
+// the block stack together; reusing scenes run the fused reuse kernel.
+// Everything is enqueued on the caller's stream.
+
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "drivecache.h"
+#include "kernels/kernels.h"
+#include "plan/planner.h"
+
+using dc::SlotMap;
+
+struct BlockW {
+  void *w_qkv, *w_o, *w_1, *w_2;
+  float *b_qkv, *b_o, *b_1, *b_2;
+  CUtensorMap tm_qkv, tm_o, tm_1, tm_2;
+};
+
+struct dc_model {
+  dc_model_desc desc{};
+  int device = 0, n_sms = 0;
+  bool bf16 = false;
+  int N = 0, C = 0, d = 0, L = 0, heads = 0, dh = 0, dhp = 0, md = 0, P = 0, Bmax = 0, Kmax = 0;
+  int mod_stride = 0;
+  size_t elt = 4;
+  // weights
+  void* wbuf = nullptr;
+  float *w_e = nullptr, *b_e = nullptr, *w_t1 = nullptr, *b_t1 = nullptr, *w_t2 = nullptr,
+        *b_t2 = nullptr, *w_traj = nullptr, *b_traj = nullptr, *b_ada = nullptr, *w_f = nullptr,
+        *b_f = nullptr;
+  void *pos = nullptr, *w_ada = nullptr;
+  std::vector<BlockW> blk;
+  // workspace
+  void* ws = nullptr;
+  float *u = nullptr, *h = nullptr, *xj = nullptr, *mod = nullptr, *silu_c = nullptr,
+        *temb_f = nullptr, *temb_h = nullptr, *temb = nullptr, *pose_f = nullptr, *traj = nullptr,
+        *drift_part = nullptr, *drift_out = nullptr, *lat_stage = nullptr;
+  void *a = nullptr, *qkv = nullptr, *o = nullptr, *m = nullptr, *r = nullptr;
+  double *poses_d = nullptr, *sig_d = nullptr;
+  int* err_d = nullptr;
+  float* drift_host = nullptr;  // pinned
+  CUtensorMap tm_a, tm_oact, tm_m;
+  long long launches = 0;
+  // per-kernel profiling (dc_profile)
+  struct ProfRec { int cat; cudaEvent_t a, b; double flops, bytes; };
+  bool prof_on = false;
+  std::vector<cudaEvent_t> ev_pool;
+  std::vector<ProfRec> prof_pending;
+  double prof_ms[DC_PROF_N] = {}, prof_flops[DC_PROF_N] = {}, prof_bytes[DC_PROF_N] = {};
+  long long prof_cnt[DC_PROF_N] = {};
+};
+
+namespace {
+
+#define DC_CK(expr)                                                                \
+  do {                                                                             \
+    cudaError_t e_ = (expr);                                                       \
+    if (e_ != cudaSuccess) {                                                       \
+      dc::set_error(std::string(#expr) + ": " + cudaGetErrorString(e_));           \
+      return DC_ERR_CUDA;                                                          \
+    }                                                                              \
+  } while (0)
+
+#define DC_TRY(expr)                    \
+  do {                                  \
+    dc_status s_ = (expr);              \
+    if (s_ != DC_OK) return s_;         \
+  } while (0)
+
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+cudaEvent_t take_event(dc_model* m) {
+  if (!m->ev_pool.empty()) {
+    cudaEvent_t e = m->ev_pool.back();
+    m->ev_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+  return e;
+}
+
+dc_status prof_start(dc_model* m, cudaStream_t st, cudaEvent_t* ev) {
+  *ev = nullptr;
+  if (!m->prof_on) return DC_OK;
+  *ev = take_event(m);
+  if (!*ev) { dc::set_error("cudaEventCreate failed"); return DC_ERR_CUDA; }
+  DC_CK(cudaEventRecord(*ev, st));
+  return DC_OK;
+}
+
+dc_status prof_stop(dc_model* m, int cat, cudaStream_t st, cudaEvent_t a, double flops,
+                    double bytes) {
+  if (!m->prof_on || !a) return DC_OK;
+  cudaEvent_t b = take_event(m);
+  if (!b) { dc::set_error("cudaEventCreate failed"); return DC_ERR_CUDA; }
+  DC_CK(cudaEventRecord(b, st));
+  m->prof_pending.push_back({cat, a, b, flops, bytes});
+  return DC_OK;
+}
+
+// after the stream has been synchronised: fold pending timings into totals
+void prof_flush(dc_model* m) {
+  for (auto& r : m->prof_pending) {
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, r.a, r.b) == cudaSuccess) {
+      m->prof_ms[r.cat] += ms;
+      m->prof_flops[r.cat] += r.flops;
+      m->prof_bytes[r.cat] += r.bytes;
+      m->prof_cnt[r.cat] += 1;
+    }
+    m->ev_pool.push_back(r.a);
+    m->ev_pool.push_back(r.b);
+  }
+  m->prof_pending.clear();
+}
+
+// Launch one kernel (or a fixed pair) with optional per-category timing.
+#define DC_LAUNCH(cat, flops, bytes, expr)                           \
+  do {                                                               \
+    cudaEvent_t ev_ = nullptr;                                       \
+    DC_TRY(prof_start(m, st, &ev_));                                 \
+    DC_CK(expr);                                                     \
+    DC_TRY(prof_stop(m, (cat), st, ev_, (double)(flops), (double)(bytes))); \
+  } while (0)
+
+PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    cudaDriverEntryPointQueryResult q;
+    void* p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 2-D bf16 K-major operand [rows][inner], box 64 x box_rows, 128-byte swizzle.
+dc_status make_map(CUtensorMap* map, const void* ptr, uint64_t inner, uint64_t rows,
+                   uint32_t box_rows) {
+  auto enc = get_encode();
+  if (!enc) {
+    dc::set_error("cuTensorMapEncodeTiled is unavailable");
+    return DC_ERR_CUDA;
+  }
+  cuuint64_t dims[2] = {inner, rows};
+  cuuint64_t strides[1] = {inner * 2};
+  cuuint32_t box[2] = {64, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides,
+                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    dc::set_error("cuTensorMapEncodeTiled failed with CUresult " + std::to_string((int)r));
+    return DC_ERR_CUDA;
+  }
+  return DC_OK;
+}
+
+uint16_t f2bf_host(float f) {
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  if ((u & 0x7F800000u) == 0x7F800000u && (u & 0x7FFFFFu)) return (uint16_t)((u >> 16) | 0x40);
+  const uint32_t lsb = (u >> 16) & 1u;
+  u += 0x7FFFu + lsb;
+  return (uint16_t)(u >> 16);
+}
+
+dc_status check_desc(const dc_model_desc* d) {
+  if (!d) { dc::set_error("desc is NULL"); return DC_ERR_INVALID_ARG; }
+  if (d->dtype != DC_DTYPE_F32 && d->dtype != DC_DTYPE_BF16) {
+    dc::set_error("dtype must be DC_DTYPE_F32 or DC_DTYPE_BF16");
+    return DC_ERR_INVALID_ARG;
+  }
+  if (d->n_blocks < 1 || d->d_model < 8 || d->n_heads < 1 || d->mlp_ratio < 1 ||
+      d->channels < 1 || d->n_tokens < 1 || d->n_poses < 1 || d->max_batch < 1 ||
+      d->max_steps < 1 || d->d_model % d->n_heads != 0) {
+    dc::set_error("model shape fields must be positive and d_model divisible by n_heads");
+    return DC_ERR_INVALID_ARG;
+  }
+  if (d->max_batch > dc::kMaxBatch) {
+    dc::set_error("max_batch above " + std::to_string(dc::kMaxBatch));
+    return DC_ERR_UNSUPPORTED;
+  }
+  if (d->channels != 4 && d->channels != 16) {
+    dc::set_error("channels must be 4 or 16");
+    return DC_ERR_UNSUPPORTED;
+  }
+  const int dh = d->d_model / d->n_heads;
+  if (d->d_model % 4 != 0 || d->d_model > 3072) {
+    dc::set_error("d_model must be a multiple of 4 and <= 3072");
+    return DC_ERR_UNSUPPORTED;
+  }
+  if (d->dtype == DC_DTYPE_BF16) {
+    if (d->d_model % 192 != 0 || (d->mlp_ratio * d->d_model) % 192 != 0 ||
+        !(dh == 64 || dh == 72 || dh == 128)) {
+      dc::set_error("bf16 kernels need d_model % 192 == 0 and head_dim in {64, 72, 128}");
+      return DC_ERR_UNSUPPORTED;
+    }
+  } else {
+    if (d->d_model % 8 != 0 || !(dh == 8 || dh == 16 || dh == 32 || dh == 64)) {
+      dc::set_error("fp32 kernels need d_model % 8 == 0 and head_dim in {8, 16, 32, 64}");
+      return DC_ERR_UNSUPPORTED;
+    }
+  }
+  return DC_OK;
+}
+
+struct WeightLayout {
+  struct T { const char* name; size_t n; bool big; };
+  std::vector<T> t;
+  size_t total = 0;
+};
+
+void weight_layout(const dc_model_desc& d, WeightLayout* w) {
+  const size_t D = d.d_model, Cc = d.channels, L = d.n_blocks, N = d.n_tokens,
+               M = (size_t)d.mlp_ratio * D, P = d.n_poses;
+  auto add = [&](const char* n, size_t cnt, bool big) { w->t.push_back({n, cnt, big}); w->total += cnt; };
+  add("w_embed", D * Cc, false); add("b_embed", D, false); add("pos", N * D, true);
+  add("w_t1", D * 256, false); add("b_t1", D, false);
+  add("w_t2", D * D, false); add("b_t2", D, false);
+  add("w_traj", D * 3 * P, false); add("b_traj", D, false);
+  add("w_ada", (6 * L + 2) * D * D, true); add("b_ada", (6 * L + 2) * D, false);
+  for (size_t l = 0; l < L; ++l) {
+    add("w_qkv", 3 * D * D, true); add("b_qkv", 3 * D, false);
+    add("w_o", D * D, true); add("b_o", D, false);
+    add("w_1", M * D, true); add("b_1", M, false);
+    add("w_2", D * M, true); add("b_2", D, false);
+  }
+  add("w_final", Cc * D, false); add("b_final", Cc, false);
+}
+
+template <typename T>
+dc_status enqueue_conditioning(dc_model* m, int B, int K, cudaStream_t st) {
+  const int d = m->d;
+  cudaEvent_t ev = nullptr;
+  DC_TRY(prof_start(m, st, &ev));
+  DC_CK(dc::launch_temb_features(m->sig_d, K, m->temb_f, st));
+  DC_CK(dc::launch_rows_linear<float>(m->temb_f, K, 256, m->w_t1, m->b_t1, d, m->temb_h, 0, st));
+  DC_CK(dc::launch_rows_linear<float>(m->temb_h, K, d, m->w_t2, m->b_t2, d, m->temb, 1, st));
+  DC_CK(dc::launch_pose_features(m->poses_d, B, m->P, m->pose_f, st));
+  DC_CK(dc::launch_rows_linear<float>(m->pose_f, B, 3 * m->P, m->w_traj, m->b_traj, d, m->traj, 0,
+                                      st));
+  DC_CK(dc::launch_cond_combine(m->temb, m->traj, K, B, d, m->silu_c, st));
+  DC_CK(dc::launch_rows_linear<T>(m->silu_c, K * B, d, static_cast<const T*>(m->w_ada), m->b_ada,
+                                  m->mod_stride, m->mod, 0, st));
+  // algorithmic bytes: the adaLN weight table read once + the table written
+  DC_TRY(prof_stop(m, DC_PROF_CONDITION, st, ev, 2.0 * K * B * d * m->mod_stride,
+                   (double)m->mod_stride * d * m->elt + 4.0 * K * B * m->mod_stride));
+  m->launches += 7;
+  return DC_OK;
+}
+
+// One full backbone pass + interface + Euler for the scenes in `map`.
+template <typename T>
+dc_status enqueue_compute(dc_model* m, float* lat, const float* mod_k, const SlotMap& map,
+                          float dsig, cudaStream_t st) {
+  const int N = m->N, d = m->d, nc = map.n, M = nc * N;
+  if (nc == 0) return DC_OK;
+  T* a = static_cast<T*>(m->a);
+  T* qkv = static_cast<T*>(m->qkv);
+  T* o = static_cast<T*>(m->o);
+  T* mm = static_cast<T*>(m->m);
+  const double Md = (double)M * d, E = (double)m->elt;
+  DC_LAUNCH(DC_PROF_EMBED, 2.0 * M * d * m->C, 4.0 * M * m->C + 8.0 * Md + (double)N * d * E,
+            dc::launch_embed<T>(lat, m->w_e, m->b_e, static_cast<const T*>(m->pos), map, N, m->C,
+                                d, m->u, m->h, st));
+  m->launches += 1;
+  const double ln_bytes = 4.0 * Md + E * Md;
+  const double attn_flops = 4.0 * nc * (double)N * N * d;
+  const double attn_bytes = E * (3.0 * Md + Md);
+  dc::EpiArgs ep{};
+  ep.M = M;
+  ep.n_tok = N;
+  ep.mod = mod_k;
+  ep.mod_stride = m->mod_stride;
+  ep.d = d;
+  ep.heads = m->heads;
+  ep.dh = m->dh;
+  ep.dhp = m->dhp;
+  ep.nslots = nc;
+  for (int l = 0; l < m->L; ++l) {
+    const BlockW& w = m->blk[l];
+    const int base = l * 6 * d;
+    DC_LAUNCH(DC_PROF_LN, 0.0, ln_bytes,
+              dc::launch_ln_mod<T>(m->h, M, N, d, mod_k, m->mod_stride, base + 0 * d, base + 1 * d,
+                                   map, a, st));
+    dc::EpiArgs e1 = ep;
+    e1.N = 3 * d; e1.bias = w.b_qkv; e1.out = qkv;
+    dc::EpiArgs e2 = ep;
+    e2.N = d; e2.bias = w.b_o; e2.h = m->h; e2.gate_off = base + 2 * d;
+    dc::EpiArgs e3 = ep;
+    e3.N = m->md; e3.bias = w.b_1; e3.out = mm;
+    dc::EpiArgs e4 = ep;
+    e4.N = d; e4.bias = w.b_2; e4.h = m->h; e4.gate_off = base + 5 * d;
+    const double f_qkv = 2.0 * M * 3.0 * d * d, f_o = 2.0 * M * (double)d * d,
+                 f_mlp = 2.0 * M * (double)m->md * d;
+    const double b_qkv = E * (Md + 3.0 * d * d + 3.0 * Md), b_o = E * (Md + (double)d * d) + 8.0 * Md,
+                 b_1 = E * (Md + (double)m->md * d + (double)M * m->md),
+                 b_2 = E * ((double)M * m->md + (double)m->md * d) + 8.0 * Md;
+    if constexpr (sizeof(T) == 2) {
+      DC_LAUNCH(DC_PROF_GEMM_QKV, f_qkv, b_qkv,
+                dc::launch_gemm_tc(dc::kEpiQKV, m->tm_a, w.tm_qkv, M, 3 * d, d, e1, map, m->err_d,
+                                   m->n_sms, st));
+      DC_LAUNCH(DC_PROF_ATTENTION, attn_flops, attn_bytes,
+                dc::launch_attention_bf16(reinterpret_cast<const __nv_bfloat16*>(qkv), nc, m->heads,
+                                          N, m->dh, m->dhp, reinterpret_cast<__nv_bfloat16*>(o), st));
+      DC_LAUNCH(DC_PROF_GEMM_OUT, f_o, b_o,
+                dc::launch_gemm_tc(dc::kEpiResid, m->tm_oact, w.tm_o, M, d, d, e2, map, m->err_d,
+                                   m->n_sms, st));
+      DC_LAUNCH(DC_PROF_LN, 0.0, ln_bytes,
+                dc::launch_ln_mod<T>(m->h, M, N, d, mod_k, m->mod_stride, base + 3 * d,
+                                     base + 4 * d, map, a, st));
+      DC_LAUNCH(DC_PROF_GEMM_MLP1, f_mlp, b_1,
+                dc::launch_gemm_tc(dc::kEpiGELU, m->tm_a, w.tm_1, M, m->md, d, e3, map, m->err_d,
+                                   m->n_sms, st));
+      DC_LAUNCH(DC_PROF_GEMM_MLP2, f_mlp, b_2,
+                dc::launch_gemm_tc(dc::kEpiResid, m->tm_m, w.tm_2, M, d, m->md, e4, map, m->err_d,
+                                   m->n_sms, st));
+    } else {
+      DC_LAUNCH(DC_PROF_GEMM_QKV, f_qkv, b_qkv,
+                dc::launch_gemm_f32(dc::kEpiQKV, reinterpret_cast<const float*>(a),
+                                    static_cast<const float*>(w.w_qkv), M, 3 * d, d, e1, map, st));
+      DC_LAUNCH(DC_PROF_ATTENTION, attn_flops, attn_bytes,
+                dc::launch_attention_f32(reinterpret_cast<const float*>(qkv), nc, m->heads, N,
+                                         m->dh, m->dhp, reinterpret_cast<float*>(o), st));
+      DC_LAUNCH(DC_PROF_GEMM_OUT, f_o, b_o,
+                dc::launch_gemm_f32(dc::kEpiResid, reinterpret_cast<const float*>(o),
+                                    static_cast<const float*>(w.w_o), M, d, d, e2, map, st));
+      DC_LAUNCH(DC_PROF_LN, 0.0, ln_bytes,
+                dc::launch_ln_mod<T>(m->h, M, N, d, mod_k, m->mod_stride, base + 3 * d,
+                                     base + 4 * d, map, a, st));
+      DC_LAUNCH(DC_PROF_GEMM_MLP1, f_mlp, b_1,
+                dc::launch_gemm_f32(dc::kEpiGELU, reinterpret_cast<const float*>(a),
+                                    static_cast<const float*>(w.w_1), M, m->md, d, e3, map, st));
+      DC_LAUNCH(DC_PROF_GEMM_MLP2, f_mlp, b_2,
+                dc::launch_gemm_f32(dc::kEpiResid, reinterpret_cast<const float*>(mm),
+                                    static_cast<const float*>(w.w_2), M, d, m->md, e4, map, st));
+    }
+    m->launches += 7;
+  }
+  DC_LAUNCH(DC_PROF_FINAL, 2.0 * M * d * m->C, 8.0 * Md + E * Md + 12.0 * M * m->C,
+            dc::launch_final_compute<T>(m->h, m->u, lat, m->xj, static_cast<T*>(m->r), map, N,
+                                        m->C, d, mod_k, m->mod_stride, 6 * m->L * d, m->w_f,
+                                        m->b_f, dsig, st));
+  m->launches += 1;
+  return DC_OK;
+}
+
+template <typename T>
+dc_status enqueue_reuse(dc_model* m, float* lat, const float* mod_k, const SlotMap& map, float dsig,
+                        cudaStream_t st) {
+  if (map.n == 0) return DC_OK;
+  const double M = (double)map.n * m->N;
+  // algorithmic bytes of a reuse scene-step: r_j (N d elements) + x_k read,
+  // x_{k+1} written and x_j read by the drift check (3 N C fp32)
+  DC_LAUNCH(DC_PROF_REUSE, 4.0 * M * m->d * m->C, M * ((double)m->d * m->elt + 12.0 * m->C),
+            dc::launch_final_reuse<T>(lat, static_cast<const T*>(m->r), m->w_e, m->b_e,
+                                      static_cast<const T*>(m->pos), map, m->N, m->C, m->d, mod_k,
+                                      m->mod_stride, 6 * m->L * m->d, m->w_f, m->b_f, dsig, st));
+  m->launches += 1;
+  return DC_OK;
+}
+
+template <typename T>
+dc_status enqueue_drift(dc_model* m, const dc::DriftItems& it, float* out, cudaStream_t st) {
+  DC_LAUNCH(DC_PROF_DRIFT, 4.0 * it.n * m->N * m->d * m->C, 8.0 * it.n * m->N * m->C,
+            dc::launch_drift<T>(it, m->w_e, m->b_e, static_cast<const T*>(m->pos), m->N, m->C,
+                                m->d, m->drift_part, out, st));
+  m->launches += 2;
+  return DC_OK;
+}
+
+dc_status check_device_error(dc_model* m, cudaStream_t st) {
+  int err = 0;
+  DC_CK(cudaMemcpyAsync(&err, m->err_d, sizeof(int), cudaMemcpyDeviceToHost, st));
+  DC_CK(cudaStreamSynchronize(st));
+  prof_flush(m);
+  if (err != 0) {
+    dc::set_error("a bounded device wait gave up (code " + std::to_string(err) + ")");
+    cudaMemsetAsync(m->err_d, 0, sizeof(int), st);
+    return DC_ERR_DEVICE_TIMEOUT;
+  }
+  return DC_OK;
+}
+
+struct SceneState {
+  double C = 0.0;
+  int j = 0, age = 0;
+};
+
+// The sampler.  trace (optional, device [K][B][N][C]) receives x_k before
+// step k.
+template <typename T>
+dc_status run_sampler(dc_model* m, float* lat, const dc_cond* cond, const dc_sched* sc,
+                      cudaStream_t st, dc_run_stats* stats, float* trace) {
+  const int B = cond->B, K = sc->K, N = m->N, C = m->C;
+  const dc_anchor_responses* anc = sc->anchors;
+  const double eps = anc ? anc->eps : 1e-6;
+  const int W = K + 1;
+  std::vector<unsigned char> acts((size_t)B * W, dc::kCompute);
+  std::vector<dc::SceneTables> tabs(B);
+  std::vector<int> supported(B, 0);
+  std::vector<double> Dv(B, 0.0);
+  const bool forced = sc->forced != nullptr;
+  for (int s = 0; s < B; ++s) {
+    unsigned char* a = &acts[(size_t)s * W];
+    a[0] = 0;
+    if (forced) {
+      for (int k = 1; k <= K; ++k) a[k] = sc->forced[(size_t)s * W + k];
+      a[1] = dc::kCompute;
+      continue;
+    }
+    double L, Th, D;
+    dc::motion_stats(cond->traj[s].poses, cond->traj[s].n_poses, &L, &Th);
+    supported[s] = dc::scene_intensity(L, Th, *anc, &D);
+    Dv[s] = D;
+    if (!supported[s]) continue;
+    dc::scene_tables(*anc, D, &tabs[s]);
+    double cost;
+    dc::plan_suffix(tabs[s], anc->legal, 1, sc->tau, a, &cost);
+  }
+  if (stats) {
+    if (stats->planned) std::memcpy(stats->planned, acts.data(), acts.size());
+    for (int s = 0; s < B; ++s) {
+      if (stats->supported) stats->supported[s] = supported[s];
+      if (stats->D) stats->D[s] = Dv[s];
+      for (int k = 0; k <= K; ++k) {
+        if (stats->d_obs) stats->d_obs[(size_t)s * W + k] = NAN;
+        if (stats->d_bar) stats->d_bar[(size_t)s * W + k] = NAN;
+        if (stats->checked) stats->checked[(size_t)s * W + k] = 0;
+        if (stats->executed) stats->executed[(size_t)s * W + k] = 0;
+      }
+      if (stats->n_compute) stats->n_compute[s] = 0;
+      if (stats->n_reuse) stats->n_reuse[s] = 0;
+      if (stats->n_veto) stats->n_veto[s] = 0;
+      if (stats->n_replan) stats->n_replan[s] = 0;
+    }
+    stats->backbone_calls = 0;
+  }
+  const long long launches0 = m->launches;
+
+  // inputs of the conditioning: poses and sigmas
+  std::vector<double> poses((size_t)B * m->P * 3);
+  for (int s = 0; s < B; ++s)
+    for (int t = 0; t < m->P; ++t) {
+      const dc_pose& p = cond->traj[s].poses[t];
+      double* q = &poses[((size_t)s * m->P + t) * 3];
+      q[0] = p.x; q[1] = p.y; q[2] = p.psi;
+    }
+  DC_CK(cudaMemcpyAsync(m->poses_d, poses.data(), poses.size() * sizeof(double),
+                        cudaMemcpyHostToDevice, st));
+  DC_CK(cudaMemcpyAsync(m->sig_d, sc->sigmas, (size_t)(K + 1) * sizeof(double),
+                        cudaMemcpyHostToDevice, st));
+  DC_TRY(enqueue_conditioning<T>(m, B, K, st));
+
+  std::vector<SceneState> state(B);
+  std::vector<unsigned char> reuse_now(B);
+  for (int k = 1; k <= K; ++k) {
+    const float dsig = (float)(sc->sigmas[k] - sc->sigmas[k - 1]);
+    const float* mod_k = m->mod + (size_t)(k - 1) * B * m->mod_stride;
+    if (trace) {
+      DC_CK(cudaMemcpyAsync(trace + (size_t)(k - 1) * B * N * C, lat, (size_t)B * N * C * 4,
+                            cudaMemcpyDeviceToDevice, st));
+    }
+    std::vector<int> chk;
+    for (int s = 0; s < B; ++s) {
+      reuse_now[s] = 0;
+      if (k == 1 || acts[(size_t)s * W + k] != dc::kReuse) continue;
+      if (forced || !sc->veto) {
+        reuse_now[s] = 1;
+        if (!forced) state[s].C = state[s].C + tabs[s].at_c(state[s].j, state[s].age + 1);
+      } else {
+        chk.push_back(s);
+      }
+    }
+    if (!chk.empty()) {
+      dc::DriftItems it{};
+      it.n = (int)chk.size();
+      for (int i = 0; i < it.n; ++i) {
+        it.now[i] = lat + (size_t)chk[i] * N * C;
+        it.ref[i] = m->xj + (size_t)chk[i] * N * C;
+      }
+      DC_TRY(enqueue_drift<T>(m, it, m->drift_out, st));
+      DC_CK(cudaMemcpyAsync(m->drift_host, m->drift_out, (size_t)2 * it.n * sizeof(float),
+                            cudaMemcpyDeviceToHost, st));
+      DC_TRY(check_device_error(m, st));  // synchronises the stream
+      for (int i = 0; i < it.n; ++i) {
+        const int s = chk[i];
+        const double Sd = m->drift_host[2 * i], Su = m->drift_host[2 * i + 1];
+        if (!std::isfinite(Sd) || !std::isfinite(Su)) {
+          dc::set_error("non-finite drift statistic for scene " + std::to_string(s) + " at step " +
+                        std::to_string(k));
+          return DC_ERR_NONFINITE;
+        }
+        SceneState& S = state[s];
+        const int h = S.age + 1, j = S.j;
+        const double d_obs = std::sqrt(Sd) / (std::sqrt(Su) + eps);
+        const double dbar = tabs[s].at_d(j, h);
+        const double c = tabs[s].at_c(j, h);
+        const bool ok = d_obs <= dbar + eps && S.C + c <= sc->tau;
+        if (stats) {
+          if (stats->d_obs) stats->d_obs[(size_t)s * W + k] = d_obs;
+          if (stats->d_bar) stats->d_bar[(size_t)s * W + k] = dbar;
+          if (stats->checked) stats->checked[(size_t)s * W + k] = ok ? 1 : 2;
+        }
+        if (ok) {
+          reuse_now[s] = 1;
+          S.C = S.C + c;
+        } else {
+          if (stats && stats->n_veto) stats->n_veto[s]++;
+          if (stats && stats->n_replan) stats->n_replan[s]++;
+          double cost;
+          dc::plan_suffix(tabs[s], anc->legal, k, sc->tau - S.C, &acts[(size_t)s * W], &cost);
+        }
+      }
+    }
+    SlotMap cm{}, rm{};
+    for (int s = 0; s < B; ++s) {
+      if (reuse_now[s]) rm.scene[rm.n++] = s;
+      else cm.scene[cm.n++] = s;
+    }
+    DC_TRY(enqueue_compute<T>(m, lat, mod_k, cm, dsig, st));
+    DC_TRY(enqueue_reuse<T>(m, lat, mod_k, rm, dsig, st));
+    for (int s = 0; s < B; ++s) {
+      if (reuse_now[s]) {
+        state[s].age += 1;
+      } else {
+        state[s].j = k;
+        state[s].age = 0;
+      }
+      if (stats) {
+        if (stats->executed) stats->executed[(size_t)s * W + k] = reuse_now[s] ? dc::kReuse : dc::kCompute;
+        if (reuse_now[s] && stats->n_reuse) stats->n_reuse[s]++;
+        if (!reuse_now[s] && stats->n_compute) stats->n_compute[s]++;
+      }
+    }
+    if (stats) stats->backbone_calls += cm.n;
+  }
+  DC_TRY(check_device_error(m, st));
+  if (stats) {
+    for (int s = 0; s < B; ++s)
+      if (stats->charge) stats->charge[s] = state[s].C;
+    stats->launches = m->launches - launches0;
+  }
+  return DC_OK;
+}
+
+dc_status check_call(dc_model* m, const dc_cond* cond, const dc_sched* sc) {
+  if (!m || !cond || !sc) { dc::set_error("NULL model/cond/sched"); return DC_ERR_INVALID_ARG; }
+  if (cond->B < 1 || cond->B > m->Bmax || !cond->traj) {
+    dc::set_error("cond->B must be in [1, max_batch] with non-NULL trajectories");
+    return DC_ERR_INVALID_ARG;
+  }
+  if (sc->K < 1 || sc->K > m->Kmax || !sc->sigmas) {
+    dc::set_error("sched->K must be in [1, max_steps] with non-NULL sigmas");
+    return DC_ERR_INVALID_ARG;
+  }
+  for (int k = 0; k <= sc->K; ++k)
+    if (!std::isfinite(sc->sigmas[k])) {
+      dc::set_error("non-finite sigma");
+      return DC_ERR_INVALID_ARG;
+    }
+  for (int s = 0; s < cond->B; ++s) {
+    const dc_trajectory& t = cond->traj[s];
+    if (!t.poses || t.n_poses != m->P) {
+      dc::set_error("trajectory " + std::to_string(s) + " must have n_poses = " + std::to_string(m->P));
+      return DC_ERR_INVALID_ARG;
+    }
+    for (int i = 0; i < t.n_poses; ++i)
+      if (!std::isfinite(t.poses[i].x) || !std::isfinite(t.poses[i].y) ||
+          !std::isfinite(t.poses[i].psi)) {
+        dc::set_error("non-finite pose");
+        return DC_ERR_INVALID_ARG;
+      }
+  }
+  if (sc->forced) {
+    for (int s = 0; s < cond->B; ++s)
+      for (int k = 1; k <= sc->K; ++k) {
+        const unsigned char a = sc->forced[(size_t)s * (sc->K + 1) + k];
+        if (a != dc::kCompute && a != dc::kReuse) {
+          dc::set_error("forced actions must be DC_ACT_COMPUTE or DC_ACT_REUSE");
+          return DC_ERR_INVALID_ARG;
+        }
+      }
+  } else {
+    dc_status s = dc::check_anchors(sc->anchors);
+    if (s != DC_OK) return s;
+    if (sc->anchors->K != sc->K || std::isnan(sc->tau)) {
+      dc::set_error("anchors->K must equal sched->K and tau must not be NaN");
+      return DC_ERR_INVALID_ARG;
+    }
+  }
+  return DC_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t dc_model_weight_count(const dc_model_desc* desc) {
+  if (!desc) return 0;
+  WeightLayout w;
+  weight_layout(*desc, &w);
+  return w.total;
+}
+
+dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, size_t n_floats,
+                          int device, dc_model** out) {
+  DC_TRY(check_desc(desc));
+  if (!host_weights || !out) { dc::set_error("NULL weights/out"); return DC_ERR_INVALID_ARG; }
+  WeightLayout lay;
+  weight_layout(*desc, &lay);
+  if (n_floats != lay.total) {
+    dc::set_error("weight blob has " + std::to_string(n_floats) + " floats, expected " +
+                  std::to_string(lay.total));
+    return DC_ERR_INVALID_ARG;
+  }
+  if (device >= 0) DC_CK(cudaSetDevice(device));
+  int dev = 0;
+  DC_CK(cudaGetDevice(&dev));
+  int major = 0, minor = 0;
+  DC_CK(cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev));
+  DC_CK(cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev));
+  if (major != 10 || minor != 3) {
+    dc::set_error("this library is built for sm_103a only (device is sm_" + std::to_string(major) +
+                  std::to_string(minor) + ")");
+    return DC_ERR_UNSUPPORTED;
+  }
+  dc_model* m = new dc_model();
+  m->desc = *desc;
+  m->device = dev;
+  DC_CK(cudaDeviceGetAttribute(&m->n_sms, cudaDevAttrMultiProcessorCount, dev));
+  m->bf16 = desc->dtype == DC_DTYPE_BF16;
+  m->elt = m->bf16 ? 2 : 4;
+  m->N = desc->n_tokens; m->C = desc->channels; m->d = desc->d_model; m->L = desc->n_blocks;
+  m->heads = desc->n_heads; m->dh = m->d / m->heads;
+  m->dhp = m->bf16 ? ((m->dh + 15) / 16) * 16 : m->dh;
+  m->md = desc->mlp_ratio * m->d; m->P = desc->n_poses; m->Bmax = desc->max_batch;
+  m->Kmax = desc->max_steps;
+  m->mod_stride = (6 * m->L + 2) * m->d;
+
+  // ---- weights
+  std::vector<size_t> off(lay.t.size());
+  size_t bytes = 0;
+  for (size_t i = 0; i < lay.t.size(); ++i) {
+    off[i] = bytes;
+    bytes += align256(lay.t[i].n * (lay.t[i].big ? m->elt : 4));
+  }
+  std::vector<uint8_t> host(bytes, 0);
+  {
+    const float* src = host_weights;
+    for (size_t i = 0; i < lay.t.size(); ++i) {
+      const size_t n = lay.t[i].n;
+      if (lay.t[i].big && m->bf16) {
+        uint16_t* dst = reinterpret_cast<uint16_t*>(host.data() + off[i]);
+        for (size_t k = 0; k < n; ++k) dst[k] = f2bf_host(src[k]);
+      } else {
+        std::memcpy(host.data() + off[i], src, n * 4);
+      }
+      src += n;
+    }
+  }
+  auto fail = [&](dc_status s) { dc_model_destroy(m); return s; };
+  if (cudaMalloc(&m->wbuf, bytes) != cudaSuccess) {
+    dc::set_error("cudaMalloc of " + std::to_string(bytes) + " weight bytes failed");
+    return fail(DC_ERR_NOMEM);
+  }
+  if (cudaMemcpy(m->wbuf, host.data(), bytes, cudaMemcpyHostToDevice) != cudaSuccess) {
+    dc::set_error("weight upload failed");
+    return fail(DC_ERR_CUDA);
+  }
+  {
+    uint8_t* b = static_cast<uint8_t*>(m->wbuf);
+    size_t i = 0;
+    auto nxt = [&]() { return b + off[i++]; };
+    m->w_e = (float*)nxt(); m->b_e = (float*)nxt(); m->pos = nxt();
+    m->w_t1 = (float*)nxt(); m->b_t1 = (float*)nxt();
+    m->w_t2 = (float*)nxt(); m->b_t2 = (float*)nxt();
+    m->w_traj = (float*)nxt(); m->b_traj = (float*)nxt();
+    m->w_ada = nxt(); m->b_ada = (float*)nxt();
+    m->blk.resize(m->L);
+    for (int l = 0; l < m->L; ++l) {
+      BlockW& w = m->blk[l];
+      w.w_qkv = nxt(); w.b_qkv = (float*)nxt();
+      w.w_o = nxt(); w.b_o = (float*)nxt();
+      w.w_1 = nxt(); w.b_1 = (float*)nxt();
+      w.w_2 = nxt(); w.b_2 = (float*)nxt();
+    }
+    m->w_f = (float*)nxt(); m->b_f = (float*)nxt();
+  }
+
+  // ---- workspace
+  const size_t B = m->Bmax, N = m->N, d = m->d, K = m->Kmax;
+  struct Buf { void** p; size_t bytes; };
+  std::vector<Buf> bufs = {
+      {(void**)&m->u, B * N * d * 4}, {(void**)&m->h, B * N * d * 4},
+      {&m->a, B * N * d * m->elt}, {&m->qkv, 3 * B * m->heads * N * m->dhp * m->elt},
+      {&m->o, B * N * d * m->elt}, {&m->m, B * N * m->md * m->elt},
+      {&m->r, B * N * d * m->elt}, {(void**)&m->xj, B * N * m->C * 4},
+      {(void**)&m->lat_stage, B * N * m->C * 4},
+      {(void**)&m->mod, K * B * m->mod_stride * 4}, {(void**)&m->silu_c, K * B * d * 4},
+      {(void**)&m->temb_f, K * 256 * 4}, {(void**)&m->temb_h, K * d * 4},
+      {(void**)&m->temb, K * d * 4}, {(void**)&m->pose_f, B * 3 * m->P * 4},
+      {(void**)&m->traj, B * d * 4},
+      {(void**)&m->drift_part, (size_t)dc::kMaxBatch * dc::kDriftParts * 2 * 4},
+      {(void**)&m->drift_out, (size_t)dc::kMaxBatch * 2 * 4},
+      {(void**)&m->poses_d, B * m->P * 3 * 8}, {(void**)&m->sig_d, (K + 1) * 8},
+      {(void**)&m->err_d, 256}};
+  size_t wsb = 0;
+  for (auto& b : bufs) wsb += align256(b.bytes);
+  if (cudaMalloc(&m->ws, wsb) != cudaSuccess) {
+    dc::set_error("cudaMalloc of " + std::to_string(wsb) + " workspace bytes failed");
+    return fail(DC_ERR_NOMEM);
+  }
+  {
+    uint8_t* p = static_cast<uint8_t*>(m->ws);
+    for (auto& b : bufs) { *b.p = p; p += align256(b.bytes); }
+  }
+  // zero everything once: the head-dim pad columns of q/k/v stay zero
+  if (cudaMemset(m->ws, 0, wsb) != cudaSuccess) return fail(DC_ERR_CUDA);
+  if (cudaMallocHost(&m->drift_host, (size_t)dc::kMaxBatch * 2 * 4) != cudaSuccess) {
+    dc::set_error("cudaMallocHost failed");
+    return fail(DC_ERR_NOMEM);
+  }
+  if (m->bf16) {
+    const uint32_t bn = (uint32_t)dc::gemm_tc_tile_n(), bm = (uint32_t)dc::gemm_tc_tile_m();
+    dc_status s;
+    if ((s = make_map(&m->tm_a, m->a, d, B * N, bm)) != DC_OK) return fail(s);
+    if ((s = make_map(&m->tm_oact, m->o, d, B * N, bm)) != DC_OK) return fail(s);
+    if ((s = make_map(&m->tm_m, m->m, m->md, B * N, bm)) != DC_OK) return fail(s);
+    for (int l = 0; l < m->L; ++l) {
+      BlockW& w = m->blk[l];
+      if ((s = make_map(&w.tm_qkv, w.w_qkv, d, 3 * d, bn)) != DC_OK) return fail(s);
+      if ((s = make_map(&w.tm_o, w.w_o, d, d, bn)) != DC_OK) return fail(s);
+      if ((s = make_map(&w.tm_1, w.w_1, d, m->md, bn)) != DC_OK) return fail(s);
+      if ((s = make_map(&w.tm_2, w.w_2, m->md, d, bn)) != DC_OK) return fail(s);
+    }
+  }
+  if (cudaDeviceSynchronize() != cudaSuccess) return fail(DC_ERR_CUDA);
+  *out = m;
+  return DC_OK;
+}
+
+void dc_model_destroy(dc_model* m) {
+  if (!m) return;
+  if (m->wbuf) cudaFree(m->wbuf);
+  if (m->ws) cudaFree(m->ws);
+  if (m->drift_host) cudaFreeHost(m->drift_host);
+  for (auto& r : m->prof_pending) { cudaEventDestroy(r.a); cudaEventDestroy(r.b); }
+  for (auto e : m->ev_pool) cudaEventDestroy(e);
+  delete m;
+}
+
+dc_status dc_denoise(dc_model* m, float* latents, const dc_cond* cond, const dc_sched* sched,
+                     void* stream, dc_run_stats* stats) {
+  DC_TRY(check_call(m, cond, sched));
+  if (!latents) { dc::set_error("latents is NULL"); return DC_ERR_INVALID_ARG; }
+  DC_CK(cudaSetDevice(m->device));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (m->bf16) return run_sampler<__nv_bfloat16>(m, latents, cond, sched, st, stats, nullptr);
+  return run_sampler<float>(m, latents, cond, sched, st, stats, nullptr);
+}
+
+dc_status dc_denoise_host(dc_model* m, float* host_latents, const dc_cond* cond,
+                          const dc_sched* sched, void* stream, dc_run_stats* stats) {
+  DC_TRY(check_call(m, cond, sched));
+  if (!host_latents) { dc::set_error("host_latents is NULL"); return DC_ERR_INVALID_ARG; }
+  DC_CK(cudaSetDevice(m->device));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t bytes = (size_t)cond->B * m->N * m->C * sizeof(float);
+  DC_CK(cudaMemcpyAsync(m->lat_stage, host_latents, bytes, cudaMemcpyHostToDevice, st));
+  dc_status s = m->bf16 ? run_sampler<__nv_bfloat16>(m, m->lat_stage, cond, sched, st, stats, nullptr)
+                        : run_sampler<float>(m, m->lat_stage, cond, sched, st, stats, nullptr);
+  if (s != DC_OK) return s;
+  DC_CK(cudaMemcpyAsync(host_latents, m->lat_stage, bytes, cudaMemcpyDeviceToHost, st));
+  DC_CK(cudaStreamSynchronize(st));
+  return DC_OK;
+}
+
+dc_status dc_anchor_drift(dc_model* m, const float* noise, const dc_trajectory* traj, int K,
+                          const double* sigmas, int H_max, double eps, double* d_out,
+                          void* stream) {
+  if (!m || !noise || !traj || !sigmas || !d_out || K < 1 || K > m->Kmax || H_max < 1 ||
+      !(eps > 0.0)) {
+    dc::set_error("dc_anchor_drift: NULL argument, K outside [1, max_steps], H_max < 1 or eps <= 0");
+    return DC_ERR_INVALID_ARG;
+  }
+  DC_CK(cudaSetDevice(m->device));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t NC = (size_t)m->N * m->C;
+  float* trace = nullptr;
+  float* x = nullptr;
+  if (cudaMalloc(&trace, (size_t)K * NC * 4) != cudaSuccess ||
+      cudaMalloc(&x, NC * 4) != cudaSuccess) {
+    if (trace) cudaFree(trace);
+    dc::set_error("dc_anchor_drift: trace allocation failed");
+    return DC_ERR_NOMEM;
+  }
+  std::vector<unsigned char> forced((size_t)K + 1, dc::kCompute);
+  dc_sched sc{};
+  sc.K = K; sc.sigmas = sigmas; sc.anchors = nullptr; sc.tau = 0.0; sc.veto = 0;
+  sc.forced = forced.data();
+  dc_cond cond{1, traj};
+  dc_status s = check_call(m, &cond, &sc);
+  if (s == DC_OK && cudaMemcpyAsync(x, noise, NC * 4, cudaMemcpyDeviceToDevice, st) != cudaSuccess) {
+    dc::set_error("dc_anchor_drift: copy failed");
+    s = DC_ERR_CUDA;
+  }
+  if (s == DC_OK)
+    s = m->bf16 ? run_sampler<__nv_bfloat16>(m, x, &cond, &sc, st, nullptr, trace)
+                : run_sampler<float>(m, x, &cond, &sc, st, nullptr, trace);
+  for (int j = 0; j < K; ++j)
+    for (int h = 0; h <= H_max; ++h) d_out[(size_t)j * (H_max + 1) + h] = 0.0;
+  // pairs (j + h, j) for j = 1..K-1, h = 1..min(H_max, K - j); trace[k-1] = x_k
+  std::vector<std::pair<int, int>> pairs;
+  for (int j = 1; j < K; ++j)
+    for (int h = 1; h <= H_max && j + h <= K; ++h) pairs.push_back({j, h});
+  for (size_t p0 = 0; s == DC_OK && p0 < pairs.size(); p0 += dc::kMaxBatch) {
+    dc::DriftItems it{};
+    it.n = (int)std::min(pairs.size() - p0, (size_t)dc::kMaxBatch);
+    for (int i = 0; i < it.n; ++i) {
+      const auto& pr = pairs[p0 + i];
+      it.now[i] = trace + (size_t)(pr.first + pr.second - 1) * NC;
+      it.ref[i] = trace + (size_t)(pr.first - 1) * NC;
+    }
+    s = m->bf16 ? enqueue_drift<__nv_bfloat16>(m, it, m->drift_out, st)
+                : enqueue_drift<float>(m, it, m->drift_out, st);
+    if (s != DC_OK) break;
+    if (cudaMemcpyAsync(m->drift_host, m->drift_out, (size_t)2 * it.n * 4, cudaMemcpyDeviceToHost,
+                        st) != cudaSuccess ||
+        cudaStreamSynchronize(st) != cudaSuccess) {
+      dc::set_error("dc_anchor_drift: readback failed");
+      s = DC_ERR_CUDA;
+      break;
+    }
+    for (int i = 0; i < it.n; ++i) {
+      const auto& pr = pairs[p0 + i];
+      const double Sd = m->drift_host[2 * i], Su = m->drift_host[2 * i + 1];
+      if (!std::isfinite(Sd) || !std::isfinite(Su)) {
+        dc::set_error("non-finite drift along the anchor trace");
+        s = DC_ERR_NONFINITE;
+        break;
+      }
+      d_out[(size_t)pr.first * (H_max + 1) + pr.second] = std::sqrt(Sd) / (std::sqrt(Su) + eps);
+    }
+  }
+  cudaStreamSynchronize(st);
+  cudaFree(trace);
+  cudaFree(x);
+  return s;
+}
+
+dc_status dc_drift_sums(dc_model* m, const float* x_now, const float* x_ref, int B, float* out,
+                        void* stream) {
+  if (!m || !x_now || !x_ref || !out || B < 1 || B > m->Bmax) {
+    dc::set_error("dc_drift_sums: NULL pointer or B outside [1, max_batch]");
+    return DC_ERR_INVALID_ARG;
+  }
+  DC_CK(cudaSetDevice(m->device));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  dc::DriftItems it{};
+  it.n = B;
+  const size_t NC = (size_t)m->N * m->C;
+  for (int i = 0; i < B; ++i) {
+    it.now[i] = x_now + i * NC;
+    it.ref[i] = x_ref + i * NC;
+  }
+  return m->bf16 ? enqueue_drift<__nv_bfloat16>(m, it, out, st) : enqueue_drift<float>(m, it, out, st);
+}
+
+dc_status dc_profile(dc_model* m, int enable) {
+  if (!m) { dc::set_error("model is NULL"); return DC_ERR_INVALID_ARG; }
+  if (enable) {
+    for (int i = 0; i < DC_PROF_N; ++i) {
+      m->prof_ms[i] = m->prof_flops[i] = m->prof_bytes[i] = 0.0;
+      m->prof_cnt[i] = 0;
+    }
+  }
+  m->prof_on = enable != 0;
+  return DC_OK;
+}
+
+dc_status dc_profile_read(dc_model* m, double* ms, long long* launches, double* flops,
+                          double* bytes) {
+  if (!m) { dc::set_error("model is NULL"); return DC_ERR_INVALID_ARG; }
+  for (int i = 0; i < DC_PROF_N; ++i) {
+    if (ms) ms[i] = m->prof_ms[i];
+    if (launches) launches[i] = m->prof_cnt[i];
+    if (flops) flops[i] = m->prof_flops[i];
+    if (bytes) bytes[i] = m->prof_bytes[i];
+  }
+  return DC_OK;
+}
+
+dc_status dc_cache_copy(dc_model* m, int scene, void* dst, size_t bytes, void* stream) {
+  if (!m || !dst || scene < 0 || scene >= m->Bmax ||
+      bytes != (size_t)m->N * m->d * m->elt) {
+    dc::set_error("dc_cache_copy: NULL pointer, scene outside [0, max_batch) or wrong size");
+    return DC_ERR_INVALID_ARG;
+  }
+  DC_CK(cudaSetDevice(m->device));
+  const uint8_t* src = static_cast<const uint8_t*>(m->r) + (size_t)scene * bytes;
+  DC_CK(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToDevice, static_cast<cudaStream_t>(stream)));
+  return DC_OK;
+}
+
+dc_status dc_attention(int dtype, const void* qkv, int slots, int heads, int n_tokens,
+                       int head_dim, void* out, void* stream) {
+  if (!qkv || !out || slots < 1 || heads < 1 || n_tokens < 1 || head_dim < 1) {
+    dc::set_error("dc_attention: NULL pointer or non-positive size");
+    return DC_ERR_INVALID_ARG;
+  }
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (dtype == DC_DTYPE_BF16) {
+    if (!(head_dim == 16 || head_dim == 64 || head_dim == 72 || head_dim == 128)) {
+      dc::set_error("dc_attention: bf16 head_dim must be 16, 64, 72 or 128");
+      return DC_ERR_UNSUPPORTED;
+    }
+    const int dhp = ((head_dim + 15) / 16) * 16;
+    DC_CK(dc::launch_attention_bf16(static_cast<const __nv_bfloat16*>(qkv), slots, heads, n_tokens,
+                                    head_dim, dhp, static_cast<__nv_bfloat16*>(out), st));
+    return DC_OK;
+  }
+  if (dtype == DC_DTYPE_F32) {
+    if (!(head_dim == 8 || head_dim == 16 || head_dim == 32 || head_dim == 64)) {
+      dc::set_error("dc_attention: fp32 head_dim must be 8, 16, 32 or 64");
+      return DC_ERR_UNSUPPORTED;
+    }
+    DC_CK(dc::launch_attention_f32(static_cast<const float*>(qkv), slots, heads, n_tokens, head_dim,
+                                   head_dim, static_cast<float*>(out), st));
+    return DC_OK;
+  }
+  dc::set_error("dc_attention: unknown dtype");
+  return DC_ERR_INVALID_ARG;
+}
+
+}  // extern "C"

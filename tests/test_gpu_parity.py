@@ -1,0 +1,367 @@
+"""GPU path vs the CPU oracle, through the C ABI.
+
+Tolerances (from the acceptance criteria): fp32 path rel-L2 <= 1e-4, bf16 path
+rel-L2 <= 2e-2 on the final latents; schedules and refresh decisions equal,
+except decisions whose oracle statistic lies within 1e-3 relative of the
+threshold, which are logged and then replayed with the oracle's decisions.
+Because x_K stays close to x_1 for a random-init backbone, the bf16 checks
+also bound the rel-L2 of the latent update x_K - x_1."""
+
+import math
+
+import numpy as np
+import pytest
+
+from oracle import controller as Ctl
+from oracle import planner as P
+from synth import WORKLOADS, gen
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+NEAR = 1e-3
+
+
+@pytest.fixture(scope="module")
+def dc():
+    from paper_2608_16354_gb300 import _build, binding
+    _build.build()
+    binding.lib()
+    return binding
+
+
+def rel(a, b):
+    return float(np.linalg.norm(np.asarray(a, np.float64) - b) / max(np.linalg.norm(b), 1e-30))
+
+
+def no_anchors(dc, K, H):
+    return dc.AnchorArgs(K, H, dict(L0=0, T0=0, L1=0, T1=0, valid=0), dict(q0=None, q1=None))
+
+
+def run_forced(dc, wl, w, x1, trajs, forced, sig):
+    model = dc.Model(wl, gen.flat_blob(wl, w), max_batch=len(x1), max_steps=len(sig) - 1)
+    lat = torch.tensor(np.asarray(x1, np.float32), device="cuda")
+    K = len(sig) - 1
+    st = dc.denoise(model, lat, list(trajs),
+                    dc.SchedArgs(K, sig, no_anchors(dc, K, wl.h_max), 0.0,
+                                 forced=np.asarray(forced, np.uint8)))
+    torch.cuda.synchronize()
+    out = lat.cpu().numpy()
+    model.close()
+    return out, st
+
+
+def check_bf16(got, ref, x1, tol=2e-2):
+    assert rel(got, ref) <= tol
+    assert rel(got - x1, ref - x1) <= tol, rel(got - x1, ref - x1)
+
+
+# --------------------------------------------------------------- fp32 path
+
+def _calibrated(wl):
+    w = gen.weights(wl)
+    om = Ctl.build(wl, w)
+    K, H = wl.steps, wl.h_max
+    sig = gen.sigmas(K)
+    q0, q1 = gen.synthetic_q_tables(K, H)
+    anc, tabs, tau, reached = Ctl.calibrate(om, wl, gen.calibration_trajectories(wl),
+                                            gen.anchor_noise(wl), sig, q0, q1, wl.target())
+    return w, om, sig, anc, tabs, tau
+
+
+def _compare_controller(dc, wl, w, om, sig, anc, tabs, tau, tol, bf16):
+    K, H = wl.steps, wl.h_max
+    x1 = gen.latents(wl)
+    trajs = gen.scene_trajectories(wl)
+    ref = Ctl.denoise(om, x1, trajs, sig, anc, tabs, tau, K, H)
+    model = dc.Model(wl, gen.flat_blob(wl, w))
+    lat = torch.tensor(x1, device="cuda")
+    st = dc.denoise(model, lat, list(trajs), dc.SchedArgs(K, sig, dc.AnchorArgs(K, H, anc, tabs), tau))
+    torch.cuda.synchronize()
+    got = lat.cpu().numpy()
+    model.close()
+    B = len(trajs)
+    near = []
+    for s in range(B):
+        assert st["planned"][s].tolist()[1:] == ref["plans"][s]["actions"][1:]
+        assert st["supported"][s] == ref["plans"][s]["supported"]
+        for e in ref["log"][s]:
+            k = e["k"]
+            thr = e["dbar"] + P.EPS
+            g_ok = st["checked"][s, k] == 1
+            assert st["checked"][s, k] in (1, 2), (s, k)
+            assert abs(st["d_obs"][s, k] - e["d_obs"]) <= (1e-4 if not bf16 else 2e-3) * e["d_obs"]
+            if g_ok != e["accept"]:
+                assert abs(e["d_obs"] - thr) <= NEAR * thr, (s, k, e, st["d_obs"][s, k])
+                near.append((s, k))
+    if near:
+        # logged near-threshold decisions: replay the oracle's decisions
+        got, _ = run_forced(dc, wl, w, x1, trajs, ref["executed"], sig)
+    else:
+        for s in range(B):
+            assert st["executed"][s].tolist()[1:] == ref["executed"][s][1:]
+            assert st["n_veto"][s] == ref["stats"][s]["n_veto"]
+            assert st["charge"][s] == ref["stats"][s]["charge"]
+    if bf16:
+        check_bf16(got, ref["x"], x1, tol)
+    else:
+        assert rel(got, ref["x"]) <= tol
+        assert rel(got - x1, ref["x"] - x1) <= 10 * tol
+    return st, ref
+
+
+def test_tiny_fp32_full_controller(dc):
+    wl = WORKLOADS["c1"]
+    w, om, sig, anc, tabs, tau = _calibrated(wl)
+    st, ref = _compare_controller(dc, wl, w, om, sig, anc, tabs, tau, 1e-4, False)
+    assert st["n_reuse"][0] == wl.target_reuses
+
+
+def test_tiny_fp32_anchor_drift_tables(dc):
+    wl = WORKLOADS["c1"]
+    w = gen.weights(wl)
+    om = Ctl.build(wl, w)
+    K, H = wl.steps, wl.h_max
+    sig = gen.sigmas(K)
+    poses = gen.calibration_trajectories(wl)[5]
+    ref, _ = Ctl.anchor_trace_drift(om, gen.anchor_noise(wl), poses, sig, K, H)
+    model = dc.Model(wl, gen.flat_blob(wl, w), max_batch=1)
+    noise = torch.tensor(gen.anchor_noise(wl), device="cuda")
+    got = dc.anchor_drift(model, noise, poses, K, sig, H)
+    model.close()
+    ref = np.array(ref)
+    mask = ref > 0
+    assert np.array_equal(got > 0, mask)
+    assert np.max(np.abs(got[mask] - ref[mask]) / ref[mask]) <= 1e-4
+
+
+def test_tiny_fp32_veto_refresh_replan(dc):
+    """Zero drift thresholds: every planned reuse is refused, refreshed and
+    replanned, identically on both sides."""
+    wl = WORKLOADS["c1"]
+    w = gen.weights(wl)
+    om = Ctl.build(wl, w)
+    K, H = wl.steps, wl.h_max
+    sig = gen.sigmas(K)
+    q0, q1 = gen.synthetic_q_tables(K, H)
+    z = np.zeros((K, H + 1))
+    tabs = dict(q0=q0, q1=q1, d0=z, d1=z)
+    anc = dict(L0=0.0, T0=0.0, L1=10.0, T1=1.0, valid=1)
+    st, ref = _compare_controller(dc, wl, w, om, sig, anc, tabs, 0.2, 1e-4, False)
+    assert st["n_veto"][0] >= 1 and st["n_reuse"][0] == 0
+
+
+def test_zero_reuse_schedule_equals_full_compute(dc):
+    """Budget 0 plans no reuse; the result is bit-identical to a forced
+    all-compute replay on the device."""
+    wl = WORKLOADS["c2"].with_(n_blocks=2, frames=1, rows=9, cols=21, batch=3, steps=4)
+    w = gen.weights(wl)
+    K, H = wl.steps, wl.h_max
+    sig = gen.sigmas(K)
+    x1 = gen.latents(wl)
+    trajs = gen.scene_trajectories(wl)
+    q0, q1 = gen.synthetic_q_tables(K, H)
+    d0, d1 = gen.synthetic_d_tables(K, H)
+    A = dc.AnchorArgs(K, H, dict(L0=0.0, T0=0.0, L1=60.0, T1=2.0, valid=1),
+                      dict(q0=q0, q1=q1, d0=d0, d1=d1))
+    model = dc.Model(wl, gen.flat_blob(wl, w))
+    lat = torch.tensor(x1, device="cuda")
+    st = dc.denoise(model, lat, list(trajs), dc.SchedArgs(K, sig, A, 0.0))
+    assert int(st["n_reuse"].sum()) == 0
+    lat2 = torch.tensor(x1, device="cuda")
+    dc.denoise(model, lat2, list(trajs),
+               dc.SchedArgs(K, sig, A, 0.0, forced=np.ones((3, K + 1), np.uint8)))
+    torch.cuda.synchronize()
+    assert torch.equal(lat, lat2)
+    model.close()
+
+
+# --------------------------------------------------------------- bf16 path
+
+@pytest.mark.parametrize("shape", [
+    # d=384 / dh 64 (bench family), ragged token count 390 = 3 x 128 + 6
+    dict(key="c2", n_blocks=2, frames=3, rows=10, cols=13, batch=3, steps=4),
+    # d=1152 / dh 72 (padded to 80)
+    dict(key="c3", n_blocks=1, frames=1, rows=10, cols=27, batch=2, steps=3),
+    # multi-view joint attention, d=1152
+    dict(key="c4", n_blocks=1, frames=1, rows=4, cols=7, batch=2, steps=2),
+    # d=3072 / dh 128
+    dict(key="c5", n_blocks=1, frames=1, rows=5, cols=31, batch=1, steps=2),
+])
+def test_bf16_forced_schedule_vs_oracle(dc, shape):
+    shape = dict(shape)
+    wl = WORKLOADS[shape.pop("key")].with_(**shape)
+    w = gen.weights(wl)
+    om = Ctl.build(wl, w)
+    K = wl.steps
+    sig = gen.sigmas(K)
+    x1 = gen.latents(wl)
+    trajs = gen.scene_trajectories(wl)
+    pattern = [0] + [P.COMPUTE if k % 2 == 1 else P.REUSE for k in range(1, K + 1)]
+    forced = [pattern] * wl.batch
+    ref = Ctl.denoise(om, x1, trajs, sig, dict(valid=0), None, 0.0, K, wl.h_max, forced=forced)
+    got, st = run_forced(dc, wl, w, x1, trajs, forced, sig)
+    assert st["executed"].tolist() == [p for p in forced]
+    check_bf16(got, ref["x"], x1)
+
+
+def test_bf16_small_full_controller(dc):
+    """The bench family (d=384, 6 heads) with the calibrated controller:
+    anchors, anchor drift tables measured on the device vs the oracle's,
+    tau, the plan, the drift checks and the latents."""
+    wl = WORKLOADS["c2"].with_(n_blocks=2, frames=3, rows=10, cols=13, batch=3, steps=10,
+                               rho_tar=0.4)
+    w, om, sig, anc, tabs, tau = _calibrated(wl)
+    K, H = wl.steps, wl.h_max
+    # the device's own anchor drift tables agree with the oracle's
+    model = dc.Model(wl, gen.flat_blob(wl, w), max_batch=wl.batch)
+    clips = gen.calibration_trajectories(wl)
+    noise = torch.tensor(gen.anchor_noise(wl), device="cuda")
+    d0 = dc.anchor_drift(model, noise, clips[anc["i0"]], K, sig, H)
+    model.close()
+    ref0 = np.array(tabs["d0"])
+    m = ref0 > 0
+    assert np.max(np.abs(d0[m] - ref0[m]) / ref0[m]) <= 2e-3
+    _compare_controller(dc, wl, w, om, sig, anc, tabs, tau, 2e-2, True)
+
+
+def test_drift_sums_vs_numpy_and_deterministic(dc):
+    wl = WORKLOADS["c2"].with_(n_blocks=1, frames=2, rows=9, cols=17, batch=5, steps=2)
+    w = gen.weights(wl)
+    rng = np.random.default_rng(3)
+    xn = rng.standard_normal((5, wl.n_tokens, wl.channels)).astype(np.float32)
+    xr = (xn + 0.05 * rng.standard_normal(xn.shape)).astype(np.float32)
+    model = dc.Model(wl, gen.flat_blob(wl, w))
+    tn, tr = torch.tensor(xn, device="cuda"), torch.tensor(xr, device="cuda")
+    out = torch.zeros(10, device="cuda")
+    dc.drift_sums(model, tn, tr, out)
+    out2 = torch.zeros(10, device="cuda")
+    dc.drift_sums(model, tn, tr, out2)
+    torch.cuda.synchronize()
+    assert torch.equal(out, out2)
+    We = w["w_embed"].astype(np.float64)
+    for s in range(5):
+        du = (xn[s].astype(np.float64) - xr[s]) @ We.T
+        u = xn[s].astype(np.float64) @ We.T + w["b_embed"] + w["pos"]
+        assert abs(out[2 * s].item() - np.sum(du * du)) <= 1e-5 * np.sum(du * du)
+        assert abs(out[2 * s + 1].item() - np.sum(u * u)) <= 1e-5 * np.sum(u * u)
+    model.close()
+
+
+def test_denoise_host_matches_device_call(dc):
+    wl = WORKLOADS["c2"].with_(n_blocks=1, frames=1, rows=8, cols=16, batch=2, steps=3)
+    w = gen.weights(wl)
+    K = wl.steps
+    sig = gen.sigmas(K)
+    x1 = gen.latents(wl)
+    trajs = gen.scene_trajectories(wl)
+    forced = np.array([[0, 1, 2, 1]] * 2, np.uint8)
+    model = dc.Model(wl, gen.flat_blob(wl, w))
+    lat = torch.tensor(x1, device="cuda")
+    sa = dc.SchedArgs(K, sig, no_anchors(dc, K, wl.h_max), 0.0, forced=forced)
+    dc.denoise(model, lat, list(trajs), sa)
+    host = torch.tensor(x1).pin_memory()
+    dc.denoise_host(model, host, list(trajs), sa)
+    torch.cuda.synchronize()
+    assert torch.equal(lat.cpu(), host)
+    model.close()
+
+
+def test_invalid_calls_fail_before_launch(dc):
+    wl = WORKLOADS["c2"].with_(n_blocks=1, frames=1, rows=8, cols=16, batch=2, steps=3)
+    w = gen.weights(wl)
+    model = dc.Model(wl, gen.flat_blob(wl, w))
+    K = wl.steps
+    sig = gen.sigmas(K)
+    lat = torch.zeros((3, wl.n_tokens, wl.channels), device="cuda")
+    trajs = list(gen.scene_trajectories(wl, batch=3))
+    sa = dc.SchedArgs(K, sig, no_anchors(dc, K, wl.h_max), 0.0,
+                      forced=np.ones((3, K + 1), np.uint8))
+    with pytest.raises(dc.DCError):  # B = 3 > max_batch = 2
+        dc.denoise(model, lat, trajs, sa)
+    bad = np.ones((2, K + 1), np.uint8)
+    bad[1, 2] = 7
+    with pytest.raises(dc.DCError):
+        dc.denoise(model, lat[:2], trajs[:2], dc.SchedArgs(K, sig, no_anchors(dc, K, wl.h_max), 0.0,
+                                                            forced=bad))
+    with pytest.raises(dc.DCError):  # wrong pose count
+        dc.denoise(model, lat[:2], [t[:5] for t in trajs[:2]], sa)
+    with pytest.raises(dc.DCError):  # unsupported head dim for bf16
+        dc.Model(wl.with_(n_heads=4), gen.flat_blob(wl, w))
+    model.close()
+
+
+# ------------------------------------------------- kernel-level stress cases
+
+@pytest.mark.parametrize("dh,N,heads,slots", [(64, 390, 2, 2), (72, 200, 3, 1), (128, 131, 2, 1),
+                                              (64, 64, 1, 1), (64, 1, 1, 1)])
+def test_attention_kernel_sharp_softmax(dc, dh, N, heads, slots):
+    """Attention alone on random q/k/v scaled so that the softmax is far from
+    uniform (logits ~ N(0, 9)), ragged token counts, all bf16 head dims."""
+    from oracle.dit import attention_core
+    rng = np.random.default_rng(dh + N)
+    dhp = (dh + 15) // 16 * 16
+    qkv = np.zeros((3, slots, heads, N, dhp), np.float32)
+    qkv[..., :dh] = rng.standard_normal((3, slots, heads, N, dh))
+    qkv[0] *= 3.0
+    t = torch.tensor(qkv, device="cuda").to(torch.bfloat16)
+    ref_in = t.float().cpu().numpy()
+    out = torch.zeros((slots, N, heads * dh), device="cuda", dtype=torch.bfloat16)
+    dc.attention(t, slots, heads, N, dh, out)
+    torch.cuda.synchronize()
+    got = out.float().cpu().numpy()
+    for s in range(slots):
+        ref = attention_core(ref_in[0, s, :, :, :dh], ref_in[1, s, :, :, :dh], ref_in[2, s, :, :, :dh])
+        ref = ref.transpose(1, 0, 2).reshape(N, heads * dh)
+        assert rel(got[s], ref) <= 1e-2, rel(got[s], ref)
+
+
+@pytest.mark.parametrize("dh,N", [(16, 128), (16, 77), (64, 50)])
+def test_attention_kernel_fp32(dc, dh, N):
+    from oracle.dit import attention_core
+    rng = np.random.default_rng(dh * N)
+    heads, slots = 2, 2
+    qkv = rng.standard_normal((3, slots, heads, N, dh)).astype(np.float32)
+    qkv[0] *= 3.0
+    t = torch.tensor(qkv, device="cuda")
+    out = torch.zeros((slots, N, heads * dh), device="cuda")
+    dc.attention(t, slots, heads, N, dh, out)
+    torch.cuda.synchronize()
+    got = out.cpu().numpy()
+    for s in range(slots):
+        ref = attention_core(qkv[0, s], qkv[1, s], qkv[2, s]).transpose(1, 0, 2).reshape(N, heads * dh)
+        assert rel(got[s], ref) <= 1e-5
+
+
+@pytest.mark.parametrize("key,shape,tol", [
+    ("c1", dict(), 1e-4),
+    ("c2", dict(n_blocks=2, frames=3, rows=10, cols=13, batch=2), 2e-2),
+    ("c3", dict(n_blocks=1, frames=1, rows=10, cols=27, batch=1), 2e-2),
+    ("c5", dict(n_blocks=1, frames=1, rows=5, cols=31, batch=1), 2e-2),
+])
+def test_cached_backbone_output_strong_weights(dc, key, shape, tol):
+    """With weights N(0, 0.05) the block stack's residual r = h_L - u is as
+    large as u and attention is sharp, so comparing the cached r of one full
+    step against the oracle checks every block kernel directly."""
+    wl = WORKLOADS[key].with_(steps=1, **shape)
+    w = gen.weights(wl, std=0.05)
+    om = Ctl.build(wl, w)
+    sig = gen.sigmas(1)
+    x1 = gen.latents(wl)
+    trajs = gen.scene_trajectories(wl)
+    model = dc.Model(wl, gen.flat_blob(wl, w), max_batch=wl.batch, max_steps=1)
+    lat = torch.tensor(x1, device="cuda")
+    dc.denoise(model, lat, list(trajs), dc.SchedArgs(1, sig, no_anchors(dc, 1, wl.h_max), 0.0,
+                                                      forced=np.ones((wl.batch, 2), np.uint8)))
+    tdt = torch.float32 if wl.dtype == "f32" else torch.bfloat16
+    for s in range(wl.batch):
+        v, u, r = om.full_step(x1[s], sig[0], trajs[s])
+        buf = torch.zeros((wl.n_tokens, wl.d_model), device="cuda", dtype=tdt)
+        dc.cache_copy(model, s, buf)
+        torch.cuda.synchronize()
+        got_r = buf.float().cpu().numpy()
+        assert np.linalg.norm(r) > 0.3 * np.linalg.norm(u)
+        assert rel(got_r, r) <= tol, rel(got_r, r)
+        x2 = x1[s] + (sig[1] - sig[0]) * v
+        assert rel(lat[s].cpu().numpy() - x1[s], x2 - x1[s]) <= tol
+    model.close()
