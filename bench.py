@@ -215,6 +215,15 @@ def run_reference(args, wl, rank, world):
 
 # ------------------------------------------------------------ main bench
 
+def ratio_summary(st):
+    """Quantiles of d_obs / d_bar over the drift checks of one call."""
+    m = st["checked"] > 0
+    if not np.any(m):
+        return None
+    r = st["d_obs"][m] / st["d_bar"][m]
+    return {"min": float(r.min()), "median": float(np.median(r)), "max": float(r.max())}
+
+
 def main():
     args = parse()
     wl = WORKLOADS[args.workload]
@@ -355,7 +364,10 @@ def main():
         "full_compute_steps_per_s": world * B * K / (full_ms / 1000.0),
         "speedup_vs_full_compute": full_ms / ms_step,
         "schedule": {"compute_scene_steps": n_comp, "reuse_scene_steps": n_reuse,
+                     "planned_reuse_scene_steps": int(np.sum(stats0["planned"][:, 1:] == dc.REUSE)),
+                     "checks": int(np.sum(stats0["checked"] > 0)),
                      "vetoes": int(np.sum(stats0["n_veto"])),
+                     "d_obs_over_d_bar": ratio_summary(stats0),
                      "unsupported_scenes": int(B - np.sum(stats0["supported"]))},
         "gpu_launches": int(launches),
         "e2e": {"value": world * B * K / (e2e_step / 1000.0), "unit": UNIT,

@@ -88,10 +88,14 @@ __global__ void cond_combine_kernel(const float* __restrict__ temb, const float*
 // ------------------------------------------------------------- embedding
 
 template <typename T>
-__global__ void embed_kernel(const float* __restrict__ x, const float* __restrict__ w_e,
+__device__ __forceinline__ float4 load4(const T* src);
+
+// u = x W_e^T + b_e + pos, one thread per 4 consecutive outputs; W_e is read
+// transposed ([C][d]) so that the threads of a warp load contiguous float4.
+template <typename T, int C>
+__global__ void embed_kernel(const float* __restrict__ x, const float* __restrict__ w_eT,
                              const float* __restrict__ b_e, const T* __restrict__ pos, SlotMap map,
-                             int N, int C, int d, float* __restrict__ u, float* __restrict__ h) {
-  // one thread per 4 consecutive outputs of one token of one slot
+                             int N, int d, float* __restrict__ u) {
   const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int d4 = d >> 2;
   const size_t total = (size_t)map.n * N * d4;
@@ -99,19 +103,22 @@ __global__ void embed_kernel(const float* __restrict__ x, const float* __restric
   const int e4 = (int)(i % d4);
   const size_t row = i / d4;  // slot * N + tok
   const int slot = (int)(row / N), tok = (int)(row - (size_t)slot * N);
-  const float* xr = x + ((size_t)map.scene[slot] * N + tok) * C;
-  float acc[4];
+  const float4* xr = reinterpret_cast<const float4*>(x + ((size_t)map.scene[slot] * N + tok) * C);
+  float xv[C];
 #pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    const int e = e4 * 4 + j;
-    float a = b_e[e] + to_f(pos[(size_t)tok * d + e]);
-    const float* w = w_e + (size_t)e * C;
-    for (int c = 0; c < C; ++c) a += w[c] * xr[c];
-    acc[j] = a;
+  for (int c = 0; c < C / 4; ++c) {
+    const float4 t = __ldg(xr + c);
+    xv[4 * c] = t.x; xv[4 * c + 1] = t.y; xv[4 * c + 2] = t.z; xv[4 * c + 3] = t.w;
   }
-  const float4 v = make_float4(acc[0], acc[1], acc[2], acc[3]);
-  reinterpret_cast<float4*>(u)[i] = v;
-  reinterpret_cast<float4*>(h)[i] = v;
+  const float4 bv = __ldg(reinterpret_cast<const float4*>(b_e) + e4);
+  const float4 pv = load4<T>(pos + (size_t)tok * d + 4 * e4);
+  float4 acc = make_float4(bv.x + pv.x, bv.y + pv.y, bv.z + pv.z, bv.w + pv.w);
+#pragma unroll
+  for (int c = 0; c < C; ++c) {
+    const float4 w = __ldg(reinterpret_cast<const float4*>(w_eT + (size_t)c * d) + e4);
+    acc.x += w.x * xv[c]; acc.y += w.y * xv[c]; acc.z += w.z * xv[c]; acc.w += w.w * xv[c];
+  }
+  reinterpret_cast<float4*>(u)[i] = acc;
 }
 
 // --------------------------------------------------------------- LN + mod
@@ -294,7 +301,7 @@ __global__ void final_compute_kernel(const float* __restrict__ hL, const float* 
 
 template <typename T, int NV, int C>
 __global__ void final_reuse_kernel(float* __restrict__ x, const T* __restrict__ r,
-                                   const float* __restrict__ w_e, const float* __restrict__ b_e,
+                                   const float* __restrict__ w_eT, const float* __restrict__ b_e,
                                    const T* __restrict__ pos, SlotMap map, int N, int d,
                                    const float* __restrict__ mod, int mod_stride, int fin_off,
                                    const float* __restrict__ w_f, const float* __restrict__ b_f,
@@ -318,15 +325,15 @@ __global__ void final_reuse_kernel(float* __restrict__ x, const T* __restrict__ 
     if (i < d4) {
       const float4 rv = load4<T>(rr + 4 * i);
       const float4 pv = load4<T>(pr + 4 * i);
-      const float4 bv = reinterpret_cast<const float4*>(b_e)[i];
-      float o[4] = {bv.x + pv.x, bv.y + pv.y, bv.z + pv.z, bv.w + pv.w};
+      const float4 bv = __ldg(reinterpret_cast<const float4*>(b_e) + i);
+      float4 o = make_float4(bv.x + pv.x + rv.x, bv.y + pv.y + rv.y, bv.z + pv.z + rv.z,
+                             bv.w + pv.w + rv.w);
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const float* w = w_e + (size_t)(4 * i + q) * C;
-#pragma unroll
-        for (int c = 0; c < C; ++c) o[q] += w[c] * xv[c];
+      for (int c = 0; c < C; ++c) {
+        const float4 w = __ldg(reinterpret_cast<const float4*>(w_eT + (size_t)c * d) + i);
+        o.x += w.x * xv[c]; o.y += w.y * xv[c]; o.z += w.z * xv[c]; o.w += w.w * xv[c];
       }
-      hv[j] = make_float4(o[0] + rv.x, o[1] + rv.y, o[2] + rv.z, o[3] + rv.w);
+      hv[j] = o;
     } else {
       hv[j] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
@@ -352,38 +359,55 @@ __global__ void final_reuse_kernel(float* __restrict__ x, const T* __restrict__ 
 
 // ------------------------------------------------------------ drift sums
 
-template <typename T, int C>
-__global__ void drift_partial_kernel(DriftItems items, const float* __restrict__ w_e,
-                                     const float* __restrict__ b_e, const T* __restrict__ pos,
-                                     int N, int d, float* __restrict__ partials) {
+// Drift sums in Gram form: with u_t = x_t W_e^T + g_t (g_t = b_e + pos_t),
+//   ||u_t - u'_t||^2 = dx_t^T G dx_t,   ||u_t||^2 = x_t^T G x_t + 2 x_t . gp_t + gs_t
+// where G = W_e^T W_e [C][C], gp_t = W_e^T g_t and gs_t = ||g_t||^2 are fixed
+// tables of the model.  One thread per token, fixed token-to-thread mapping
+// and fixed reduction trees: the sums are deterministic.
+template <int C>
+__global__ void drift_partial_kernel(DriftItems items, const float* __restrict__ gram,
+                                     const float* __restrict__ gp, const float* __restrict__ gs,
+                                     int N, float* __restrict__ partials) {
+  __shared__ float sG[C * C];
+  __shared__ float red[32][2];
+  for (int i = threadIdx.x; i < C * C; i += blockDim.x) sG[i] = gram[i];
+  __syncthreads();
   const int part = blockIdx.x, item = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nw = blockDim.x >> 5;
   const int per = (N + kDriftParts - 1) / kDriftParts;
   const int t0 = part * per, t1 = min(N, t0 + per);
-  const float* xn = items.now[item];
-  const float* xr = items.ref[item];
+  const float4* xn = reinterpret_cast<const float4*>(items.now[item]);
+  const float4* xr = reinterpret_cast<const float4*>(items.ref[item]);
   float sd = 0.f, su = 0.f;
-  for (int t = t0 + warp; t < t1; t += nw) {
-    float xv[C], dv[C];
+  for (int t = t0 + (int)threadIdx.x; t < t1; t += blockDim.x) {
+    float xv[C], dv[C], gv[C];
 #pragma unroll
-    for (int c = 0; c < C; ++c) {
-      xv[c] = xn[(size_t)t * C + c];
-      dv[c] = xv[c] - xr[(size_t)t * C + c];
+    for (int c = 0; c < C / 4; ++c) {
+      const float4 a = __ldg(xn + (size_t)t * (C / 4) + c);
+      const float4 b = __ldg(xr + (size_t)t * (C / 4) + c);
+      const float4 g = __ldg(reinterpret_cast<const float4*>(gp) + (size_t)t * (C / 4) + c);
+      xv[4 * c] = a.x; xv[4 * c + 1] = a.y; xv[4 * c + 2] = a.z; xv[4 * c + 3] = a.w;
+      dv[4 * c] = a.x - b.x; dv[4 * c + 1] = a.y - b.y; dv[4 * c + 2] = a.z - b.z;
+      dv[4 * c + 3] = a.w - b.w;
+      gv[4 * c] = g.x; gv[4 * c + 1] = g.y; gv[4 * c + 2] = g.z; gv[4 * c + 3] = g.w;
     }
-    for (int e = lane; e < d; e += 32) {
-      const float* w = w_e + (size_t)e * C;
-      float du = 0.f, uu = b_e[e] + to_f(pos[(size_t)t * d + e]);
+    float qd = 0.f, qx = 0.f, lin = 0.f;
 #pragma unroll
-      for (int c = 0; c < C; ++c) {
-        du += w[c] * dv[c];
-        uu += w[c] * xv[c];
+    for (int a = 0; a < C; ++a) {
+      float md = 0.f, mx = 0.f;
+#pragma unroll
+      for (int b = 0; b < C; ++b) {
+        md += sG[a * C + b] * dv[b];
+        mx += sG[a * C + b] * xv[b];
       }
-      sd += du * du;
-      su += uu * uu;
+      qd += dv[a] * md;
+      qx += xv[a] * mx;
+      lin += xv[a] * gv[a];
     }
+    sd += qd;
+    su += qx + 2.f * lin + __ldg(gs + t);
   }
-  __shared__ float red[32][2];
   sd = warp_sum(sd);
   su = warp_sum(su);
   if (lane == 0) { red[warp][0] = sd; red[warp][1] = su; }
@@ -465,19 +489,25 @@ cudaError_t launch_cond_combine(const float* temb, const float* traj, int K, int
 }
 
 template <typename T>
-cudaError_t launch_embed(const float* x, const float* w_e, const float* b_e, const T* pos,
-                         const SlotMap& map, int N, int C, int d, float* u, float* h,
-                         cudaStream_t st) {
+cudaError_t launch_embed(const float* x, const float* w_eT, const float* b_e, const T* pos,
+                         const SlotMap& map, int N, int C, int d, float* u, cudaStream_t st) {
   if (map.n <= 0) return cudaSuccess;
   const size_t n = (size_t)map.n * N * (d / 4);
-  embed_kernel<T><<<(unsigned)((n + 255) / 256), 256, 0, st>>>(x, w_e, b_e, pos, map, N, C, d, u, h);
+  const unsigned blocks = (unsigned)((n + 255) / 256);
+  if (C == 16) {
+    embed_kernel<T, 16><<<blocks, 256, 0, st>>>(x, w_eT, b_e, pos, map, N, d, u);
+  } else if (C == 4) {
+    embed_kernel<T, 4><<<blocks, 256, 0, st>>>(x, w_eT, b_e, pos, map, N, d, u);
+  } else {
+    return cudaErrorInvalidValue;
+  }
   return cudaGetLastError();
 }
 template cudaError_t launch_embed<float>(const float*, const float*, const float*, const float*,
-                                         const SlotMap&, int, int, int, float*, float*, cudaStream_t);
+                                         const SlotMap&, int, int, int, float*, cudaStream_t);
 template cudaError_t launch_embed<__nv_bfloat16>(const float*, const float*, const float*,
                                                  const __nv_bfloat16*, const SlotMap&, int, int,
-                                                 int, float*, float*, cudaStream_t);
+                                                 int, float*, cudaStream_t);
 
 template <typename T>
 cudaError_t launch_ln_mod(const float* h, int rows, int N, int d, const float* mod, int mod_stride,
@@ -553,15 +583,15 @@ template cudaError_t launch_final_reuse<__nv_bfloat16>(float*, const __nv_bfloat
                                                        int, int, const float*, const float*, float,
                                                        cudaStream_t);
 
-template <typename T>
-cudaError_t launch_drift(const DriftItems& items, const float* w_e, const float* b_e, const T* pos,
-                         int N, int C, int d, float* partials, float* out, cudaStream_t st) {
+cudaError_t launch_drift(const DriftItems& items, const float* gram, const float* gp,
+                         const float* gs, int N, int C, float* partials, float* out,
+                         cudaStream_t st) {
   if (items.n <= 0) return cudaSuccess;
   dim3 grid(kDriftParts, items.n);
   if (C == 16) {
-    drift_partial_kernel<T, 16><<<grid, 256, 0, st>>>(items, w_e, b_e, pos, N, d, partials);
+    drift_partial_kernel<16><<<grid, 128, 0, st>>>(items, gram, gp, gs, N, partials);
   } else if (C == 4) {
-    drift_partial_kernel<T, 4><<<grid, 256, 0, st>>>(items, w_e, b_e, pos, N, d, partials);
+    drift_partial_kernel<4><<<grid, 128, 0, st>>>(items, gram, gp, gs, N, partials);
   } else {
     return cudaErrorInvalidValue;
   }
@@ -570,10 +600,5 @@ cudaError_t launch_drift(const DriftItems& items, const float* w_e, const float*
   drift_final_kernel<<<(items.n + 63) / 64, 64, 0, st>>>(partials, items.n, out);
   return cudaGetLastError();
 }
-template cudaError_t launch_drift<float>(const DriftItems&, const float*, const float*, const float*,
-                                         int, int, int, float*, float*, cudaStream_t);
-template cudaError_t launch_drift<__nv_bfloat16>(const DriftItems&, const float*, const float*,
-                                                 const __nv_bfloat16*, int, int, int, float*,
-                                                 float*, cudaStream_t);
 
 }  // namespace dc

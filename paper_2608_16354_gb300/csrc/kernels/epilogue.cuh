@@ -19,7 +19,8 @@ struct EpiArgs {
   const float* bias;   // [N]
   void* out;           // QKV: q/k/v base; GELU: [M][N]
   int d, heads, dh, dhp, nslots;  // QKV layout
-  float* h;            // Resid: fp32 residual [M][N]
+  float* h;            // Resid: fp32 residual written [M][N]
+  const float* h_in;   // Resid: residual read (== h, or the block-stack input u)
   const float* mod;    // Resid: modulation table of this step [B][mod_stride]
   int mod_stride;      // floats per scene in the table
   int gate_off;        // offset of this block's gate vector inside a scene's row
@@ -60,19 +61,82 @@ __device__ __forceinline__ void epilogue8(const EpiArgs& e, const SlotMap& map, 
     Pack8<T>::store(dst, v);
   } else if constexpr (MODE == kEpiGELU) {
 #pragma unroll
-    for (int i = 0; i < 8; ++i) v[i] = gelu_tanh(v[i]);
+    for (int i = 0; i < 8; ++i) v[i] = sizeof(T) == 2 ? gelu_tanh_bf16(v[i]) : gelu_tanh(v[i]);
     Pack8<T>::store(reinterpret_cast<T*>(e.out) + (size_t)row * e.N + col, v);
   } else {
     const int slot = row / e.n_tok;
     const float* g = e.mod + (size_t)map.scene[slot] * e.mod_stride + e.gate_off + col;
     const float4 g0 = *reinterpret_cast<const float4*>(g);
     const float4 g1 = *reinterpret_cast<const float4*>(g + 4);
+    const float4* hi = reinterpret_cast<const float4*>(e.h_in + (size_t)row * e.N + col);
     float4* hp = reinterpret_cast<float4*>(e.h + (size_t)row * e.N + col);
-    float4 h0 = hp[0], h1 = hp[1];
+    float4 h0 = hi[0], h1 = hi[1];
     h0.x += g0.x * v[0]; h0.y += g0.y * v[1]; h0.z += g0.z * v[2]; h0.w += g0.w * v[3];
     h1.x += g1.x * v[4]; h1.y += g1.y * v[5]; h1.z += g1.z * v[6]; h1.w += g1.w * v[7];
     hp[0] = h0;
     hp[1] = h1;
+  }
+}
+
+// Epilogue of one 32 x 32 block staged in shared memory (stg[r * 33 + c],
+// r = row within the block, c = column within the block).  The warp writes
+// whole rows: fp32 residual rows of 128 B, bf16 rows of 64 B (two rows per
+// instruction), so every store and load is coalesced.
+template <int MODE>
+__device__ __forceinline__ void epilogue_block32(const EpiArgs& e, const SlotMap& map,
+                                                 const float* stg, int row0, int col0, int lane) {
+  if constexpr (MODE == kEpiResid) {
+    // all 32 residual loads are issued before any store (h and h_in may
+    // alias, so the compiler would otherwise serialise load -> store pairs)
+    const int col = col0 + lane;
+    const float b = e.bias[col];
+    const int nrow = min(32, e.M - row0);
+    const int s_first = row0 / e.n_tok;
+    const int s_last = (row0 + nrow - 1) / e.n_tok;
+    const float g_first = e.mod[(size_t)map.scene[s_first] * e.mod_stride + e.gate_off + col];
+    const float g_last = e.mod[(size_t)map.scene[s_last] * e.mod_stride + e.gate_off + col];
+    const int row_split = (s_first + 1) * e.n_tok;  // first row of the next slot
+    float hv[32];
+#pragma unroll
+    for (int r = 0; r < 32; ++r)
+      hv[r] = r < nrow ? __ldcs(e.h_in + (size_t)(row0 + r) * e.N + col) : 0.f;
+#pragma unroll
+    for (int r = 0; r < 32; ++r) {
+      if (r < nrow) {
+        const float g = row0 + r < row_split ? g_first : g_last;
+        e.h[(size_t)(row0 + r) * e.N + col] = hv[r] + g * (stg[r * 33 + lane] + b);
+      }
+    }
+  } else {
+    const int cc = 2 * (lane & 15);
+    const int col = col0 + cc;
+    const float b0 = e.bias[col], b1 = e.bias[col + 1];
+    int which = 0, head = 0, c = 0;
+    if constexpr (MODE == kEpiQKV) {
+      which = col / e.d;
+      const int within = col - which * e.d;
+      head = within / e.dh;
+      c = within - head * e.dh;
+    }
+    for (int i = 0; i < 16; ++i) {
+      const int r = 2 * i + (lane >> 4);
+      const int row = row0 + r;
+      if (row >= e.M) break;
+      float v0 = stg[r * 33 + cc] + b0, v1 = stg[r * 33 + cc + 1] + b1;
+      if constexpr (MODE == kEpiGELU) {
+        v0 = gelu_tanh(v0);
+        v1 = gelu_tanh(v1);
+        *reinterpret_cast<__nv_bfloat162*>(reinterpret_cast<__nv_bfloat16*>(e.out) +
+                                           (size_t)row * e.N + col) = __floats2bfloat162_rn(v0, v1);
+      } else {
+        const int slot = row / e.n_tok;
+        const int tok = row - slot * e.n_tok;
+        __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(e.out) +
+                             ((((size_t)which * e.nslots + slot) * e.heads + head) * e.n_tok + tok) *
+                                 e.dhp + c;
+        *reinterpret_cast<__nv_bfloat162*>(dst) = __floats2bfloat162_rn(v0, v1);
+      }
+    }
   }
 }
 

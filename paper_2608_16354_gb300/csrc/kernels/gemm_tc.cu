@@ -28,7 +28,9 @@ constexpr int kTmemCols = 512;                // two 192-column accumulators at 
 constexpr int kThreads = 320;                 // 10 warps
 constexpr int kEpiWarps = 8;
 constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, kBN);
-constexpr size_t kSmemBytes = 1024 + (size_t)kStages * kStageBytes + 256;
+constexpr int kStgFloats = 32 * 33;           // per epilogue warp: 32 x 32 block, padded
+constexpr size_t kSmemBytes =
+    1024 + (size_t)kStages * kStageBytes + 256 + (size_t)kEpiWarps * kStgFloats * 4;
 
 struct __align__(8) Barriers {
   uint64_t full[kStages];
@@ -50,6 +52,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* sA = smem;
   uint8_t* sB = smem + (size_t)kStages * kABytes;
   Barriers* bar = reinterpret_cast<Barriers*>(smem + (size_t)kStages * kStageBytes);
+  float* stg_all = reinterpret_cast<float*>(smem + (size_t)kStages * kStageBytes + 256);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -58,6 +61,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int n_tiles = tiles_m * tiles_n;
   const int KB = K / kBK;
 
+  // a bounded wait of an earlier launch gave up: do nothing (the host
+  // reports DC_ERR_DEVICE_TIMEOUT at its next check)
+  if (*(volatile int*)err != 0) return;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&bar->full[s], 1);
@@ -149,7 +155,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       const int m0 = (tile / tiles_n) * kBM;
       const int n0 = (tile % tiles_n) * kBN;
-      const int row = m0 + q * 32 + lane;
       float acc[3][32];
 #pragma unroll
       for (int c = 0; c < 3; ++c) {
@@ -161,15 +166,35 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&bar->tmem_empty[b]);
-      if (row < M) {
+      const int row0 = m0 + q * 32;
+      if constexpr (MODE == kEpiResid) {
+        // fp32 read-modify-write of the residual: transpose each 32 x 32
+        // block through shared memory so that the warp reads and writes
+        // whole 128-byte rows
+        float* stg = stg_all + (warp - 2) * kStgFloats;
+        if (row0 < M) {
 #pragma unroll
-        for (int c = 0; c < 3; ++c) {
+          for (int c = 0; c < 3; ++c) {
 #pragma unroll
-          for (int g = 0; g < 4; ++g) {
-            float v[8];
+            for (int i = 0; i < 32; ++i) stg[lane * 33 + i] = acc[c][i];
+            __syncwarp();
+            epilogue_block32<MODE>(ep, map, stg, row0, n0 + half * 96 + c * 32, lane);
+            __syncwarp();
+          }
+        }
+      } else {
+        // bf16 outputs: each thread stores 16-byte pieces of its own row
+        const int row = row0 + lane;
+        if (row < M) {
 #pragma unroll
-            for (int i = 0; i < 8; ++i) v[i] = acc[c][g * 8 + i];
-            epilogue8<MODE, __nv_bfloat16>(ep, map, row, n0 + half * 96 + c * 32 + g * 8, v);
+          for (int c = 0; c < 3; ++c) {
+#pragma unroll
+            for (int g = 0; g < 4; ++g) {
+              float v[8];
+#pragma unroll
+              for (int i = 0; i < 8; ++i) v[i] = acc[c][g * 8 + i];
+              epilogue8<MODE, __nv_bfloat16>(ep, map, row, n0 + half * 96 + c * 32 + g * 8, v);
+            }
           }
         }
       }

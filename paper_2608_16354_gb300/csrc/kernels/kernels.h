@@ -24,11 +24,10 @@ cudaError_t launch_cond_combine(const float* temb, const float* traj, int K, int
                                 float* silu_c, cudaStream_t st);
 
 // ---- per-step kernels --------------------------------------------------
-// u = x W_e^T + b_e + pos (fp32) for each compute slot; h = u
+// u = x W_e^T + b_e + pos (fp32) for each compute slot; w_eT = W_e^T [C][d]
 template <typename T>
-cudaError_t launch_embed(const float* x, const float* w_e, const float* b_e, const T* pos,
-                         const SlotMap& map, int N, int C, int d, float* u, float* h,
-                         cudaStream_t st);
+cudaError_t launch_embed(const float* x, const float* w_eT, const float* b_e, const T* pos,
+                         const SlotMap& map, int N, int C, int d, float* u, cudaStream_t st);
 // a = LN(h) * (1 + scale) + shift  (per-slot modulation)  -> T
 template <typename T>
 cudaError_t launch_ln_mod(const float* h, int rows, int N, int d, const float* mod, int mod_stride,
@@ -48,30 +47,37 @@ cudaError_t launch_attention_bf16(const __nv_bfloat16* qkv, int slots, int heads
                                   int dhp, __nv_bfloat16* o, cudaStream_t st);
 cudaError_t launch_attention_f32(const float* qkv, int slots, int heads, int N, int dh, int dhp,
                                  float* o, cudaStream_t st);
+// tcgen05 attention (dh = dhp = 64 or 128): tm is a 2-D bf16 map over the
+// q/k/v buffer viewed as [3 * slots * heads * N][dhp], box 64 x 128, 128-byte
+// swizzle; err receives a code if a bounded wait gives up
+bool attention_tc_supported(int dh);
+cudaError_t launch_attention_tc(const CUtensorMap& tm, int nslots, int heads, int N, int dh,
+                                __nv_bfloat16* o, int* err, cudaStream_t st);
 // compute-step interface + Euler: v = head(h_L); x_j <- x; x += dsig v; r <- h_L - u
 template <typename T>
 cudaError_t launch_final_compute(const float* hL, const float* u, float* x, float* xj, T* r,
                                  const SlotMap& map, int N, int C, int d, const float* mod,
                                  int mod_stride, int fin_off, const float* w_f, const float* b_f,
                                  float dsig, cudaStream_t st);
-// reuse step: u = embed(x); h = u + r_j; v = head(h); x += dsig v
+// reuse step: u = embed(x); h = u + r_j; v = head(h); x += dsig v  (w_eT = W_e^T [C][d])
 template <typename T>
-cudaError_t launch_final_reuse(float* x, const T* r, const float* w_e, const float* b_e,
+cudaError_t launch_final_reuse(float* x, const T* r, const float* w_eT, const float* b_e,
                                const T* pos, const SlotMap& map, int N, int C, int d,
                                const float* mod, int mod_stride, int fin_off, const float* w_f,
                                const float* b_f, float dsig, cudaStream_t st);
 
 // drift sums over items: out[2i] = sum ||(now_i - ref_i) W_e^T||^2,
-// out[2i+1] = sum ||now_i W_e^T + b_e + pos||^2   (deterministic order)
+// out[2i+1] = sum ||now_i W_e^T + b_e + pos||^2   (deterministic order),
+// evaluated with the Gram tables gram = W_e^T W_e [C][C],
+// gp[t] = W_e^T (b_e + pos_t) [N][C] and gs[t] = ||b_e + pos_t||^2 [N]
 struct DriftItems {
   int n;
   const float* now[kMaxBatch];
   const float* ref[kMaxBatch];
 };
 constexpr int kDriftParts = 64;
-template <typename T>
-cudaError_t launch_drift(const DriftItems& items, const float* w_e, const float* b_e, const T* pos,
-                         int N, int C, int d, float* partials /* [n][kDriftParts][2] */,
+cudaError_t launch_drift(const DriftItems& items, const float* gram, const float* gp,
+                         const float* gs, int N, int C, float* partials /* [n][kDriftParts][2] */,
                          float* out /* [2n] */, cudaStream_t st);
 
 }  // namespace dc

@@ -54,7 +54,9 @@ struct dc_model {
   double *poses_d = nullptr, *sig_d = nullptr;
   int* err_d = nullptr;
   float* drift_host = nullptr;  // pinned
-  CUtensorMap tm_a, tm_oact, tm_m;
+  // derived tables: W_e^T [C][d] and the Gram tables of the drift sums
+  float *w_eT = nullptr, *gram = nullptr, *gp = nullptr, *gs = nullptr;
+  CUtensorMap tm_a, tm_oact, tm_m, tm_qkv;
   long long launches = 0;
   // per-kernel profiling (dc_profile)
   struct ProfRec { int cat; cudaEvent_t a, b; double flops, bytes; };
@@ -279,9 +281,9 @@ dc_status enqueue_compute(dc_model* m, float* lat, const float* mod_k, const Slo
   T* o = static_cast<T*>(m->o);
   T* mm = static_cast<T*>(m->m);
   const double Md = (double)M * d, E = (double)m->elt;
-  DC_LAUNCH(DC_PROF_EMBED, 2.0 * M * d * m->C, 4.0 * M * m->C + 8.0 * Md + (double)N * d * E,
-            dc::launch_embed<T>(lat, m->w_e, m->b_e, static_cast<const T*>(m->pos), map, N, m->C,
-                                d, m->u, m->h, st));
+  DC_LAUNCH(DC_PROF_EMBED, 2.0 * M * d * m->C, 4.0 * M * m->C + 4.0 * Md + (double)N * d * E,
+            dc::launch_embed<T>(lat, m->w_eT, m->b_e, static_cast<const T*>(m->pos), map, N, m->C,
+                                d, m->u, st));
   m->launches += 1;
   const double ln_bytes = 4.0 * Md + E * Md;
   const double attn_flops = 4.0 * nc * (double)N * N * d;
@@ -299,17 +301,19 @@ dc_status enqueue_compute(dc_model* m, float* lat, const float* mod_k, const Slo
   for (int l = 0; l < m->L; ++l) {
     const BlockW& w = m->blk[l];
     const int base = l * 6 * d;
+    // block 0 reads the block-stack input u directly (h = u is never copied)
+    const float* h_in = l == 0 ? m->u : m->h;
     DC_LAUNCH(DC_PROF_LN, 0.0, ln_bytes,
-              dc::launch_ln_mod<T>(m->h, M, N, d, mod_k, m->mod_stride, base + 0 * d, base + 1 * d,
+              dc::launch_ln_mod<T>(h_in, M, N, d, mod_k, m->mod_stride, base + 0 * d, base + 1 * d,
                                    map, a, st));
     dc::EpiArgs e1 = ep;
     e1.N = 3 * d; e1.bias = w.b_qkv; e1.out = qkv;
     dc::EpiArgs e2 = ep;
-    e2.N = d; e2.bias = w.b_o; e2.h = m->h; e2.gate_off = base + 2 * d;
+    e2.N = d; e2.bias = w.b_o; e2.h = m->h; e2.h_in = h_in; e2.gate_off = base + 2 * d;
     dc::EpiArgs e3 = ep;
     e3.N = m->md; e3.bias = w.b_1; e3.out = mm;
     dc::EpiArgs e4 = ep;
-    e4.N = d; e4.bias = w.b_2; e4.h = m->h; e4.gate_off = base + 5 * d;
+    e4.N = d; e4.bias = w.b_2; e4.h = m->h; e4.h_in = m->h; e4.gate_off = base + 5 * d;
     const double f_qkv = 2.0 * M * 3.0 * d * d, f_o = 2.0 * M * (double)d * d,
                  f_mlp = 2.0 * M * (double)m->md * d;
     const double b_qkv = E * (Md + 3.0 * d * d + 3.0 * Md), b_o = E * (Md + (double)d * d) + 8.0 * Md,
@@ -319,9 +323,16 @@ dc_status enqueue_compute(dc_model* m, float* lat, const float* mod_k, const Slo
       DC_LAUNCH(DC_PROF_GEMM_QKV, f_qkv, b_qkv,
                 dc::launch_gemm_tc(dc::kEpiQKV, m->tm_a, w.tm_qkv, M, 3 * d, d, e1, map, m->err_d,
                                    m->n_sms, st));
-      DC_LAUNCH(DC_PROF_ATTENTION, attn_flops, attn_bytes,
-                dc::launch_attention_bf16(reinterpret_cast<const __nv_bfloat16*>(qkv), nc, m->heads,
-                                          N, m->dh, m->dhp, reinterpret_cast<__nv_bfloat16*>(o), st));
+      if (dc::attention_tc_supported(m->dh)) {
+        DC_LAUNCH(DC_PROF_ATTENTION, attn_flops, attn_bytes,
+                  dc::launch_attention_tc(m->tm_qkv, nc, m->heads, N, m->dh,
+                                          reinterpret_cast<__nv_bfloat16*>(o), m->err_d, st));
+      } else {
+        DC_LAUNCH(DC_PROF_ATTENTION, attn_flops, attn_bytes,
+                  dc::launch_attention_bf16(reinterpret_cast<const __nv_bfloat16*>(qkv), nc,
+                                            m->heads, N, m->dh, m->dhp,
+                                            reinterpret_cast<__nv_bfloat16*>(o), st));
+      }
       DC_LAUNCH(DC_PROF_GEMM_OUT, f_o, b_o,
                 dc::launch_gemm_tc(dc::kEpiResid, m->tm_oact, w.tm_o, M, d, d, e2, map, m->err_d,
                                    m->n_sms, st));
@@ -372,7 +383,7 @@ dc_status enqueue_reuse(dc_model* m, float* lat, const float* mod_k, const SlotM
   // algorithmic bytes of a reuse scene-step: r_j (N d elements) + x_k read,
   // x_{k+1} written and x_j read by the drift check (3 N C fp32)
   DC_LAUNCH(DC_PROF_REUSE, 4.0 * M * m->d * m->C, M * ((double)m->d * m->elt + 12.0 * m->C),
-            dc::launch_final_reuse<T>(lat, static_cast<const T*>(m->r), m->w_e, m->b_e,
+            dc::launch_final_reuse<T>(lat, static_cast<const T*>(m->r), m->w_eT, m->b_e,
                                       static_cast<const T*>(m->pos), map, m->N, m->C, m->d, mod_k,
                                       m->mod_stride, 6 * m->L * m->d, m->w_f, m->b_f, dsig, st));
   m->launches += 1;
@@ -381,9 +392,9 @@ dc_status enqueue_reuse(dc_model* m, float* lat, const float* mod_k, const SlotM
 
 template <typename T>
 dc_status enqueue_drift(dc_model* m, const dc::DriftItems& it, float* out, cudaStream_t st) {
-  DC_LAUNCH(DC_PROF_DRIFT, 4.0 * it.n * m->N * m->d * m->C, 8.0 * it.n * m->N * m->C,
-            dc::launch_drift<T>(it, m->w_e, m->b_e, static_cast<const T*>(m->pos), m->N, m->C,
-                                m->d, m->drift_part, out, st));
+  // algorithmic bytes: x_now and x_ref of every item (2 N C fp32)
+  DC_LAUNCH(DC_PROF_DRIFT, 4.0 * it.n * m->N * m->C * m->C, 8.0 * it.n * m->N * m->C,
+            dc::launch_drift(it, m->gram, m->gp, m->gs, m->N, m->C, m->drift_part, out, st));
   m->launches += 2;
   return DC_OK;
 }
@@ -723,7 +734,9 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
       {(void**)&m->drift_part, (size_t)dc::kMaxBatch * dc::kDriftParts * 2 * 4},
       {(void**)&m->drift_out, (size_t)dc::kMaxBatch * 2 * 4},
       {(void**)&m->poses_d, B * m->P * 3 * 8}, {(void**)&m->sig_d, (K + 1) * 8},
-      {(void**)&m->err_d, 256}};
+      {(void**)&m->err_d, 256}, {(void**)&m->w_eT, (size_t)m->C * d * 4},
+      {(void**)&m->gram, (size_t)m->C * m->C * 4}, {(void**)&m->gp, N * m->C * 4},
+      {(void**)&m->gs, N * 4}};
   size_t wsb = 0;
   for (auto& b : bufs) wsb += align256(b.bytes);
   if (cudaMalloc(&m->ws, wsb) != cudaSuccess) {
@@ -736,6 +749,49 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
   }
   // zero everything once: the head-dim pad columns of q/k/v stay zero
   if (cudaMemset(m->ws, 0, wsb) != cudaSuccess) return fail(DC_ERR_CUDA);
+  {
+    // W_e^T and the Gram tables of the drift sums (fp64 on the host, from the
+    // values the device uses: pos rounded to bf16 for bf16 models)
+    const int C = m->C, D = (int)d;
+    const float* we = host_weights;                 // w_embed [d][C]
+    const float* be = host_weights + (size_t)D * C;  // b_embed [d]
+    const float* ps = be + D;                        // pos [N][d]
+    std::vector<float> weT((size_t)C * D), gram((size_t)C * C), gp(N * C), gs(N);
+    for (int e = 0; e < D; ++e)
+      for (int c = 0; c < C; ++c) weT[(size_t)c * D + e] = we[(size_t)e * C + c];
+    for (int a = 0; a < C; ++a)
+      for (int b = 0; b < C; ++b) {
+        double acc = 0.0;
+        for (int e = 0; e < D; ++e) acc += (double)we[(size_t)e * C + a] * we[(size_t)e * C + b];
+        gram[(size_t)a * C + b] = (float)acc;
+      }
+    std::vector<double> g(D);
+    for (size_t t = 0; t < N; ++t) {
+      double sq = 0.0;
+      for (int e = 0; e < D; ++e) {
+        float pv = ps[t * D + e];
+        if (m->bf16) {
+          const uint32_t bits = (uint32_t)f2bf_host(pv) << 16;
+          std::memcpy(&pv, &bits, 4);
+        }
+        g[e] = (double)be[e] + (double)pv;
+        sq += g[e] * g[e];
+      }
+      gs[t] = (float)sq;
+      for (int c = 0; c < C; ++c) {
+        double acc = 0.0;
+        for (int e = 0; e < D; ++e) acc += (double)we[(size_t)e * C + c] * g[e];
+        gp[t * C + c] = (float)acc;
+      }
+    }
+    if (cudaMemcpy(m->w_eT, weT.data(), weT.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaMemcpy(m->gram, gram.data(), gram.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaMemcpy(m->gp, gp.data(), gp.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaMemcpy(m->gs, gs.data(), gs.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess) {
+      dc::set_error("upload of the derived tables failed");
+      return fail(DC_ERR_CUDA);
+    }
+  }
   if (cudaMallocHost(&m->drift_host, (size_t)dc::kMaxBatch * 2 * 4) != cudaSuccess) {
     dc::set_error("cudaMallocHost failed");
     return fail(DC_ERR_NOMEM);
@@ -746,6 +802,9 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
     if ((s = make_map(&m->tm_a, m->a, d, B * N, bm)) != DC_OK) return fail(s);
     if ((s = make_map(&m->tm_oact, m->o, d, B * N, bm)) != DC_OK) return fail(s);
     if ((s = make_map(&m->tm_m, m->m, m->md, B * N, bm)) != DC_OK) return fail(s);
+    if (dc::attention_tc_supported(m->dh) &&
+        (s = make_map(&m->tm_qkv, m->qkv, m->dhp, 3 * B * m->heads * N, 128)) != DC_OK)
+      return fail(s);
     for (int l = 0; l < m->L; ++l) {
       BlockW& w = m->blk[l];
       if ((s = make_map(&w.tm_qkv, w.w_qkv, d, 3 * d, bn)) != DC_OK) return fail(s);
@@ -935,6 +994,25 @@ dc_status dc_attention(int dtype, const void* qkv, int slots, int heads, int n_t
       return DC_ERR_UNSUPPORTED;
     }
     const int dhp = ((head_dim + 15) / 16) * 16;
+    if (dc::attention_tc_supported(head_dim)) {
+      // the tensor-core kernel: a TMA map over the caller's buffer and a
+      // library-owned error word; the call waits for the kernel to report
+      static int* err_d = nullptr;
+      if (!err_d) DC_CK(cudaMalloc(&err_d, sizeof(int)));
+      DC_CK(cudaMemsetAsync(err_d, 0, sizeof(int), st));
+      CUtensorMap tm;
+      DC_TRY(make_map(&tm, qkv, dhp, (uint64_t)3 * slots * heads * n_tokens, 128));
+      DC_CK(dc::launch_attention_tc(tm, slots, heads, n_tokens, head_dim,
+                                    static_cast<__nv_bfloat16*>(out), err_d, st));
+      int err = 0;
+      DC_CK(cudaMemcpyAsync(&err, err_d, sizeof(int), cudaMemcpyDeviceToHost, st));
+      DC_CK(cudaStreamSynchronize(st));
+      if (err) {
+        dc::set_error("dc_attention: a bounded device wait gave up");
+        return DC_ERR_DEVICE_TIMEOUT;
+      }
+      return DC_OK;
+    }
     DC_CK(dc::launch_attention_bf16(static_cast<const __nv_bfloat16*>(qkv), slots, heads, n_tokens,
                                     head_dim, dhp, static_cast<__nv_bfloat16*>(out), st));
     return DC_OK;

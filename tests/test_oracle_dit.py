@@ -14,11 +14,8 @@ from oracle import controller as Ctl
 from oracle import planner as P
 from synth import gen
 
-torch.set_default_dtype(torch.float64)
-
-
 def _t(a):
-    return torch.tensor(np.asarray(a, np.float64))
+    return torch.tensor(np.asarray(a, np.float64), dtype=torch.float64)
 
 
 def test_layer_norm_vs_torch():
@@ -50,7 +47,7 @@ def test_attention_vs_torch_multihead(n, d, heads):
     w_o = rng.standard_normal((d, d)) * 0.2
     b_o = rng.standard_normal(d) * 0.1
     ours = O.linear(O.attention(a, w_qkv, b_qkv, heads), w_o, b_o)
-    mha = torch.nn.MultiheadAttention(d, heads, bias=True, batch_first=True)
+    mha = torch.nn.MultiheadAttention(d, heads, bias=True, batch_first=True, dtype=torch.float64)
     with torch.no_grad():
         mha.in_proj_weight.copy_(_t(w_qkv))
         mha.in_proj_bias.copy_(_t(b_qkv))
@@ -64,10 +61,11 @@ def _torch_block(wb, h, mod, heads):
     """The block written with torch modules (LayerNorm without affine,
     MultiheadAttention, Linear, GELU(tanh))."""
     d = h.shape[1]
-    ln = torch.nn.LayerNorm(d, eps=1e-6, elementwise_affine=False)
-    mha = torch.nn.MultiheadAttention(d, heads, bias=True, batch_first=True)
-    fc1 = torch.nn.Linear(d, wb["w_1"].shape[0])
-    fc2 = torch.nn.Linear(wb["w_1"].shape[0], d)
+    f64 = dict(dtype=torch.float64)
+    ln = torch.nn.LayerNorm(d, eps=1e-6, elementwise_affine=False, **f64)
+    mha = torch.nn.MultiheadAttention(d, heads, bias=True, batch_first=True, **f64)
+    fc1 = torch.nn.Linear(d, wb["w_1"].shape[0], **f64)
+    fc2 = torch.nn.Linear(wb["w_1"].shape[0], d, **f64)
     with torch.no_grad():
         mha.in_proj_weight.copy_(_t(wb["w_qkv"]))
         mha.in_proj_bias.copy_(_t(wb["b_qkv"]))
