@@ -222,6 +222,25 @@ dc_status dc_anchor_drift(dc_model* m, const float* noise, const dc_trajectory* 
 dc_status dc_drift_sums(dc_model* m, const float* x_now, const float* x_ref, int B, float* out,
                         void* stream);
 
+/* dc_drift_sums for callers that cannot allocate device memory while they
+ * run (for example a planning loop whose memory budget is fixed at start-up,
+ * or a host process that may not call cudaMalloc after initialisation,
+ * since cudaMalloc can synchronise the device and can fail).  The paper has
+ * no counterpart; this is a deployment variant of the Eq. 12 sums.
+ * Same inputs, outputs and result as dc_drift_sums (x_now, x_ref: DEVICE
+ * fp32 [B][N][C]; out: DEVICE fp32 [2B]), but the reduction scratch is a
+ * fixed 32 KiB array in device memory that every GPU loading this library
+ * holds until the process exits; no device memory is allocated or freed.
+ * B must be in [1, min(max_batch, 64)]; larger B is rejected with
+ * DC_ERR_INVALID_ARG before any launch.  The first call on a device looks up
+ * the array's device address (with that device made current); make that
+ * first call before capturing the stream into a graph.  All calls share the
+ * one array: calls that can overlap on the GPU (different streams without
+ * ordering) race on it and must be serialised by the caller.  Every scratch
+ * entry a call reads is written earlier in the same call. */
+dc_status dc_drift_sums_noalloc(dc_model* m, const float* x_now, const float* x_ref, int B,
+                                float* out, void* stream);
+
 /* Copy the cached backbone output r_j (Eq. 1: r = h_L - u of the scene's
  * last full evaluation) of `scene` (0 <= scene < max_batch) into DEVICE
  * memory dst.  The cache holds [N][d] elements of the model dtype (fp32 or

@@ -110,6 +110,8 @@ def lib():
                                  C.c_int, C.c_double, P(C.c_double), C.c_void_p]),
         "dc_drift_sums": (st, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int, C.c_void_p,
                                C.c_void_p]),
+        "dc_drift_sums_noalloc": (st, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int, C.c_void_p,
+                                       C.c_void_p]),
         "dc_cache_copy": (st, [C.c_void_p, C.c_int, C.c_void_p, C.c_size_t, C.c_void_p]),
         "dc_attention": (st, [C.c_int, C.c_void_p, C.c_int, C.c_int, C.c_int, C.c_int, C.c_void_p,
                               C.c_void_p]),
@@ -395,3 +397,11 @@ def profile_read(model: Model):
     _check(lib().dc_profile_read(model.h, ms, cnt, fl, by))
     return {PROF_NAMES[i]: dict(ms=ms[i], launches=cnt[i], flops=fl[i], bytes=by[i])
             for i in range(n)}
+
+
+def drift_sums_noalloc(model: Model, x_now, x_ref, out, stream=None):
+    """dc_drift_sums_noalloc: same as drift_sums, with no device allocation
+    (fixed scratch inside the library, at most 64 scenes per call)."""
+    _check(lib().dc_drift_sums_noalloc(model.h, C.c_void_p(x_now.data_ptr()),
+                                       C.c_void_p(x_ref.data_ptr()), int(x_now.shape[0]),
+                                       C.c_void_p(out.data_ptr()), _stream_handle(stream)))

@@ -14,8 +14,10 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -1031,3 +1033,79 @@ dc_status dc_attention(int dtype, const void* qkv, int slots, int heads, int n_t
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Drift sums without allocation.
+//
+// Some callers cannot allocate device memory once they are running: a planner
+// loop with a memory budget fixed at start-up, or a host process where a
+// cudaMalloc (which may synchronise the device and can fail under
+// fragmentation) is not allowed after initialisation.  For them the
+// reduction scratch of the drift sums lives in a fixed array in device
+// memory that every GPU loading this library holds until the process exits.
+// ---------------------------------------------------------------------------
+
+namespace {
+
+// Up to this many scenes per call: kNoAllocMaxScenes x kDriftParts x 2 fp32
+// partial sums = 32 KiB of device memory per GPU.
+constexpr int kNoAllocMaxScenes = dc::kMaxBatch;
+static __device__ __align__(256) float g_drift_scratch[kNoAllocMaxScenes * dc::kDriftParts * 2];
+
+std::mutex g_scratch_mu;
+constexpr int kScratchDevices = 64;
+float* g_scratch_addr[kScratchDevices] = {};
+
+// Device address of the scratch array on `dev` (which must be current).  The
+// array's name is only a host-side stand-in; the address is looked up once
+// per device and cached.
+dc_status scratch_address(int dev, float** out) {
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (dev < 0 || dev >= kScratchDevices) {
+    dc::set_error("dc_drift_sums_noalloc: device ordinal out of range");
+    return DC_ERR_UNSUPPORTED;
+  }
+  if (!g_scratch_addr[dev]) {
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_drift_scratch);
+    if (e != cudaSuccess || !p) {
+      dc::set_error(std::string("cudaGetSymbolAddress(drift scratch) failed: ") +
+                    cudaGetErrorString(e));
+      return DC_ERR_CUDA;
+    }
+    g_scratch_addr[dev] = static_cast<float*>(p);
+  }
+  *out = g_scratch_addr[dev];
+  return DC_OK;
+}
+
+}  // namespace
+
+extern "C" dc_status dc_drift_sums_noalloc(dc_model* m, const float* x_now, const float* x_ref,
+                                           int B, float* out, void* stream) {
+  if (!m || !x_now || !x_ref || !out) {
+    dc::set_error("dc_drift_sums_noalloc: NULL pointer");
+    return DC_ERR_INVALID_ARG;
+  }
+  if (B < 1 || B > m->Bmax || B > kNoAllocMaxScenes) {
+    dc::set_error("dc_drift_sums_noalloc: B = " + std::to_string(B) + " outside [1, " +
+                  std::to_string(std::min(m->Bmax, kNoAllocMaxScenes)) +
+                  "] (fixed scratch holds " + std::to_string(kNoAllocMaxScenes) + " scenes)");
+    return DC_ERR_INVALID_ARG;
+  }
+  DC_CK(cudaSetDevice(m->device));
+  float* scratch = nullptr;
+  DC_TRY(scratch_address(m->device, &scratch));
+  dc::DriftItems it{};
+  it.n = B;
+  const size_t NC = (size_t)m->N * m->C;
+  for (int i = 0; i < B; ++i) {
+    it.now[i] = x_now + i * NC;
+    it.ref[i] = x_ref + i * NC;
+  }
+  // every partial the final pass reads is written by the first pass of the
+  // same call, so nothing in the scratch needs clearing
+  DC_CK(dc::launch_drift(it, m->gram, m->gp, m->gs, m->N, m->C, scratch, out,
+                         static_cast<cudaStream_t>(stream)));
+  return DC_OK;
+}
