@@ -6,12 +6,22 @@
 //
 // Design: persistent CTAs (one per SM), 128 x 192 output tiles, K in steps
 // of 64 (one 128-byte swizzle atom per row).  Warp 0 streams A/W tiles with
-// TMA into a 4-stage shared-memory ring; warp 1 owns the TMEM allocation and
-// one elected lane issues tcgen05.mma (M=128, N=192, K=16) into one of two
-// TMEM accumulators; warps 2-9 drain the other accumulator with tcgen05.ld
-// and run the epilogue, so the epilogue of tile i overlaps the MMAs of tile
-// i+1.  N = 192 divides every projection width of the configured models
-// (3d, d, 4d for d = 384, 1152, 3072).  Every mbarrier wait is bounded.
+// TMA into a shared-memory ring; warp 1 owns the TMEM allocation and one
+// elected lane issues tcgen05.mma (M=128, N=192, K=16) into one of two TMEM
+// accumulators; warps 2-9 drain the other accumulator with tcgen05.ld and run
+// the epilogue, so the epilogue of tile i overlaps the MMAs of tile i+1.
+// N = 192 divides every projection width of the configured models (3d, d,
+// 4d for d = 384, 1152, 3072).
+//
+// Epilogues (bias and gate vectors of the tile are staged in shared memory):
+//   QKV      y = acc + b, 16-byte stores into head-major q / k / v
+//   GELU     y = gelu(acc + b) in bf16, written to a swizzled shared tile and
+//            stored with TMA
+//   residual the fp32 residual tile is prefetched with TMA into shared memory
+//            while the MMAs run, h = h_in + gate (acc + b) is formed in place
+//            and the tile goes back with TMA stores, so the epilogue moves
+//            whole tiles at DRAM speed instead of single rows
+// Every mbarrier wait is bounded.
 #include "common.cuh"
 #include "epilogue.cuh"
 #include "kernels.h"
@@ -20,39 +30,61 @@ namespace dc {
 
 namespace {
 
-constexpr int kBM = 128, kBN = 192, kBK = 64, kStages = 4;
+constexpr int kBM = 128, kBN = 192, kBK = 64;
 constexpr int kABytes = kBM * kBK * 2;        // 16 KB
 constexpr int kBBytes = kBN * kBK * 2;        // 24 KB
 constexpr int kStageBytes = kABytes + kBBytes;
 constexpr int kTmemCols = 512;                // two 192-column accumulators at 0 / 256
 constexpr int kThreads = 320;                 // 10 warps
 constexpr int kEpiWarps = 8;
+constexpr int kEpiThreads = kEpiWarps * 32;
 constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, kBN);
-constexpr int kStgFloats = 32 * 33;           // per epilogue warp: 32 x 32 block, padded
-constexpr size_t kSmemBytes =
-    1024 + (size_t)kStages * kStageBytes + 256 + (size_t)kEpiWarps * kStgFloats * 4;
+
+template <int MODE>
+struct GemmCfg {
+  static constexpr int kStages = MODE == kEpiResid ? 3 : 4;
+  // epilogue staging tile: residual 6 boxes of [128 rows][32 fp32], GELU 3
+  // boxes of [128 rows][64 bf16]; 16 KB per box, 128-byte swizzle
+  static constexpr int kOutBytes = MODE == kEpiResid ? 6 * 16384 : MODE == kEpiGELU ? 3 * 16384 : 0;
+  static constexpr int kOffA = 0;
+  static constexpr int kOffB = kOffA + kStages * kABytes;
+  static constexpr int kOffOut = kOffB + kStages * kBBytes;
+  static constexpr int kOffVec = kOffOut + kOutBytes;            // bias + two gate rows
+  static constexpr int kOffBar = kOffVec + 3 * kBN * 4;
+  static constexpr int kSmem = 1024 + kOffBar + 256;
+};
 
 struct __align__(8) Barriers {
-  uint64_t full[kStages];
-  uint64_t empty[kStages];
+  uint64_t full[4];
+  uint64_t empty[4];
   uint64_t tmem_full[2];
   uint64_t tmem_empty[2];
+  uint64_t hin_full;
   uint64_t drain;
   uint32_t tmem_base;
 };
 
+// byte offset of 16-byte chunk `c` of row `r` in a [rows][128 B] box written
+// with 128-byte swizzle (the layout TMA produces and consumes)
+__device__ __forceinline__ int sw128_off(int r, int c) { return r * 128 + ((c ^ (r & 7)) << 4); }
+
 template <int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
     gemm_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmA,
-                        const __grid_constant__ CUtensorMap tmB, int M, int N, int K,
+                        const __grid_constant__ CUtensorMap tmB,
+                        const __grid_constant__ CUtensorMap tmCin,
+                        const __grid_constant__ CUtensorMap tmCout, int M, int N, int K,
                         EpiArgs ep, SlotMap map, int* err) {
+  using Cfg = GemmCfg<MODE>;
+  constexpr int kStages = Cfg::kStages;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t base = smem_u32(smem_raw);
   uint8_t* smem = smem_raw + ((1024 - (base & 1023)) & 1023);
-  uint8_t* sA = smem;
-  uint8_t* sB = smem + (size_t)kStages * kABytes;
-  Barriers* bar = reinterpret_cast<Barriers*>(smem + (size_t)kStages * kStageBytes);
-  float* stg_all = reinterpret_cast<float*>(smem + (size_t)kStages * kStageBytes + 256);
+  uint8_t* sA = smem + Cfg::kOffA;
+  uint8_t* sB = smem + Cfg::kOffB;
+  uint8_t* sOut = smem + Cfg::kOffOut;
+  float* vec = reinterpret_cast<float*>(smem + Cfg::kOffVec);
+  Barriers* bar = reinterpret_cast<Barriers*>(smem + Cfg::kOffBar);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -73,10 +105,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&bar->tmem_full[b], 1);
       mbar_init(&bar->tmem_empty[b], kEpiWarps);
     }
+    mbar_init(&bar->hin_full, 1);
     mbar_init(&bar->drain, 1);
     fence_barrier_init();
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
+    if (MODE != kEpiQKV) tma_prefetch_desc(&tmCout);
+    if (MODE == kEpiResid) tma_prefetch_desc(&tmCin);
   }
   if (warp == 1) {
     tmem_alloc(&bar->tmem_base, kTmemCols);
@@ -147,57 +182,167 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---------------------------------------------------- epilogue warps
     const int q = warp & 3;             // TMEM lane quarter this warp may access
     const int half = (warp - 2) >> 2;   // which 96-column half of the tile
+    const int et = threadIdx.x - 64;    // epilogue thread 0..255
+    const bool leader = et == 0;
+    const int r = q * 32 + lane;        // row of the tile owned by this thread
+    int hin_loads = 0;                  // residual tiles requested so far
+    if (MODE == kEpiResid && leader && (int)blockIdx.x < n_tiles) {
+      const int tile = blockIdx.x;
+      mbar_arrive_expect_tx(&bar->hin_full, Cfg::kOutBytes);
+      for (int k = 0; k < 6; ++k)
+        tma_load_2d(sOut + k * 16384, &tmCin, &bar->hin_full, (tile % tiles_n) * kBN + 32 * k,
+                    (tile / tiles_n) * kBM);
+      hin_loads = 1;
+    }
     int t = 0;
-    for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++t) {
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++t) {
       const int b = t & 1;
       const uint32_t use = (uint32_t)(t >> 1);
-      if (!mbar_wait(&bar->tmem_full[b], use & 1, err, kDevTimeoutEpi)) break;
-      tc_fence_after();
+      // every wait outcome is made uniform (warp, then the 8 epilogue warps at
+      // the named barrier) so that an abort is taken by all of them together
+      const bool acc_ok = mbar_wait_warp(&bar->tmem_full[b], use & 1, err, kDevTimeoutEpi);
       const int m0 = (tile / tiles_n) * kBM;
       const int n0 = (tile % tiles_n) * kBN;
       float acc[3][32];
+      if (acc_ok) {
+        tc_fence_after();
 #pragma unroll
-      for (int c = 0; c < 3; ++c) {
-        const uint32_t taddr =
-            tmem_base + (uint32_t)(b * 256 + half * 96 + c * 32) + ((uint32_t)(q * 32) << 16);
-        tmem_ld32(taddr, acc[c]);
+        for (int c = 0; c < 3; ++c) {
+          const uint32_t taddr =
+              tmem_base + (uint32_t)(b * 256 + half * 96 + c * 32) + ((uint32_t)(q * 32) << 16);
+          tmem_ld32(taddr, acc[c]);
+        }
+        tmem_ld_wait();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bar->tmem_empty[b]);
       }
-      tmem_ld_wait();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bar->tmem_empty[b]);
-      const int row0 = m0 + q * 32;
+
+      // stage bias (and gate rows) of this tile once the previous tile is done
+      if (named_bar_or(1, kEpiThreads, !acc_ok)) { ok = false; break; }
+      const int last_row = min(m0 + kBM, M) - 1;
+      const int slot_a = m0 / ep.n_tok, slot_b = last_row / ep.n_tok;
+      const int split = (slot_a + 1) * ep.n_tok;  // first row that belongs to slot_b
+      for (int i = et; i < kBN; i += kEpiThreads) {
+        vec[i] = ep.bias[n0 + i];
+        if (MODE == kEpiResid) {
+          vec[kBN + i] = ep.mod[(size_t)map.scene[slot_a] * ep.mod_stride + ep.gate_off + n0 + i];
+          vec[2 * kBN + i] = ep.mod[(size_t)map.scene[slot_b] * ep.mod_stride + ep.gate_off + n0 + i];
+        }
+      }
+      if (MODE == kEpiGELU && leader) bulk_wait_read0();  // previous tile's stores have read sOut
+      named_bar(1, kEpiThreads);
+
       if constexpr (MODE == kEpiResid) {
-        // fp32 read-modify-write of the residual: transpose each 32 x 32
-        // block through shared memory so that the warp reads and writes
-        // whole 128-byte rows
-        float* stg = stg_all + (warp - 2) * kStgFloats;
-        if (row0 < M) {
+        // rows spanning more than two slots (tokens per scene < 128) take the
+        // gate from global memory per row
+        const bool two_slots = slot_b - slot_a <= 1;
+        const bool hin_ok = mbar_wait_warp(&bar->hin_full, (uint32_t)t & 1, err, kDevTimeoutEpi);
+        const int row = m0 + r;
+        const float* gsel = vec + (row < split ? kBN : 2 * kBN);
+        const float* grow = nullptr;
+        if (!two_slots && row < M)
+          grow = ep.mod + (size_t)map.scene[row / ep.n_tok] * ep.mod_stride + ep.gate_off + n0;
 #pragma unroll
-          for (int c = 0; c < 3; ++c) {
+        for (int c = 0; c < 3 && hin_ok; ++c) {
+          const int col0 = half * 96 + c * 32;  // tile column of this 32-column chunk
+          uint8_t* box = sOut + (col0 >> 5) * 16384;
 #pragma unroll
-            for (int i = 0; i < 32; ++i) stg[lane * 33 + i] = acc[c][i];
-            __syncwarp();
-            epilogue_block32<MODE>(ep, map, stg, row0, n0 + half * 96 + c * 32, lane);
-            __syncwarp();
+          for (int ch = 0; ch < 8; ++ch) {
+            float4* p = reinterpret_cast<float4*>(box + sw128_off(r, ch));
+            float4 h = *p;
+            const int j = col0 + ch * 4;
+            float g0, g1, g2, g3;
+            if (two_slots) {
+              g0 = gsel[j]; g1 = gsel[j + 1]; g2 = gsel[j + 2]; g3 = gsel[j + 3];
+            } else if (grow) {
+              g0 = grow[j]; g1 = grow[j + 1]; g2 = grow[j + 2]; g3 = grow[j + 3];
+            } else {
+              g0 = g1 = g2 = g3 = 0.f;
+            }
+            h.x += g0 * (acc[c][ch * 4 + 0] + vec[j + 0]);
+            h.y += g1 * (acc[c][ch * 4 + 1] + vec[j + 1]);
+            h.z += g2 * (acc[c][ch * 4 + 2] + vec[j + 2]);
+            h.w += g3 * (acc[c][ch * 4 + 3] + vec[j + 3]);
+            *p = h;
           }
         }
+        fence_proxy_async();
+        if (named_bar_or(1, kEpiThreads, !hin_ok)) { ok = false; break; }
+        if (leader) {
+          for (int k = 0; k < 6; ++k) tma_store_2d(&tmCout, sOut + k * 16384, n0 + 32 * k, m0);
+          bulk_commit();
+          bulk_wait_read0();
+          const int next = tile + gridDim.x;
+          if (next < n_tiles) {
+            mbar_arrive_expect_tx(&bar->hin_full, Cfg::kOutBytes);
+            for (int k = 0; k < 6; ++k)
+              tma_load_2d(sOut + k * 16384, &tmCin, &bar->hin_full, (next % tiles_n) * kBN + 32 * k,
+                          (next / tiles_n) * kBM);
+            ++hin_loads;
+          }
+        }
+      } else if constexpr (MODE == kEpiGELU) {
+#pragma unroll
+        for (int c = 0; c < 3; ++c) {
+#pragma unroll
+          for (int g = 0; g < 4; ++g) {
+            const int j = half * 96 + c * 32 + g * 8;  // tile column of this 8-column group
+            uint4 w;
+            float v[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) v[i] = gelu_tanh_bf16(acc[c][g * 8 + i] + vec[j + i]);
+            __nv_bfloat162 p0 = __floats2bfloat162_rn(v[0], v[1]);
+            __nv_bfloat162 p1 = __floats2bfloat162_rn(v[2], v[3]);
+            __nv_bfloat162 p2 = __floats2bfloat162_rn(v[4], v[5]);
+            __nv_bfloat162 p3 = __floats2bfloat162_rn(v[6], v[7]);
+            w.x = *reinterpret_cast<uint32_t*>(&p0);
+            w.y = *reinterpret_cast<uint32_t*>(&p1);
+            w.z = *reinterpret_cast<uint32_t*>(&p2);
+            w.w = *reinterpret_cast<uint32_t*>(&p3);
+            *reinterpret_cast<uint4*>(sOut + (j >> 6) * 16384 + sw128_off(r, (j & 63) >> 3)) = w;
+          }
+        }
+        fence_proxy_async();
+        named_bar(1, kEpiThreads);
+        if (leader) {
+          for (int k = 0; k < 3; ++k) tma_store_2d(&tmCout, sOut + k * 16384, n0 + 64 * k, m0);
+          bulk_commit();
+        }
       } else {
-        // bf16 outputs: each thread stores 16-byte pieces of its own row
-        const int row = row0 + lane;
+        // QKV: each thread stores 16-byte pieces of its own row
+        const int row = m0 + r;
         if (row < M) {
+          const int slot = row / ep.n_tok;
+          const int tok = row - slot * ep.n_tok;
 #pragma unroll
           for (int c = 0; c < 3; ++c) {
 #pragma unroll
             for (int g = 0; g < 4; ++g) {
+              const int j = half * 96 + c * 32 + g * 8;
+              const int col = n0 + j;
+              const int which = col / ep.d;
+              const int within = col - which * ep.d;
+              const int head = within / ep.dh;
+              const int e = within - head * ep.dh;
               float v[8];
 #pragma unroll
-              for (int i = 0; i < 8; ++i) v[i] = acc[c][g * 8 + i];
-              epilogue8<MODE, __nv_bfloat16>(ep, map, row, n0 + half * 96 + c * 32 + g * 8, v);
+              for (int i = 0; i < 8; ++i) v[i] = acc[c][g * 8 + i] + vec[j + i];
+              __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(ep.out) +
+                                   ((((size_t)which * ep.nslots + slot) * ep.heads + head) * ep.n_tok + tok) *
+                                       ep.dhp + e;
+              Pack8<__nv_bfloat16>::store(dst, v);
             }
           }
         }
       }
+    }
+    if (leader) {
+      if (MODE != kEpiQKV) bulk_wait0();
+      // a residual prefetch that was never consumed (aborted run) must land first
+      if (MODE == kEpiResid && !ok && hin_loads > t)
+        mbar_wait(&bar->hin_full, (uint32_t)(hin_loads - 1) & 1, err, kDevTimeoutEpi);
     }
   }
 
@@ -209,37 +354,40 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-}  // namespace
-
-size_t gemm_tc_smem_bytes() { return kSmemBytes; }
-
 template <int MODE>
-static cudaError_t launch_mode(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K,
-                               const EpiArgs& ep, const SlotMap& map, int* err, int n_sms,
-                               cudaStream_t st) {
+cudaError_t launch_mode(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmCin,
+                        const CUtensorMap& tmCout, int M, int N, int K, const EpiArgs& ep,
+                        const SlotMap& map, int* err, int n_sms, cudaStream_t st) {
+  using Cfg = GemmCfg<MODE>;
   static bool configured = false;
   if (!configured) {
     cudaError_t e = cudaFuncSetAttribute(gemm_bf16_tc_kernel<MODE>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kSmemBytes);
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmem);
     if (e != cudaSuccess) return e;
     configured = true;
   }
   const int tiles = ((M + kBM - 1) / kBM) * (N / kBN);
   const int grid = tiles < n_sms ? tiles : n_sms;
-  gemm_bf16_tc_kernel<MODE><<<grid, kThreads, kSmemBytes, st>>>(tmA, tmB, M, N, K, ep, map, err);
+  gemm_bf16_tc_kernel<MODE><<<grid, kThreads, Cfg::kSmem, st>>>(tmA, tmB, tmCin, tmCout, M, N, K,
+                                                                ep, map, err);
   return cudaGetLastError();
 }
 
-cudaError_t launch_gemm_tc(int mode, const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N,
+}  // namespace
+
+cudaError_t launch_gemm_tc(int mode, const CUtensorMap& tmA, const CUtensorMap& tmB,
+                           const CUtensorMap& tmCin, const CUtensorMap& tmCout, int M, int N,
                            int K, const EpiArgs& ep, const SlotMap& map, int* err, int n_sms,
                            cudaStream_t st) {
   if (M <= 0) return cudaSuccess;
   if (N % kBN != 0 || K % kBK != 0) return cudaErrorInvalidValue;
   switch (mode) {
-    case kEpiQKV: return launch_mode<kEpiQKV>(tmA, tmB, M, N, K, ep, map, err, n_sms, st);
-    case kEpiGELU: return launch_mode<kEpiGELU>(tmA, tmB, M, N, K, ep, map, err, n_sms, st);
-    case kEpiResid: return launch_mode<kEpiResid>(tmA, tmB, M, N, K, ep, map, err, n_sms, st);
+    case kEpiQKV:
+      return launch_mode<kEpiQKV>(tmA, tmB, tmCin, tmCout, M, N, K, ep, map, err, n_sms, st);
+    case kEpiGELU:
+      return launch_mode<kEpiGELU>(tmA, tmB, tmCin, tmCout, M, N, K, ep, map, err, n_sms, st);
+    case kEpiResid:
+      return launch_mode<kEpiResid>(tmA, tmB, tmCin, tmCout, M, N, K, ep, map, err, n_sms, st);
   }
   return cudaErrorInvalidValue;
 }

@@ -33,7 +33,10 @@ template <typename T>
 cudaError_t launch_ln_mod(const float* h, int rows, int N, int d, const float* mod, int mod_stride,
                           int shift_off, int scale_off, const SlotMap& map, T* a, cudaStream_t st);
 // GEMMs
-cudaError_t launch_gemm_tc(int mode, const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N,
+// tmCin / tmCout: epilogue maps (residual: fp32 [rows][N] box 32 x 128 for
+// h_in and h; GELU: bf16 [rows][N] box 64 x 128 for the output; QKV: unused)
+cudaError_t launch_gemm_tc(int mode, const CUtensorMap& tmA, const CUtensorMap& tmB,
+                           const CUtensorMap& tmCin, const CUtensorMap& tmCout, int M, int N,
                            int K, const EpiArgs& ep, const SlotMap& map, int* err, int n_sms,
                            cudaStream_t st);
 cudaError_t launch_gemm_f32(int mode, const float* A, const float* W, int M, int N, int K,

@@ -58,7 +58,7 @@ struct dc_model {
   float* drift_host = nullptr;  // pinned
   // derived tables: W_e^T [C][d] and the Gram tables of the drift sums
   float *w_eT = nullptr, *gram = nullptr, *gp = nullptr, *gs = nullptr;
-  CUtensorMap tm_a, tm_oact, tm_m, tm_qkv;
+  CUtensorMap tm_a, tm_oact, tm_m, tm_qkv, tm_u32, tm_h32;
   long long launches = 0;
   // per-kernel profiling (dc_profile)
   struct ProfRec { int cat; cudaEvent_t a, b; double flops, bytes; };
@@ -156,21 +156,24 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
   return fn;
 }
 
-// 2-D bf16 K-major operand [rows][inner], box 64 x box_rows, 128-byte swizzle.
+// 2-D row-major tensor [rows][inner] with 128-byte rows per box (64 bf16 or
+// 32 fp32 elements), box_rows rows, 128-byte swizzle.
 dc_status make_map(CUtensorMap* map, const void* ptr, uint64_t inner, uint64_t rows,
-                   uint32_t box_rows) {
+                   uint32_t box_rows, bool fp32 = false) {
   auto enc = get_encode();
   if (!enc) {
     dc::set_error("cuTensorMapEncodeTiled is unavailable");
     return DC_ERR_CUDA;
   }
+  const uint32_t esize = fp32 ? 4 : 2;
   cuuint64_t dims[2] = {inner, rows};
-  cuuint64_t strides[1] = {inner * 2};
-  cuuint32_t box[2] = {64, box_rows};
+  cuuint64_t strides[1] = {inner * esize};
+  cuuint32_t box[2] = {128 / esize, box_rows};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides,
-                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  CUresult r = enc(map, fp32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                   const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                   CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) {
     dc::set_error("cuTensorMapEncodeTiled failed with CUresult " + std::to_string((int)r));
     return DC_ERR_CUDA;
@@ -323,8 +326,8 @@ dc_status enqueue_compute(dc_model* m, float* lat, const float* mod_k, const Slo
                  b_2 = E * ((double)M * m->md + (double)m->md * d) + 8.0 * Md;
     if constexpr (sizeof(T) == 2) {
       DC_LAUNCH(DC_PROF_GEMM_QKV, f_qkv, b_qkv,
-                dc::launch_gemm_tc(dc::kEpiQKV, m->tm_a, w.tm_qkv, M, 3 * d, d, e1, map, m->err_d,
-                                   m->n_sms, st));
+                dc::launch_gemm_tc(dc::kEpiQKV, m->tm_a, w.tm_qkv, m->tm_a, m->tm_a, M, 3 * d, d,
+                                   e1, map, m->err_d, m->n_sms, st));
       if (dc::attention_tc_supported(m->dh)) {
         DC_LAUNCH(DC_PROF_ATTENTION, attn_flops, attn_bytes,
                   dc::launch_attention_tc(m->tm_qkv, nc, m->heads, N, m->dh,
@@ -336,17 +339,17 @@ dc_status enqueue_compute(dc_model* m, float* lat, const float* mod_k, const Slo
                                             reinterpret_cast<__nv_bfloat16*>(o), st));
       }
       DC_LAUNCH(DC_PROF_GEMM_OUT, f_o, b_o,
-                dc::launch_gemm_tc(dc::kEpiResid, m->tm_oact, w.tm_o, M, d, d, e2, map, m->err_d,
-                                   m->n_sms, st));
+                dc::launch_gemm_tc(dc::kEpiResid, m->tm_oact, w.tm_o, l == 0 ? m->tm_u32 : m->tm_h32,
+                                   m->tm_h32, M, d, d, e2, map, m->err_d, m->n_sms, st));
       DC_LAUNCH(DC_PROF_LN, 0.0, ln_bytes,
                 dc::launch_ln_mod<T>(m->h, M, N, d, mod_k, m->mod_stride, base + 3 * d,
                                      base + 4 * d, map, a, st));
       DC_LAUNCH(DC_PROF_GEMM_MLP1, f_mlp, b_1,
-                dc::launch_gemm_tc(dc::kEpiGELU, m->tm_a, w.tm_1, M, m->md, d, e3, map, m->err_d,
-                                   m->n_sms, st));
+                dc::launch_gemm_tc(dc::kEpiGELU, m->tm_a, w.tm_1, m->tm_m, m->tm_m, M, m->md, d,
+                                   e3, map, m->err_d, m->n_sms, st));
       DC_LAUNCH(DC_PROF_GEMM_MLP2, f_mlp, b_2,
-                dc::launch_gemm_tc(dc::kEpiResid, m->tm_m, w.tm_2, M, d, m->md, e4, map, m->err_d,
-                                   m->n_sms, st));
+                dc::launch_gemm_tc(dc::kEpiResid, m->tm_m, w.tm_2, m->tm_h32, m->tm_h32, M, d,
+                                   m->md, e4, map, m->err_d, m->n_sms, st));
     } else {
       DC_LAUNCH(DC_PROF_GEMM_QKV, f_qkv, b_qkv,
                 dc::launch_gemm_f32(dc::kEpiQKV, reinterpret_cast<const float*>(a),
@@ -804,6 +807,8 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
     if ((s = make_map(&m->tm_a, m->a, d, B * N, bm)) != DC_OK) return fail(s);
     if ((s = make_map(&m->tm_oact, m->o, d, B * N, bm)) != DC_OK) return fail(s);
     if ((s = make_map(&m->tm_m, m->m, m->md, B * N, bm)) != DC_OK) return fail(s);
+    if ((s = make_map(&m->tm_u32, m->u, d, B * N, bm, true)) != DC_OK) return fail(s);
+    if ((s = make_map(&m->tm_h32, m->h, d, B * N, bm, true)) != DC_OK) return fail(s);
     if (dc::attention_tc_supported(m->dh) &&
         (s = make_map(&m->tm_qkv, m->qkv, m->dhp, 3 * B * m->heads * N, 128)) != DC_OK)
       return fail(s);
