@@ -280,6 +280,8 @@ def main():
     barrier()
     torch.cuda.synchronize()
     clocks.start()
+    # the timed region is the profiler range (ncu --profile-from-start off)
+    torch.cuda.profiler.start()
     ms_list, launches, calls = [], 0, 0
     for _ in range(args.steps):
         ms, st = one_call()
@@ -291,6 +293,7 @@ def main():
             stats0 = st
         assert np.array_equal(ref_exec, st["executed"]), "schedule changed between steps"
     torch.cuda.synchronize()
+    torch.cuda.profiler.stop()
     barrier()
     clk = clocks.stop()
     dc.profile(model, False)

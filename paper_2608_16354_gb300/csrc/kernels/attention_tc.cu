@@ -52,7 +52,8 @@ struct AttCfg {
 template <int NQ>
 struct __align__(8) AttBars {
   uint64_t q_full;
-  uint64_t kv_full[2], kv_empty[2];
+  uint64_t k_full[2], k_empty[2];   // key ring: loader <-> S MMAs
+  uint64_t v_full[2], v_empty[2];   // value ring: loader <-> PV MMAs
   uint64_t s_full[NQ][2];    // MMA -> softmax: S ready in buffer
   uint64_t p_full[NQ][2];    // softmax -> MMA: P written, S consumed
   uint64_t o_full[NQ][2];    // MMA -> softmax: PV ready in buffer (P buffer free again)
@@ -212,8 +213,10 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
   if (threadIdx.x == 0) {
     mbar_init(&bar->q_full, 1);
     for (int b = 0; b < 2; ++b) {
-      mbar_init(&bar->kv_full[b], 1);
-      mbar_init(&bar->kv_empty[b], 1);
+      mbar_init(&bar->k_full[b], 1);
+      mbar_init(&bar->k_empty[b], 1);
+      mbar_init(&bar->v_full[b], 1);
+      mbar_init(&bar->v_empty[b], 1);
       for (int t = 0; t < NQ; ++t) {
         mbar_init(&bar->s_full[t][b], 1);
         mbar_init(&bar->p_full[t][b], 4);
@@ -238,29 +241,61 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------------------ TMA
+      // K and V have rings of their own: K_j is released as soon as every
+      // S_{t,j} is issued, so the next key tile streams in while the PV
+      // products on V_j are still pending.
       bool ok = true;
-      int last[2] = {-1, -1};
+      int last_k[2] = {-1, -1}, last_v[2] = {-1, -1};
       mbar_arrive_expect_tx(&bar->q_full, NQ * Cfg::kTileBytes);
       for (int t = 0; t < NQ; ++t)
         for (int a = 0; a < Cfg::kAtoms; ++a)
           tma_load_2d(smem + Cfg::kOffQ + t * Cfg::kTileBytes + a * 16384, &tm, &bar->q_full,
                       a * 64, row_q + t * 128);
-      for (int j = 0; j < n_kv && ok; ++j) {
-        const int b = j & 1;
-        const uint32_t u = (uint32_t)(j >> 1);
-        if (!mbar_wait(&bar->kv_empty[b], (u & 1) ^ 1, err, kDevTimeoutTma)) { ok = false; break; }
-        mbar_arrive_expect_tx(&bar->kv_full[b], 2 * Cfg::kTileBytes);
-        for (int a = 0; a < Cfg::kAtoms; ++a) {
-          tma_load_2d(smem + Cfg::kOffK + b * Cfg::kTileBytes + a * 16384, &tm, &bar->kv_full[b],
-                      a * 64, row_k + j * 128);
-          tma_load_2d(smem + Cfg::kOffV + b * Cfg::kTileBytes + a * 16384, &tm, &bar->kv_full[b],
-                      a * 64, row_v + j * 128);
+      int nk = 0, nv = 0;
+      unsigned long long t_idle = global_ns();
+      while (ok && nv < n_kv) {
+        bool progressed = false;
+        if (nk < n_kv) {
+          const int b = nk & 1;
+          const uint32_t u = (uint32_t)(nk >> 1);
+          if (mbar_test(&bar->k_empty[b], (u & 1) ^ 1)) {
+            mbar_arrive_expect_tx(&bar->k_full[b], Cfg::kTileBytes);
+            for (int a = 0; a < Cfg::kAtoms; ++a)
+              tma_load_2d(smem + Cfg::kOffK + b * Cfg::kTileBytes + a * 16384, &tm,
+                          &bar->k_full[b], a * 64, row_k + nk * 128);
+            last_k[b] = (int)(u & 1);
+            ++nk;
+            progressed = true;
+          }
         }
-        last[b] = (int)(u & 1);
+        if (nv < nk) {
+          const int b = nv & 1;
+          const uint32_t u = (uint32_t)(nv >> 1);
+          if (mbar_test(&bar->v_empty[b], (u & 1) ^ 1)) {
+            mbar_arrive_expect_tx(&bar->v_full[b], Cfg::kTileBytes);
+            for (int a = 0; a < Cfg::kAtoms; ++a)
+              tma_load_2d(smem + Cfg::kOffV + b * Cfg::kTileBytes + a * 16384, &tm,
+                          &bar->v_full[b], a * 64, row_v + nv * 128);
+            last_v[b] = (int)(u & 1);
+            ++nv;
+            progressed = true;
+          }
+        }
+        if (progressed) {
+          t_idle = global_ns();
+        } else if (*(volatile int*)err != 0) {
+          ok = false;
+        } else if (global_ns() - t_idle > kWaitLimitNs) {
+          atomicCAS(err, 0, kDevTimeoutTma);
+          ok = false;
+        }
       }
+      // every copy in flight lands before the CTA can exit
       mbar_wait(&bar->q_full, 0, err, kDevTimeoutTma);
-      for (int b = 0; b < 2; ++b)
-        if (last[b] >= 0) mbar_wait(&bar->kv_full[b], (uint32_t)last[b], err, kDevTimeoutTma);
+      for (int b = 0; b < 2; ++b) {
+        if (last_k[b] >= 0) mbar_wait(&bar->k_full[b], (uint32_t)last_k[b], err, kDevTimeoutTma);
+        if (last_v[b] >= 0) mbar_wait(&bar->v_full[b], (uint32_t)last_v[b], err, kDevTimeoutTma);
+      }
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -272,7 +307,7 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
       bool ok = mbar_wait(&bar->q_full, 0, err, kDevTimeoutMma);
       int next_s[NQ], next_pv[NQ];
       for (int t = 0; t < NQ; ++t) next_s[t] = next_pv[t] = 0;
-      int released = 0;  // key tiles whose stage has been handed back to the loader
+      int released = 0, k_released = 0;  // stages handed back to the loader (V, K)
       unsigned long long t_idle = global_ns();
       while (ok) {
         bool progressed = false, done = true;
@@ -282,7 +317,7 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
             done = false;
             const int b = js & 1;
             const uint32_t u = (uint32_t)(js >> 1);
-            if (mbar_test(&bar->kv_full[b], u & 1) && mbar_test(&bar->buf_free[t][b], (u & 1) ^ 1)) {
+            if (mbar_test(&bar->k_full[b], u & 1) && mbar_test(&bar->buf_free[t][b], (u & 1) ^ 1)) {
               tc_fence_after();
               const uint32_t sK = smem_u32(smem + Cfg::kOffK + b * Cfg::kTileBytes);
               const uint32_t sQ = smem_u32(smem + Cfg::kOffQ + t * Cfg::kTileBytes);
@@ -302,7 +337,8 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
             done = false;
             const int b = jp & 1;
             const uint32_t u = (uint32_t)(jp >> 1);
-            if (jp < next_s[t] && mbar_test(&bar->p_full[t][b], u & 1)) {
+            if (jp < next_s[t] && mbar_test(&bar->p_full[t][b], u & 1) &&
+                mbar_test(&bar->v_full[b], u & 1)) {
               tc_fence_after();
               const uint32_t sV = smem_u32(smem + Cfg::kOffV + b * Cfg::kTileBytes);
               const uint32_t sP = smem_u32(smem + Cfg::kOffP + (2 * t + b) * Cfg::kPBytes);
@@ -321,11 +357,19 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
             }
           }
         }
-        // a key stage goes back to the loader once every tile's PV on it is issued
-        int min_pv = n_kv;
-        for (int t = 0; t < NQ; ++t) min_pv = min(min_pv, next_pv[t]);
+        // a K stage goes back to the loader once every tile's S on it is
+        // issued, a V stage once every tile's PV on it is
+        int min_s = n_kv, min_pv = n_kv;
+        for (int t = 0; t < NQ; ++t) {
+          min_s = min(min_s, next_s[t]);
+          min_pv = min(min_pv, next_pv[t]);
+        }
+        while (k_released < min_s) {
+          tc_commit(&bar->k_empty[k_released & 1]);
+          ++k_released;
+        }
         while (released < min_pv) {
-          tc_commit(&bar->kv_empty[released & 1]);
+          tc_commit(&bar->v_empty[released & 1]);
           ++released;
         }
         if (done) break;
