@@ -2,26 +2,30 @@
 // o = softmax(q k^T / sqrt(dh)) v for head dims 64 and 128.
 //
 // One CTA per (slot, head, NQ x 128 queries); keys stream in tiles of 128.
-//   warp 0        TMA: the NQ query tiles once, K_j and V_j into a 2-stage ring
-//   warp 1        owns TMEM and issues tcgen05.mma for every query tile t:
-//                   S_{t,j}  = Q_t K_j^T  -> TMEM buffer (t, j % 2)  (M=128, N=128, K=dh)
-//                   PV_{t,j} = P_{t,j} V_j -> the same buffer once S_{t,j} has been
-//                                             read (M=128, N=64 per MMA, K=128)
-//   warps 2..     one softmax warpgroup per query tile, one query row per
+//   warp 0        TMA: the NQ query tiles once; K_j and V_j into two rings of
+//                 their own (kStages stages each)
+//   warp 1        owns TMEM and issues, in a fixed order, for key tile j:
+//                   S_{t,j}    = Q_t K_j^T   (M=128, N=128, K=dh; Q, K from shared memory)
+//                   O_t       += P_{t,j-1} V_{j-1}  (M=128, N=64 per MMA, K=128;
+//                                P from TMEM, V from shared memory)
+//   warps 2, 3    idle (they complete the control warpgroup)
+//   warps 4..     one softmax warpgroup per query tile, one query row per
 //                 thread.
-// Softmax of tile j (per row): P = exp2(s * scale - ref) against a reference
-// max `ref` that only moves when the row's max exceeds it by more than 8
-// (log2 units), so one pass over S suffices; P is written as bf16 into shared
-// memory (double-buffered) in the 128-byte-swizzled K-major layout the MMA
-// reads.  Halfway through the pass the thread folds PV_{j-1} into its
-// register accumulator (O = (O + PV) * c, c = exp2(ref_old - ref_new)) and
-// frees that TMEM buffer, so S_{j+1} is computed during the second half and
-// PV_j during the first half of the next tile.  Both softmax warpgroups share
-// the tensor core.  A quarter of the exponentials run on the FMA pipe
-// (Cody-Waite split into integer and fraction, degree-3 minimax polynomial
-// for 2^r on [0, 1], max relative error 8.6e-5) to relieve the MUFU unit.
-// V is consumed as an MN-major operand straight from its [keys][dh] layout.
-// Keys beyond N are masked (last tile only).  Every mbarrier wait is bounded.
+// TMEM per query tile t: O_t (dh columns), S_t (128), P_t (64: 128 bf16 keys).
+// Keeping P in TMEM means the PV products read only V from shared memory,
+// which halves the shared-memory traffic per key tile (the MMA operand path
+// shares shared-memory bandwidth with TMA writes and the mbarriers).
+// Softmax of tile j (per row): the whole 128-column S row is loaded into
+// registers and S_t handed straight back, so S_{t,j+1} is computed while this
+// tile's exponentials run.  P = exp2(s * scale - ref) against a reference max
+// `ref` that only moves when the row's max exceeds it by more than 8 (log2
+// units); when it moves, the row of O_t (and the row sum) is rescaled by
+// exp2(ref_old - ref_new) once PV_{t,j-1} has landed and before P_{t,j} is
+// released.  3/8 of the exponentials run on the FMA/ALU pipes (Cody-Waite
+// split into integer and fraction, degree-3 minimax polynomial for 2^r on
+// [0, 1], max relative error 8.6e-5) to relieve the MUFU unit.  V is consumed
+// as an MN-major operand straight from its [keys][dh] layout.  Keys beyond N
+// are masked (last tile only).  Every mbarrier wait is bounded.
 #include <math.h>
 
 #include "common.cuh"
@@ -31,35 +35,47 @@ namespace dc {
 
 namespace {
 
-constexpr float kRefSlack = 8.0f;    // move the reference max only beyond this (log2 units)
-constexpr float kRedoExcess = 64.0f; // larger jumps redo the tile against the new max
+constexpr float kRefSlack = 8.0f;  // move the reference max only beyond this (log2 units)
+constexpr int kPoly8 = 3;          // of every 8 exponentials, this many on the FMA pipe
+constexpr int kStages = 3;         // K and V ring depth
 
 template <int DHP, int NQ>
 struct AttCfg {
   static constexpr int kAtoms = DHP / 64;             // 64-element swizzle atoms along dh
   static constexpr int kTileBytes = kAtoms * 16384;   // 128 rows x DHP bf16
-  static constexpr int kPBytes = 2 * 16384;           // 128 queries x 128 keys bf16
-  static constexpr int kOffQ = 0;                           // NQ tiles
-  static constexpr int kOffK = kOffQ + NQ * kTileBytes;     // 2 stages
-  static constexpr int kOffV = kOffK + 2 * kTileBytes;      // 2 stages
-  static constexpr int kOffP = kOffV + 2 * kTileBytes;      // NQ x 2 buffers
-  static constexpr int kOffBar = kOffP + NQ * 2 * kPBytes;
+  static constexpr int kOffQ = 0;                              // NQ tiles
+  static constexpr int kOffK = kOffQ + NQ * kTileBytes;        // kStages stages
+  static constexpr int kOffV = kOffK + kStages * kTileBytes;   // kStages stages
+  static constexpr int kOffBar = kOffV + kStages * kTileBytes;
   static constexpr int kSmem = 1024 + kOffBar + 256;
-  static constexpr int kThreads = 64 + NQ * 128;
-  static constexpr int kTmemCols = NQ * 256;  // two 128-column buffers per query tile
+  static constexpr int kThreads = 128 + NQ * 128;   // control warpgroup + softmax
+  // two query tiles: the control warpgroup gives registers to the softmax
+  // warpgroups (128 x 72 + 256 x 216 = 384 x 168, the launch allocation)
+  static constexpr bool kSplitRegs = NQ == 2;
+  static constexpr int kRegsLaunch = 168, kRegsCtl = 72, kRegsSoftmax = 216;
+  static_assert(!kSplitRegs || 128 * kRegsCtl + NQ * 128 * kRegsSoftmax <= kThreads * kRegsLaunch,
+                "register split exceeds the launch allocation");
+  // TMEM columns
+  static constexpr int kColO = 0;                     // O_t at t * DHP
+  static constexpr int kColS = NQ * DHP;              // S_t at kColS + t * 128
+  static constexpr int kColP = kColS + NQ * 128;      // P_t at kColP + t * 64
+  static constexpr int kTmemCols = 512;
+  static_assert(kColP + NQ * 64 <= kTmemCols, "TMEM budget");
+  static_assert(kSmem <= 232448, "shared memory budget");
 };
 
 template <int NQ>
 struct __align__(8) AttBars {
   uint64_t q_full;
-  uint64_t k_full[2], k_empty[2];   // key ring: loader <-> S MMAs
-  uint64_t v_full[2], v_empty[2];   // value ring: loader <-> PV MMAs
-  uint64_t s_full[NQ][2];    // MMA -> softmax: S ready in buffer
-  uint64_t p_full[NQ][2];    // softmax -> MMA: P written, S consumed
-  uint64_t o_full[NQ][2];    // MMA -> softmax: PV ready in buffer (P buffer free again)
-  uint64_t buf_free[NQ][2];  // softmax -> MMA: PV folded, buffer free
+  uint64_t k_full[kStages], k_empty[kStages];   // key ring: loader <-> S MMAs
+  uint64_t v_full[kStages], v_empty[kStages];   // value ring: loader <-> PV MMAs
+  uint64_t s_full[NQ];    // MMA -> softmax: S_{t,j} ready
+  uint64_t s_free[NQ];    // softmax -> MMA: S_{t,j} read into registers
+  uint64_t p_full[NQ];    // softmax -> MMA: P_{t,j} in TMEM (and O_t rescaled)
+  uint64_t p_free[NQ];    // MMA -> softmax: PV_{t,j} done (P_t free, O_t current)
   uint64_t drain;
   uint32_t tmem_base;
+  int abort;              // the error word was set before this CTA started
 };
 
 // Descriptor of an MN-major operand tile written by TMA with 128-byte swizzle
@@ -100,22 +116,28 @@ __device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
       : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
   return r;
 }
-__device__ __forceinline__ float2 fmul2(float2 a, float2 b) {
-  float2 r;
-  asm("{\n .reg .b64 a, b, d;\n mov.b64 a, {%2, %3};\n mov.b64 b, {%4, %5};\n"
-      " mul.rn.f32x2 d, a, b;\n mov.b64 {%0, %1}, d;\n}\n"
-      : "=f"(r.x), "=f"(r.y)
-      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
-  return r;
+__device__ __forceinline__ uint32_t pack2(float a, float b) {
+  __nv_bfloat162 t = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<uint32_t*>(&t);
 }
 
-// 2^x for a pair, on the FMA/ALU pipes, given y = x - 1/2 (x <= kRedoExcess):
-// n = round(y) = floor(x) from the rounding against 1.5 * 2^23, r' = y - n in
-// [-1/2, 1/2], 2^(r' + 1/2) by a degree-3 minimax polynomial (the [0, 1]
-// minimax for 2^r re-expanded around 1/2), and n (clamped at -126 so tiny
-// values stay tiny) added to the exponent bits.
-__device__ __forceinline__ float2 ex2_poly2(float2 y) {
+
+// max of three (one instruction on sm_100 and later)
+__device__ __forceinline__ float fmax3f(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+// 2^x for a pair on the FMA/ALU pipes, given y = x - 1/2 (x <= kRefSlack):
+// y is clamped at -126.5 so the result stays a tiny normal/subnormal, n =
+// round(y) = floor(x) comes from rounding against 1.5 * 2^23 (whose bit
+// pattern, shifted left by 23, is n << 23), r' = y - n in [-1/2, 1/2], and
+// 2^(r' + 1/2) is a degree-3 minimax polynomial (the [0, 1] minimax for 2^r
+// re-expanded around 1/2) whose exponent field receives n.
+__device__ __forceinline__ float2 ex2_poly2c(float2 y) {
   const float magic = 12582912.0f;  // 1.5 * 2^23
+  y = make_float2(fmaxf(y.x, -126.5f), fmaxf(y.y, -126.5f));
   const float2 t = fadd2(y, make_float2(magic, magic));
   const float2 n = fadd2(t, make_float2(-magic, -magic));
   const float2 r = fadd2(y, make_float2(-n.x, -n.y));
@@ -123,67 +145,57 @@ __device__ __forceinline__ float2 ex2_poly2(float2 y) {
                    make_float2(3.432455659e-01f, 3.432455659e-01f));
   q = ffma2(q, r, make_float2(9.805620313e-01f, 9.805620313e-01f));
   q = ffma2(q, r, make_float2(1.414103031e+00f, 1.414103031e+00f));
-  const int n0 = max(__float_as_int(t.x) - 0x4B400000, -126);
-  const int n1 = max(__float_as_int(t.y) - 0x4B400000, -126);
-  return make_float2(__int_as_float(__float_as_int(q.x) + (n0 << 23)),
-                     __int_as_float(__float_as_int(q.y) + (n1 << 23)));
+  return make_float2(__uint_as_float(__float_as_uint(q.x) + (__float_as_uint(t.x) << 23)),
+                     __uint_as_float(__float_as_uint(q.y) + (__float_as_uint(t.y) << 23)));
 }
 
-__device__ __forceinline__ uint32_t pack2(float a, float b) {
-  __nv_bfloat162 t = __floats2bfloat162_rn(a, b);
-  return *reinterpret_cast<uint32_t*>(&t);
-}
-
-// One 32-column chunk of the softmax pass: p = 2^(s * scale - ref) (chunk 3
-// on the FMA pipe), masked beyond `valid`, raw max and row sum updated on
-// four independent chains, P chunk written to shared memory.
+// One 32-column chunk: p = 2^(s * scale - ref) (kPoly8 of every 8 on the FMA
+// pipe), masked beyond `valid`, row sum on two packed chains, and the chunk
+// packed into 16 bf16 pairs (even key in the low half) for P in TMEM.
 template <bool MASKED>
-__device__ __forceinline__ void softmax_chunk(const uint32_t (&raw)[32], int c, int valid,
-                                              float scale_log2, float neg_ref, float (&tmax)[4],
-                                              float2 (&rs)[2], uint8_t* P, int row) {
+__device__ __forceinline__ void p_chunk(const uint32_t (&v)[32], int c, int valid,
+                                        float scale_log2, float neg_ref, float2 (&rs)[2],
+                                        uint32_t* pk) {
   const float2 sc = make_float2(scale_log2, scale_log2);
-  float v[32];
-  if (c == 3) {
-    const float2 nr = make_float2(neg_ref - 0.5f, neg_ref - 0.5f);
+  const float2 nr = make_float2(neg_ref, neg_ref);
+  const float2 nrh = make_float2(neg_ref - 0.5f, neg_ref - 0.5f);
 #pragma unroll
-    for (int e = 0; e < 32; e += 2) {
-      const float2 y = ffma2(make_float2(__uint_as_float(raw[e]), __uint_as_float(raw[e + 1])), sc, nr);
-      const float2 p = ex2_poly2(y);
-      v[e] = p.x;
-      v[e + 1] = p.y;
-    }
-  } else {
-    const float2 nr = make_float2(neg_ref, neg_ref);
-#pragma unroll
-    for (int e = 0; e < 32; e += 2) {
-      const float2 x = ffma2(make_float2(__uint_as_float(raw[e]), __uint_as_float(raw[e + 1])), sc, nr);
-      v[e] = ex2_mufu(x.x);
-      v[e + 1] = ex2_mufu(x.y);
-    }
-  }
-#pragma unroll
-  for (int e = 0; e < 32; ++e) {
-    if (!MASKED || c * 32 + e < valid) {
-      tmax[e & 3] = fmaxf(tmax[e & 3], __uint_as_float(raw[e]));
+  for (int e = 0; e < 32; e += 2) {
+    const float2 s2 = make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1]));
+    float2 p;
+    if (((e >> 1) & 7) >= 8 - kPoly8) {
+      p = ex2_poly2c(ffma2(s2, sc, nrh));
     } else {
-      v[e] = 0.f;
+      const float2 x = ffma2(s2, sc, nr);
+      p = make_float2(ex2_mufu(x.x), ex2_mufu(x.y));
     }
+    if (MASKED) {
+      if (c * 32 + e >= valid) p.x = 0.f;
+      if (c * 32 + e + 1 >= valid) p.y = 0.f;
+    }
+    rs[(e >> 1) & 1] = fadd2(rs[(e >> 1) & 1], p);
+    pk[e >> 1] = pack2(p.x, p.y);
   }
+}
+
+// Raw max of a 32-column chunk (columns at or beyond `valid` ignored).
+template <bool MASKED>
+__device__ __forceinline__ float chunk_max(const uint32_t (&raw)[32], int c, int valid, float m) {
+  float m0 = m, m1 = -INFINITY;
 #pragma unroll
   for (int e = 0; e < 32; e += 4) {
-    rs[0] = fadd2(rs[0], make_float2(v[e], v[e + 1]));
-    rs[1] = fadd2(rs[1], make_float2(v[e + 2], v[e + 3]));
+    float a = __uint_as_float(raw[e]), b = __uint_as_float(raw[e + 1]);
+    float x = __uint_as_float(raw[e + 2]), y = __uint_as_float(raw[e + 3]);
+    if (MASKED) {
+      if (c * 32 + e >= valid) a = -INFINITY;
+      if (c * 32 + e + 1 >= valid) b = -INFINITY;
+      if (c * 32 + e + 2 >= valid) x = -INFINITY;
+      if (c * 32 + e + 3 >= valid) y = -INFINITY;
+    }
+    m0 = fmax3f(m0, a, b);
+    m1 = fmax3f(m1, x, y);
   }
-#pragma unroll
-  for (int g = 0; g < 4; ++g) {
-    const int ch = c * 4 + g;  // 16-byte chunk of the row (8 keys)
-    uint4 w;
-    w.x = pack2(v[g * 8 + 0], v[g * 8 + 1]);
-    w.y = pack2(v[g * 8 + 2], v[g * 8 + 3]);
-    w.z = pack2(v[g * 8 + 4], v[g * 8 + 5]);
-    w.w = pack2(v[g * 8 + 6], v[g * 8 + 7]);
-    *reinterpret_cast<uint4*>(P + (ch >> 3) * 16384 + row * 128 + (((ch & 7) ^ (row & 7)) << 4)) = w;
-  }
+  return fmaxf(m0, m1);
 }
 
 template <int DHP, int NQ>
@@ -194,9 +206,10 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
   constexpr uint32_t kIdS = idesc_bf16_f32(128, 128);
   constexpr uint32_t kIdPV = idesc_bf16_f32(128, 64) | (1u << 16);  // B (= V) MN-major
   extern __shared__ uint8_t smem_raw[];
-  const uint32_t base = smem_u32(smem_raw);
-  uint8_t* smem = smem_raw + ((1024 - (base & 1023)) & 1023);
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
   AttBars<NQ>* bar = reinterpret_cast<AttBars<NQ>*>(smem + Cfg::kOffBar);
+  static_assert(sizeof(AttBars<NQ>) <= 256, "barrier block exceeds its reserve");
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int bh = blockIdx.y;
@@ -207,22 +220,21 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
   const int row_k = ((1 * nslots + slot) * heads + head) * N;
   const int row_v = ((2 * nslots + slot) * heads + head) * N;
 
-  // a bounded wait of an earlier launch gave up: do nothing (the host
-  // reports DC_ERR_DEVICE_TIMEOUT at its next check)
-  if (*(volatile int*)err != 0) return;
   if (threadIdx.x == 0) {
+    // read once, so that the whole CTA takes the same decision below
+    bar->abort = *(volatile int*)err;
     mbar_init(&bar->q_full, 1);
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < kStages; ++b) {
       mbar_init(&bar->k_full[b], 1);
       mbar_init(&bar->k_empty[b], 1);
       mbar_init(&bar->v_full[b], 1);
       mbar_init(&bar->v_empty[b], 1);
-      for (int t = 0; t < NQ; ++t) {
-        mbar_init(&bar->s_full[t][b], 1);
-        mbar_init(&bar->p_full[t][b], 4);
-        mbar_init(&bar->o_full[t][b], 1);
-        mbar_init(&bar->buf_free[t][b], 4);
-      }
+    }
+    for (int t = 0; t < NQ; ++t) {
+      mbar_init(&bar->s_full[t], 1);
+      mbar_init(&bar->s_free[t], 4);
+      mbar_init(&bar->p_full[t], 4);
+      mbar_init(&bar->p_free[t], 1);
     }
     mbar_init(&bar->drain, 1);
     fence_barrier_init();
@@ -236,299 +248,297 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = bar->tmem_base;
-  // TMEM buffer (t, b) = columns (2 t + b) * 128 .. + 127
+  if (bar->abort != 0) {
+    // a bounded wait of an earlier launch gave up: do nothing (the host
+    // reports DC_ERR_DEVICE_TIMEOUT at its next check)
+    if (warp == 1) tmem_dealloc(tmem, Cfg::kTmemCols);
+    return;
+  }
 
-  if (warp == 0) {
-    if (lane == 0) {
+  // Each register region runs to its own end: the control warpgroup and the
+  // softmax warpgroups meet only at the named barrier before TMEM is freed.
+  if (warp < 4) {
+    if constexpr (Cfg::kSplitRegs)
+      asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(Cfg::kRegsCtl));
+    if (warp == 0) {
       // ------------------------------------------------------------ TMA
-      // K and V have rings of their own: K_j is released as soon as every
-      // S_{t,j} is issued, so the next key tile streams in while the PV
-      // products on V_j are still pending.
+      // The whole warp runs the loop (warp-uniform decisions, taken by lane
+      // 0 and broadcast); one elected lane issues the copies.  K and V have
+      // rings of their own: K_j is released as soon as every S_{t,j} is
+      // issued, so later key tiles stream in while the PV products on V_j
+      // are still pending.
       bool ok = true;
-      int last_k[2] = {-1, -1}, last_v[2] = {-1, -1};
-      mbar_arrive_expect_tx(&bar->q_full, NQ * Cfg::kTileBytes);
-      for (int t = 0; t < NQ; ++t)
-        for (int a = 0; a < Cfg::kAtoms; ++a)
-          tma_load_2d(smem + Cfg::kOffQ + t * Cfg::kTileBytes + a * 16384, &tm, &bar->q_full,
-                      a * 64, row_q + t * 128);
+      int last_k[kStages], last_v[kStages];
+      for (int b = 0; b < kStages; ++b) last_k[b] = last_v[b] = -1;
+      if (elect_one()) {
+        mbar_arrive_expect_tx(&bar->q_full, NQ * Cfg::kTileBytes);
+        for (int t = 0; t < NQ; ++t)
+          for (int a = 0; a < Cfg::kAtoms; ++a)
+            tma_load_2d(smem + Cfg::kOffQ + t * Cfg::kTileBytes + a * 16384, &tm, &bar->q_full,
+                        a * 64, row_q + t * 128);
+      }
+      __syncwarp();
       int nk = 0, nv = 0;
-      unsigned long long t_idle = global_ns();
+      long long t_idle = clock64();
       while (ok && nv < n_kv) {
         bool progressed = false;
         if (nk < n_kv) {
-          const int b = nk & 1;
-          const uint32_t u = (uint32_t)(nk >> 1);
-          if (mbar_test(&bar->k_empty[b], (u & 1) ^ 1)) {
-            mbar_arrive_expect_tx(&bar->k_full[b], Cfg::kTileBytes);
-            for (int a = 0; a < Cfg::kAtoms; ++a)
-              tma_load_2d(smem + Cfg::kOffK + b * Cfg::kTileBytes + a * 16384, &tm,
-                          &bar->k_full[b], a * 64, row_k + nk * 128);
+          const int b = nk % kStages;
+          const uint32_t u = (uint32_t)(nk / kStages);
+          int ready = 0;
+          if (lane == 0) ready = mbar_test(&bar->k_empty[b], (u & 1) ^ 1);
+          if (__shfl_sync(0xffffffffu, ready, 0)) {
+            if (elect_one()) {
+              mbar_arrive_expect_tx(&bar->k_full[b], Cfg::kTileBytes);
+              for (int a = 0; a < Cfg::kAtoms; ++a)
+                tma_load_2d(smem + Cfg::kOffK + b * Cfg::kTileBytes + a * 16384, &tm,
+                            &bar->k_full[b], a * 64, row_k + nk * 128);
+            }
+            __syncwarp();
             last_k[b] = (int)(u & 1);
             ++nk;
             progressed = true;
           }
         }
         if (nv < nk) {
-          const int b = nv & 1;
-          const uint32_t u = (uint32_t)(nv >> 1);
-          if (mbar_test(&bar->v_empty[b], (u & 1) ^ 1)) {
-            mbar_arrive_expect_tx(&bar->v_full[b], Cfg::kTileBytes);
-            for (int a = 0; a < Cfg::kAtoms; ++a)
-              tma_load_2d(smem + Cfg::kOffV + b * Cfg::kTileBytes + a * 16384, &tm,
-                          &bar->v_full[b], a * 64, row_v + nv * 128);
+          const int b = nv % kStages;
+          const uint32_t u = (uint32_t)(nv / kStages);
+          int ready = 0;
+          if (lane == 0) ready = mbar_test(&bar->v_empty[b], (u & 1) ^ 1);
+          if (__shfl_sync(0xffffffffu, ready, 0)) {
+            if (elect_one()) {
+              mbar_arrive_expect_tx(&bar->v_full[b], Cfg::kTileBytes);
+              for (int a = 0; a < Cfg::kAtoms; ++a)
+                tma_load_2d(smem + Cfg::kOffV + b * Cfg::kTileBytes + a * 16384, &tm,
+                            &bar->v_full[b], a * 64, row_v + nv * 128);
+            }
+            __syncwarp();
             last_v[b] = (int)(u & 1);
             ++nv;
             progressed = true;
           }
         }
         if (progressed) {
-          t_idle = global_ns();
-        } else if (*(volatile int*)err != 0) {
-          ok = false;
-        } else if (global_ns() - t_idle > kWaitLimitNs) {
-          atomicCAS(err, 0, kDevTimeoutTma);
-          ok = false;
+          t_idle = clock64();
+        } else {
+          int stop = 0;
+          if (lane == 0) {
+            if (*(volatile int*)err != 0) {
+              stop = 1;
+            } else if (clock64() - t_idle > kWaitLimitCycles) {
+              atomicCAS(err, 0, kDevTimeoutTma);
+              stop = 1;
+            }
+          }
+          if (__shfl_sync(0xffffffffu, stop, 0)) ok = false;
         }
       }
       // every copy in flight lands before the CTA can exit
-      mbar_wait(&bar->q_full, 0, err, kDevTimeoutTma);
-      for (int b = 0; b < 2; ++b) {
-        if (last_k[b] >= 0) mbar_wait(&bar->k_full[b], (uint32_t)last_k[b], err, kDevTimeoutTma);
-        if (last_v[b] >= 0) mbar_wait(&bar->v_full[b], (uint32_t)last_v[b], err, kDevTimeoutTma);
+      mbar_wait_warp(&bar->q_full, 0, err, kDevTimeoutTma);
+      for (int b = 0; b < kStages; ++b) {
+        if (last_k[b] >= 0) mbar_wait_warp(&bar->k_full[b], (uint32_t)last_k[b], err, kDevTimeoutTma);
+        if (last_v[b] >= 0) mbar_wait_warp(&bar->v_full[b], (uint32_t)last_v[b], err, kDevTimeoutTma);
       }
-    }
-  } else if (warp == 1) {
-    if (lane == 0) {
+    } else if (warp == 1) {
       // ------------------------------------------------------------ MMA
-      // Issue whichever operation is ready (non-blocking tests), so that a
-      // lagging softmax warpgroup never holds up the other one:
-      //   S_{t,j}  needs K_j loaded and buffer (t, j % 2) freed (PV_{t,j-2} folded)
-      //   PV_{t,j} needs P_{t,j} written (S_{t,j} consumed) and V_j loaded
-      bool ok = mbar_wait(&bar->q_full, 0, err, kDevTimeoutMma);
-      int next_s[NQ], next_pv[NQ];
-      for (int t = 0; t < NQ; ++t) next_s[t] = next_pv[t] = 0;
-      int released = 0, k_released = 0;  // stages handed back to the loader (V, K)
-      unsigned long long t_idle = global_ns();
-      while (ok) {
-        bool progressed = false, done = true;
-        for (int t = 0; t < NQ; ++t) {
-          const int js = next_s[t];
-          if (js < n_kv) {
-            done = false;
-            const int b = js & 1;
-            const uint32_t u = (uint32_t)(js >> 1);
-            if (mbar_test(&bar->k_full[b], u & 1) && mbar_test(&bar->buf_free[t][b], (u & 1) ^ 1)) {
-              tc_fence_after();
-              const uint32_t sK = smem_u32(smem + Cfg::kOffK + b * Cfg::kTileBytes);
-              const uint32_t sQ = smem_u32(smem + Cfg::kOffQ + t * Cfg::kTileBytes);
+      // Fixed order with blocking waits.  Round j issues S_{t,j} for every
+      // query tile (each needs K_j and S_{t,j-1} read by its softmax, which
+      // happens at the start of that softmax tile), then PV_{t,j-1} (each
+      // needs P_{t,j-1} and V_{j-1}).  Nothing waited for here depends on a
+      // later issue, so the order cannot deadlock.  The whole warp runs the
+      // loop with uniform descriptors; one elected lane (the same one
+      // throughout, as tcgen05.commit tracks the issuing thread) issues.
+      bool ok = mbar_wait_warp(&bar->q_full, 0, err, kDevTimeoutMma);
+      // descriptor + (byte offset >> 4) moves the start address (no carry:
+      // shared-memory addresses are below 256 KB)
+      const uint64_t dQ = sw128_kmajor_desc(smem_u32(smem + Cfg::kOffQ));
+      const uint64_t dK = sw128_kmajor_desc(smem_u32(smem + Cfg::kOffK));
+      const uint64_t dV = sw128_mnmajor_desc(smem_u32(smem + Cfg::kOffV));
+      for (int j = 0; j <= n_kv && ok; ++j) {
+        if (j < n_kv) {
+          const int kb = j % kStages;
+          ok = mbar_wait_warp(&bar->k_full[kb], (uint32_t)(j / kStages) & 1, err, kDevTimeoutMma);
+          for (int t = 0; t < NQ && ok; ++t) {
+            ok = mbar_wait_warp(&bar->s_free[t], ((uint32_t)j & 1) ^ 1, err, kDevTimeoutMma);
+            if (!ok) break;
+            tc_fence_after();
+            if (elect_one()) {
 #pragma unroll
               for (int kk = 0; kk < DHP / 16; ++kk) {
                 const uint32_t off = (kk >> 2) * 16384 + (kk & 3) * 32;
-                tc_mma_f16(tmem + (2 * t + b) * 128, sw128_kmajor_desc(sQ + off),
-                           sw128_kmajor_desc(sK + off), kIdS, kk > 0 ? 1u : 0u);
+                tc_mma_f16(tmem + Cfg::kColS + t * 128,
+                           dQ + ((uint32_t)(t * Cfg::kTileBytes + off) >> 4),
+                           dK + ((uint32_t)(kb * Cfg::kTileBytes + off) >> 4), kIdS,
+                           kk > 0 ? 1u : 0u);
               }
-              tc_commit(&bar->s_full[t][b]);
-              next_s[t] = js + 1;
-              progressed = true;
+              tc_commit(&bar->s_full[t]);
             }
+            __syncwarp();
           }
-          const int jp = next_pv[t];
-          if (jp < n_kv) {
-            done = false;
-            const int b = jp & 1;
-            const uint32_t u = (uint32_t)(jp >> 1);
-            if (jp < next_s[t] && mbar_test(&bar->p_full[t][b], u & 1) &&
-                mbar_test(&bar->v_full[b], u & 1)) {
-              tc_fence_after();
-              const uint32_t sV = smem_u32(smem + Cfg::kOffV + b * Cfg::kTileBytes);
-              const uint32_t sP = smem_u32(smem + Cfg::kOffP + (2 * t + b) * Cfg::kPBytes);
+          if (!ok) break;
+          if (elect_one()) tc_commit(&bar->k_empty[kb]);
+          __syncwarp();
+        }
+        if (j >= 1) {
+          const int jp = j - 1;
+          const int vb = jp % kStages;
+          ok = mbar_wait_warp(&bar->v_full[vb], (uint32_t)(jp / kStages) & 1, err, kDevTimeoutMma);
+          for (int t = 0; t < NQ && ok; ++t) {
+            ok = mbar_wait_warp(&bar->p_full[t], (uint32_t)jp & 1, err, kDevTimeoutMma);
+            if (!ok) break;
+            tc_fence_after();
+            if (elect_one()) {
 #pragma unroll
               for (int kk = 0; kk < 8; ++kk) {
-                const uint64_t ad = sw128_kmajor_desc(sP + (kk >> 2) * 16384 + (kk & 3) * 32);
 #pragma unroll
                 for (int a = 0; a < Cfg::kAtoms; ++a)
-                  tc_mma_f16(tmem + (2 * t + b) * 128 + a * 64, ad,
-                             sw128_mnmajor_desc(sV + a * 16384 + kk * 2048), kIdPV,
-                             kk > 0 ? 1u : 0u);
+                  tc_mma_f16_ta(tmem + Cfg::kColO + t * DHP + a * 64,
+                                tmem + Cfg::kColP + t * 64 + kk * 8,
+                                dV + ((uint32_t)(vb * Cfg::kTileBytes + a * 16384 + kk * 2048) >> 4),
+                                kIdPV, (jp > 0 || kk > 0) ? 1u : 0u);
               }
-              tc_commit(&bar->o_full[t][b]);
-              next_pv[t] = jp + 1;
-              progressed = true;
+              tc_commit(&bar->p_free[t]);
             }
+            __syncwarp();
           }
-        }
-        // a K stage goes back to the loader once every tile's S on it is
-        // issued, a V stage once every tile's PV on it is
-        int min_s = n_kv, min_pv = n_kv;
-        for (int t = 0; t < NQ; ++t) {
-          min_s = min(min_s, next_s[t]);
-          min_pv = min(min_pv, next_pv[t]);
-        }
-        while (k_released < min_s) {
-          tc_commit(&bar->k_empty[k_released & 1]);
-          ++k_released;
-        }
-        while (released < min_pv) {
-          tc_commit(&bar->v_empty[released & 1]);
-          ++released;
-        }
-        if (done) break;
-        if (progressed) {
-          t_idle = global_ns();
-        } else if (global_ns() - t_idle > kWaitLimitNs) {
-          atomicCAS(err, 0, kDevTimeoutMma);
-          ok = false;
+          if (!ok) break;
+          if (elect_one()) tc_commit(&bar->v_empty[vb]);
+          __syncwarp();
         }
       }
-      tc_commit(&bar->drain);
-      mbar_wait(&bar->drain, 0, err, kDevTimeoutMma);
+      if (elect_one()) tc_commit(&bar->drain);
+      __syncwarp();
+      mbar_wait_warp(&bar->drain, 0, err, kDevTimeoutMma);
+    }
+    tc_fence_before();
+    named_bar(1, Cfg::kThreads);
+    if (warp == 1) {
+      tc_fence_after();
+      tmem_dealloc(tmem, Cfg::kTmemCols);
     }
   } else {
+    if constexpr (Cfg::kSplitRegs)
+      asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(Cfg::kRegsSoftmax));
     // ------------------------------------------------------------ softmax
-    const int t = (warp - 2) >> 2;  // query tile of this warpgroup
+    const int t = (warp - 4) >> 2;  // query tile of this warpgroup
     const int q = warp & 3;         // TMEM lane quarter
     const int row = q * 32 + lane;
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
-    float O[DHP];
-#pragma unroll
-    for (int i = 0; i < DHP; ++i) O[i] = 0.f;
-    float ref = -INFINITY, l = 0.f, c_prev = 1.f;
+    const uint32_t tO = tmem + Cfg::kColO + t * DHP + lane_off;
+    const uint32_t tS = tmem + Cfg::kColS + t * 128 + lane_off;
+    const uint32_t tP = tmem + Cfg::kColP + t * 64 + lane_off;
+    float ref = -INFINITY, l = 0.f;
     bool ok = true;
-    // fold PV_{t,i} (relative to the reference of tile i) and free its buffer
-    auto fold = [&](int i, float c) -> bool {
-      const int b = i & 1;
-      if (!mbar_wait_warp(&bar->o_full[t][b], (uint32_t)(i >> 1) & 1, err, kDevTimeoutEpi)) return false;
-      tc_fence_after();
-      const uint32_t tb = tmem + (2 * t + b) * 128 + lane_off;
-      const bool scale = __any_sync(0xffffffffu, c != 1.f);
-      const float2 c2 = make_float2(c, c);
-#pragma unroll
-      for (int ch = 0; ch < DHP / 32; ++ch) {
-        uint32_t r[32];
-        tmem_ld32_async(tb + ch * 32, r);
-        tmem_ld_wait_regs(r);
-#pragma unroll
-        for (int e = 0; e < 32; e += 2) {
-          float2 acc = fadd2(make_float2(O[ch * 32 + e], O[ch * 32 + e + 1]),
-                             make_float2(__uint_as_float(r[e]), __uint_as_float(r[e + 1])));
-          if (scale) acc = fmul2(acc, c2);
-          O[ch * 32 + e] = acc.x;
-          O[ch * 32 + e + 1] = acc.y;
-        }
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bar->buf_free[t][b]);
-      return true;
-    };
     for (int j = 0; j < n_kv && ok; ++j) {
-      const int b = j & 1;
-      if (!mbar_wait_warp(&bar->s_full[t][b], (uint32_t)(j >> 1) & 1, err, kDevTimeoutEpi)) {
+      if (!mbar_wait_warp(&bar->s_full[t], (uint32_t)j & 1, err, kDevTimeoutEpi)) {
         ok = false;
         break;
       }
       tc_fence_after();
-      const uint32_t tS = tmem + (2 * t + b) * 128 + lane_off;
-      uint8_t* Pb = smem + Cfg::kOffP + (2 * t + b) * Cfg::kPBytes;
+      uint32_t s0[32], s1[32], s2[32], s3[32];
+      tmem_ld32_async(tS + 0, s0);
+      tmem_ld32_async(tS + 32, s1);
+      tmem_ld32_async(tS + 64, s2);
+      tmem_ld32_async(tS + 96, s3);
+      tmem_ld_wait_regs(s0);
+      tmem_ld_wait_regs(s1);
+      tmem_ld_wait_regs(s2);
+      tmem_ld_wait_regs(s3);
+      // S is in registers: hand S_t back to the MMA warp
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bar->s_free[t]);
+
       const int valid = min(128, N - j * 128);
-      if (j == 0) {
-        // the first tile sets the reference max
-        float mx = -INFINITY;
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          uint32_t r[32];
-          tmem_ld32_async(tS + c * 32, r);
-          tmem_ld_wait_regs(r);
-#pragma unroll
-          for (int e = 0; e < 32; ++e)
-            if (c * 32 + e < valid) mx = fmaxf(mx, __uint_as_float(r[e]));
-        }
-        ref = mx * scale_log2;
+      float mx;
+      if (valid == 128) {
+        mx = chunk_max<false>(s0, 0, valid, -INFINITY);
+        mx = chunk_max<false>(s1, 1, valid, mx);
+        mx = chunk_max<false>(s2, 2, valid, mx);
+        mx = chunk_max<false>(s3, 3, valid, mx);
+      } else {
+        mx = chunk_max<true>(s0, 0, valid, -INFINITY);
+        mx = chunk_max<true>(s1, 1, valid, mx);
+        mx = chunk_max<true>(s2, 2, valid, mx);
+        mx = chunk_max<true>(s3, 3, valid, mx);
       }
-      float tmax4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+      const float tm = mx * scale_log2;
+      float c = 1.f;
+      if (j == 0) {
+        ref = tm;
+      } else if (tm > ref + kRefSlack) {
+        c = ex2_mufu(ref - tm);
+        ref = tm;
+      }
+      uint32_t pk[64];
       float2 rs2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
       const float neg_ref = -ref;
-      uint32_t ra[32], rb[32];
-      // first half: chunks 0 and 1
-      tmem_ld32_async(tS + 0, ra);
-      tmem_ld_wait_regs(ra);
-      tmem_ld32_async(tS + 32, rb);
-      if (valid == 128) softmax_chunk<false>(ra, 0, valid, scale_log2, neg_ref, tmax4, rs2, Pb, row);
-      else softmax_chunk<true>(ra, 0, valid, scale_log2, neg_ref, tmax4, rs2, Pb, row);
-      tmem_ld_wait_regs(rb);
-      if (valid == 128) softmax_chunk<false>(rb, 1, valid, scale_log2, neg_ref, tmax4, rs2, Pb, row);
-      else softmax_chunk<true>(rb, 1, valid, scale_log2, neg_ref, tmax4, rs2, Pb, row);
-      // fold PV_{j-1} (issued at the end of the previous tile)
-      if (j >= 1 && !fold(j - 1, c_prev)) { ok = false; break; }
-      // second half: chunks 2 and 3
-      tmem_ld32_async(tS + 64, ra);
-      tmem_ld_wait_regs(ra);
-      tmem_ld32_async(tS + 96, rb);
-      if (valid == 128) softmax_chunk<false>(ra, 2, valid, scale_log2, neg_ref, tmax4, rs2, Pb, row);
-      else softmax_chunk<true>(ra, 2, valid, scale_log2, neg_ref, tmax4, rs2, Pb, row);
-      tmem_ld_wait_regs(rb);
-      if (valid == 128) softmax_chunk<false>(rb, 3, valid, scale_log2, neg_ref, tmax4, rs2, Pb, row);
-      else softmax_chunk<true>(rb, 3, valid, scale_log2, neg_ref, tmax4, rs2, Pb, row);
-      const float tmax = fmaxf(fmaxf(tmax4[0], tmax4[1]), fmaxf(tmax4[2], tmax4[3]));
-      float rs = (rs2[0].x + rs2[0].y) + (rs2[1].x + rs2[1].y);
-      const float tm = tmax * scale_log2;
-      if (__any_sync(0xffffffffu, tm - ref > kRedoExcess)) {
-        // rare: a row's max jumped far above its reference; rescale what is
-        // accumulated to the new max and redo this tile against it
-        if (tm > ref) {
-          const float c = ex2_mufu(ref - tm);
-#pragma unroll
-          for (int i = 0; i < DHP; ++i) O[i] *= c;
-          l *= c;
-          ref = tm;
-        }
-        float dummy[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-        float2 rr[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          tmem_ld32_async(tS + c * 32, ra);
-          tmem_ld_wait_regs(ra);
-          softmax_chunk<true>(ra, c, valid, scale_log2, -ref, dummy, rr, Pb, row);
-        }
-        l += (rr[0].x + rr[0].y) + (rr[1].x + rr[1].y);
-        c_prev = 1.f;
+      if (valid == 128) {
+        p_chunk<false>(s0, 0, valid, scale_log2, neg_ref, rs2, pk + 0);
+        p_chunk<false>(s1, 1, valid, scale_log2, neg_ref, rs2, pk + 16);
+        p_chunk<false>(s2, 2, valid, scale_log2, neg_ref, rs2, pk + 32);
+        p_chunk<false>(s3, 3, valid, scale_log2, neg_ref, rs2, pk + 48);
       } else {
-        float c = 1.f;
-        if (tm > ref + kRefSlack) {
-          c = ex2_mufu(ref - tm);
-          ref = tm;
-        }
-        l = (l + rs) * c;
-        c_prev = c;
+        p_chunk<true>(s0, 0, valid, scale_log2, neg_ref, rs2, pk + 0);
+        p_chunk<true>(s1, 1, valid, scale_log2, neg_ref, rs2, pk + 16);
+        p_chunk<true>(s2, 2, valid, scale_log2, neg_ref, rs2, pk + 32);
+        p_chunk<true>(s3, 3, valid, scale_log2, neg_ref, rs2, pk + 48);
       }
-      // S consumed, P written: hand the buffer to the PV MMA
+      l = l * c + ((rs2[0].x + rs2[0].y) + (rs2[1].x + rs2[1].y));
+      // P_t and O_t are free once PV_{t,j-1} has landed
+      if (!mbar_wait_warp(&bar->p_free[t], ((uint32_t)j & 1) ^ 1, err, kDevTimeoutEpi)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      if (__any_sync(0xffffffffu, c != 1.f)) {
+        // the reference moved for some row of this warp: rescale the warp's
+        // 32 rows of O_t (c = 1 elsewhere) before PV_{t,j} accumulates
+#pragma unroll
+        for (int ch = 0; ch < DHP / 32; ++ch) {
+          uint32_t r[32];
+          tmem_ld32_async(tO + ch * 32, r);
+          tmem_ld_wait_regs(r);
+#pragma unroll
+          for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * c);
+          tmem_st32(tO + ch * 32, r);
+        }
+      }
+      tmem_st32(tP + 0, *reinterpret_cast<const uint32_t(*)[32]>(pk));
+      tmem_st32(tP + 32, *reinterpret_cast<const uint32_t(*)[32]>(pk + 32));
+      tmem_st_wait();
+      // P in TMEM (and O rescaled): hand both to the PV MMA
       tc_fence_before();
-      fence_proxy_async();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&bar->p_full[t][b]);
+      if (lane == 0) mbar_arrive(&bar->p_full[t]);
     }
-    if (ok) ok = fold(n_kv - 1, c_prev);
+    // the last PV product of this query tile completes O_t
+    if (ok) ok = mbar_wait_warp(&bar->p_free[t], (uint32_t)(n_kv - 1) & 1, err, kDevTimeoutEpi);
     const int qrow = q0 + t * 128 + row;
-    if (ok && qrow < N) {
+    if (ok) {
+      tc_fence_after();
       const float inv = 1.f / l;
       __nv_bfloat16* dst = o + ((size_t)slot * N + qrow) * ((size_t)heads * DHP) + head * DHP;
 #pragma unroll
-      for (int e = 0; e < DHP; e += 8) {
-        uint4 w;
-        w.x = pack2(O[e] * inv, O[e + 1] * inv);
-        w.y = pack2(O[e + 2] * inv, O[e + 3] * inv);
-        w.z = pack2(O[e + 4] * inv, O[e + 5] * inv);
-        w.w = pack2(O[e + 6] * inv, O[e + 7] * inv);
-        *reinterpret_cast<uint4*>(dst + e) = w;
+      for (int ch = 0; ch < DHP / 32; ++ch) {
+        uint32_t r[32];
+        tmem_ld32_async(tO + ch * 32, r);
+        tmem_ld_wait_regs(r);
+        if (qrow < N) {
+#pragma unroll
+          for (int e = 0; e < 32; e += 8) {
+            uint4 w;
+            w.x = pack2(__uint_as_float(r[e]) * inv, __uint_as_float(r[e + 1]) * inv);
+            w.y = pack2(__uint_as_float(r[e + 2]) * inv, __uint_as_float(r[e + 3]) * inv);
+            w.z = pack2(__uint_as_float(r[e + 4]) * inv, __uint_as_float(r[e + 5]) * inv);
+            w.w = pack2(__uint_as_float(r[e + 6]) * inv, __uint_as_float(r[e + 7]) * inv);
+            *reinterpret_cast<uint4*>(dst + ch * 32 + e) = w;
+          }
+        }
       }
     }
-  }
-
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 1) {
-    tc_fence_after();
-    tmem_dealloc(tmem, Cfg::kTmemCols);
+    tc_fence_before();
+    named_bar(1, Cfg::kThreads);
   }
 }
 
@@ -541,6 +551,12 @@ cudaError_t launch_tc(const CUtensorMap& tm, int nslots, int heads, int N, __nv_
     cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<DHP, NQ>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmem);
     if (e != cudaSuccess) return e;
+    // setmaxnreg.inc waits until the CTA's launch allocation can serve it:
+    // never launch a build whose allocation is not the one the split assumes
+    cudaFuncAttributes fa;
+    e = cudaFuncGetAttributes(&fa, attn_tc_kernel<DHP, NQ>);
+    if (e != cudaSuccess) return e;
+    if (Cfg::kSplitRegs && fa.numRegs != Cfg::kRegsLaunch) return cudaErrorInvalidConfiguration;
     configured = true;
   }
   dim3 grid((N + 128 * NQ - 1) / (128 * NQ), nslots * heads);

@@ -62,6 +62,7 @@ struct __align__(8) Barriers {
   uint64_t hin_full;
   uint64_t drain;
   uint32_t tmem_base;
+  int abort;  // the error word was set before this CTA started
 };
 
 // byte offset of 16-byte chunk `c` of row `r` in a [rows][128 B] box written
@@ -85,6 +86,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* sOut = smem + Cfg::kOffOut;
   float* vec = reinterpret_cast<float*>(smem + Cfg::kOffVec);
   Barriers* bar = reinterpret_cast<Barriers*>(smem + Cfg::kOffBar);
+  static_assert(sizeof(Barriers) <= 256, "barrier block exceeds its reserve");
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -93,10 +95,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int n_tiles = tiles_m * tiles_n;
   const int KB = K / kBK;
 
-  // a bounded wait of an earlier launch gave up: do nothing (the host
-  // reports DC_ERR_DEVICE_TIMEOUT at its next check)
-  if (*(volatile int*)err != 0) return;
   if (threadIdx.x == 0) {
+    // read once, so that the whole CTA takes the same decision below
+    bar->abort = *(volatile int*)err;
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&bar->full[s], 1);
       mbar_init(&bar->empty[s], 1);
@@ -121,6 +122,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = bar->tmem_base;
+  if (bar->abort != 0) {
+    // a bounded wait of an earlier launch gave up: do nothing (the host
+    // reports DC_ERR_DEVICE_TIMEOUT at its next check)
+    if (warp == 1) tmem_dealloc(tmem_base, kTmemCols);
+    return;
+  }
 
   if (warp == 0) {
     if (lane == 0) {

@@ -328,6 +328,31 @@ def test_attention_kernel_sharp_softmax(dc, dh, N, heads, slots):
         assert rel(got[s], ref) <= 1e-2, rel(got[s], ref)
 
 
+@pytest.mark.parametrize("dh,N,heads,slots", [(64, 700, 2, 2), (128, 517, 1, 2)])
+def test_attention_kernel_growing_logits(dc, dh, N, heads, slots):
+    """Key norms ramp up 1 -> 5 along the sequence, so each row's running max
+    keeps rising tile after tile: the running reference moves (and the
+    accumulated output is rescaled) many times per row, and the last, ragged
+    tile holds the largest logits."""
+    from oracle.dit import attention_core
+    rng = np.random.default_rng(3 * dh + N)
+    qkv = np.zeros((3, slots, heads, N, dh), np.float32)
+    qkv[...] = rng.standard_normal((3, slots, heads, N, dh))
+    qkv[0] *= 2.0
+    qkv[1] *= np.linspace(1.0, 5.0, N, dtype=np.float32)[None, None, :, None]
+    t = torch.tensor(qkv, device="cuda").to(torch.bfloat16)
+    ref_in = t.float().cpu().numpy()
+    out = torch.zeros((slots, N, heads * dh), device="cuda", dtype=torch.bfloat16)
+    dc.attention(t, slots, heads, N, dh, out)
+    torch.cuda.synchronize()
+    got = out.float().cpu().numpy()
+    for s in range(slots):
+        ref = attention_core(ref_in[0, s], ref_in[1, s], ref_in[2, s])
+        ref = ref.transpose(1, 0, 2).reshape(N, heads * dh)
+        record(f"attn_bf16_growing_dh{dh}_N{N}", dict(rel=rel(got[s], ref)))
+        assert rel(got[s], ref) <= 1e-2, rel(got[s], ref)
+
+
 @pytest.mark.parametrize("dh,N", [(16, 128), (16, 77), (64, 50)])
 def test_attention_kernel_fp32(dc, dh, N):
     from oracle.dit import attention_core
