@@ -24,6 +24,9 @@ struct EpiArgs {
   const float* mod;    // Resid: modulation table of this step [B][mod_stride]
   int mod_stride;      // floats per scene in the table
   int gate_off;        // offset of this block's gate vector inside a scene's row
+  int qkv_tma;         // QKV (tcgen05 GEMM): the output map covers q/k/v viewed as
+                       // [3 * slots * heads * tokens][dh_pad] with 64 x 128 boxes, and
+                       // dh is a multiple of 64: tiles inside one slot go out by TMA
 };
 
 template <typename T> struct Pack8;

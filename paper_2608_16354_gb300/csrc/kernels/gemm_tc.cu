@@ -43,9 +43,9 @@ constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, kBN);
 template <int MODE>
 struct GemmCfg {
   static constexpr int kStages = MODE == kEpiResid ? 3 : 4;
-  // epilogue staging tile: residual 6 boxes of [128 rows][32 fp32], GELU 3
-  // boxes of [128 rows][64 bf16]; 16 KB per box, 128-byte swizzle
-  static constexpr int kOutBytes = MODE == kEpiResid ? 6 * 16384 : MODE == kEpiGELU ? 3 * 16384 : 0;
+  // epilogue staging tile: residual 6 boxes of [128 rows][32 fp32], GELU and
+  // QKV 3 boxes of [128 rows][64 bf16]; 16 KB per box, 128-byte swizzle
+  static constexpr int kOutBytes = MODE == kEpiResid ? 6 * 16384 : 3 * 16384;
   static constexpr int kOffA = 0;
   static constexpr int kOffB = kOffA + kStages * kABytes;
   static constexpr int kOffOut = kOffB + kStages * kBBytes;
@@ -130,61 +130,74 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 
   if (warp == 0) {
-    if (lane == 0) {
-      // ------------------------------------------------ TMA producer
-      int stage = 0;
-      uint32_t phase = 0;
-      int last_phase[kStages];
-      for (int s = 0; s < kStages; ++s) last_phase[s] = -1;
-      bool ok = true;
-      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
-        const int m0 = (tile / tiles_n) * kBM;
-        const int n0 = (tile % tiles_n) * kBN;
-        for (int kb = 0; kb < KB; ++kb) {
-          if (!mbar_wait(&bar->empty[stage], phase ^ 1, err, kDevTimeoutTma)) { ok = false; break; }
+    // -------------------------------------------------- TMA producer
+    // The whole warp runs the loop (uniform waits); one elected lane issues.
+    int stage = 0;
+    uint32_t phase = 0;
+    int last_phase[kStages];
+    for (int s = 0; s < kStages; ++s) last_phase[s] = -1;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+      const int m0 = (tile / tiles_n) * kBM;
+      const int n0 = (tile % tiles_n) * kBN;
+      for (int kb = 0; kb < KB; ++kb) {
+        if (!mbar_wait_warp(&bar->empty[stage], phase ^ 1, err, kDevTimeoutTma)) { ok = false; break; }
+        if (elect_one()) {
           mbar_arrive_expect_tx(&bar->full[stage], kStageBytes);
           tma_load_2d(sA + (size_t)stage * kABytes, &tmA, &bar->full[stage], kb * kBK, m0);
           tma_load_2d(sB + (size_t)stage * kBBytes, &tmB, &bar->full[stage], kb * kBK, n0);
-          last_phase[stage] = (int)phase;
-          if (++stage == kStages) { stage = 0; phase ^= 1; }
         }
+        __syncwarp();
+        last_phase[stage] = (int)phase;
+        if (++stage == kStages) { stage = 0; phase ^= 1; }
       }
-      // do not leave the CTA with copies still landing in shared memory
-      for (int s = 0; s < kStages; ++s)
-        if (last_phase[s] >= 0) mbar_wait(&bar->full[s], (uint32_t)last_phase[s], err, kDevTimeoutTma);
     }
+    // do not leave the CTA with copies still landing in shared memory
+    for (int s = 0; s < kStages; ++s)
+      if (last_phase[s] >= 0) mbar_wait_warp(&bar->full[s], (uint32_t)last_phase[s], err, kDevTimeoutTma);
   } else if (warp == 1) {
-    if (lane == 0) {
-      // ------------------------------------------------ MMA issuer
-      int stage = 0;
-      uint32_t phase = 0;
-      bool ok = true;
-      int t = 0;
-      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++t) {
-        const int b = t & 1;
-        const uint32_t use = (uint32_t)(t >> 1);
-        if (!mbar_wait(&bar->tmem_empty[b], (use & 1) ^ 1, err, kDevTimeoutMma)) { ok = false; break; }
+    // -------------------------------------------------- MMA issuer
+    // The whole warp runs the loop with uniform descriptors; one elected lane
+    // (the same one throughout: tcgen05.commit tracks the issuing thread)
+    // issues the MMAs and commits.
+    int stage = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    int t = 0;
+    // descriptor + (byte offset >> 4) moves the start address (no carry:
+    // shared-memory addresses are below 256 KB)
+    const uint64_t dA = sw128_kmajor_desc(smem_u32(sA));
+    const uint64_t dB = sw128_kmajor_desc(smem_u32(sB));
+    for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++t) {
+      const int b = t & 1;
+      const uint32_t use = (uint32_t)(t >> 1);
+      if (!mbar_wait_warp(&bar->tmem_empty[b], (use & 1) ^ 1, err, kDevTimeoutMma)) { ok = false; break; }
+      tc_fence_after();
+      const uint32_t d_tmem = tmem_base + (uint32_t)(b * 256);
+      for (int kb = 0; kb < KB; ++kb) {
+        if (!mbar_wait_warp(&bar->full[stage], phase, err, kDevTimeoutMma)) { ok = false; break; }
         tc_fence_after();
-        const uint32_t d_tmem = tmem_base + (uint32_t)(b * 256);
-        for (int kb = 0; kb < KB; ++kb) {
-          if (!mbar_wait(&bar->full[stage], phase, err, kDevTimeoutMma)) { ok = false; break; }
-          tc_fence_after();
-          const uint32_t a0 = smem_u32(sA + (size_t)stage * kABytes);
-          const uint32_t b0 = smem_u32(sB + (size_t)stage * kBBytes);
+        if (elect_one()) {
 #pragma unroll
           for (int kk = 0; kk < kBK / 16; ++kk) {
-            tc_mma_f16(d_tmem, sw128_kmajor_desc(a0 + kk * 32), sw128_kmajor_desc(b0 + kk * 32),
-                       kIdesc, (kb | kk) != 0 ? 1u : 0u);
+            tc_mma_f16(d_tmem, dA + ((uint32_t)(stage * kABytes + kk * 32) >> 4),
+                       dB + ((uint32_t)(stage * kBBytes + kk * 32) >> 4), kIdesc,
+                       (kb | kk) != 0 ? 1u : 0u);
           }
           tc_commit(&bar->empty[stage]);
-          if (++stage == kStages) { stage = 0; phase ^= 1; }
         }
-        if (ok) tc_commit(&bar->tmem_full[b]);
+        __syncwarp();
+        if (++stage == kStages) { stage = 0; phase ^= 1; }
       }
-      // every MMA this thread issued has completed once `drain` flips
-      tc_commit(&bar->drain);
-      mbar_wait(&bar->drain, 0, err, kDevTimeoutMma);
+      if (ok) {
+        if (elect_one()) tc_commit(&bar->tmem_full[b]);
+        __syncwarp();
+      }
     }
+    // every MMA this warp issued has completed once `drain` flips
+    if (elect_one()) tc_commit(&bar->drain);
+    __syncwarp();
+    mbar_wait_warp(&bar->drain, 0, err, kDevTimeoutMma);
   } else {
     // ---------------------------------------------------- epilogue warps
     const int q = warp & 3;             // TMEM lane quarter this warp may access
@@ -201,6 +214,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                     (tile / tiles_n) * kBM);
       hin_loads = 1;
     }
+    // bias (and gate rows) of the next tile are loaded into registers while
+    // the current tile is processed, and staged to shared memory at its start
+    float nb = 0.f, nga = 0.f, ngb = 0.f;
+    auto fetch_vec = [&](int tile) {
+      if (tile < n_tiles && et < kBN) {
+        const int fm0 = (tile / tiles_n) * kBM, fn0 = (tile % tiles_n) * kBN;
+        nb = ep.bias[fn0 + et];
+        if (MODE == kEpiResid) {
+          const int sa = fm0 / ep.n_tok, sb = (min(fm0 + kBM, M) - 1) / ep.n_tok;
+          nga = ep.mod[(size_t)map.scene[sa] * ep.mod_stride + ep.gate_off + fn0 + et];
+          ngb = ep.mod[(size_t)map.scene[sb] * ep.mod_stride + ep.gate_off + fn0 + et];
+        }
+      }
+    };
+    fetch_vec(blockIdx.x);
     int t = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++t) {
@@ -231,14 +259,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int last_row = min(m0 + kBM, M) - 1;
       const int slot_a = m0 / ep.n_tok, slot_b = last_row / ep.n_tok;
       const int split = (slot_a + 1) * ep.n_tok;  // first row that belongs to slot_b
-      for (int i = et; i < kBN; i += kEpiThreads) {
-        vec[i] = ep.bias[n0 + i];
+      if (et < kBN) {
+        vec[et] = nb;
         if (MODE == kEpiResid) {
-          vec[kBN + i] = ep.mod[(size_t)map.scene[slot_a] * ep.mod_stride + ep.gate_off + n0 + i];
-          vec[2 * kBN + i] = ep.mod[(size_t)map.scene[slot_b] * ep.mod_stride + ep.gate_off + n0 + i];
+          vec[kBN + et] = nga;
+          vec[2 * kBN + et] = ngb;
         }
       }
-      if (MODE == kEpiGELU && leader) bulk_wait_read0();  // previous tile's stores have read sOut
+      fetch_vec(tile + gridDim.x);
+      if (MODE != kEpiResid && leader) bulk_wait_read0();  // previous tile's stores have read sOut
       named_bar(1, kEpiThreads);
 
       if constexpr (MODE == kEpiResid) {
@@ -317,6 +346,37 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int k = 0; k < 3; ++k) tma_store_2d(&tmCout, sOut + k * 16384, n0 + 64 * k, m0);
           bulk_commit();
         }
+      } else if (ep.qkv_tma && m0 + kBM <= M && (m0 + kBM - 1) / ep.n_tok == slot_a) {
+        // QKV, tile inside one slot: each 64-column group is one head's
+        // [128 tokens][64] block of q, k or v, contiguous in the head-major
+        // layout; stage the bf16 tile swizzled and store it with TMA
+#pragma unroll
+        for (int c = 0; c < 3; ++c) {
+#pragma unroll
+          for (int g = 0; g < 4; ++g) {
+            const int j = half * 96 + c * 32 + g * 8;  // tile column of this 8-column group
+            float v[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) v[i] = acc[c][g * 8 + i] + vec[j + i];
+            Pack8<__nv_bfloat16>::store(
+                reinterpret_cast<__nv_bfloat16*>(sOut + (j >> 6) * 16384 + sw128_off(r, (j & 63) >> 3)), v);
+          }
+        }
+        fence_proxy_async();
+        named_bar(1, kEpiThreads);
+        if (leader) {
+          const int tok0 = m0 - slot_a * ep.n_tok;
+          for (int k = 0; k < 3; ++k) {
+            const int col = n0 + 64 * k;
+            const int which = col / ep.d;
+            const int within = col - which * ep.d;
+            const int head = within / ep.dh;
+            const int e = within - head * ep.dh;
+            tma_store_2d(&tmCout, sOut + k * 16384, e,
+                         ((which * ep.nslots + slot_a) * ep.heads + head) * ep.n_tok + tok0);
+          }
+          bulk_commit();
+        }
       } else {
         // QKV: each thread stores 16-byte pieces of its own row
         const int row = m0 + r;
@@ -346,7 +406,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     if (leader) {
-      if (MODE != kEpiQKV) bulk_wait0();
+      bulk_wait0();
       // a residual prefetch that was never consumed (aborted run) must land first
       if (MODE == kEpiResid && !ok && hin_loads > t)
         mbar_wait(&bar->hin_full, (uint32_t)(hin_loads - 1) & 1, err, kDevTimeoutEpi);

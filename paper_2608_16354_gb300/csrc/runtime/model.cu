@@ -313,6 +313,8 @@ dc_status enqueue_compute(dc_model* m, float* lat, const float* mod_k, const Slo
                                    map, a, st));
     dc::EpiArgs e1 = ep;
     e1.N = 3 * d; e1.bias = w.b_qkv; e1.out = qkv;
+    // q/k/v tiles go out by TMA through the attention's map when dh = 64 or 128
+    e1.qkv_tma = dc::attention_tc_supported(m->dh) ? 1 : 0;
     dc::EpiArgs e2 = ep;
     e2.N = d; e2.bias = w.b_o; e2.h = m->h; e2.h_in = h_in; e2.gate_off = base + 2 * d;
     dc::EpiArgs e3 = ep;
@@ -326,7 +328,7 @@ dc_status enqueue_compute(dc_model* m, float* lat, const float* mod_k, const Slo
                  b_2 = E * ((double)M * m->md + (double)m->md * d) + 8.0 * Md;
     if constexpr (sizeof(T) == 2) {
       DC_LAUNCH(DC_PROF_GEMM_QKV, f_qkv, b_qkv,
-                dc::launch_gemm_tc(dc::kEpiQKV, m->tm_a, w.tm_qkv, m->tm_a, m->tm_a, M, 3 * d, d,
+                dc::launch_gemm_tc(dc::kEpiQKV, m->tm_a, w.tm_qkv, m->tm_a, m->tm_qkv, M, 3 * d, d,
                                    e1, map, m->err_d, m->n_sms, st));
       if (dc::attention_tc_supported(m->dh)) {
         DC_LAUNCH(DC_PROF_ATTENTION, attn_flops, attn_bytes,
