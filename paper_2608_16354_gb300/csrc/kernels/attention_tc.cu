@@ -263,7 +263,8 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
     if (warp == 0) {
       // ------------------------------------------------------------ TMA
       // The whole warp runs the loop (warp-uniform decisions, taken by lane
-      // 0 and broadcast); one elected lane issues the copies.  K and V have
+      // 0 and broadcast).  Copies issued by one thread complete one after
+      // another, so K_j and V_j go out from lanes that rotate over 0-7.  K and V have
       // rings of their own: K_j is released as soon as every S_{t,j} is
       // issued, so later key tiles stream in while the PV products on V_j
       // are still pending.
@@ -288,7 +289,7 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
           int ready = 0;
           if (lane == 0) ready = mbar_test(&bar->k_empty[b], (u & 1) ^ 1);
           if (__shfl_sync(0xffffffffu, ready, 0)) {
-            if (elect_one()) {
+            if (lane == ((2 * nk) & 7)) {
               mbar_arrive_expect_tx(&bar->k_full[b], Cfg::kTileBytes);
               for (int a = 0; a < Cfg::kAtoms; ++a)
                 tma_load_2d(smem + Cfg::kOffK + b * Cfg::kTileBytes + a * 16384, &tm,
@@ -306,7 +307,7 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
           int ready = 0;
           if (lane == 0) ready = mbar_test(&bar->v_empty[b], (u & 1) ^ 1);
           if (__shfl_sync(0xffffffffu, ready, 0)) {
-            if (elect_one()) {
+            if (lane == ((2 * nv + 1) & 7)) {
               mbar_arrive_expect_tx(&bar->v_full[b], Cfg::kTileBytes);
               for (int a = 0; a < Cfg::kAtoms; ++a)
                 tma_load_2d(smem + Cfg::kOffV + b * Cfg::kTileBytes + a * 16384, &tm,

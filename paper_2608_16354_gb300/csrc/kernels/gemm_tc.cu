@@ -4,12 +4,17 @@
 //   weights, both K-major bf16), fp32 accumulation in TMEM, followed by one
 //   of the fused DiT epilogues (QKV scatter, GELU, gated residual).
 //
-// Design: persistent CTAs (one per SM), 128 x 192 output tiles, K in steps
-// of 64 (one 128-byte swizzle atom per row).  Warp 0 streams A/W tiles with
-// TMA into a shared-memory ring; warp 1 owns the TMEM allocation and one
-// elected lane issues tcgen05.mma (M=128, N=192, K=16) into one of two TMEM
-// accumulators; warps 2-9 drain the other accumulator with tcgen05.ld and run
-// the epilogue, so the epilogue of tile i overlaps the MMAs of tile i+1.
+// Design: persistent CTAs (one per SM) in clusters of two, 128 x 192 output
+// tiles, K in steps of 64 (one 128-byte swizzle atom per row).  The two CTAs
+// of a cluster work on vertically adjacent tiles with the same W columns:
+// each loads its own A tile and half of the W tile, multicast into both, so
+// every CTA pulls 28 KB instead of 40 KB per K step from L2 (the loads, not
+// the tensor core, bound these GEMMs).  Warp 0 streams the tiles with TMA
+// into a shared-memory ring whose stages are released by both CTAs' MMAs;
+// warp 1 owns the TMEM allocation and one elected lane issues tcgen05.mma
+// (M=128, N=192, K=16) into one of two TMEM accumulators; warps 2-9 drain the
+// other accumulator with tcgen05.ld and run the epilogue, so the epilogue of
+// tile i overlaps the MMAs of tile i+1.
 // N = 192 divides every projection width of the configured models (3d, d,
 // 4d for d = 384, 1152, 3072).
 //
@@ -70,7 +75,7 @@ struct __align__(8) Barriers {
 __device__ __forceinline__ int sw128_off(int r, int c) { return r * 128 + ((c ^ (r & 7)) << 4); }
 
 template <int MODE>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     gemm_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmA,
                         const __grid_constant__ CUtensorMap tmB,
                         const __grid_constant__ CUtensorMap tmCin,
@@ -92,15 +97,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int lane = threadIdx.x & 31;
   const int tiles_n = N / kBN;
   const int tiles_m = (M + kBM - 1) / kBM;
-  const int n_tiles = tiles_m * tiles_n;
   const int KB = K / kBK;
+  // pair tiles: (pair of m tiles, n tile); this CTA takes m tile 2 p + rank
+  const int rank = (int)cluster_rank();
+  const int n_pt = ((tiles_m + 1) / 2) * tiles_n;
+  const int pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
+  auto m0_of = [&](int pt) { return ((pt / tiles_n) * 2 + rank) * kBM; };
+  auto n0_of = [&](int pt) { return (pt % tiles_n) * kBN; };
 
   if (threadIdx.x == 0) {
     // read once, so that the whole CTA takes the same decision below
     bar->abort = *(volatile int*)err;
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&bar->full[s], 1);
-      mbar_init(&bar->empty[s], 1);
+      mbar_init(&bar->empty[s], 2);  // released by the MMAs of both CTAs
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bar->tmem_full[b], 1);
@@ -118,36 +128,42 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_alloc(&bar->tmem_base, kTmemCols);
     tmem_relinquish();
   }
+  // the peer's barriers are initialised before any multicast or remote arrive
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();
   tc_fence_after();
   const uint32_t tmem_base = bar->tmem_base;
+  // a bounded wait of an earlier launch gave up: do nothing (the host reports
+  // DC_ERR_DEVICE_TIMEOUT at its next check), but still meet the peer at the
+  // final cluster barrier
   if (bar->abort != 0) {
-    // a bounded wait of an earlier launch gave up: do nothing (the host
-    // reports DC_ERR_DEVICE_TIMEOUT at its next check)
-    if (warp == 1) tmem_dealloc(tmem_base, kTmemCols);
-    return;
-  }
-
-  if (warp == 0) {
+  } else if (warp == 0) {
     // -------------------------------------------------- TMA producer
-    // The whole warp runs the loop (uniform waits); one elected lane issues.
-    int stage = 0;
+    // The whole warp runs the loop (uniform waits).  Copies issued by one
+    // thread complete one after another (about one box per 300-400 cycles
+    // whatever its size), so the boxes of successive stages rotate over
+    // lanes 0-7: A from an even lane, the W half from the next odd one.
+    int stage = 0, issued = 0;
     uint32_t phase = 0;
     int last_phase[kStages];
     for (int s = 0; s < kStages; ++s) last_phase[s] = -1;
     bool ok = true;
-    for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
-      const int m0 = (tile / tiles_n) * kBM;
-      const int n0 = (tile % tiles_n) * kBN;
+    for (int pt = pair; pt < n_pt && ok; pt += n_pairs) {
+      const int m0 = m0_of(pt);
+      const int n0 = n0_of(pt);
       for (int kb = 0; kb < KB; ++kb) {
+        // the stage is free once both CTAs' MMAs have read it (the W half
+        // goes into both)
         if (!mbar_wait_warp(&bar->empty[stage], phase ^ 1, err, kDevTimeoutTma)) { ok = false; break; }
-        if (elect_one()) {
-          mbar_arrive_expect_tx(&bar->full[stage], kStageBytes);
-          tma_load_2d(sA + (size_t)stage * kABytes, &tmA, &bar->full[stage], kb * kBK, m0);
-          tma_load_2d(sB + (size_t)stage * kBBytes, &tmB, &bar->full[stage], kb * kBK, n0);
-        }
+        const int la = (2 * issued) & 7;
+        if (lane == la) mbar_arrive_expect_tx(&bar->full[stage], kStageBytes);
         __syncwarp();
+        if (lane == la) tma_load_2d(sA + (size_t)stage * kABytes, &tmA, &bar->full[stage], kb * kBK, m0);
+        if (lane == la + 1)
+          tma_load_2d_mc(sB + (size_t)stage * kBBytes + rank * (kBBytes / 2), &tmB, &bar->full[stage],
+                         kb * kBK, n0 + rank * (kBN / 2), (uint16_t)0x3);
+        __syncwarp();
+        ++issued;
         last_phase[stage] = (int)phase;
         if (++stage == kStages) { stage = 0; phase ^= 1; }
       }
@@ -168,7 +184,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // shared-memory addresses are below 256 KB)
     const uint64_t dA = sw128_kmajor_desc(smem_u32(sA));
     const uint64_t dB = sw128_kmajor_desc(smem_u32(sB));
-    for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++t) {
+    for (int pt = pair; pt < n_pt && ok; pt += n_pairs, ++t) {
       const int b = t & 1;
       const uint32_t use = (uint32_t)(t >> 1);
       if (!mbar_wait_warp(&bar->tmem_empty[b], (use & 1) ^ 1, err, kDevTimeoutMma)) { ok = false; break; }
@@ -184,7 +200,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                        dB + ((uint32_t)(stage * kBBytes + kk * 32) >> 4), kIdesc,
                        (kb | kk) != 0 ? 1u : 0u);
           }
-          tc_commit(&bar->empty[stage]);
+          tc_commit_mc(&bar->empty[stage], (uint16_t)0x3);  // release it in both CTAs
         }
         __syncwarp();
         if (++stage == kStages) { stage = 0; phase ^= 1; }
@@ -203,23 +219,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int q = warp & 3;             // TMEM lane quarter this warp may access
     const int half = (warp - 2) >> 2;   // which 96-column half of the tile
     const int et = threadIdx.x - 64;    // epilogue thread 0..255
-    const bool leader = et == 0;
+    const bool copy_warp = warp == 2;   // issues the tile's bulk copies, one box per lane
     const int r = q * 32 + lane;        // row of the tile owned by this thread
     int hin_loads = 0;                  // residual tiles requested so far
-    if (MODE == kEpiResid && leader && (int)blockIdx.x < n_tiles) {
-      const int tile = blockIdx.x;
-      mbar_arrive_expect_tx(&bar->hin_full, Cfg::kOutBytes);
-      for (int k = 0; k < 6; ++k)
-        tma_load_2d(sOut + k * 16384, &tmCin, &bar->hin_full, (tile % tiles_n) * kBN + 32 * k,
-                    (tile / tiles_n) * kBM);
+    if (MODE == kEpiResid && copy_warp && pair < n_pt) {
+      if (lane == 0) mbar_arrive_expect_tx(&bar->hin_full, Cfg::kOutBytes);
+      __syncwarp();
+      if (lane < 6)
+        tma_load_2d(sOut + lane * 16384, &tmCin, &bar->hin_full, n0_of(pair) + 32 * lane, m0_of(pair));
       hin_loads = 1;
     }
     // bias (and gate rows) of the next tile are loaded into registers while
     // the current tile is processed, and staged to shared memory at its start
     float nb = 0.f, nga = 0.f, ngb = 0.f;
-    auto fetch_vec = [&](int tile) {
-      if (tile < n_tiles && et < kBN) {
-        const int fm0 = (tile / tiles_n) * kBM, fn0 = (tile % tiles_n) * kBN;
+    auto fetch_vec = [&](int pt) {
+      if (pt < n_pt && et < kBN && m0_of(pt) < M) {
+        const int fm0 = m0_of(pt), fn0 = n0_of(pt);
         nb = ep.bias[fn0 + et];
         if (MODE == kEpiResid) {
           const int sa = fm0 / ep.n_tok, sb = (min(fm0 + kBM, M) - 1) / ep.n_tok;
@@ -228,17 +243,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     };
-    fetch_vec(blockIdx.x);
+    fetch_vec(pair);
     int t = 0;
     bool ok = true;
-    for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++t) {
+    for (int pt = pair; pt < n_pt && ok; pt += n_pairs, ++t) {
       const int b = t & 1;
       const uint32_t use = (uint32_t)(t >> 1);
       // every wait outcome is made uniform (warp, then the 8 epilogue warps at
       // the named barrier) so that an abort is taken by all of them together
       const bool acc_ok = mbar_wait_warp(&bar->tmem_full[b], use & 1, err, kDevTimeoutEpi);
-      const int m0 = (tile / tiles_n) * kBM;
-      const int n0 = (tile % tiles_n) * kBN;
+      const int m0 = m0_of(pt);
+      const int n0 = n0_of(pt);
+      // the second tile of the last pair may lie below M: it runs (its A rows
+      // are zero) but writes nothing
+      const bool live = m0 < M;
       float acc[3][32];
       if (acc_ok) {
         tc_fence_after();
@@ -256,7 +274,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
       // stage bias (and gate rows) of this tile once the previous tile is done
       if (named_bar_or(1, kEpiThreads, !acc_ok)) { ok = false; break; }
-      const int last_row = min(m0 + kBM, M) - 1;
+      const int last_row = live ? min(m0 + kBM, M) - 1 : m0;
       const int slot_a = m0 / ep.n_tok, slot_b = last_row / ep.n_tok;
       const int split = (slot_a + 1) * ep.n_tok;  // first row that belongs to slot_b
       if (et < kBN) {
@@ -266,8 +284,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           vec[2 * kBN + et] = ngb;
         }
       }
-      fetch_vec(tile + gridDim.x);
-      if (MODE != kEpiResid && leader) bulk_wait_read0();  // previous tile's stores have read sOut
+      fetch_vec(pt + n_pairs);
+      if (MODE != kEpiResid && copy_warp && lane < 3) bulk_wait_read0();  // previous stores read sOut
       named_bar(1, kEpiThreads);
 
       if constexpr (MODE == kEpiResid) {
@@ -306,16 +324,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         fence_proxy_async();
         if (named_bar_or(1, kEpiThreads, !hin_ok)) { ok = false; break; }
-        if (leader) {
-          for (int k = 0; k < 6; ++k) tma_store_2d(&tmCout, sOut + k * 16384, n0 + 32 * k, m0);
-          bulk_commit();
-          bulk_wait_read0();
-          const int next = tile + gridDim.x;
-          if (next < n_tiles) {
-            mbar_arrive_expect_tx(&bar->hin_full, Cfg::kOutBytes);
-            for (int k = 0; k < 6; ++k)
-              tma_load_2d(sOut + k * 16384, &tmCin, &bar->hin_full, (next % tiles_n) * kBN + 32 * k,
-                          (next / tiles_n) * kBM);
+        if (copy_warp) {
+          if (live && lane < 6) {
+            tma_store_2d(&tmCout, sOut + lane * 16384, n0 + 32 * lane, m0);
+            bulk_commit();
+            bulk_wait_read0();
+          }
+          __syncwarp();  // every box has been read out before the next tile lands
+          const int next = pt + n_pairs;
+          if (next < n_pt) {
+            if (lane == 0) mbar_arrive_expect_tx(&bar->hin_full, Cfg::kOutBytes);
+            __syncwarp();
+            if (lane < 6)
+              tma_load_2d(sOut + lane * 16384, &tmCin, &bar->hin_full, n0_of(next) + 32 * lane,
+                          m0_of(next));
             ++hin_loads;
           }
         }
@@ -342,11 +364,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         fence_proxy_async();
         named_bar(1, kEpiThreads);
-        if (leader) {
-          for (int k = 0; k < 3; ++k) tma_store_2d(&tmCout, sOut + k * 16384, n0 + 64 * k, m0);
+        if (copy_warp && live && lane < 3) {
+          tma_store_2d(&tmCout, sOut + lane * 16384, n0 + 64 * lane, m0);
           bulk_commit();
         }
-      } else if (ep.qkv_tma && m0 + kBM <= M && (m0 + kBM - 1) / ep.n_tok == slot_a) {
+      } else if (ep.qkv_tma && (!live || (m0 + kBM <= M && (m0 + kBM - 1) / ep.n_tok == slot_a))) {
         // QKV, tile inside one slot: each 64-column group is one head's
         // [128 tokens][64] block of q, k or v, contiguous in the head-major
         // layout; stage the bf16 tile swizzled and store it with TMA
@@ -364,17 +386,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         fence_proxy_async();
         named_bar(1, kEpiThreads);
-        if (leader) {
+        if (copy_warp && live && lane < 3) {
           const int tok0 = m0 - slot_a * ep.n_tok;
-          for (int k = 0; k < 3; ++k) {
-            const int col = n0 + 64 * k;
-            const int which = col / ep.d;
-            const int within = col - which * ep.d;
-            const int head = within / ep.dh;
-            const int e = within - head * ep.dh;
-            tma_store_2d(&tmCout, sOut + k * 16384, e,
-                         ((which * ep.nslots + slot_a) * ep.heads + head) * ep.n_tok + tok0);
-          }
+          const int col = n0 + 64 * lane;
+          const int which = col / ep.d;
+          const int within = col - which * ep.d;
+          const int head = within / ep.dh;
+          const int e = within - head * ep.dh;
+          tma_store_2d(&tmCout, sOut + lane * 16384, e,
+                       ((which * ep.nslots + slot_a) * ep.heads + head) * ep.n_tok + tok0);
           bulk_commit();
         }
       } else {
@@ -405,10 +425,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-    if (leader) {
-      bulk_wait0();
+    if (copy_warp) {
+      if (lane < 6) bulk_wait0();
       // a residual prefetch that was never consumed (aborted run) must land first
-      if (MODE == kEpiResid && !ok && hin_loads > t)
+      if (MODE == kEpiResid && lane == 0 && !ok && hin_loads > t)
         mbar_wait(&bar->hin_full, (uint32_t)(hin_loads - 1) & 1, err, kDevTimeoutEpi);
     }
   }
@@ -419,6 +439,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem_base, kTmemCols);
   }
+  // no CTA leaves while its peer may still multicast into it or arrive on
+  // its barriers
+  cluster_sync();
 }
 
 template <int MODE>
@@ -433,8 +456,9 @@ cudaError_t launch_mode(const CUtensorMap& tmA, const CUtensorMap& tmB, const CU
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  const int tiles = ((M + kBM - 1) / kBM) * (N / kBN);
-  const int grid = tiles < n_sms ? tiles : n_sms;
+  // clusters of two CTAs over pairs of m tiles (the grid is even)
+  const int pair_tiles = ((M + kBM - 1) / kBM + 1) / 2 * (N / kBN);
+  const int grid = 2 * (pair_tiles < n_sms / 2 ? pair_tiles : n_sms / 2);
   gemm_bf16_tc_kernel<MODE><<<grid, kThreads, Cfg::kSmem, st>>>(tmA, tmB, tmCin, tmCout, M, N, K,
                                                                 ep, map, err);
   return cudaGetLastError();
@@ -460,6 +484,7 @@ cudaError_t launch_gemm_tc(int mode, const CUtensorMap& tmA, const CUtensorMap& 
 }
 
 int gemm_tc_tile_n() { return kBN; }
+int gemm_tc_w_box_rows() { return kBN / 2; }
 int gemm_tc_tile_k() { return kBK; }
 int gemm_tc_tile_m() { return kBM; }
 

@@ -43,6 +43,7 @@ cudaError_t launch_gemm_f32(int mode, const float* A, const float* W, int M, int
                             const EpiArgs& ep, const SlotMap& map, cudaStream_t st);
 size_t gemm_tc_smem_bytes();
 int gemm_tc_tile_n();
+int gemm_tc_w_box_rows();  // rows of the W box: each CTA of a cluster loads half the tile
 int gemm_tc_tile_k();
 int gemm_tc_tile_m();
 // attention: q/k/v [3][slots][heads][N][dhp] -> o [slots][N][heads*dh]

@@ -804,7 +804,7 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
     return fail(DC_ERR_NOMEM);
   }
   if (m->bf16) {
-    const uint32_t bn = (uint32_t)dc::gemm_tc_tile_n(), bm = (uint32_t)dc::gemm_tc_tile_m();
+    const uint32_t bn = (uint32_t)dc::gemm_tc_w_box_rows(), bm = (uint32_t)dc::gemm_tc_tile_m();
     dc_status s;
     if ((s = make_map(&m->tm_a, m->a, d, B * N, bm)) != DC_OK) return fail(s);
     if ((s = make_map(&m->tm_oact, m->o, d, B * N, bm)) != DC_OK) return fail(s);
