@@ -54,13 +54,20 @@ def calibrate(model, wl, calib_poses, noise, sig, q0, q1, target, eps=P.EPS):
 
 
 def denoise(model, x1, trajs, sig, anc, tables, tau, K, H, veto=True, forced=None,
-            eps=P.EPS, keep_trace=False):
+            eps=P.EPS, keep_trace=False, variant=P.DRIVECACHE):
     """Run the sampler over B scenes with the causal controller.
 
     forced: optional [B][K+1] actions to replay verbatim (no planning, no
-    checks).  Returns dict(x, plans, executed, log, stats, trace)."""
+    checks).  variant: a planner variant of oracle.planner (Table 3
+    ablations, fixed-interval baseline); SHUFFLED plans scene s from the
+    trajectory of scene (s+1) mod B, FIXED_INTERVAL runs its schedule with no
+    charge and no checks, and refusals under FIXED_PLACEMENT keep the fixed
+    pattern (no replan).  Returns dict(x, plans, executed, log, stats, trace)."""
     B = len(trajs)
-    plans = [P.plan_scene(trajs[s], anc, tables, tau, K, H, eps) for s in range(B)]
+    plan_traj = [trajs[(s + 1) % B] if variant == P.SHUFFLED else trajs[s] for s in range(B)]
+    plans = [P.plan_scene_variant(plan_traj[s], anc, tables, tau, K, H, variant, eps)
+             for s in range(B)]
+    fixed = variant == P.FIXED_INTERVAL
     acts = [list(p["actions"]) for p in plans]
     if forced is not None:
         acts = [[0] + [int(forced[s][k]) for k in range(1, K + 1)] for s in range(B)]
@@ -78,9 +85,9 @@ def denoise(model, x1, trajs, sig, anc, tables, tau, K, H, veto=True, forced=Non
             S = st[s]
             reuse = False
             if k > 1 and acts[s][k] == P.REUSE:
-                if forced is not None or not veto:
+                if forced is not None or not veto or fixed:
                     reuse = True
-                    if forced is None:
+                    if forced is None and not fixed:
                         tabs = plans[s]["tabs"]
                         S["C"] = S["C"] + tabs["c"][S["j"]][S["age"] + 1]
                 else:
@@ -99,10 +106,11 @@ def denoise(model, x1, trajs, sig, anc, tables, tau, K, H, veto=True, forced=Non
                         S["C"] = S["C"] + c_inc
                     else:
                         stats[s]["n_veto"] += 1
-                        stats[s]["n_replan"] += 1
-                        a, _, _ = P.plan_suffix(tabs["c"], K, H, k, tau - S["C"])
-                        for kk in range(k, K + 1):
-                            acts[s][kk] = a[kk]
+                        if variant != P.FIXED_PLACEMENT:
+                            stats[s]["n_replan"] += 1
+                            a, _, _ = P.plan_suffix(tabs["c"], K, H, k, tau - S["C"])
+                            for kk in range(k, K + 1):
+                                acts[s][kk] = a[kk]
             if reuse:
                 v, _ = model.reuse_step(x[s], S["r"], sig[k - 1], trajs[s])
                 S["age"] += 1

@@ -18,6 +18,9 @@ Sections followed:
   Eq. 10  DP transitions, Eq. 11 maximal reuse count, backtracking (Sec. 3.2)
   Sec. 3.2 budget calibration tau(rho_tar)
   Eq. 12 / Sec. 3.2 causal acceptance test and suffix replanning
+  Table 3 ablations (no motion prior, shuffled trajectory, translation only,
+          rotation only, fixed placement) and the fixed-interval baseline of
+          Table 1, as planner variants
 """
 
 import math
@@ -350,3 +353,135 @@ def accept_reuse(d_obs, dbar, c_inc, charge, tau, eps=EPS):
     """Sec. 3.2: accept the h-th reuse of the run from j only when
     d_obs <= d_bar_{j,h} + eps and C_k + c_hat_{j,h} <= tau."""
     return d_obs <= dbar + eps and charge + c_inc <= tau
+
+
+# ------------------------------------- Table 3 ablations, Table 1 baseline
+#
+# The paper names these variants without defining them; the READINGS below
+# are the ones the library implements (variant ids match include/drivecache.h).
+
+DRIVECACHE = 0         # the method as published
+NO_MOTION_PRIOR = 1    # READING: every scene is planned at D = 1/2, no support gate
+SHUFFLED = 2           # READING: scene s is planned from the trajectory of scene (s+1) mod B
+TRANSLATION_ONLY = 3   # READING: D = z^L, supported iff 0 <= z^L <= 1
+ROTATION_ONLY = 4      # READING: D = z^Theta, supported iff 0 <= z^Theta <= 1
+FIXED_PLACEMENT = 5    # READING: B* of the method, spread evenly (no DP placement), no replan
+FIXED_INTERVAL = 6     # READING: `budget` reuses spread evenly for every scene; no charge, no veto
+
+
+def variant_intensity(L, T, anc, variant, eps=EPS):
+    """(supported, D) of a scene under a planner variant (Eq. 3-4 for the
+    method itself)."""
+    if not anc["valid"]:
+        return 0, 0.0
+    if variant == NO_MOTION_PRIOR:
+        return 1, 0.5
+    zL, zT = normalize(L, T, anc, eps)
+    if variant == TRANSLATION_ONLY:
+        return (1, zL) if 0.0 <= zL <= 1.0 else (0, 0.0)
+    if variant == ROTATION_ONLY:
+        return (1, zT) if 0.0 <= zT <= 1.0 else (0, 0.0)
+    if not is_supported(zL, zT):
+        return 0, 0.0
+    return 1, intensity(zL, zT)
+
+
+def even_schedule(n, K, H, legal=None):
+    """READING of fixed placement and of the fixed-interval baseline: n reuses
+    spread evenly over steps 2..K -- step k is a reuse iff
+    floor((k-1) n / (K-1)) > floor((k-2) n / (K-1)) -- except that a reuse
+    whose cache age would be illegal (L(k, h), default 1 <= h <= H_max) is a
+    full evaluation instead.  Returns the action list (index 0 unused)."""
+    leg = legal or (lambda k, h: default_legal(k, h, H))
+    acts = [0] * (K + 1)
+    acts[1] = COMPUTE
+    age = 0
+    for k in range(2, K + 1):
+        want = K > 1 and (k - 1) * n // (K - 1) > (k - 2) * n // (K - 1)
+        if want and leg(k, age + 1):
+            acts[k] = REUSE
+            age += 1
+        else:
+            acts[k] = COMPUTE
+            age = 0
+    return acts
+
+
+def schedule_cost(acts, c, K):
+    """Sum of c_hat_{j,h} over the reuses of a schedule (j = last full
+    evaluation, h = age), in step order."""
+    total = 0.0
+    j, age = 1, 0
+    for k in range(2, K + 1):
+        if acts[k] == REUSE:
+            age += 1
+            total = total + c[j][age]
+        else:
+            j, age = k, 0
+    return total
+
+
+def plan_scene_variant(poses, anc, tables, budget, K, H, variant, eps=EPS, legal=None):
+    """dc_plan under a planner variant.  `budget` is tau, except for
+    FIXED_INTERVAL where it is the number of reuses."""
+    if variant == FIXED_INTERVAL:
+        L, T = motion_stats(poses)
+        acts = even_schedule(int(budget), K, H, legal)
+        n = sum(1 for k in range(2, K + 1) if acts[k] == REUSE)
+        return dict(actions=acts, n_reuse=n, cost=0.0, supported=1, D=0.0, L=L, T=T, tabs=None)
+    if variant in (DRIVECACHE, SHUFFLED, FIXED_PLACEMENT):
+        res = plan_scene(poses, anc, tables, budget, K, H, eps, legal)
+        if variant == FIXED_PLACEMENT and res["supported"]:
+            acts = even_schedule(res["n_reuse"], K, H, legal)
+            res["actions"] = acts
+            res["n_reuse"] = sum(1 for k in range(2, K + 1) if acts[k] == REUSE)
+            res["cost"] = schedule_cost(acts, res["tabs"]["c"], K)
+        return res
+    L, T = motion_stats(poses)
+    acts = [0] + [COMPUTE] * K
+    res = dict(actions=acts, n_reuse=0, cost=0.0, supported=0, D=0.0, L=L, T=T, tabs=None)
+    sup, D = variant_intensity(L, T, anc, variant, eps)
+    if not sup:
+        return res
+    tabs = scene_tables(tables, D, K, H)
+    a, n, cost = plan_suffix(tabs["c"], K, H, 1, budget, legal)
+    for k in range(1, K + 1):
+        acts[k] = a[k]
+    res.update(n_reuse=n, cost=cost, supported=1, D=D, tabs=tabs)
+    return res
+
+
+def calibrate_budget_variant(clip_poses, anc, tables, target, K, H, variant, eps=EPS, legal=None):
+    """Sec. 3.2 calibration under a planner variant: the motion variants use
+    their own intensity; FIXED_PLACEMENT keeps the method's tau (it changes
+    placement, not count); FIXED_INTERVAL returns the reuse count itself
+    (reached iff the even schedule holds `target` reuses)."""
+    if variant == FIXED_INTERVAL:
+        acts = even_schedule(target, K, H, legal)
+        n = sum(1 for k in range(2, K + 1) if acts[k] == REUSE)
+        return float(target), 1 if n >= target else 0
+    if variant in (DRIVECACHE, SHUFFLED, FIXED_PLACEMENT):
+        return calibrate_budget(clip_poses, anc, tables, target, K, H, eps, legal)
+    curves = []
+    cands = set()
+    for poses in clip_poses:
+        L, T = motion_stats(poses)
+        sup, D = variant_intensity(L, T, anc, variant, eps)
+        if not sup:
+            curves.append(None)
+            continue
+        tabs = scene_tables(tables, D, K, H)
+        J, _ = dp_tables(tabs["c"], K, H, 1, legal)
+        m = cost_curve(J, K, H)
+        curves.append(m)
+        for v in m:
+            if v < INF:
+                cands.add(v)
+    if not cands:
+        return 0.0, 0
+    ordered = sorted(cands)
+    for tau in ordered:
+        counts = [0 if m is None else best_count(m, tau) for m in curves]
+        if _median([float(x) for x in counts]) >= target:
+            return tau, 1
+    return ordered[-1], 0
