@@ -51,6 +51,36 @@ typedef struct { double x, y, psi; } dc_pose;
 /* A planned trajectory: n_poses consecutive poses (host memory). */
 typedef struct { const dc_pose* poses; int n_poses; } dc_trajectory;
 
+/* Planner variants: the method itself, the ablations of Table 3 and the
+ * fixed-interval baseline of Table 1 (Sec. 4).  The paper names them without
+ * formulas; the readings implemented are:
+ *  DC_VAR_DRIVECACHE        the method as published (Sec. 3.1-3.2);
+ *  DC_VAR_NO_MOTION_PRIOR   every scene planned at D = 1/2, no support gate;
+ *  DC_VAR_SHUFFLED          dc_denoise plans scene s from the trajectory of
+ *                           scene (s+1) mod B (the backbone still sees its
+ *                           own); dc_plan plans the trajectory it is given;
+ *  DC_VAR_TRANSLATION_ONLY  D = z^L, supported iff 0 <= z^L <= 1;
+ *  DC_VAR_ROTATION_ONLY     D = z^Theta, supported iff 0 <= z^Theta <= 1;
+ *  DC_VAR_FIXED_PLACEMENT   the method's B* reuses spread evenly over steps
+ *                           2..T (below) instead of the DP placement; a
+ *                           refused reuse is computed and the pattern kept;
+ *  DC_VAR_FIXED_INTERVAL    `budget` (an integer) reuses spread evenly for
+ *                           every scene, whatever its motion or support; no
+ *                           charge and no drift check.
+ * Even spreading: step k (2 <= k <= T) is a reuse iff
+ * floor((k-1) n / (T-1)) > floor((k-2) n / (T-1)), except that a reuse whose
+ * cache age would be illegal (the mask below, or h > H_max) is a full
+ * evaluation instead. */
+enum {
+  DC_VAR_DRIVECACHE = 0,
+  DC_VAR_NO_MOTION_PRIOR = 1,
+  DC_VAR_SHUFFLED = 2,
+  DC_VAR_TRANSLATION_ONLY = 3,
+  DC_VAR_ROTATION_ONLY = 4,
+  DC_VAR_FIXED_PLACEMENT = 5,
+  DC_VAR_FIXED_INTERVAL = 6
+};
+
 /* Calibrated anchor responses (Sec. 3.1-3.2).
  *  (L0,T0), (L1,T1): low-motion and moving-turn anchor statistics (Eq. 2);
  *  valid = 0 means no moving-turn anchor exists -> every scene runs full
@@ -60,7 +90,8 @@ typedef struct { const dc_pose* poses; int n_poses; } dc_trajectory;
  *  legal: optional [K+1][H_max+1] bytes, legal[k][h] != 0 iff reusing at
  *  step k with cache age h is allowed (the L(k,h) mask of Eq. 10); NULL means
  *  every age 1..H_max at every step k >= 2.  eps: the epsilon of Eq. 3 and of
- *  the veto slack (1e-6 by default). */
+ *  the veto slack (1e-6 by default).  variant: a DC_VAR_* planner variant
+ *  (0 = the method). */
 typedef struct {
   int K, H_max;
   double L0, T0, L1, T1;
@@ -68,6 +99,7 @@ typedef struct {
   const double *q0, *q1, *d0, *d1;
   const unsigned char* legal;
   double eps;
+  int variant;
 } dc_anchor_responses;
 
 /* A per-scene schedule.  action: caller-owned [T+1] bytes (index 0 unused). */
@@ -99,7 +131,10 @@ dc_status dc_select_anchors(const double* L, const double* Theta, int n,
  * Eq. 8/9 scene tables -> Eq. 10 DP from J_1(0,0) = 0 -> Eq. 11 B* under
  * `budget` (tau) -> backtracking (ties: smallest final age, then smallest
  * age before each refresh).  T must equal anc->K; out->action must hold T+1
- * bytes.  An unsupported scene gets an all-COMPUTE schedule. */
+ * bytes.  An unsupported scene gets an all-COMPUTE schedule.  Under
+ * anc->variant the intensity and placement follow the variant (see DC_VAR_*);
+ * for DC_VAR_FIXED_INTERVAL `budget` is the reuse count, an integer in
+ * [0, T-1], and cost is 0. */
 dc_status dc_plan(const dc_trajectory* traj, const dc_anchor_responses* anc, double budget,
                   int T, dc_schedule* out);
 
@@ -108,7 +143,9 @@ dc_status dc_plan(const dc_trajectory* traj, const dc_anchor_responses* anc, dou
  * `remaining` (= tau - C_k) with the scene tables of intensity D.  Overwrites
  * inout->action[k_refresh..T] (action[k_refresh] = COMPUTE) and leaves the
  * prefix untouched; sets inout->n_reuse to the REUSE count of the whole
- * action array and inout->cost to the suffix plan's cost. */
+ * action array and inout->cost to the suffix plan's cost.  The fixed
+ * variants (DC_VAR_FIXED_PLACEMENT, DC_VAR_FIXED_INTERVAL) never replan: the
+ * actions are left as they are and cost is set to 0. */
 dc_status dc_replan(const dc_anchor_responses* anc, double D, int k_refresh, double remaining,
                     dc_schedule* inout);
 
@@ -117,7 +154,11 @@ dc_status dc_replan(const dc_anchor_responses* anc, double D, int k_refresh, dou
  * pass target = ceil(rho_tar (T-1))).  Candidates are the finite
  * min_h J_T(n, h) of every supported clip; unsupported clips count as zero
  * reuses.  *reached = 0 if no candidate reaches the target, in which case
- * *tau is the largest candidate. */
+ * *tau is the largest candidate.  The motion variants calibrate on their own
+ * intensities; DC_VAR_SHUFFLED and DC_VAR_FIXED_PLACEMENT give the method's
+ * tau (they change which trajectory or which steps, not the count);
+ * DC_VAR_FIXED_INTERVAL returns *tau = target (its reuse count), reached iff
+ * the even schedule holds `target` reuses. */
 dc_status dc_calibrate_budget(const dc_trajectory* clips, int n, const dc_anchor_responses* anc,
                               int target, int T, double* tau, int* reached);
 
@@ -159,7 +200,10 @@ typedef struct { int B; const dc_trajectory* traj; } dc_cond;
  *  sigmas: [K+1] host doubles, sigma_1 .. sigma_{K+1} stored 0-based.
  *  anchors: calibrated responses (anchors->K must equal K); tau: budget.
  *  veto: 1 = check drift and charge before every planned reuse (Eq. 12);
- *        0 = execute the plan as made.
+ *        0 = execute the plan as made (the no-veto ablation of Table 3).
+ *  The planner variant is anchors->variant (DC_VAR_*).  The reduced-steps
+ *  baseline of Table 2 is a plain call with fewer steps (K and sigmas of the
+ *  shorter schedule) and a forced all-COMPUTE schedule.
  *  forced: NULL, or [B][K+1] actions replayed verbatim (no planning, no
  *        checks; step 1 is always computed). */
 typedef struct {

@@ -15,6 +15,9 @@ _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libdrivecache.so")
 
 COMPUTE, REUSE = 1, 2
+# planner variants (DC_VAR_* in include/drivecache.h)
+(VAR_DRIVECACHE, VAR_NO_MOTION_PRIOR, VAR_SHUFFLED, VAR_TRANSLATION_ONLY, VAR_ROTATION_ONLY,
+ VAR_FIXED_PLACEMENT, VAR_FIXED_INTERVAL) = range(7)
 DTYPE_F32, DTYPE_BF16 = 0, 1
 
 STATUS = {0: "DC_OK", 1: "DC_ERR_INVALID_ARG", 2: "DC_ERR_NOMEM", 3: "DC_ERR_CUDA",
@@ -41,7 +44,7 @@ class AnchorResponses(C.Structure):
                 ("valid", C.c_int),
                 ("q0", C.POINTER(C.c_double)), ("q1", C.POINTER(C.c_double)),
                 ("d0", C.POINTER(C.c_double)), ("d1", C.POINTER(C.c_double)),
-                ("legal", C.POINTER(C.c_ubyte)), ("eps", C.c_double)]
+                ("legal", C.POINTER(C.c_ubyte)), ("eps", C.c_double), ("variant", C.c_int)]
 
 
 class Schedule(C.Structure):
@@ -163,7 +166,7 @@ class AnchorArgs:
     """dc_anchor_responses built from Python tables ([K][H+1] nested lists or
     arrays) and anchor statistics."""
 
-    def __init__(self, K, H, anc, tables, legal=None, eps=1e-6):
+    def __init__(self, K, H, anc, tables, legal=None, eps=1e-6, variant=VAR_DRIVECACHE):
         def tab(t):
             if t is None:
                 return np.zeros((K, H + 1), np.float64)
@@ -180,6 +183,7 @@ class AnchorArgs:
         s.q0, s.q1, s.d0, s.d1 = _dptr(self.q0), _dptr(self.q1), _dptr(self.d0), _dptr(self.d1)
         s.legal = _bptr(self.legal) if self.legal is not None else None
         s.eps = eps
+        s.variant = int(variant)
         self.s = s
 
     def ptr(self):

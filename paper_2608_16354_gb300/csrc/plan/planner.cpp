@@ -121,10 +121,86 @@ void motion_stats(const dc_pose* p, int n, double* L, double* T) {
 int scene_intensity(double L, double T, const dc_anchor_responses& a, double* D) {
   *D = 0.0;
   if (!a.valid) return 0;
+  if (a.variant == DC_VAR_NO_MOTION_PRIOR) {  // no motion prior: one intensity for all
+    *D = 0.5;
+    return 1;
+  }
   double zL = (L - a.L0) / std::max(a.L1 - a.L0, a.eps);
   double zT = (T - a.T0) / std::max(a.T1 - a.T0, a.eps);
+  if (a.variant == DC_VAR_TRANSLATION_ONLY) {
+    if (!(0.0 <= zL && zL <= 1.0)) return 0;
+    *D = zL;
+    return 1;
+  }
+  if (a.variant == DC_VAR_ROTATION_ONLY) {
+    if (!(0.0 <= zT && zT <= 1.0)) return 0;
+    *D = zT;
+    return 1;
+  }
   if (!(0.0 <= zL && zL <= 1.0 && 0.0 <= zT && zT <= 1.0)) return 0;
-  *D = std::sqrt(zL * zL + zT * zT) / std::sqrt(2.0);
+  *D = std::sqrt(zL * zL + zT * zT) / std::sqrt(2.0);  // Eq. 4
+  return 1;
+}
+
+void even_schedule(int n, int T, int H, const unsigned char* legal, unsigned char* acts) {
+  acts[1] = kCompute;
+  int age = 0;
+  for (int k = 2; k <= T; ++k) {
+    const bool want =
+        T > 1 && (long long)(k - 1) * n / (T - 1) > (long long)(k - 2) * n / (T - 1);
+    if (want && legal_at(legal, H, k, age + 1)) {
+      acts[k] = kReuse;
+      ++age;
+    } else {
+      acts[k] = kCompute;
+      age = 0;
+    }
+  }
+}
+
+namespace {
+// Sum of c_hat_{j,h} over the reuses of a schedule, in step order.
+double schedule_cost(const unsigned char* acts, const SceneTables& t) {
+  double total = 0.0;
+  int j = 1, age = 0;
+  for (int k = 2; k <= t.K; ++k) {
+    if (acts[k] == kReuse) {
+      ++age;
+      total = total + t.at_c(j, age);
+    } else {
+      j = k;
+      age = 0;
+    }
+  }
+  return total;
+}
+int count_reuse(const unsigned char* acts, int T) {
+  int n = 0;
+  for (int k = 1; k <= T; ++k) n += acts[k] == kReuse;
+  return n;
+}
+}  // namespace
+
+int plan_scene(double L, double Th, const dc_anchor_responses& a, double budget,
+               unsigned char* acts, int* n_reuse, double* cost, double* D, SceneTables* tabs) {
+  const int T = a.K;
+  for (int k = 1; k <= T; ++k) acts[k] = kCompute;
+  *n_reuse = 0;
+  *cost = 0.0;
+  *D = 0.0;
+  if (a.variant == DC_VAR_FIXED_INTERVAL) {  // no motion, no budget: a fixed pattern
+    even_schedule((int)budget, T, a.H_max, a.legal, acts);
+    *n_reuse = count_reuse(acts, T);
+    return 1;
+  }
+  if (!scene_intensity(L, Th, a, D)) return 0;
+  scene_tables(a, *D, tabs);
+  *n_reuse = plan_suffix(*tabs, a.legal, 1, budget, acts, cost);
+  if (a.variant == DC_VAR_FIXED_PLACEMENT) {  // the DP's count, evenly placed
+    even_schedule(*n_reuse, T, a.H_max, a.legal, acts);
+    *n_reuse = count_reuse(acts, T);
+    *cost = schedule_cost(acts, *tabs);
+  }
   return 1;
 }
 
@@ -194,6 +270,15 @@ void cost_curve(const SceneTables& t, const unsigned char* legal, std::vector<do
     for (int h = 0; h <= t.H; ++h) (*m)[n] = std::min((*m)[n], r.Jfin[(size_t)n * W + h]);
 }
 
+dc_status check_reuse_count(const dc_anchor_responses& a, double budget) {
+  if (a.variant != DC_VAR_FIXED_INTERVAL) return DC_OK;
+  if (!(budget >= 0.0 && budget <= a.K - 1) || budget != std::floor(budget)) {
+    set_error("fixed-interval variant: the budget is the reuse count, an integer in [0, K-1]");
+    return DC_ERR_INVALID_ARG;
+  }
+  return DC_OK;
+}
+
 dc_status check_anchors(const dc_anchor_responses* a) {
   if (!a) { set_error("anchors is NULL"); return DC_ERR_INVALID_ARG; }
   if (a->K < 1 || a->K > 100000 || a->H_max < 1 || a->H_max > 4096) {
@@ -202,6 +287,10 @@ dc_status check_anchors(const dc_anchor_responses* a) {
   }
   if (!(a->eps > 0.0) || !std::isfinite(a->eps)) {
     set_error("anchors: eps must be finite and > 0");
+    return DC_ERR_INVALID_ARG;
+  }
+  if (a->variant < DC_VAR_DRIVECACHE || a->variant > DC_VAR_FIXED_INTERVAL) {
+    set_error("anchors: variant must be one of DC_VAR_*");
     return DC_ERR_INVALID_ARG;
   }
   if (!a->valid) return DC_OK;
@@ -312,20 +401,16 @@ dc_status dc_plan(const dc_trajectory* traj, const dc_anchor_responses* anc, dou
     dc::set_error("dc_plan: out/action NULL, T != anchors.K, out->T != T, or NaN budget");
     return DC_ERR_INVALID_ARG;
   }
+  if ((s = dc::check_reuse_count(*anc, budget)) != DC_OK) return s;
   double L, Th, D;
   dc::motion_stats(traj->poses, traj->n_poses, &L, &Th);
   out->L = L;
   out->Theta = Th;
   out->action[0] = 0;
-  for (int k = 1; k <= T; ++k) out->action[k] = dc::kCompute;
-  out->n_reuse = 0;
-  out->cost = 0.0;
-  out->supported = dc::scene_intensity(L, Th, *anc, &D);
-  out->D = D;
-  if (!out->supported) return DC_OK;
   dc::SceneTables t;
-  dc::scene_tables(*anc, D, &t);
-  out->n_reuse = dc::plan_suffix(t, anc->legal, 1, budget, out->action, &out->cost);
+  out->supported = dc::plan_scene(L, Th, *anc, budget, out->action, &out->n_reuse, &out->cost,
+                                  &D, &t);
+  out->D = D;
   return DC_OK;
 }
 
@@ -337,6 +422,14 @@ dc_status dc_replan(const dc_anchor_responses* anc, double D, int k_refresh, dou
       !(D >= 0.0 && D <= 1.0) || std::isnan(remaining)) {
     dc::set_error("dc_replan: bad schedule, k_refresh outside 1..K, D outside [0,1] or NaN budget");
     return DC_ERR_INVALID_ARG;
+  }
+  if (anc->variant == DC_VAR_FIXED_PLACEMENT || anc->variant == DC_VAR_FIXED_INTERVAL) {
+    // the fixed variants keep their pattern
+    int n = 0;
+    for (int k = 1; k <= inout->T; ++k) n += inout->action[k] == dc::kReuse;
+    inout->n_reuse = n;
+    inout->cost = 0.0;
+    return DC_OK;
   }
   if (!anc->valid) {
     dc::set_error("dc_replan: anchors are invalid (full inference, nothing to replan)");
@@ -361,6 +454,20 @@ dc_status dc_calibrate_budget(const dc_trajectory* clips, int n, const dc_anchor
   }
   for (int i = 0; i < n; ++i)
     if ((s = check_traj(&clips[i])) != DC_OK) return s;
+  if (anc->variant == DC_VAR_FIXED_INTERVAL) {
+    // the reuse count is the budget itself
+    if (target > T - 1) {
+      dc::set_error("dc_calibrate_budget: fixed-interval target must be in [0, T-1]");
+      return DC_ERR_INVALID_ARG;
+    }
+    std::vector<unsigned char> acts((size_t)T + 1, 0);
+    dc::even_schedule(target, T, anc->H_max, anc->legal, acts.data());
+    int got = 0;
+    for (int k = 1; k <= T; ++k) got += acts[k] == dc::kReuse;
+    *tau = (double)target;
+    if (reached) *reached = got >= target ? 1 : 0;
+    return DC_OK;
+  }
   std::vector<std::vector<double>> curves(n);
   std::vector<char> has(n, 0);
   std::set<double> cands;

@@ -37,6 +37,19 @@ int plan_suffix(const SceneTables& t, const unsigned char* legal, int k0, double
 // Cost curve m(n) = min_h J_K(n, h) from k0 = 1 (INF where infeasible).
 void cost_curve(const SceneTables& t, const unsigned char* legal, std::vector<double>* m);
 
+// The fixed variants' schedule: n reuses spread evenly over steps 2..T,
+// an illegal age turning the reuse into a full evaluation.  acts[1..T].
+void even_schedule(int n, int T, int H, const unsigned char* legal, unsigned char* acts);
+
+// One scene's initial plan under anchors.variant (dc_plan and the sampler):
+// fills acts[1..K], *n_reuse, *cost and *D, and *tabs when the variant uses
+// scene tables; returns 1 when the scene is planned (supported).
+int plan_scene(double L, double Th, const dc_anchor_responses& a, double budget,
+               unsigned char* acts, int* n_reuse, double* cost, double* D, SceneTables* tabs);
+
 dc_status check_anchors(const dc_anchor_responses* a);
+
+// DC_VAR_FIXED_INTERVAL: the budget is a reuse count, an integer in [0, K-1].
+dc_status check_reuse_count(const dc_anchor_responses& a, double budget);
 
 }  // namespace dc

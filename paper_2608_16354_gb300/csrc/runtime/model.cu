@@ -446,15 +446,16 @@ dc_status run_sampler(dc_model* m, float* lat, const dc_cond* cond, const dc_sch
       a[1] = dc::kCompute;
       continue;
     }
-    double L, Th, D;
-    dc::motion_stats(cond->traj[s].poses, cond->traj[s].n_poses, &L, &Th);
-    supported[s] = dc::scene_intensity(L, Th, *anc, &D);
+    // the shuffled-trajectory ablation plans scene s from scene s+1's poses
+    const dc_trajectory& pt = cond->traj[anc->variant == DC_VAR_SHUFFLED ? (s + 1) % B : s];
+    double L, Th, D, cost;
+    int n_reuse;
+    dc::motion_stats(pt.poses, pt.n_poses, &L, &Th);
+    supported[s] = dc::plan_scene(L, Th, *anc, sc->tau, a, &n_reuse, &cost, &D, &tabs[s]);
     Dv[s] = D;
-    if (!supported[s]) continue;
-    dc::scene_tables(*anc, D, &tabs[s]);
-    double cost;
-    dc::plan_suffix(tabs[s], anc->legal, 1, sc->tau, a, &cost);
   }
+  // the fixed-interval baseline runs its pattern with no charge and no checks
+  const bool unchecked = !forced && anc->variant == DC_VAR_FIXED_INTERVAL;
   if (stats) {
     if (stats->planned) std::memcpy(stats->planned, acts.data(), acts.size());
     for (int s = 0; s < B; ++s) {
@@ -502,9 +503,9 @@ dc_status run_sampler(dc_model* m, float* lat, const dc_cond* cond, const dc_sch
     for (int s = 0; s < B; ++s) {
       reuse_now[s] = 0;
       if (k == 1 || acts[(size_t)s * W + k] != dc::kReuse) continue;
-      if (forced || !sc->veto) {
+      if (forced || !sc->veto || unchecked) {
         reuse_now[s] = 1;
-        if (!forced) state[s].C = state[s].C + tabs[s].at_c(state[s].j, state[s].age + 1);
+        if (!forced && !unchecked) state[s].C = state[s].C + tabs[s].at_c(state[s].j, state[s].age + 1);
       } else {
         chk.push_back(s);
       }
@@ -544,9 +545,11 @@ dc_status run_sampler(dc_model* m, float* lat, const dc_cond* cond, const dc_sch
           S.C = S.C + c;
         } else {
           if (stats && stats->n_veto) stats->n_veto[s]++;
-          if (stats && stats->n_replan) stats->n_replan[s]++;
-          double cost;
-          dc::plan_suffix(tabs[s], anc->legal, k, sc->tau - S.C, &acts[(size_t)s * W], &cost);
+          if (anc->variant != DC_VAR_FIXED_PLACEMENT) {  // the fixed pattern is kept
+            if (stats && stats->n_replan) stats->n_replan[s]++;
+            double cost;
+            dc::plan_suffix(tabs[s], anc->legal, k, sc->tau - S.C, &acts[(size_t)s * W], &cost);
+          }
         }
       }
     }
@@ -625,6 +628,7 @@ dc_status check_call(dc_model* m, const dc_cond* cond, const dc_sched* sc) {
       dc::set_error("anchors->K must equal sched->K and tau must not be NaN");
       return DC_ERR_INVALID_ARG;
     }
+    if ((s = dc::check_reuse_count(*sc->anchors, sc->tau)) != DC_OK) return s;
   }
   return DC_OK;
 }

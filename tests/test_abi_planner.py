@@ -182,3 +182,77 @@ def test_invalid_anchor_set_is_full_inference(dc):
     A = dc.AnchorArgs(K, H, dict(L0=0, T0=0, L1=0, T1=0, valid=0), tabs)
     r = dc.plan(gen.unicycle(5, 0, 8), A, 10.0, K)
     assert r["supported"] == 0 and r["n_reuse"] == 0 and r["actions"][1:] == [1] * K
+
+
+# ------------------------------------------- planner variants (Table 1, 3)
+
+VARIANTS = range(7)
+
+
+@pytest.mark.parametrize("variant", VARIANTS)
+def test_plan_variants_bit_exact(dc, variant):
+    rng = random.Random(500 + variant)
+    for trial in range(12):
+        K = rng.randint(2, 40)
+        H = rng.randint(1, 5)
+        tabs = _rand_tables(rng, K, H, dyadic=trial % 2 == 0)
+        anc = dict(L0=rng.uniform(0, 5), T0=rng.uniform(0, 0.3), L1=rng.uniform(20, 100),
+                   T1=rng.uniform(1, 3), valid=int(trial % 5 != 4))
+        A = dc.AnchorArgs(K, H, anc, tabs, variant=variant)
+        for _ in range(6):
+            poses = gen.unicycle(rng.uniform(0, 30), rng.uniform(-0.6, 0.6), 29, 0.1,
+                                 rng.uniform(-3, 3))
+            if variant == P.FIXED_INTERVAL:
+                budget = rng.randint(0, K - 1)
+            else:
+                budget = rng.choice([0.0, rng.uniform(0, 0.5), rng.uniform(0, 3), math.inf])
+            got = dc.plan(poses, A, budget, K)
+            ref = P.plan_scene_variant(poses, anc, tabs, budget, K, H, variant)
+            assert got["supported"] == ref["supported"]
+            assert got["actions"][1:] == ref["actions"][1:]
+            assert got["n_reuse"] == ref["n_reuse"]
+            assert got["cost"] == ref["cost"]
+            assert got["D"] == ref["D"]
+
+
+@pytest.mark.parametrize("variant", VARIANTS)
+def test_calibrate_variants_bit_exact(dc, variant):
+    wl = WORKLOADS["c2"]
+    K, H = wl.steps, wl.h_max
+    clips = gen.calibration_trajectories(wl)
+    stats = [P.motion_stats(c) for c in clips]
+    anc = P.select_anchors([s[0] for s in stats], [s[1] for s in stats])
+    q0, q1 = gen.synthetic_q_tables(K, H)
+    d0, d1 = gen.synthetic_d_tables(K, H)
+    tabs = dict(q0=q0, q1=q1, d0=d0, d1=d1)
+    A = dc.AnchorArgs(K, H, anc, tabs, variant=variant)
+    got = dc.calibrate_budget(list(clips), A, wl.target(), K)
+    ref = P.calibrate_budget_variant(list(clips), anc, tabs, wl.target(), K, H, variant)
+    assert got == ref
+    assert got[1] == 1
+
+
+def test_fixed_variants_do_not_replan(dc):
+    K, H = 12, 3
+    tabs = dict(q0=np.full((K, H + 1), 0.1), q1=np.full((K, H + 1), 0.2),
+                d0=np.full((K, H + 1), 0.1), d1=np.full((K, H + 1), 0.1))
+    anc = dict(L0=0.0, T0=0.0, L1=5.0, T1=1.0, valid=1)
+    prefix = [0] + [1, 2, 1, 2, 2, 1, 2, 1, 2, 1, 2, 2]
+    for v in (P.FIXED_PLACEMENT, P.FIXED_INTERVAL):
+        got = dc.replan(dc.AnchorArgs(K, H, anc, tabs, variant=v), 0.5, 4, 0.1, prefix)
+        assert got["actions"] == prefix and got["cost"] == 0.0
+
+
+def test_variant_arguments_are_checked(dc):
+    K, H = 6, 2
+    tabs = dict(q0=np.full((K, H + 1), 0.1), q1=np.full((K, H + 1), 0.2),
+                d0=np.full((K, H + 1), 0.1), d1=np.full((K, H + 1), 0.1))
+    anc = dict(L0=0.0, T0=0.0, L1=5.0, T1=1.0, valid=1)
+    poses = gen.unicycle(3.0, 0.1, 8)
+    with pytest.raises(dc.DCError):
+        dc.plan(poses, dc.AnchorArgs(K, H, anc, tabs, variant=7), 1.0, K)
+    fi = dc.AnchorArgs(K, H, anc, tabs, variant=P.FIXED_INTERVAL)
+    for bad in (2.5, -1.0, float(K), math.inf):
+        with pytest.raises(dc.DCError):
+            dc.plan(poses, fi, bad, K)
+    assert dc.plan(poses, fi, 2.0, K)["n_reuse"] == 2

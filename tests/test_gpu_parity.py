@@ -80,14 +80,16 @@ def _calibrated(wl):
     return w, om, sig, anc, tabs, tau
 
 
-def _compare_controller(dc, wl, w, om, sig, anc, tabs, tau, tol, bf16):
+def _compare_controller(dc, wl, w, om, sig, anc, tabs, tau, tol, bf16, variant=P.DRIVECACHE,
+                        trajs=None):
     K, H = wl.steps, wl.h_max
     x1 = gen.latents(wl)
-    trajs = gen.scene_trajectories(wl)
-    ref = Ctl.denoise(om, x1, trajs, sig, anc, tabs, tau, K, H)
+    trajs = gen.scene_trajectories(wl) if trajs is None else trajs
+    ref = Ctl.denoise(om, x1, trajs, sig, anc, tabs, tau, K, H, variant=variant)
     model = dc.Model(wl, gen.flat_blob(wl, w))
     lat = torch.tensor(x1, device="cuda")
-    st = dc.denoise(model, lat, list(trajs), dc.SchedArgs(K, sig, dc.AnchorArgs(K, H, anc, tabs), tau))
+    st = dc.denoise(model, lat, list(trajs),
+                    dc.SchedArgs(K, sig, dc.AnchorArgs(K, H, anc, tabs, variant=variant), tau))
     torch.cuda.synchronize()
     got = lat.cpu().numpy()
     model.close()
@@ -105,6 +107,8 @@ def _compare_controller(dc, wl, w, om, sig, anc, tabs, tau, tol, bf16):
             if g_ok != e["accept"]:
                 assert abs(e["d_obs"] - thr) <= NEAR * thr, (s, k, e, st["d_obs"][s, k])
                 near.append((s, k))
+    for s in range(B):
+        assert st["n_replan"][s] == ref["stats"][s]["n_replan"] or near
     if near:
         # logged near-threshold decisions: replay the oracle's decisions
         got, _ = run_forced(dc, wl, w, x1, trajs, ref["executed"], sig)
@@ -126,6 +130,28 @@ def test_tiny_fp32_full_controller(dc):
     w, om, sig, anc, tabs, tau = _calibrated(wl)
     st, ref = _compare_controller(dc, wl, w, om, sig, anc, tabs, tau, 1e-4, False)
     assert st["n_reuse"][0] == wl.target_reuses
+
+
+@pytest.mark.parametrize("variant", range(7))
+def test_tiny_fp32_controller_variants(dc, variant):
+    """Every planner variant (Table 3 ablations, Table 1 fixed interval)
+    through dc_denoise on three scenes of different motion, against the
+    oracle's controller under the same variant and its own calibrated tau."""
+    base = WORKLOADS["c1"]
+    w, om, sig, anc, tabs, _ = _calibrated(base)
+    wl = base.with_(batch=3)
+    K, H = wl.steps, wl.h_max
+    tau, reached = P.calibrate_budget_variant(gen.calibration_trajectories(base), anc, tabs,
+                                              wl.target(), K, H, variant)
+    assert reached == 1
+    trajs = [gen.unicycle(2.0, 0.0, wl.n_poses), gen.unicycle(5.0, 0.15, wl.n_poses),
+             gen.unicycle(1.0, 0.4, wl.n_poses)]
+    st, ref = _compare_controller(dc, wl, w, om, sig, anc, tabs, tau, 1e-4, False, variant=variant,
+                                  trajs=trajs)
+    if variant == P.FIXED_INTERVAL:
+        assert int(np.sum(st["checked"])) == 0
+        for s in range(3):
+            assert st["executed"][s].tolist()[1:] == P.even_schedule(int(tau), K, H)[1:]
 
 
 def test_tiny_fp32_anchor_drift_tables(dc):
