@@ -257,6 +257,25 @@ dc_status dc_denoise_host(dc_model* m, float* host_latents, const dc_cond* cond,
 dc_status dc_anchor_drift(dc_model* m, const float* noise, const dc_trajectory* traj, int K,
                           const double* sigmas, int H_max, double eps, double* d_out, void* stream);
 
+/* Eq. 6-7 along one full trace: the joint run responses of one anchor.
+ * Runs all K steps as full evaluations from `noise` (DEVICE fp32 [N][C], not
+ * modified) under `traj` (the anchor trace x_1..x_{K+1} with its cached
+ * r_1..r_K), forms e_{j,l} = H_{j+l}(x_{j+l}, r_j) - H_{j+l}(x_{j+l}, r_{j+l})
+ * with the reuse interface H (Eq. 6), carries each through the rest of the
+ * run with Jacobian-vector products of the model along the frozen trace --
+ * dx_{t+1} = dsig_t e, dx_{m+1} = dx_m + dsig_m J_m dx_m for m = t+1..K,
+ * J_m = dv_m/dx_m -- and writes
+ *   q_out[j*(H_max+1)+h] = ||sum_{l<=h} dx_{K+1}(e_{j,l})|| / (||x_{K+1}|| + eps)
+ * for j = 1..K-1, h = 1..min(H_max, K-j), other entries 0 (host q_out, fp64
+ * sums).  The tangents run in fp32 on the model's weights (any model dtype);
+ * the calibration cost is O(K^2 H_max) tangent passes, batched per trace
+ * point.  Device workspace is allocated and freed inside the call (about
+ * 8 GB at most for the tangents plus the stored activations); the call
+ * synchronises `stream`.  head_dim must be 8, 16, 32, 64, 72 or 128. */
+dc_status dc_anchor_response(dc_model* m, const float* noise, const dc_trajectory* traj, int K,
+                             const double* sigmas, int H_max, double eps, double* q_out,
+                             void* stream);
+
 /* Drift sums for Eq. 12 on B scenes: for each scene s, out[2s] =
  * sum ||u(x_now_s) - u(x_ref_s)||^2 = sum ||(x_now_s - x_ref_s) W_e^T||^2 and
  * out[2s+1] = sum ||u(x_now_s)||^2 with u(x) = x W_e^T + b_e + pos, summed

@@ -111,6 +111,9 @@ def lib():
                                  P(RunStats)]),
         "dc_anchor_drift": (st, [C.c_void_p, C.c_void_p, P(Trajectory), C.c_int, P(C.c_double),
                                  C.c_int, C.c_double, P(C.c_double), C.c_void_p]),
+        "dc_anchor_response": (st, [C.c_void_p, C.c_void_p, P(Trajectory), C.c_int,
+                                    P(C.c_double), C.c_int, C.c_double, P(C.c_double),
+                                    C.c_void_p]),
         "dc_drift_sums": (st, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int, C.c_void_p,
                                C.c_void_p]),
         "dc_drift_sums_noalloc": (st, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int, C.c_void_p,
@@ -363,6 +366,18 @@ def anchor_drift(model: Model, noise, poses, K, sigmas, H, eps=1e-6, stream=None
                                  _stream_handle(stream)))
     return out
 
+
+
+def anchor_response(model: Model, noise, poses, K, sigmas, H, eps=1e-6, stream=None):
+    """dc_anchor_response (Eq. 6-7): noise is a CUDA fp32 tensor [N, C];
+    returns the joint run responses q [K][H+1]."""
+    ta = TrajectoryArgs([poses])
+    sig = np.ascontiguousarray(sigmas, np.float64)
+    out = np.zeros((K, H + 1), np.float64)
+    _check(lib().dc_anchor_response(model.h, C.c_void_p(noise.data_ptr()), ta.ptr(), int(K),
+                                    _dptr(sig), int(H), float(eps), _dptr(out),
+                                    _stream_handle(stream)))
+    return out
 
 def drift_sums(model: Model, x_now, x_ref, out, stream=None):
     """dc_drift_sums on CUDA fp32 tensors x_now/x_ref [B, N, C], out [2B]."""

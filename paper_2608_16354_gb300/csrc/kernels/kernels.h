@@ -84,4 +84,41 @@ cudaError_t launch_drift(const DriftItems& items, const float* gram, const float
                          const float* gs, int N, int C, float* partials /* [n][kDriftParts][2] */,
                          float* out /* [2n] */, cudaStream_t st);
 
+// ---- fp32 forward-mode kernels for the joint run responses (Eq. 6-7) ----
+// C[M][N] = A[M][K] W[N][K]^T + epilogue (W fp32 or bf16, fp32 accumulate):
+enum { kJStore = 0, kJGatedAdd = 1, kJGeluPrimal = 2, kJGeluGrad = 3 };
+struct JEpi {
+  int mode;
+  const float* bias;   // optional [N], added to the product first
+  const float* gate;   // kJGatedAdd: out = base + gate (acc + bias)
+  const float* base;   // kJGatedAdd: [M][N], may equal out
+  float* out;          // [M][N]
+  float* out2;         // kJGeluPrimal: out = z = acc + bias, out2 = gelu(z)
+  const float* z;      // kJGeluGrad: out = gelu'(z[row % zrows]) acc
+  int zrows;
+};
+template <typename TW>
+cudaError_t launch_gemm_f32w(const float* A, const TW* W, int M, int N, int K, const JEpi& ep,
+                             cudaStream_t st);
+// out = LN(h) (1 + scale) + shift per row of d
+cudaError_t launch_ln_mod_f32(const float* h, int R, int d, const float* shift, const float* scale,
+                              float* out, cudaStream_t st);
+// tangent of the modulated LayerNorm at primal rows h [N][d] for dh [T][N][d]
+cudaError_t launch_ln_jvp_f32(const float* h, const float* dh, int N, int T, int d,
+                              const float* scale, float* out, cudaStream_t st);
+// u = x W_e^T (+ b_e + pos when b_e != NULL), x [R][C], rows r use pos[r % N]
+template <typename TP>
+cudaError_t launch_embed_f32(const float* x, const float* w_eT, const float* b_e, const TP* pos,
+                             int R, int N, int C, int d, float* out, cudaStream_t st);
+// attention of one scene (qkv [N][3d] fp32 rows) -> o [N][d]; with dqkv
+// [T][N][3d] (non-NULL) the tangent -> dout [T][N][d] instead
+bool attention_f32_jvp_supported(int dh);
+cudaError_t launch_attention_f32_jvp(const float* qkv, const float* dqkv, int N, int d, int heads,
+                                     int dh, int T, float* o, float* dout, cudaStream_t st);
+cudaError_t launch_axpy_f32(float* y, const float* x, float a, size_t n, cudaStream_t st);
+template <typename T>
+cudaError_t launch_add_cache(const float* a, const T* r, float* out, size_t n, cudaStream_t st);
+cudaError_t launch_scaled_diff(const float* a, const float* b, float s, float* out, size_t n,
+                               cudaStream_t st);
+
 }  // namespace dc

@@ -425,10 +425,12 @@ struct SceneState {
 };
 
 // The sampler.  trace (optional, device [K][B][N][C]) receives x_k before
-// step k.
+// step k; r_trace (optional, device [K][N][d] of the cache type) receives
+// scene 0's cached r after step k.
 template <typename T>
 dc_status run_sampler(dc_model* m, float* lat, const dc_cond* cond, const dc_sched* sc,
-                      cudaStream_t st, dc_run_stats* stats, float* trace) {
+                      cudaStream_t st, dc_run_stats* stats, float* trace,
+                      void* r_trace = nullptr) {
   const int B = cond->B, K = sc->K, N = m->N, C = m->C;
   const dc_anchor_responses* anc = sc->anchors;
   const double eps = anc ? anc->eps : 1e-6;
@@ -560,6 +562,11 @@ dc_status run_sampler(dc_model* m, float* lat, const dc_cond* cond, const dc_sch
     }
     DC_TRY(enqueue_compute<T>(m, lat, mod_k, cm, dsig, st));
     DC_TRY(enqueue_reuse<T>(m, lat, mod_k, rm, dsig, st));
+    if (r_trace) {
+      const size_t rb = (size_t)N * m->d * m->elt;
+      DC_CK(cudaMemcpyAsync(static_cast<uint8_t*>(r_trace) + (size_t)(k - 1) * rb, m->r, rb,
+                            cudaMemcpyDeviceToDevice, st));
+    }
     for (int s = 0; s < B; ++s) {
       if (reuse_now[s]) {
         state[s].age += 1;
@@ -629,6 +636,227 @@ dc_status check_call(dc_model* m, const dc_cond* cond, const dc_sched* sc) {
       return DC_ERR_INVALID_ARG;
     }
     if ((s = dc::check_reuse_count(*sc->anchors, sc->tau)) != DC_OK) return s;
+  }
+  return DC_OK;
+}
+
+// ------------------------------------------- joint run responses (Eq. 6-7)
+
+// Device buffers of one dc_anchor_response call, freed on every exit.
+struct DevBufs {
+  std::vector<void*> p;
+  ~DevBufs() {
+    for (void* q : p) cudaFree(q);
+  }
+  template <typename X>
+  bool get(X** out, size_t bytes) {
+    void* q = nullptr;
+    if (cudaMalloc(&q, bytes ? bytes : 16) != cudaSuccess) return false;
+    p.push_back(q);
+    *out = static_cast<X*>(q);
+    return true;
+  }
+};
+
+template <typename T>
+struct ResponseWork {
+  int N, C, d, L, md, heads, dh;
+  // trace and interface outputs
+  float *xs, *vbar, *e, *vtmp;
+  T* rs;
+  // primal activations at one trace point
+  float *hin, *qkv, *h1, *z, *hcur, *hL, *abuf, *obuf, *mbuf;
+  // tangents
+  float *th, *ta, *tqkv, *tout, *tm, *tv;
+};
+
+// v = H_t(x, r): u(x) + r through the step's final modulated LayerNorm and
+// head (the reuse interface of Eq. 1).
+template <typename T>
+dc_status interface_f32(dc_model* m, ResponseWork<T>& w, const float* x, const T* r,
+                        const float* mod, float* v, cudaStream_t st) {
+  const size_t Nd = (size_t)w.N * w.d;
+  const float* fsh = mod + (size_t)6 * w.L * w.d;
+  DC_CK(dc::launch_embed_f32<T>(x, m->w_eT, m->b_e, static_cast<const T*>(m->pos), w.N, w.N, w.C,
+                                w.d, w.hcur, st));
+  DC_CK(dc::launch_add_cache<T>(w.hcur, r, w.hcur, Nd, st));
+  DC_CK(dc::launch_ln_mod_f32(w.hcur, w.N, w.d, fsh, fsh + w.d, w.abuf, st));
+  dc::JEpi ep{};
+  ep.mode = dc::kJStore; ep.bias = m->b_f; ep.out = v;
+  DC_CK(dc::launch_gemm_f32w<float>(w.abuf, m->w_f, w.N, w.C, w.d, ep, st));
+  return DC_OK;
+}
+
+// Full evaluation at one trace point, keeping what the tangents need.
+template <typename T>
+dc_status primal_f32(dc_model* m, ResponseWork<T>& w, const float* x, const float* mod,
+                     cudaStream_t st) {
+  const int N = w.N, d = w.d, md = w.md;
+  const size_t Nd = (size_t)N * d;
+  DC_CK(dc::launch_embed_f32<T>(x, m->w_eT, m->b_e, static_cast<const T*>(m->pos), N, N, w.C, d,
+                                w.hcur, st));
+  for (int l = 0; l < w.L; ++l) {
+    const BlockW& b = m->blk[l];
+    const float* mb = mod + (size_t)l * 6 * d;
+    float* qkv = w.qkv + (size_t)l * N * 3 * d;
+    DC_CK(cudaMemcpyAsync(w.hin + l * Nd, w.hcur, Nd * 4, cudaMemcpyDeviceToDevice, st));
+    DC_CK(dc::launch_ln_mod_f32(w.hcur, N, d, mb, mb + d, w.abuf, st));
+    dc::JEpi e1{};
+    e1.mode = dc::kJStore; e1.bias = b.b_qkv; e1.out = qkv;
+    DC_CK(dc::launch_gemm_f32w<T>(w.abuf, static_cast<const T*>(b.w_qkv), N, 3 * d, d, e1, st));
+    DC_CK(dc::launch_attention_f32_jvp(qkv, nullptr, N, d, w.heads, w.dh, 1, w.obuf, nullptr, st));
+    dc::JEpi e2{};
+    e2.mode = dc::kJGatedAdd; e2.bias = b.b_o; e2.gate = mb + 2 * d; e2.base = w.hcur; e2.out = w.hcur;
+    DC_CK(dc::launch_gemm_f32w<T>(w.obuf, static_cast<const T*>(b.w_o), N, d, d, e2, st));
+    DC_CK(cudaMemcpyAsync(w.h1 + l * Nd, w.hcur, Nd * 4, cudaMemcpyDeviceToDevice, st));
+    DC_CK(dc::launch_ln_mod_f32(w.hcur, N, d, mb + 3 * d, mb + 4 * d, w.abuf, st));
+    dc::JEpi e3{};
+    e3.mode = dc::kJGeluPrimal; e3.bias = b.b_1; e3.out = w.z + (size_t)l * N * md; e3.out2 = w.mbuf;
+    DC_CK(dc::launch_gemm_f32w<T>(w.abuf, static_cast<const T*>(b.w_1), N, md, d, e3, st));
+    dc::JEpi e4{};
+    e4.mode = dc::kJGatedAdd; e4.bias = b.b_2; e4.gate = mb + 5 * d; e4.base = w.hcur; e4.out = w.hcur;
+    DC_CK(dc::launch_gemm_f32w<T>(w.mbuf, static_cast<const T*>(b.w_2), N, d, md, e4, st));
+  }
+  DC_CK(cudaMemcpyAsync(w.hL, w.hcur, Nd * 4, cudaMemcpyDeviceToDevice, st));
+  return DC_OK;
+}
+
+// dv = J dx for T perturbations dx [T][N][C] of the last primal point.
+template <typename T>
+dc_status tangent_f32(dc_model* m, ResponseWork<T>& w, const float* dx, int Tn, const float* mod,
+                      float* dv, cudaStream_t st) {
+  const int N = w.N, d = w.d, md = w.md, R = Tn * N;
+  const size_t Nd = (size_t)N * d;
+  DC_CK(dc::launch_embed_f32<T>(dx, m->w_eT, nullptr, static_cast<const T*>(nullptr), R, N, w.C, d,
+                                w.th, st));
+  for (int l = 0; l < w.L; ++l) {
+    const BlockW& b = m->blk[l];
+    const float* mb = mod + (size_t)l * 6 * d;
+    DC_CK(dc::launch_ln_jvp_f32(w.hin + l * Nd, w.th, N, Tn, d, mb + d, w.ta, st));
+    dc::JEpi e1{};
+    e1.mode = dc::kJStore; e1.out = w.tqkv;
+    DC_CK(dc::launch_gemm_f32w<T>(w.ta, static_cast<const T*>(b.w_qkv), R, 3 * d, d, e1, st));
+    DC_CK(dc::launch_attention_f32_jvp(w.qkv + (size_t)l * N * 3 * d, w.tqkv, N, d, w.heads, w.dh,
+                                       Tn, nullptr, w.tout, st));
+    dc::JEpi e2{};
+    e2.mode = dc::kJGatedAdd; e2.gate = mb + 2 * d; e2.base = w.th; e2.out = w.th;
+    DC_CK(dc::launch_gemm_f32w<T>(w.tout, static_cast<const T*>(b.w_o), R, d, d, e2, st));
+    DC_CK(dc::launch_ln_jvp_f32(w.h1 + l * Nd, w.th, N, Tn, d, mb + 4 * d, w.ta, st));
+    dc::JEpi e3{};
+    e3.mode = dc::kJGeluGrad; e3.out = w.tm; e3.z = w.z + (size_t)l * N * md; e3.zrows = N;
+    DC_CK(dc::launch_gemm_f32w<T>(w.ta, static_cast<const T*>(b.w_1), R, md, d, e3, st));
+    dc::JEpi e4{};
+    e4.mode = dc::kJGatedAdd; e4.gate = mb + 5 * d; e4.base = w.th; e4.out = w.th;
+    DC_CK(dc::launch_gemm_f32w<T>(w.tm, static_cast<const T*>(b.w_2), R, d, md, e4, st));
+  }
+  const float* fsh = mod + (size_t)6 * w.L * d;
+  DC_CK(dc::launch_ln_jvp_f32(w.hL, w.th, N, Tn, d, fsh + d, w.ta, st));
+  dc::JEpi ef{};
+  ef.mode = dc::kJStore; ef.out = dv;
+  DC_CK(dc::launch_gemm_f32w<float>(w.ta, m->w_f, R, w.C, d, ef, st));
+  return DC_OK;
+}
+
+template <typename T>
+dc_status anchor_response_impl(dc_model* m, const float* noise, const dc_trajectory* traj, int K,
+                               const double* sig, int H, double eps, double* q_out,
+                               cudaStream_t st) {
+  ResponseWork<T> w{};
+  w.N = m->N; w.C = m->C; w.d = m->d; w.L = m->L; w.md = m->md; w.heads = m->heads; w.dh = m->dh;
+  const int N = w.N, C = w.C, d = w.d, md = w.md;
+  const size_t NC = (size_t)N * C, Nd = (size_t)N * d;
+  // perturbation chains (j, l), injected after step t = j + l, ordered by t
+  std::vector<std::pair<int, int>> chains;
+  std::vector<int> first_at(K + 2, 0);
+  for (int t = 2; t <= K; ++t) {
+    first_at[t] = (int)chains.size();
+    for (int l = 1; l <= std::min(H, t - 1); ++l) chains.push_back({t - l, l});
+  }
+  first_at[K + 1] = (int)chains.size();
+  const int nch = (int)chains.size();
+  // tangent batch: at most 64, within about 8 GB of tangent workspace
+  const size_t per_tan = (size_t)N * (6 * (size_t)d + md + 2 * (size_t)C) * 4;
+  const int Tmax = (int)std::max<size_t>(1, std::min<size_t>(64, (size_t)8e9 / per_tan));
+  DevBufs buf;
+  const bool ok =
+      buf.get(&w.xs, (size_t)(K + 1) * NC * 4) && buf.get(&w.rs, (size_t)K * Nd * sizeof(T)) &&
+      buf.get(&w.vbar, (size_t)K * NC * 4) && buf.get(&w.e, NC * 4) && buf.get(&w.vtmp, NC * 4) &&
+      buf.get(&w.hin, (size_t)w.L * Nd * 4) && buf.get(&w.qkv, (size_t)w.L * Nd * 3 * 4) &&
+      buf.get(&w.h1, (size_t)w.L * Nd * 4) && buf.get(&w.z, (size_t)w.L * N * md * 4) &&
+      buf.get(&w.hcur, Nd * 4) && buf.get(&w.hL, Nd * 4) && buf.get(&w.abuf, Nd * 4) &&
+      buf.get(&w.obuf, Nd * 4) && buf.get(&w.mbuf, (size_t)N * md * 4) &&
+      buf.get(&w.th, (size_t)Tmax * Nd * 4) && buf.get(&w.ta, (size_t)Tmax * Nd * 4) &&
+      buf.get(&w.tqkv, (size_t)Tmax * Nd * 3 * 4) && buf.get(&w.tout, (size_t)Tmax * Nd * 4) &&
+      buf.get(&w.tm, (size_t)Tmax * N * md * 4) && buf.get(&w.tv, (size_t)Tmax * NC * 4);
+  float* dxs = nullptr;
+  if (!ok || !buf.get(&dxs, (size_t)std::max(nch, 1) * NC * 4)) {
+    dc::set_error("dc_anchor_response: device allocation failed");
+    return DC_ERR_NOMEM;
+  }
+  // the frozen full trace: x_1..x_K, the cached r_1..r_K, then x_{K+1}
+  std::vector<unsigned char> forced((size_t)K + 1, dc::kCompute);
+  dc_sched sc{};
+  sc.K = K; sc.sigmas = sig; sc.anchors = nullptr; sc.tau = 0.0; sc.veto = 0;
+  sc.forced = forced.data();
+  dc_cond cond{1, traj};
+  DC_TRY(check_call(m, &cond, &sc));
+  float* lat = w.xs + (size_t)K * NC;
+  DC_CK(cudaMemcpyAsync(lat, noise, NC * 4, cudaMemcpyDeviceToDevice, st));
+  DC_TRY(run_sampler<T>(m, lat, &cond, &sc, st, nullptr, w.xs, w.rs));
+  auto x_at = [&](int k) { return w.xs + (size_t)(k - 1) * NC; };      // x_k, k = 1..K+1
+  auto r_at = [&](int k) { return w.rs + (size_t)(k - 1) * Nd; };      // r_k, k = 1..K
+  auto mod_at = [&](int k) { return m->mod + (size_t)(k - 1) * m->mod_stride; };
+  // H_t(x_t, r_t) of every step (the second term of Eq. 6)
+  for (int t = 1; t <= K; ++t)
+    DC_TRY(interface_f32<T>(m, w, x_at(t), r_at(t), mod_at(t), w.vbar + (size_t)(t - 1) * NC, st));
+  for (int step = 2; step <= K + 1; ++step) {
+    // chains injected after step t = step - 1: dx_{t+1} = dsig_t e_{j,l} (Eq. 6)
+    const int t = step - 1;
+    const float dsig_t = (float)(sig[t] - sig[t - 1]);
+    for (int c = first_at[t]; c < first_at[t + 1]; ++c) {
+      DC_TRY(interface_f32<T>(m, w, x_at(t), r_at(chains[c].first), mod_at(t), w.vtmp, st));
+      DC_CK(dc::launch_scaled_diff(w.vtmp, w.vbar + (size_t)(t - 1) * NC, dsig_t, dxs + c * NC, NC,
+                                   st));
+    }
+    if (step > K) break;
+    // carry every live chain through step `step`: dx += dsig J dx
+    const int live = first_at[step];
+    if (live == 0) continue;
+    DC_TRY(primal_f32<T>(m, w, x_at(step), mod_at(step), st));
+    const float dsig = (float)(sig[step] - sig[step - 1]);
+    for (int g0 = 0; g0 < live; g0 += Tmax) {
+      const int Tn = std::min(Tmax, live - g0);
+      DC_TRY(tangent_f32<T>(m, w, dxs + (size_t)g0 * NC, Tn, mod_at(step), w.tv, st));
+      DC_CK(dc::launch_axpy_f32(dxs + (size_t)g0 * NC, w.tv, dsig, (size_t)Tn * NC, st));
+    }
+  }
+  // Eq. 7 on the host in fp64: G_{j,h} = sum_{l<=h} P_{j+l} e_{j,l}
+  std::vector<float> Y((size_t)nch * NC), xK(NC);
+  if (nch) DC_CK(cudaMemcpyAsync(Y.data(), dxs, Y.size() * 4, cudaMemcpyDeviceToHost, st));
+  DC_CK(cudaMemcpyAsync(xK.data(), x_at(K + 1), NC * 4, cudaMemcpyDeviceToHost, st));
+  DC_TRY(check_device_error(m, st));
+  double nx = 0.0;
+  for (float v : xK) nx += (double)v * v;
+  const double den = std::sqrt(nx) + eps;
+  for (size_t i = 0; i < (size_t)K * (H + 1); ++i) q_out[i] = 0.0;
+  std::vector<int> idx((size_t)(K + 1) * (H + 1), -1);
+  for (int c = 0; c < nch; ++c) idx[(size_t)chains[c].first * (H + 1) + chains[c].second] = c;
+  std::vector<double> G(NC);
+  for (int j = 1; j < K; ++j) {
+    std::fill(G.begin(), G.end(), 0.0);
+    for (int l = 1; l <= std::min(H, K - j); ++l) {
+      const float* y = Y.data() + (size_t)idx[(size_t)j * (H + 1) + l] * NC;
+      double g2 = 0.0;
+      for (size_t i = 0; i < NC; ++i) {
+        G[i] += y[i];
+        g2 += G[i] * G[i];
+      }
+      if (!std::isfinite(g2)) {
+        dc::set_error("dc_anchor_response: non-finite response");
+        return DC_ERR_NONFINITE;
+      }
+      q_out[(size_t)j * (H + 1) + l] = std::sqrt(g2) / den;
+    }
   }
   return DC_OK;
 }
@@ -937,6 +1165,28 @@ dc_status dc_anchor_drift(dc_model* m, const float* noise, const dc_trajectory* 
   cudaStreamSynchronize(st);
   cudaFree(trace);
   cudaFree(x);
+  return s;
+}
+
+dc_status dc_anchor_response(dc_model* m, const float* noise, const dc_trajectory* traj, int K,
+                             const double* sigmas, int H_max, double eps, double* q_out,
+                             void* stream) {
+  if (!m || !noise || !traj || !sigmas || !q_out || K < 1 || K > m->Kmax || H_max < 1 ||
+      !(eps > 0.0)) {
+    dc::set_error("dc_anchor_response: NULL argument, K outside [1, max_steps], H_max < 1 or eps <= 0");
+    return DC_ERR_INVALID_ARG;
+  }
+  if (!dc::attention_f32_jvp_supported(m->dh)) {
+    dc::set_error("dc_anchor_response: head_dim must be 8, 16, 32, 64, 72 or 128");
+    return DC_ERR_UNSUPPORTED;
+  }
+  DC_CK(cudaSetDevice(m->device));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  dc_status s = m->bf16 ? anchor_response_impl<__nv_bfloat16>(m, noise, traj, K, sigmas, H_max, eps,
+                                                               q_out, st)
+                        : anchor_response_impl<float>(m, noise, traj, K, sigmas, H_max, eps, q_out,
+                                                      st);
+  cudaStreamSynchronize(st);
   return s;
 }
 

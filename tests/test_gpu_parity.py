@@ -434,3 +434,50 @@ def test_cached_backbone_output_strong_weights(dc, key, shape, std, tol):
         assert e_r <= tol, e_r
         assert e_x <= (tol if wl.dtype == "f32" else 2e-2), e_x
     model.close()
+
+
+# ------------------------------------------- joint run responses (Eq. 6-7)
+
+def _response_case(dc, wl, w, K, H, strong):
+    from oracle import dit as O
+    from oracle import response as R
+    if strong:
+        w = {k: (np.asarray(v) * 8 if k.startswith("blk") else v) for k, v in w.items()}
+    sig = gen.sigmas(K)
+    poses = gen.unicycle(4.0, 0.2, wl.n_poses)
+    noise = gen.latents(wl.with_(batch=1))[0]
+    ref, _, _ = R.response_table(O.Model(wl, w), noise, poses, sig, K, H)
+    ref = np.asarray(ref)
+    model = dc.Model(wl.with_(batch=1), gen.flat_blob(wl, w), max_batch=1, max_steps=K)
+    got = dc.anchor_response(model, torch.tensor(noise, device="cuda"), poses, K, sig, H)
+    model.close()
+    return got, ref
+
+
+@pytest.mark.parametrize("strong", [False, True])
+def test_anchor_response_fp32_vs_oracle(dc, strong):
+    """dc_anchor_response (fp32 trace, fp32 JVPs) against the fp64 oracle:
+    every entry of the q table and the zero pattern."""
+    wl = WORKLOADS["c1"]
+    K, H = wl.steps, wl.h_max
+    got, ref = _response_case(dc, wl, gen.weights(wl), K, H, strong)
+    mask = ref > 0
+    assert np.array_equal(got > 0, mask)
+    relmax = float(np.max(np.abs(got[mask] - ref[mask]) / ref[mask]))
+    record(f"anchor_response_fp32_strong{int(strong)}", dict(rel_max=relmax, rel=rel(got, ref)))
+    assert relmax <= 1e-3 and rel(got, ref) <= 2e-4
+
+
+def test_anchor_response_bf16_small_vs_oracle(dc):
+    """bf16 model (bf16 trace, fp32 JVPs on the bf16 weights) on a small
+    c2-shaped case: the trace itself is bf16, so the table agrees to the
+    bf16 latent tolerance."""
+    wl = WORKLOADS["c2"].with_(n_blocks=2, frames=2, rows=8, cols=8, steps=6, batch=1,
+                               n_poses=5)
+    K, H = wl.steps, wl.h_max
+    got, ref = _response_case(dc, wl, gen.weights(wl), K, H, False)
+    mask = ref > 0
+    assert np.array_equal(got > 0, mask)
+    record("anchor_response_bf16", dict(rel=rel(got, ref),
+                                         rel_max=float(np.max(np.abs(got[mask] - ref[mask]) / ref[mask]))))
+    assert rel(got, ref) <= 2e-2
