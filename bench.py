@@ -52,6 +52,8 @@ def parse():
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--workload", default="c2", choices=sorted(WORKLOADS))
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--calibration", action="store_true",
+                   help="time the joint run responses (Eq. 6-7) of one anchor instead")
     return p.parse_args()
 
 
@@ -243,6 +245,99 @@ def ratio_summary(st):
     return {"min": float(r.min()), "median": float(np.median(r)), "max": float(r.max())}
 
 
+# SM count and FP32 lanes per SM of the part (the ALU roofline of the fp32
+# tangent kernels): 152 SMs x 4 schedulers x 32 lanes, one FMA (2 flops) each
+SMS, FP32_LANES = 152, 128
+
+
+def tangent_passes(K, H):
+    """Tangent evaluations of dc_anchor_response: at step m every chain
+    injected after a step t < m is carried once (Eq. 7)."""
+    n = 0
+    for m in range(2, K + 1):
+        n += sum(min(H, t - 1) for t in range(2, m))
+    return n
+
+
+def oracle_block_jvp_seconds(wl, rounds=1):
+    """The oracle's tangent of one DiT block at full size (fp64 NumPy)."""
+    from oracle import dit as O
+    from oracle import response as R
+    w = gen.weights(wl)
+    rng = np.random.default_rng(0)
+    h = rng.standard_normal((wl.n_tokens, wl.d_model))
+    dh = rng.standard_normal(h.shape)
+    mod = {k: rng.standard_normal(wl.d_model) * 0.1 for k in
+           ("shift1", "scale1", "gate1", "shift2", "scale2", "gate2")}
+    t0 = time.perf_counter()
+    for _ in range(rounds):
+        R.block_jvp(O.block_weights(w, 0), h, dh, mod, wl.n_heads)
+    return (time.perf_counter() - t0) / rounds
+
+
+def run_calibration(args, wl):
+    """One anchor's joint run responses on the GPU (dc_anchor_response) at the
+    bench workload, its dominant kernel against the FP32 ALU peak, and the
+    oracle's tangent of one block scaled to the same number of passes."""
+    import torch
+    from paper_2608_16354_gb300 import binding as dc
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    dc.lib()
+    K, H = wl.steps, wl.h_max
+    one = wl.with_(batch=1)
+    model = dc.Model(one, gen.flat_blob(wl, gen.weights(wl)), max_batch=1, max_steps=K)
+    clips = gen.calibration_trajectories(wl)
+    from oracle import planner as P
+    stats = [P.motion_stats(c) for c in clips]
+    anc = dc.select_anchors([s_[0] for s_ in stats], [s_[1] for s_ in stats])
+    poses = clips[anc["i1"] if anc["valid"] else 0]
+    noise = torch.tensor(gen.anchor_noise(wl), device=dev)
+    dc.anchor_response(model, noise, poses, 3, gen.sigmas(3), H)  # warm-up (3 steps)
+    torch.cuda.synchronize()
+    clocks = Clocks(0)
+    dc.profile(model, True)
+    clocks.start()
+    t0 = time.perf_counter()
+    q = dc.anchor_response(model, noise, poses, K, gen.sigmas(K), H)
+    torch.cuda.synchronize()
+    secs = time.perf_counter() - t0
+    clk = clocks.stop()
+    dc.profile(model, False)
+    prof = dc.profile_read(model)
+    model.close()
+    pk, pk_src = peaks()
+    mhz = float(pk.get("sm_max_mhz", 2070.0))
+    peak = SMS * FP32_LANES * 2 * mhz * 1e6 / 1e12
+    p = prof["jvp_attention"]
+    achieved = p["flops"] / (p["ms"] / 1000.0) / 1e12
+    passes = tangent_passes(K, H)
+    line = {
+        "metric": "joint run response calibration (Eq. 6-7), seconds per anchor", "value": secs,
+        "unit": "s", "n_gpus": 1, "steps": 1, "warmup": 1, "higher_is_better": False,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": wl.name, "steps": K, "h_max": H, "tokens": wl.n_tokens,
+                   "blocks": wl.n_blocks, "tangent_passes": passes, "anchor": "moving-turn"},
+        "q_table_max": float(np.max(q)),
+        "kernels": {k: {"ms": v["ms"], "launches": v["launches"],
+                        "tflops": (v["flops"] / (v["ms"] / 1000.0) / 1e12) if v["ms"] > 0 and v["flops"] else None}
+                    for k, v in prof.items() if k.startswith("jvp") and v["launches"]},
+        "roofline": {"kernel": "jvp_attention", "bound": "alu", "achieved": achieved, "peak": peak,
+                     "unit": "TFLOP/s", "frac": achieved / peak, "traffic": None,
+                     "peak_source": f"{SMS} SMs x {FP32_LANES} FP32 lanes x 2 flops x {mhz:.0f} MHz ({pk_src} clock)"},
+        "clocks": clk,
+    }
+    if not args.no_cpu_baseline:
+        blk = oracle_block_jvp_seconds(wl)
+        # every pass runs L block tangents; the primal points cost about as much again
+        est = blk * wl.n_blocks * (passes + K)
+        line["cpu_baseline"] = {"value": est, "unit": "s", "cores": cpu_threads(), "kind": "oracle",
+                                "sample": (f"one block tangent at full size ({blk:.2f} s, fp64 NumPy), "
+                                           f"scaled by {wl.n_blocks} blocks x ({passes} tangent passes "
+                                           f"+ {K} primal points)")}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse()
     wl = WORKLOADS[args.workload]
@@ -251,6 +346,8 @@ def main():
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
         return run_reference(args, wl, rank, world)
+    if args.calibration:
+        return run_calibration(args, wl)
 
     import torch
     import torch.distributed as dist

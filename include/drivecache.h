@@ -340,6 +340,9 @@ enum {
   DC_PROF_FINAL,         /* interface + Euler + cache write (compute steps) */
   DC_PROF_REUSE,         /* reuse step: cached r + interface + Euler */
   DC_PROF_DRIFT,         /* drift sums of Eq. 12 */
+  DC_PROF_JVP_ATTENTION, /* dc_anchor_response: attention and its tangent (fp32) */
+  DC_PROF_JVP_GEMM,      /* dc_anchor_response: linear layers and their tangents (fp32) */
+  DC_PROF_JVP_OTHER,     /* dc_anchor_response: LayerNorm, embedding, interface, updates */
   DC_PROF_N
 };
 dc_status dc_profile(dc_model* m, int enable);

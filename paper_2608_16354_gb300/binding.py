@@ -402,7 +402,8 @@ def attention(qkv, slots, heads, n_tokens, head_dim, out, stream=None):
 
 
 PROF_NAMES = ["condition", "embed", "ln_mod", "gemm_qkv", "attention", "gemm_out", "gemm_mlp1",
-              "gemm_mlp2", "final_compute", "reuse", "drift"]
+              "gemm_mlp2", "final_compute", "reuse", "drift", "jvp_attention", "jvp_gemm",
+              "jvp_other"]
 
 
 def profile(model: Model, enable):

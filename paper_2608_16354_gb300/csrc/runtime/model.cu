@@ -677,13 +677,17 @@ dc_status interface_f32(dc_model* m, ResponseWork<T>& w, const float* x, const T
                         const float* mod, float* v, cudaStream_t st) {
   const size_t Nd = (size_t)w.N * w.d;
   const float* fsh = mod + (size_t)6 * w.L * w.d;
-  DC_CK(dc::launch_embed_f32<T>(x, m->w_eT, m->b_e, static_cast<const T*>(m->pos), w.N, w.N, w.C,
+  DC_LAUNCH(DC_PROF_JVP_OTHER, 0.0, 0.0,
+              dc::launch_embed_f32<T>(x, m->w_eT, m->b_e, static_cast<const T*>(m->pos), w.N, w.N, w.C,
                                 w.d, w.hcur, st));
-  DC_CK(dc::launch_add_cache<T>(w.hcur, r, w.hcur, Nd, st));
-  DC_CK(dc::launch_ln_mod_f32(w.hcur, w.N, w.d, fsh, fsh + w.d, w.abuf, st));
+  DC_LAUNCH(DC_PROF_JVP_OTHER, 0.0, 0.0,
+              dc::launch_add_cache<T>(w.hcur, r, w.hcur, Nd, st));
+  DC_LAUNCH(DC_PROF_JVP_OTHER, 0.0, 0.0,
+              dc::launch_ln_mod_f32(w.hcur, w.N, w.d, fsh, fsh + w.d, w.abuf, st));
   dc::JEpi ep{};
   ep.mode = dc::kJStore; ep.bias = m->b_f; ep.out = v;
-  DC_CK(dc::launch_gemm_f32w<float>(w.abuf, m->w_f, w.N, w.C, w.d, ep, st));
+  DC_LAUNCH(DC_PROF_JVP_GEMM, 2.0 * (w.N) * (w.C) * (w.d), 0.0,
+              dc::launch_gemm_f32w<float>(w.abuf, m->w_f, w.N, w.C, w.d, ep, st));
   return DC_OK;
 }
 
@@ -693,29 +697,39 @@ dc_status primal_f32(dc_model* m, ResponseWork<T>& w, const float* x, const floa
                      cudaStream_t st) {
   const int N = w.N, d = w.d, md = w.md;
   const size_t Nd = (size_t)N * d;
-  DC_CK(dc::launch_embed_f32<T>(x, m->w_eT, m->b_e, static_cast<const T*>(m->pos), N, N, w.C, d,
-                                w.hcur, st));
+  DC_LAUNCH(DC_PROF_JVP_OTHER, 0.0, 0.0,
+            dc::launch_embed_f32<T>(x, m->w_eT, m->b_e, static_cast<const T*>(m->pos), N, N, w.C,
+                                    d, w.hcur, st));
   for (int l = 0; l < w.L; ++l) {
     const BlockW& b = m->blk[l];
     const float* mb = mod + (size_t)l * 6 * d;
     float* qkv = w.qkv + (size_t)l * N * 3 * d;
     DC_CK(cudaMemcpyAsync(w.hin + l * Nd, w.hcur, Nd * 4, cudaMemcpyDeviceToDevice, st));
-    DC_CK(dc::launch_ln_mod_f32(w.hcur, N, d, mb, mb + d, w.abuf, st));
+    DC_LAUNCH(DC_PROF_JVP_OTHER, 0.0, 0.0,
+              dc::launch_ln_mod_f32(w.hcur, N, d, mb, mb + d, w.abuf, st));
     dc::JEpi e1{};
     e1.mode = dc::kJStore; e1.bias = b.b_qkv; e1.out = qkv;
-    DC_CK(dc::launch_gemm_f32w<T>(w.abuf, static_cast<const T*>(b.w_qkv), N, 3 * d, d, e1, st));
-    DC_CK(dc::launch_attention_f32_jvp(qkv, nullptr, N, d, w.heads, w.dh, 1, w.obuf, nullptr, st));
+    DC_LAUNCH(DC_PROF_JVP_GEMM, 2.0 * (N) * (3 * d) * (d), 0.0,
+              dc::launch_gemm_f32w<T>(w.abuf, static_cast<const T*>(b.w_qkv), N, 3 * d, d, e1, st));
+    // primal attention: 4 N^2 dh flops per head (scores and weighted sum)
+    DC_LAUNCH(DC_PROF_JVP_ATTENTION, 4.0 * w.heads * (double)N * N * w.dh, 0.0,
+              dc::launch_attention_f32_jvp(qkv, nullptr, N, d, w.heads, w.dh, 1, w.obuf, nullptr,
+                                           st));
     dc::JEpi e2{};
     e2.mode = dc::kJGatedAdd; e2.bias = b.b_o; e2.gate = mb + 2 * d; e2.base = w.hcur; e2.out = w.hcur;
-    DC_CK(dc::launch_gemm_f32w<T>(w.obuf, static_cast<const T*>(b.w_o), N, d, d, e2, st));
+    DC_LAUNCH(DC_PROF_JVP_GEMM, 2.0 * (N) * (d) * (d), 0.0,
+              dc::launch_gemm_f32w<T>(w.obuf, static_cast<const T*>(b.w_o), N, d, d, e2, st));
     DC_CK(cudaMemcpyAsync(w.h1 + l * Nd, w.hcur, Nd * 4, cudaMemcpyDeviceToDevice, st));
-    DC_CK(dc::launch_ln_mod_f32(w.hcur, N, d, mb + 3 * d, mb + 4 * d, w.abuf, st));
+    DC_LAUNCH(DC_PROF_JVP_OTHER, 0.0, 0.0,
+              dc::launch_ln_mod_f32(w.hcur, N, d, mb + 3 * d, mb + 4 * d, w.abuf, st));
     dc::JEpi e3{};
     e3.mode = dc::kJGeluPrimal; e3.bias = b.b_1; e3.out = w.z + (size_t)l * N * md; e3.out2 = w.mbuf;
-    DC_CK(dc::launch_gemm_f32w<T>(w.abuf, static_cast<const T*>(b.w_1), N, md, d, e3, st));
+    DC_LAUNCH(DC_PROF_JVP_GEMM, 2.0 * (N) * (md) * (d), 0.0,
+              dc::launch_gemm_f32w<T>(w.abuf, static_cast<const T*>(b.w_1), N, md, d, e3, st));
     dc::JEpi e4{};
     e4.mode = dc::kJGatedAdd; e4.bias = b.b_2; e4.gate = mb + 5 * d; e4.base = w.hcur; e4.out = w.hcur;
-    DC_CK(dc::launch_gemm_f32w<T>(w.mbuf, static_cast<const T*>(b.w_2), N, d, md, e4, st));
+    DC_LAUNCH(DC_PROF_JVP_GEMM, 2.0 * (N) * (d) * (md), 0.0,
+              dc::launch_gemm_f32w<T>(w.mbuf, static_cast<const T*>(b.w_2), N, d, md, e4, st));
   }
   DC_CK(cudaMemcpyAsync(w.hL, w.hcur, Nd * 4, cudaMemcpyDeviceToDevice, st));
   return DC_OK;
@@ -727,33 +741,44 @@ dc_status tangent_f32(dc_model* m, ResponseWork<T>& w, const float* dx, int Tn, 
                       float* dv, cudaStream_t st) {
   const int N = w.N, d = w.d, md = w.md, R = Tn * N;
   const size_t Nd = (size_t)N * d;
-  DC_CK(dc::launch_embed_f32<T>(dx, m->w_eT, nullptr, static_cast<const T*>(nullptr), R, N, w.C, d,
-                                w.th, st));
+  DC_LAUNCH(DC_PROF_JVP_OTHER, 0.0, 0.0,
+            dc::launch_embed_f32<T>(dx, m->w_eT, nullptr, static_cast<const T*>(nullptr), R, N,
+                                    w.C, d, w.th, st));
   for (int l = 0; l < w.L; ++l) {
     const BlockW& b = m->blk[l];
     const float* mb = mod + (size_t)l * 6 * d;
-    DC_CK(dc::launch_ln_jvp_f32(w.hin + l * Nd, w.th, N, Tn, d, mb + d, w.ta, st));
+    DC_LAUNCH(DC_PROF_JVP_OTHER, 0.0, 0.0,
+              dc::launch_ln_jvp_f32(w.hin + l * Nd, w.th, N, Tn, d, mb + d, w.ta, st));
     dc::JEpi e1{};
     e1.mode = dc::kJStore; e1.out = w.tqkv;
-    DC_CK(dc::launch_gemm_f32w<T>(w.ta, static_cast<const T*>(b.w_qkv), R, 3 * d, d, e1, st));
-    DC_CK(dc::launch_attention_f32_jvp(w.qkv + (size_t)l * N * 3 * d, w.tqkv, N, d, w.heads, w.dh,
-                                       Tn, nullptr, w.tout, st));
+    DC_LAUNCH(DC_PROF_JVP_GEMM, 2.0 * (R) * (3 * d) * (d), 0.0,
+              dc::launch_gemm_f32w<T>(w.ta, static_cast<const T*>(b.w_qkv), R, 3 * d, d, e1, st));
+    // tangent: scores, their tangent and the three weighted sums, 12 N^2 dh
+    DC_LAUNCH(DC_PROF_JVP_ATTENTION, 12.0 * Tn * w.heads * (double)N * N * w.dh, 0.0,
+              dc::launch_attention_f32_jvp(w.qkv + (size_t)l * N * 3 * d, w.tqkv, N, d, w.heads,
+                                           w.dh, Tn, nullptr, w.tout, st));
     dc::JEpi e2{};
     e2.mode = dc::kJGatedAdd; e2.gate = mb + 2 * d; e2.base = w.th; e2.out = w.th;
-    DC_CK(dc::launch_gemm_f32w<T>(w.tout, static_cast<const T*>(b.w_o), R, d, d, e2, st));
-    DC_CK(dc::launch_ln_jvp_f32(w.h1 + l * Nd, w.th, N, Tn, d, mb + 4 * d, w.ta, st));
+    DC_LAUNCH(DC_PROF_JVP_GEMM, 2.0 * (R) * (d) * (d), 0.0,
+              dc::launch_gemm_f32w<T>(w.tout, static_cast<const T*>(b.w_o), R, d, d, e2, st));
+    DC_LAUNCH(DC_PROF_JVP_OTHER, 0.0, 0.0,
+              dc::launch_ln_jvp_f32(w.h1 + l * Nd, w.th, N, Tn, d, mb + 4 * d, w.ta, st));
     dc::JEpi e3{};
     e3.mode = dc::kJGeluGrad; e3.out = w.tm; e3.z = w.z + (size_t)l * N * md; e3.zrows = N;
-    DC_CK(dc::launch_gemm_f32w<T>(w.ta, static_cast<const T*>(b.w_1), R, md, d, e3, st));
+    DC_LAUNCH(DC_PROF_JVP_GEMM, 2.0 * (R) * (md) * (d), 0.0,
+              dc::launch_gemm_f32w<T>(w.ta, static_cast<const T*>(b.w_1), R, md, d, e3, st));
     dc::JEpi e4{};
     e4.mode = dc::kJGatedAdd; e4.gate = mb + 5 * d; e4.base = w.th; e4.out = w.th;
-    DC_CK(dc::launch_gemm_f32w<T>(w.tm, static_cast<const T*>(b.w_2), R, d, md, e4, st));
+    DC_LAUNCH(DC_PROF_JVP_GEMM, 2.0 * (R) * (d) * (md), 0.0,
+              dc::launch_gemm_f32w<T>(w.tm, static_cast<const T*>(b.w_2), R, d, md, e4, st));
   }
   const float* fsh = mod + (size_t)6 * w.L * d;
-  DC_CK(dc::launch_ln_jvp_f32(w.hL, w.th, N, Tn, d, fsh + d, w.ta, st));
+  DC_LAUNCH(DC_PROF_JVP_OTHER, 0.0, 0.0,
+              dc::launch_ln_jvp_f32(w.hL, w.th, N, Tn, d, fsh + d, w.ta, st));
   dc::JEpi ef{};
   ef.mode = dc::kJStore; ef.out = dv;
-  DC_CK(dc::launch_gemm_f32w<float>(w.ta, m->w_f, R, w.C, d, ef, st));
+  DC_LAUNCH(DC_PROF_JVP_GEMM, 2.0 * (R) * (w.C) * (d), 0.0,
+              dc::launch_gemm_f32w<float>(w.ta, m->w_f, R, w.C, d, ef, st));
   return DC_OK;
 }
 
@@ -815,8 +840,9 @@ dc_status anchor_response_impl(dc_model* m, const float* noise, const dc_traject
     const float dsig_t = (float)(sig[t] - sig[t - 1]);
     for (int c = first_at[t]; c < first_at[t + 1]; ++c) {
       DC_TRY(interface_f32<T>(m, w, x_at(t), r_at(chains[c].first), mod_at(t), w.vtmp, st));
-      DC_CK(dc::launch_scaled_diff(w.vtmp, w.vbar + (size_t)(t - 1) * NC, dsig_t, dxs + c * NC, NC,
-                                   st));
+      DC_LAUNCH(DC_PROF_JVP_OTHER, 0.0, 0.0,
+                dc::launch_scaled_diff(w.vtmp, w.vbar + (size_t)(t - 1) * NC, dsig_t, dxs + c * NC,
+                                       NC, st));
     }
     if (step > K) break;
     // carry every live chain through step `step`: dx += dsig J dx
@@ -827,7 +853,8 @@ dc_status anchor_response_impl(dc_model* m, const float* noise, const dc_traject
     for (int g0 = 0; g0 < live; g0 += Tmax) {
       const int Tn = std::min(Tmax, live - g0);
       DC_TRY(tangent_f32<T>(m, w, dxs + (size_t)g0 * NC, Tn, mod_at(step), w.tv, st));
-      DC_CK(dc::launch_axpy_f32(dxs + (size_t)g0 * NC, w.tv, dsig, (size_t)Tn * NC, st));
+      DC_LAUNCH(DC_PROF_JVP_OTHER, 0.0, 0.0,
+                dc::launch_axpy_f32(dxs + (size_t)g0 * NC, w.tv, dsig, (size_t)Tn * NC, st));
     }
   }
   // Eq. 7 on the host in fp64: G_{j,h} = sum_{l<=h} P_{j+l} e_{j,l}
