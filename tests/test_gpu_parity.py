@@ -481,3 +481,51 @@ def test_anchor_response_bf16_small_vs_oracle(dc):
     record("anchor_response_bf16", dict(rel=rel(got, ref),
                                          rel_max=float(np.max(np.abs(got[mask] - ref[mask]) / ref[mask]))))
     assert rel(got, ref) <= 2e-2
+
+
+def test_measured_responses_end_to_end(dc):
+    """The method with measured responses instead of synthetic ones, on the
+    fp32 workload: anchors -> q tables (dc_anchor_response) and drift tables
+    (dc_anchor_drift) for both anchors -> tau (dc_calibrate_budget) ->
+    dc_denoise, against the oracle doing the same with its own tables."""
+    from oracle import dit as O
+    from oracle import response as R
+    wl = WORKLOADS["c1"]
+    K, H = wl.steps, wl.h_max
+    w = gen.weights(wl)
+    om = Ctl.build(wl, w)
+    sig = gen.sigmas(K)
+    clips = gen.calibration_trajectories(wl)
+    stats = [P.motion_stats(c) for c in clips]
+    anc = P.select_anchors([s[0] for s in stats], [s[1] for s in stats])
+    noise = gen.anchor_noise(wl)
+    ref_tabs = {}
+    for i, key in ((anc["i0"], "0"), (anc["i1"], "1")):
+        ref_tabs["q" + key] = R.response_table(om, noise, clips[i], sig, K, H)[0]
+        ref_tabs["d" + key] = Ctl.anchor_trace_drift(om, noise, clips[i], sig, K, H)[0]
+    tau_ref, reached = P.calibrate_budget(list(clips), anc, ref_tabs, wl.target(), K, H)
+    assert reached == 1
+
+    model = dc.Model(wl, gen.flat_blob(wl, w))
+    nz = torch.tensor(noise, device="cuda")
+    tabs = {}
+    for i, key in ((anc["i0"], "0"), (anc["i1"], "1")):
+        tabs["q" + key] = dc.anchor_response(model, nz, clips[i], K, sig, H)
+        tabs["d" + key] = dc.anchor_drift(model, nz, clips[i], K, sig, H)
+    for k in ("q0", "q1", "d0", "d1"):
+        assert rel(tabs[k], np.asarray(ref_tabs[k])) <= 1e-4, k
+    A = dc.AnchorArgs(K, H, anc, tabs)
+    tau, reached = dc.calibrate_budget(list(clips), A, wl.target(), K)
+    assert reached == 1 and abs(tau - tau_ref) <= 1e-4 * tau_ref
+    x1 = gen.latents(wl)
+    trajs = gen.scene_trajectories(wl)
+    ref = Ctl.denoise(om, x1, trajs, sig, anc, ref_tabs, tau_ref, K, H)
+    lat = torch.tensor(x1, device="cuda")
+    st = dc.denoise(model, lat, list(trajs), dc.SchedArgs(K, sig, A, tau))
+    torch.cuda.synchronize()
+    model.close()
+    for s in range(len(trajs)):
+        assert st["planned"][s].tolist()[1:] == ref["plans"][s]["actions"][1:]
+    record("measured_responses_end_to_end", dict(tau=tau, tau_ref=tau_ref,
+                                                  rel_x=rel(lat.cpu().numpy(), ref["x"])))
+    assert rel(lat.cpu().numpy(), ref["x"]) <= 1e-4
