@@ -21,9 +21,9 @@
 // `ref` that only moves when the row's max exceeds it by more than 8 (log2
 // units); when it moves, the row of O_t (and the row sum) is rescaled by
 // exp2(ref_old - ref_new) once PV_{t,j-1} has landed and before P_{t,j} is
-// released.  3/8 of the exponentials run on the FMA/ALU pipes (Cody-Waite
-// split into integer and fraction, degree-3 minimax polynomial for 2^r on
-// [0, 1], max relative error 8.6e-5) to relieve the MUFU unit.  V is consumed
+// released.  Every exponential runs on MUFU (ex2.approx): moving a share of
+// them to a polynomial on the FMA pipe, as done on other parts, measured
+// slower here (the softmax is bound by issue slots, not by MUFU).  V is consumed
 // as an MN-major operand straight from its [keys][dh] layout.  Keys beyond N
 // are masked (last tile only).  Every mbarrier wait is bounded.
 #include <math.h>
@@ -36,7 +36,6 @@ namespace dc {
 namespace {
 
 constexpr float kRefSlack = 8.0f;  // move the reference max only beyond this (log2 units)
-constexpr int kPoly8 = 3;          // of every 8 exponentials, this many on the FMA pipe
 constexpr int kStages = 3;         // K and V ring depth
 
 template <int DHP, int NQ>
@@ -129,46 +128,20 @@ __device__ __forceinline__ float fmax3f(float a, float b, float c) {
   return d;
 }
 
-// 2^x for a pair on the FMA/ALU pipes, given y = x - 1/2 (x <= kRefSlack):
-// y is clamped at -126.5 so the result stays a tiny normal/subnormal, n =
-// round(y) = floor(x) comes from rounding against 1.5 * 2^23 (whose bit
-// pattern, shifted left by 23, is n << 23), r' = y - n in [-1/2, 1/2], and
-// 2^(r' + 1/2) is a degree-3 minimax polynomial (the [0, 1] minimax for 2^r
-// re-expanded around 1/2) whose exponent field receives n.
-__device__ __forceinline__ float2 ex2_poly2c(float2 y) {
-  const float magic = 12582912.0f;  // 1.5 * 2^23
-  y = make_float2(fmaxf(y.x, -126.5f), fmaxf(y.y, -126.5f));
-  const float2 t = fadd2(y, make_float2(magic, magic));
-  const float2 n = fadd2(t, make_float2(-magic, -magic));
-  const float2 r = fadd2(y, make_float2(-n.x, -n.y));
-  float2 q = ffma2(make_float2(7.706703991e-02f, 7.706703991e-02f), r,
-                   make_float2(3.432455659e-01f, 3.432455659e-01f));
-  q = ffma2(q, r, make_float2(9.805620313e-01f, 9.805620313e-01f));
-  q = ffma2(q, r, make_float2(1.414103031e+00f, 1.414103031e+00f));
-  return make_float2(__uint_as_float(__float_as_uint(q.x) + (__float_as_uint(t.x) << 23)),
-                     __uint_as_float(__float_as_uint(q.y) + (__float_as_uint(t.y) << 23)));
-}
-
-// One 32-column chunk: p = 2^(s * scale - ref) (kPoly8 of every 8 on the FMA
-// pipe), masked beyond `valid`, row sum on two packed chains, and the chunk
-// packed into 16 bf16 pairs (even key in the low half) for P in TMEM.
+// One 32-column chunk: p = 2^(s * scale - ref), masked beyond `valid`, row
+// sum on two packed chains, and the chunk packed into 16 bf16 pairs (even
+// key in the low half) for P in TMEM.
 template <bool MASKED>
 __device__ __forceinline__ void p_chunk(const uint32_t (&v)[32], int c, int valid,
                                         float scale_log2, float neg_ref, float2 (&rs)[2],
                                         uint32_t* pk) {
   const float2 sc = make_float2(scale_log2, scale_log2);
   const float2 nr = make_float2(neg_ref, neg_ref);
-  const float2 nrh = make_float2(neg_ref - 0.5f, neg_ref - 0.5f);
 #pragma unroll
   for (int e = 0; e < 32; e += 2) {
     const float2 s2 = make_float2(__uint_as_float(v[e]), __uint_as_float(v[e + 1]));
-    float2 p;
-    if (((e >> 1) & 7) >= 8 - kPoly8) {
-      p = ex2_poly2c(ffma2(s2, sc, nrh));
-    } else {
-      const float2 x = ffma2(s2, sc, nr);
-      p = make_float2(ex2_mufu(x.x), ex2_mufu(x.y));
-    }
+    const float2 x = ffma2(s2, sc, nr);
+    float2 p = make_float2(ex2_mufu(x.x), ex2_mufu(x.y));
     if (MASKED) {
       if (c * 32 + e >= valid) p.x = 0.f;
       if (c * 32 + e + 1 >= valid) p.y = 0.f;
