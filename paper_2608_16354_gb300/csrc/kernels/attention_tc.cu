@@ -199,9 +199,9 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
     mbar_init(&bar->q_full, 1);
     for (int b = 0; b < kStages; ++b) {
       mbar_init(&bar->k_full[b], 1);
-      mbar_init(&bar->k_empty[b], 1);
+      mbar_init(&bar->k_empty[b], NQ);  // every query tile's MMA warp releases it
       mbar_init(&bar->v_full[b], 1);
-      mbar_init(&bar->v_empty[b], 1);
+      mbar_init(&bar->v_empty[b], NQ);
     }
     for (int t = 0; t < NQ; ++t) {
       mbar_init(&bar->s_full[t], 1);
@@ -209,7 +209,7 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
       mbar_init(&bar->p_full[t], 4);
       mbar_init(&bar->p_free[t], 1);
     }
-    mbar_init(&bar->drain, 1);
+    mbar_init(&bar->drain, NQ);
     fence_barrier_init();
     tma_prefetch_desc(&tm);
   }
@@ -313,70 +313,63 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
         if (last_k[b] >= 0) mbar_wait_warp(&bar->k_full[b], (uint32_t)last_k[b], err, kDevTimeoutTma);
         if (last_v[b] >= 0) mbar_wait_warp(&bar->v_full[b], (uint32_t)last_v[b], err, kDevTimeoutTma);
       }
-    } else if (warp == 1) {
+    } else if (warp >= 1 && warp <= NQ) {
       // ------------------------------------------------------------ MMA
-      // Fixed order with blocking waits.  Round j issues S_{t,j} for every
-      // query tile (each needs K_j and S_{t,j-1} read by its softmax, which
-      // happens at the start of that softmax tile), then PV_{t,j-1} (each
-      // needs P_{t,j-1} and V_{j-1}).  Nothing waited for here depends on a
-      // later issue, so the order cannot deadlock.  The whole warp runs the
-      // loop with uniform descriptors; one elected lane (the same one
-      // throughout, as tcgen05.commit tracks the issuing thread) issues.
+      // One warp per query tile t, fixed order with blocking waits.  Round j
+      // issues S_{t,j} (needs K_j and S_{t,j-1} read by the softmax, which
+      // happens at the start of that softmax tile), then PV_{t,j-1} (needs
+      // P_{t,j-1} and V_{j-1}).  Nothing waited for depends on a later issue
+      // of this warp or on the other tile's warp, so the order cannot
+      // deadlock.  The whole warp runs the loop with uniform descriptors; one
+      // elected lane (the same one throughout, as tcgen05.commit tracks the
+      // issuing thread) issues.
+      const int t = warp - 1;
       bool ok = mbar_wait_warp(&bar->q_full, 0, err, kDevTimeoutMma);
       // descriptor + (byte offset >> 4) moves the start address (no carry:
       // shared-memory addresses are below 256 KB)
-      const uint64_t dQ = sw128_kmajor_desc(smem_u32(smem + Cfg::kOffQ));
+      const uint64_t dQ = sw128_kmajor_desc(smem_u32(smem + Cfg::kOffQ + t * Cfg::kTileBytes));
       const uint64_t dK = sw128_kmajor_desc(smem_u32(smem + Cfg::kOffK));
       const uint64_t dV = sw128_mnmajor_desc(smem_u32(smem + Cfg::kOffV));
       for (int j = 0; j <= n_kv && ok; ++j) {
         if (j < n_kv) {
           const int kb = j % kStages;
-          ok = mbar_wait_warp(&bar->k_full[kb], (uint32_t)(j / kStages) & 1, err, kDevTimeoutMma);
-          for (int t = 0; t < NQ && ok; ++t) {
-            ok = mbar_wait_warp(&bar->s_free[t], ((uint32_t)j & 1) ^ 1, err, kDevTimeoutMma);
-            if (!ok) break;
-            tc_fence_after();
-            if (elect_one()) {
-#pragma unroll
-              for (int kk = 0; kk < DHP / 16; ++kk) {
-                const uint32_t off = (kk >> 2) * 16384 + (kk & 3) * 32;
-                tc_mma_f16(tmem + Cfg::kColS + t * 128,
-                           dQ + ((uint32_t)(t * Cfg::kTileBytes + off) >> 4),
-                           dK + ((uint32_t)(kb * Cfg::kTileBytes + off) >> 4), kIdS,
-                           kk > 0 ? 1u : 0u);
-              }
-              tc_commit(&bar->s_full[t]);
-            }
-            __syncwarp();
-          }
+          ok = mbar_wait_warp(&bar->k_full[kb], (uint32_t)(j / kStages) & 1, err, kDevTimeoutMma) &&
+               mbar_wait_warp(&bar->s_free[t], ((uint32_t)j & 1) ^ 1, err, kDevTimeoutMma);
           if (!ok) break;
-          if (elect_one()) tc_commit(&bar->k_empty[kb]);
+          tc_fence_after();
+          if (elect_one()) {
+#pragma unroll
+            for (int kk = 0; kk < DHP / 16; ++kk) {
+              const uint32_t off = (kk >> 2) * 16384 + (kk & 3) * 32;
+              tc_mma_f16(tmem + Cfg::kColS + t * 128, dQ + (off >> 4),
+                         dK + ((uint32_t)(kb * Cfg::kTileBytes + off) >> 4), kIdS,
+                         kk > 0 ? 1u : 0u);
+            }
+            tc_commit(&bar->s_full[t]);
+            tc_commit(&bar->k_empty[kb]);
+          }
           __syncwarp();
         }
         if (j >= 1) {
           const int jp = j - 1;
           const int vb = jp % kStages;
-          ok = mbar_wait_warp(&bar->v_full[vb], (uint32_t)(jp / kStages) & 1, err, kDevTimeoutMma);
-          for (int t = 0; t < NQ && ok; ++t) {
-            ok = mbar_wait_warp(&bar->p_full[t], (uint32_t)jp & 1, err, kDevTimeoutMma);
-            if (!ok) break;
-            tc_fence_after();
-            if (elect_one()) {
-#pragma unroll
-              for (int kk = 0; kk < 8; ++kk) {
-#pragma unroll
-                for (int a = 0; a < Cfg::kAtoms; ++a)
-                  tc_mma_f16_ta(tmem + Cfg::kColO + t * DHP + a * 64,
-                                tmem + Cfg::kColP + t * 64 + kk * 8,
-                                dV + ((uint32_t)(vb * Cfg::kTileBytes + a * 16384 + kk * 2048) >> 4),
-                                kIdPV, (jp > 0 || kk > 0) ? 1u : 0u);
-              }
-              tc_commit(&bar->p_free[t]);
-            }
-            __syncwarp();
-          }
+          ok = mbar_wait_warp(&bar->v_full[vb], (uint32_t)(jp / kStages) & 1, err, kDevTimeoutMma) &&
+               mbar_wait_warp(&bar->p_full[t], (uint32_t)jp & 1, err, kDevTimeoutMma);
           if (!ok) break;
-          if (elect_one()) tc_commit(&bar->v_empty[vb]);
+          tc_fence_after();
+          if (elect_one()) {
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk) {
+#pragma unroll
+              for (int a = 0; a < Cfg::kAtoms; ++a)
+                tc_mma_f16_ta(tmem + Cfg::kColO + t * DHP + a * 64,
+                              tmem + Cfg::kColP + t * 64 + kk * 8,
+                              dV + ((uint32_t)(vb * Cfg::kTileBytes + a * 16384 + kk * 2048) >> 4),
+                              kIdPV, (jp > 0 || kk > 0) ? 1u : 0u);
+            }
+            tc_commit(&bar->p_free[t]);
+            tc_commit(&bar->v_empty[vb]);
+          }
           __syncwarp();
         }
       }
