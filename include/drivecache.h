@@ -162,6 +162,19 @@ dc_status dc_replan(const dc_anchor_responses* anc, double D, int k_refresh, dou
 dc_status dc_calibrate_budget(const dc_trajectory* clips, int n, const dc_anchor_responses* anc,
                               int target, int T, double* tau, int* reached);
 
+/* Sec. 3.2 model-specific legality as the L(k, h) mask of Eq. 10: writes
+ * out[k*(H_max+1)+h] = 1 iff reusing at step k with cache age h (refresh at
+ * j = k - h) is allowed, for k = 0..K, h = 0..H_max (caller-owned
+ * [K+1][H_max+1] bytes).  Always 1 <= h <= H_max and k >= 2; in addition
+ *  expert_boundary b > 0: two experts (steps 1..b, b+1..K) and no run
+ *    crosses from one to the other (j and k in the same expert);
+ *  segment_len T > 0: autoregressive segments of T steps with caches local
+ *    to one segment ((j-1)/T == (k-1)/T), so every segment starts computed;
+ *  no_cache_until p > 0: steps 1..p are native no-cache steps (k > p).
+ * 0 disables a rule.  Pass the result as dc_anchor_responses.legal. */
+dc_status dc_legal_mask(int K, int H_max, int expert_boundary, int segment_len,
+                        int no_cache_until, unsigned char* out);
+
 /* ------------------------------------------------------------------ model */
 
 /* Shape of the synthetic DiT.  n_tokens = views x frames x rows x cols

@@ -54,7 +54,7 @@ def calibrate(model, wl, calib_poses, noise, sig, q0, q1, target, eps=P.EPS):
 
 
 def denoise(model, x1, trajs, sig, anc, tables, tau, K, H, veto=True, forced=None,
-            eps=P.EPS, keep_trace=False, variant=P.DRIVECACHE):
+            eps=P.EPS, keep_trace=False, variant=P.DRIVECACHE, legal=None):
     """Run the sampler over B scenes with the causal controller.
 
     forced: optional [B][K+1] actions to replay verbatim (no planning, no
@@ -62,10 +62,11 @@ def denoise(model, x1, trajs, sig, anc, tables, tau, K, H, veto=True, forced=Non
     ablations, fixed-interval baseline); SHUFFLED plans scene s from the
     trajectory of scene (s+1) mod B, FIXED_INTERVAL runs its schedule with no
     charge and no checks, and refusals under FIXED_PLACEMENT keep the fixed
-    pattern (no replan).  Returns dict(x, plans, executed, log, stats, trace)."""
+    pattern (no replan).  legal: optional L(k, h) callable for planning and
+    replanning.  Returns dict(x, plans, executed, log, stats, trace)."""
     B = len(trajs)
     plan_traj = [trajs[(s + 1) % B] if variant == P.SHUFFLED else trajs[s] for s in range(B)]
-    plans = [P.plan_scene_variant(plan_traj[s], anc, tables, tau, K, H, variant, eps)
+    plans = [P.plan_scene_variant(plan_traj[s], anc, tables, tau, K, H, variant, eps, legal)
              for s in range(B)]
     fixed = variant == P.FIXED_INTERVAL
     acts = [list(p["actions"]) for p in plans]
@@ -108,7 +109,7 @@ def denoise(model, x1, trajs, sig, anc, tables, tau, K, H, veto=True, forced=Non
                         stats[s]["n_veto"] += 1
                         if variant != P.FIXED_PLACEMENT:
                             stats[s]["n_replan"] += 1
-                            a, _, _ = P.plan_suffix(tabs["c"], K, H, k, tau - S["C"])
+                            a, _, _ = P.plan_suffix(tabs["c"], K, H, k, tau - S["C"], legal)
                             for kk in range(k, K + 1):
                                 acts[s][kk] = a[kk]
             if reuse:

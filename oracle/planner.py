@@ -21,6 +21,8 @@ Sections followed:
   Table 3 ablations (no motion prior, shuffled trajectory, translation only,
           rotation only, fixed placement) and the fixed-interval baseline of
           Table 1, as planner variants
+  Sec. 3.2 model-specific legality: expert boundaries, segment-local caches
+          and no-cache steps as masks L(k, h)
 """
 
 import math
@@ -485,3 +487,37 @@ def calibrate_budget_variant(clip_poses, anc, tables, target, K, H, variant, eps
         if _median([float(x) for x in counts]) >= target:
             return tau, 1
     return ordered[-1], 0
+
+
+# ------------------------------------------ Sec. 3.2 model-specific legality
+
+def legal_mask(K, H, expert_boundary=0, segment_len=0, no_cache_until=0):
+    """L(k, h) of Eq. 10 for the model-specific rules of Sec. 3.2, as a
+    [K+1][H+1] 0/1 list (index [k][h]).  A reuse at step k with cache age h
+    refreshes at j = k - h.  READINGS:
+      * always: 1 <= h <= H_max and k >= 2 (the first step is computed);
+      * expert_boundary b > 0 (two experts, steps 1..b and b+1..K): j and k
+        lie in the same expert -- no run crosses the boundary;
+      * segment_len T > 0 (autoregressive segments of T steps, caches local
+        to one denoising call): floor((j-1)/T) == floor((k-1)/T), so the
+        first step of every segment is computed;
+      * no_cache_until p > 0 (native no-cache steps 1..p): k > p."""
+    m = [[0] * (H + 1) for _ in range(K + 1)]
+    for k in range(2, K + 1):
+        for h in range(1, H + 1):
+            j = k - h
+            if j < 1:
+                continue
+            if expert_boundary > 0 and (j <= expert_boundary) != (k <= expert_boundary):
+                continue
+            if segment_len > 0 and (j - 1) // segment_len != (k - 1) // segment_len:
+                continue
+            if no_cache_until > 0 and k <= no_cache_until:
+                continue
+            m[k][h] = 1
+    return m
+
+
+def legal_fn(mask):
+    """The callable form plan_suffix and dp_tables take."""
+    return lambda k, h: 1 <= h < len(mask[0]) and k >= 2 and mask[k][h] != 0

@@ -109,6 +109,7 @@ def lib():
         "dc_denoise": (st, [C.c_void_p, C.c_void_p, P(Cond), P(Sched), C.c_void_p, P(RunStats)]),
         "dc_denoise_host": (st, [C.c_void_p, P(C.c_float), P(Cond), P(Sched), C.c_void_p,
                                  P(RunStats)]),
+        "dc_legal_mask": (st, [C.c_int, C.c_int, C.c_int, C.c_int, C.c_int, P(C.c_ubyte)]),
         "dc_anchor_drift": (st, [C.c_void_p, C.c_void_p, P(Trajectory), C.c_int, P(C.c_double),
                                  C.c_int, C.c_double, P(C.c_double), C.c_void_p]),
         "dc_anchor_response": (st, [C.c_void_p, C.c_void_p, P(Trajectory), C.c_int,
@@ -191,6 +192,15 @@ class AnchorArgs:
 
     def ptr(self):
         return C.pointer(self.s)
+
+
+def legal_mask(K, H, expert_boundary=0, segment_len=0, no_cache_until=0):
+    """dc_legal_mask: the L(k, h) mask [K+1][H+1] (uint8) of the model-specific
+    rules (expert boundary, segment-local caches, no-cache steps)."""
+    out = np.zeros((K + 1, H + 1), np.uint8)
+    _check(lib().dc_legal_mask(int(K), int(H), int(expert_boundary), int(segment_len),
+                               int(no_cache_until), out.ctypes.data_as(C.POINTER(C.c_ubyte))))
+    return out
 
 
 def motion_stats(poses):

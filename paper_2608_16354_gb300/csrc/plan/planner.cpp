@@ -507,6 +507,26 @@ dc_status dc_calibrate_budget(const dc_trajectory* clips, int n, const dc_anchor
   return DC_OK;
 }
 
+dc_status dc_legal_mask(int K, int H_max, int expert_boundary, int segment_len,
+                        int no_cache_until, unsigned char* out) {
+  if (!out || K < 1 || K > 100000 || H_max < 1 || H_max > 4096 || expert_boundary < 0 ||
+      segment_len < 0 || no_cache_until < 0) {
+    dc::set_error("dc_legal_mask: NULL out, K or H_max out of range, or a negative rule");
+    return DC_ERR_INVALID_ARG;
+  }
+  const int W = H_max + 1;
+  for (int k = 0; k <= K; ++k)
+    for (int h = 0; h <= H_max; ++h) {
+      const int j = k - h;  // refresh step of the run this reuse extends
+      bool ok = k >= 2 && h >= 1 && j >= 1;
+      if (ok && expert_boundary > 0) ok = (j <= expert_boundary) == (k <= expert_boundary);
+      if (ok && segment_len > 0) ok = (j - 1) / segment_len == (k - 1) / segment_len;
+      if (ok && no_cache_until > 0) ok = k > no_cache_until;
+      out[(size_t)k * W + h] = ok ? 1 : 0;
+    }
+  return DC_OK;
+}
+
 const char* dc_status_string(dc_status s) {
   switch (s) {
     case DC_OK: return "ok";

@@ -256,3 +256,28 @@ def test_variant_arguments_are_checked(dc):
         with pytest.raises(dc.DCError):
             dc.plan(poses, fi, bad, K)
     assert dc.plan(poses, fi, 2.0, K)["n_reuse"] == 2
+
+
+# ---------------------------------- model-specific legality (Sec. 3.2)
+
+@pytest.mark.parametrize("rules", [(0, 0, 0), (7, 0, 0), (0, 5, 0), (0, 0, 4), (9, 6, 2)])
+def test_legal_mask_bit_exact_and_planning(dc, rules):
+    K, H = 25, 4
+    m = dc.legal_mask(K, H, *rules)
+    assert m.tolist() == P.legal_mask(K, H, *rules)
+    rng = random.Random(sum(rules))
+    tabs = _rand_tables(rng, K, H, dyadic=True)
+    anc = dict(L0=0.0, T0=0.0, L1=40.0, T1=1.5, valid=1)
+    A = dc.AnchorArgs(K, H, anc, tabs, legal=m)
+    for v in (6.0, 12.0):
+        poses = gen.unicycle(v, 0.2, 29)
+        got = dc.plan(poses, A, math.inf, K)
+        ref = P.plan_scene(poses, anc, tabs, math.inf, K, H, legal=P.legal_fn(P.legal_mask(K, H, *rules)))
+        assert got["actions"][1:] == ref["actions"][1:] and got["cost"] == ref["cost"]
+
+
+def test_legal_mask_arguments(dc):
+    with pytest.raises(dc.DCError):
+        dc.legal_mask(0, 4)
+    with pytest.raises(dc.DCError):
+        dc.legal_mask(10, 4, expert_boundary=-1)

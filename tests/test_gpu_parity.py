@@ -81,15 +81,18 @@ def _calibrated(wl):
 
 
 def _compare_controller(dc, wl, w, om, sig, anc, tabs, tau, tol, bf16, variant=P.DRIVECACHE,
-                        trajs=None):
+                        trajs=None, rules=None):
     K, H = wl.steps, wl.h_max
     x1 = gen.latents(wl)
     trajs = gen.scene_trajectories(wl) if trajs is None else trajs
-    ref = Ctl.denoise(om, x1, trajs, sig, anc, tabs, tau, K, H, variant=variant)
+    legal = None if rules is None else P.legal_fn(P.legal_mask(K, H, *rules))
+    ref = Ctl.denoise(om, x1, trajs, sig, anc, tabs, tau, K, H, variant=variant, legal=legal)
     model = dc.Model(wl, gen.flat_blob(wl, w))
     lat = torch.tensor(x1, device="cuda")
+    mask = None if rules is None else dc.legal_mask(K, H, *rules)
     st = dc.denoise(model, lat, list(trajs),
-                    dc.SchedArgs(K, sig, dc.AnchorArgs(K, H, anc, tabs, variant=variant), tau))
+                    dc.SchedArgs(K, sig, dc.AnchorArgs(K, H, anc, tabs, legal=mask, variant=variant),
+                                 tau))
     torch.cuda.synchronize()
     got = lat.cpu().numpy()
     model.close()
@@ -152,6 +155,32 @@ def test_tiny_fp32_controller_variants(dc, variant):
         assert int(np.sum(st["checked"])) == 0
         for s in range(3):
             assert st["executed"][s].tolist()[1:] == P.even_schedule(int(tau), K, H)[1:]
+
+
+@pytest.mark.parametrize("rules", [(5, 0, 0), (0, 4, 0), (0, 0, 3), (6, 3, 2)])
+def test_tiny_fp32_controller_with_legality(dc, rules):
+    """Model-specific legality (expert boundary, segment-local caches,
+    no-cache steps): the sampler plans and replans under the mask exactly as
+    the oracle does, and no executed run breaks it."""
+    base = WORKLOADS["c1"]
+    w, om, sig, anc, tabs, _ = _calibrated(base)
+    wl = base.with_(batch=3)
+    K, H = wl.steps, wl.h_max
+    tau, _ = P.calibrate_budget(gen.calibration_trajectories(base), anc, tabs, wl.target(), K, H,
+                                legal=P.legal_fn(P.legal_mask(K, H, *rules)))
+    trajs = [gen.unicycle(2.0, 0.0, wl.n_poses), gen.unicycle(5.0, 0.15, wl.n_poses),
+             gen.unicycle(1.0, 0.4, wl.n_poses)]
+    st, ref = _compare_controller(dc, wl, w, om, sig, anc, tabs, tau, 1e-4, False, trajs=trajs,
+                                  rules=rules)
+    mask = P.legal_mask(K, H, *rules)
+    for s in range(3):
+        ex = st["executed"][s].tolist()
+        j = 1
+        for k in range(2, K + 1):
+            if ex[k] == P.REUSE:
+                assert mask[k][k - j] == 1, (s, k, j)
+            else:
+                j = k
 
 
 def test_tiny_fp32_anchor_drift_tables(dc):
