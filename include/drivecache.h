@@ -217,6 +217,13 @@ typedef struct { int B; const dc_trajectory* traj; } dc_cond;
  *  The planner variant is anchors->variant (DC_VAR_*).  The reduced-steps
  *  baseline of Table 2 is a plain call with fewer steps (K and sigmas of the
  *  shorter schedule) and a forced all-COMPUTE schedule.
+ *  cfg_scale: 0 = one branch; otherwise classifier-free guidance with
+ *        separate guidance branches (Sec. 3.2): every scene also runs an
+ *        unconditional branch (the null trajectory: all poses at the origin,
+ *        so its trajectory features vanish), each branch with its own cache
+ *        of r, and v = v_u + cfg_scale (v_c - v_u) drives the Euler step.  The
+ *        plan, the drift check (on x) and the charge stay per scene; both
+ *        branches compute or reuse together.  Needs 2 B <= max_batch.
  *  forced: NULL, or [B][K+1] actions replayed verbatim (no planning, no
  *        checks; step 1 is always computed). */
 typedef struct {
@@ -226,6 +233,7 @@ typedef struct {
   double tau;
   int veto;
   const unsigned char* forced;
+  double cfg_scale;
 } dc_sched;
 
 /* Optional per-call record (every pointer may be NULL; arrays caller-owned).

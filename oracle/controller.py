@@ -54,7 +54,7 @@ def calibrate(model, wl, calib_poses, noise, sig, q0, q1, target, eps=P.EPS):
 
 
 def denoise(model, x1, trajs, sig, anc, tables, tau, K, H, veto=True, forced=None,
-            eps=P.EPS, keep_trace=False, variant=P.DRIVECACHE, legal=None):
+            eps=P.EPS, keep_trace=False, variant=P.DRIVECACHE, legal=None, cfg_scale=0.0):
     """Run the sampler over B scenes with the causal controller.
 
     forced: optional [B][K+1] actions to replay verbatim (no planning, no
@@ -63,7 +63,11 @@ def denoise(model, x1, trajs, sig, anc, tables, tau, K, H, veto=True, forced=Non
     trajectory of scene (s+1) mod B, FIXED_INTERVAL runs its schedule with no
     charge and no checks, and refusals under FIXED_PLACEMENT keep the fixed
     pattern (no replan).  legal: optional L(k, h) callable for planning and
-    replanning.  Returns dict(x, plans, executed, log, stats, trace)."""
+    replanning.  cfg_scale != 0: separate guidance branches (Sec. 3.2) --
+    each scene also runs the unconditional branch (READING: the null
+    trajectory, every pose at the origin), each branch keeps its own cached
+    r, both compute or reuse together, and v = v_u + g (v_c - v_u).
+    Returns dict(x, plans, executed, log, stats, trace)."""
     B = len(trajs)
     plan_traj = [trajs[(s + 1) % B] if variant == P.SHUFFLED else trajs[s] for s in range(B)]
     plans = [P.plan_scene_variant(plan_traj[s], anc, tables, tau, K, H, variant, eps, legal)
@@ -75,7 +79,11 @@ def denoise(model, x1, trajs, sig, anc, tables, tau, K, H, veto=True, forced=Non
         for s in range(B):
             acts[s][1] = P.COMPUTE
     x = f64(x1).copy()
-    st = [dict(C=0.0, j=0, age=0, r=None, u_ref=None) for _ in range(B)]
+    st = [dict(C=0.0, j=0, age=0, r=None, r_u=None, u_ref=None) for _ in range(B)]
+    null = [np.zeros_like(np.asarray(trajs[s], np.float64)) for s in range(B)]
+
+    def guided(v_c, v_u):
+        return v_u + cfg_scale * (v_c - v_u)
     executed = [[0] * (K + 1) for _ in range(B)]
     log = [[] for _ in range(B)]
     stats = [dict(n_compute=0, n_reuse=0, n_veto=0, n_replan=0) for _ in range(B)]
@@ -114,11 +122,16 @@ def denoise(model, x1, trajs, sig, anc, tables, tau, K, H, veto=True, forced=Non
                                 acts[s][kk] = a[kk]
             if reuse:
                 v, _ = model.reuse_step(x[s], S["r"], sig[k - 1], trajs[s])
+                if cfg_scale != 0.0:
+                    v = guided(v, model.reuse_step(x[s], S["r_u"], sig[k - 1], null[s])[0])
                 S["age"] += 1
                 executed[s][k] = P.REUSE
                 stats[s]["n_reuse"] += 1
             else:
                 v, u, r = model.full_step(x[s], sig[k - 1], trajs[s])
+                if cfg_scale != 0.0:
+                    v_u, _, S["r_u"] = model.full_step(x[s], sig[k - 1], null[s])
+                    v = guided(v, v_u)
                 S["j"], S["age"], S["r"], S["u_ref"] = k, 0, r, u
                 executed[s][k] = P.COMPUTE
                 stats[s]["n_compute"] += 1

@@ -67,7 +67,7 @@ class Cond(C.Structure):
 class Sched(C.Structure):
     _fields_ = [("K", C.c_int), ("sigmas", C.POINTER(C.c_double)),
                 ("anchors", C.POINTER(AnchorResponses)), ("tau", C.c_double),
-                ("veto", C.c_int), ("forced", C.POINTER(C.c_ubyte))]
+                ("veto", C.c_int), ("forced", C.POINTER(C.c_ubyte)), ("cfg_scale", C.c_double)]
 
 
 class RunStats(C.Structure):
@@ -326,7 +326,7 @@ class StatsArgs:
 
 
 class SchedArgs:
-    def __init__(self, K, sigmas, anchors: AnchorArgs, tau, veto=True, forced=None):
+    def __init__(self, K, sigmas, anchors: AnchorArgs, tau, veto=True, forced=None, cfg_scale=0.0):
         self.sig = np.ascontiguousarray(sigmas, np.float64)
         assert self.sig.size == K + 1
         self.forced = None if forced is None else np.ascontiguousarray(forced, np.uint8)
@@ -335,6 +335,7 @@ class SchedArgs:
         s.anchors = anchors.ptr()
         s.tau, s.veto = float(tau), int(veto)
         s.forced = _bptr(self.forced) if self.forced is not None else None
+        s.cfg_scale = float(cfg_scale)
         self.anchors = anchors
         self.s = s
 

@@ -260,7 +260,7 @@ __global__ void final_compute_kernel(const float* __restrict__ hL, const float* 
                                      T* __restrict__ r, SlotMap map, int N, int d,
                                      const float* __restrict__ mod, int mod_stride, int fin_off,
                                      const float* __restrict__ w_f, const float* __restrict__ b_f,
-                                     float dsig) {
+                                     float dsig, float* __restrict__ vout) {
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;  // slot * N + tok
   const int lane = threadIdx.x & 31;
   if (row >= map.n * N) return;
@@ -295,7 +295,8 @@ __global__ void final_compute_kernel(const float* __restrict__ hL, const float* 
     const size_t xi = ((size_t)scene * N + tok) * C + lane;
     const float xo = x[xi];
     xj[xi] = xo;
-    x[xi] = xo + dsig * vc;
+    if (vout) vout[xi] = vc;  // the caller combines velocities (guidance)
+    else x[xi] = xo + dsig * vc;
   }
 }
 
@@ -305,7 +306,7 @@ __global__ void final_reuse_kernel(float* __restrict__ x, const T* __restrict__ 
                                    const T* __restrict__ pos, SlotMap map, int N, int d,
                                    const float* __restrict__ mod, int mod_stride, int fin_off,
                                    const float* __restrict__ w_f, const float* __restrict__ b_f,
-                                   float dsig) {
+                                   float dsig, float* __restrict__ vout) {
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (row >= map.n * N) return;
@@ -353,8 +354,19 @@ __global__ void final_reuse_kernel(float* __restrict__ x, const T* __restrict__ 
 #pragma unroll
     for (int c = 1; c < C; ++c)
       if (lane == c) xo = xv[c];
-    x[((size_t)scene * N + tok) * C + lane] = xo + dsig * vc;
+    const size_t xi = ((size_t)scene * N + tok) * C + lane;
+    if (vout) vout[xi] = vc;
+    else x[xi] = xo + dsig * vc;
   }
+}
+
+// Guidance: x_s += dsig (v_u + g (v_c - v_u)) with v_c = v[s], v_u = v[B + s].
+__global__ void cfg_combine_kernel(float* __restrict__ x, const float* __restrict__ v, int B,
+                                   size_t per_scene, float g, float dsig) {
+  const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (size_t)B * per_scene) return;
+  const float vc = v[i], vu = v[(size_t)B * per_scene + i];
+  x[i] = x[i] + dsig * (vu + g * (vc - vu));
 }
 
 // ------------------------------------------------------------ drift sums
@@ -529,17 +541,19 @@ template <typename T>
 cudaError_t launch_final_compute(const float* hL, const float* u, float* x, float* xj, T* r,
                                  const SlotMap& map, int N, int C, int d, const float* mod,
                                  int mod_stride, int fin_off, const float* w_f, const float* b_f,
-                                 float dsig, cudaStream_t st) {
+                                 float dsig, cudaStream_t st, float* vout) {
   if (map.n <= 0) return cudaSuccess;
   const int rows = map.n * N;
   const int threads = 256;
   const int blocks = (int)(((size_t)rows * 32 + threads - 1) / threads);
   if (C == 16) {
     DC_NV_SWITCH(nv_for(d), (final_compute_kernel<T, NV, 16><<<blocks, threads, 0, st>>>(
-                                hL, u, x, xj, r, map, N, d, mod, mod_stride, fin_off, w_f, b_f, dsig)));
+                                hL, u, x, xj, r, map, N, d, mod, mod_stride, fin_off, w_f, b_f, dsig,
+                                vout)));
   } else if (C == 4) {
     DC_NV_SWITCH(nv_for(d), (final_compute_kernel<T, NV, 4><<<blocks, threads, 0, st>>>(
-                                hL, u, x, xj, r, map, N, d, mod, mod_stride, fin_off, w_f, b_f, dsig)));
+                                hL, u, x, xj, r, map, N, d, mod, mod_stride, fin_off, w_f, b_f, dsig,
+                                vout)));
   } else {
     return cudaErrorInvalidValue;
   }
@@ -547,27 +561,30 @@ cudaError_t launch_final_compute(const float* hL, const float* u, float* x, floa
 }
 template cudaError_t launch_final_compute<float>(const float*, const float*, float*, float*, float*,
                                                  const SlotMap&, int, int, int, const float*, int,
-                                                 int, const float*, const float*, float, cudaStream_t);
+                                                 int, const float*, const float*, float, cudaStream_t,
+                                                 float*);
 template cudaError_t launch_final_compute<__nv_bfloat16>(const float*, const float*, float*, float*,
                                                          __nv_bfloat16*, const SlotMap&, int, int,
                                                          int, const float*, int, int, const float*,
-                                                         const float*, float, cudaStream_t);
+                                                         const float*, float, cudaStream_t, float*);
 
 template <typename T>
 cudaError_t launch_final_reuse(float* x, const T* r, const float* w_e, const float* b_e,
                                const T* pos, const SlotMap& map, int N, int C, int d,
                                const float* mod, int mod_stride, int fin_off, const float* w_f,
-                               const float* b_f, float dsig, cudaStream_t st) {
+                               const float* b_f, float dsig, cudaStream_t st, float* vout) {
   if (map.n <= 0) return cudaSuccess;
   const int rows = map.n * N;
   const int threads = 256;
   const int blocks = (int)(((size_t)rows * 32 + threads - 1) / threads);
   if (C == 16) {
     DC_NV_SWITCH(nv_for(d), (final_reuse_kernel<T, NV, 16><<<blocks, threads, 0, st>>>(
-                                x, r, w_e, b_e, pos, map, N, d, mod, mod_stride, fin_off, w_f, b_f, dsig)));
+                                x, r, w_e, b_e, pos, map, N, d, mod, mod_stride, fin_off, w_f, b_f, dsig,
+                                vout)));
   } else if (C == 4) {
     DC_NV_SWITCH(nv_for(d), (final_reuse_kernel<T, NV, 4><<<blocks, threads, 0, st>>>(
-                                x, r, w_e, b_e, pos, map, N, d, mod, mod_stride, fin_off, w_f, b_f, dsig)));
+                                x, r, w_e, b_e, pos, map, N, d, mod, mod_stride, fin_off, w_f, b_f, dsig,
+                                vout)));
   } else {
     return cudaErrorInvalidValue;
   }
@@ -576,12 +593,20 @@ cudaError_t launch_final_reuse(float* x, const T* r, const float* w_e, const flo
 template cudaError_t launch_final_reuse<float>(float*, const float*, const float*, const float*,
                                                const float*, const SlotMap&, int, int, int,
                                                const float*, int, int, const float*, const float*,
-                                               float, cudaStream_t);
+                                               float, cudaStream_t, float*);
 template cudaError_t launch_final_reuse<__nv_bfloat16>(float*, const __nv_bfloat16*, const float*,
                                                        const float*, const __nv_bfloat16*,
                                                        const SlotMap&, int, int, int, const float*,
                                                        int, int, const float*, const float*, float,
-                                                       cudaStream_t);
+                                                       cudaStream_t, float*);
+
+cudaError_t launch_cfg_combine(float* x, const float* v, int B, size_t per_scene, float g,
+                               float dsig, cudaStream_t st) {
+  const size_t n = (size_t)B * per_scene;
+  if (n == 0) return cudaSuccess;
+  cfg_combine_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(x, v, B, per_scene, g, dsig);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_drift(const DriftItems& items, const float* gram, const float* gp,
                          const float* gs, int N, int C, float* partials, float* out,

@@ -62,13 +62,19 @@ template <typename T>
 cudaError_t launch_final_compute(const float* hL, const float* u, float* x, float* xj, T* r,
                                  const SlotMap& map, int N, int C, int d, const float* mod,
                                  int mod_stride, int fin_off, const float* w_f, const float* b_f,
-                                 float dsig, cudaStream_t st);
+                                 float dsig, cudaStream_t st, float* vout = nullptr);
 // reuse step: u = embed(x); h = u + r_j; v = head(h); x += dsig v  (w_eT = W_e^T [C][d])
 template <typename T>
 cudaError_t launch_final_reuse(float* x, const T* r, const float* w_eT, const float* b_e,
                                const T* pos, const SlotMap& map, int N, int C, int d,
                                const float* mod, int mod_stride, int fin_off, const float* w_f,
-                               const float* b_f, float dsig, cudaStream_t st);
+                               const float* b_f, float dsig, cudaStream_t st,
+                               float* vout = nullptr);
+// vout != NULL (both): write the velocity v[scene][tok][c] instead of the
+// Euler update (x is left as it is; the compute step still sets x_j = x).
+// guidance: x_s += dsig (v_u + g (v_c - v_u)), v_c = v[s], v_u = v[B + s]
+cudaError_t launch_cfg_combine(float* x, const float* v, int B, size_t per_scene, float g,
+                               float dsig, cudaStream_t st);
 
 // drift sums over items: out[2i] = sum ||(now_i - ref_i) W_e^T||^2,
 // out[2i+1] = sum ||now_i W_e^T + b_e + pos||^2   (deterministic order),

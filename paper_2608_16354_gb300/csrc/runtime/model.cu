@@ -51,7 +51,8 @@ struct dc_model {
   void* ws = nullptr;
   float *u = nullptr, *h = nullptr, *xj = nullptr, *mod = nullptr, *silu_c = nullptr,
         *temb_f = nullptr, *temb_h = nullptr, *temb = nullptr, *pose_f = nullptr, *traj = nullptr,
-        *drift_part = nullptr, *drift_out = nullptr, *lat_stage = nullptr;
+        *drift_part = nullptr, *drift_out = nullptr, *lat_stage = nullptr,
+        *cfg_x = nullptr, *cfg_v = nullptr;  // guidance: latents and velocities of both branches
   void *a = nullptr, *qkv = nullptr, *o = nullptr, *m = nullptr, *r = nullptr;
   double *poses_d = nullptr, *sig_d = nullptr;
   int* err_d = nullptr;
@@ -278,7 +279,7 @@ dc_status enqueue_conditioning(dc_model* m, int B, int K, cudaStream_t st) {
 // One full backbone pass + interface + Euler for the scenes in `map`.
 template <typename T>
 dc_status enqueue_compute(dc_model* m, float* lat, const float* mod_k, const SlotMap& map,
-                          float dsig, cudaStream_t st) {
+                          float dsig, cudaStream_t st, float* vout = nullptr) {
   const int N = m->N, d = m->d, nc = map.n, M = nc * N;
   if (nc == 0) return DC_OK;
   T* a = static_cast<T*>(m->a);
@@ -377,14 +378,14 @@ dc_status enqueue_compute(dc_model* m, float* lat, const float* mod_k, const Slo
   DC_LAUNCH(DC_PROF_FINAL, 2.0 * M * d * m->C, 8.0 * Md + E * Md + 12.0 * M * m->C,
             dc::launch_final_compute<T>(m->h, m->u, lat, m->xj, static_cast<T*>(m->r), map, N,
                                         m->C, d, mod_k, m->mod_stride, 6 * m->L * d, m->w_f,
-                                        m->b_f, dsig, st));
+                                        m->b_f, dsig, st, vout));
   m->launches += 1;
   return DC_OK;
 }
 
 template <typename T>
 dc_status enqueue_reuse(dc_model* m, float* lat, const float* mod_k, const SlotMap& map, float dsig,
-                        cudaStream_t st) {
+                        cudaStream_t st, float* vout = nullptr) {
   if (map.n == 0) return DC_OK;
   const double M = (double)map.n * m->N;
   // algorithmic bytes of a reuse scene-step: r_j (N d elements) + x_k read,
@@ -392,7 +393,8 @@ dc_status enqueue_reuse(dc_model* m, float* lat, const float* mod_k, const SlotM
   DC_LAUNCH(DC_PROF_REUSE, 4.0 * M * m->d * m->C, M * ((double)m->d * m->elt + 12.0 * m->C),
             dc::launch_final_reuse<T>(lat, static_cast<const T*>(m->r), m->w_eT, m->b_e,
                                       static_cast<const T*>(m->pos), map, m->N, m->C, m->d, mod_k,
-                                      m->mod_stride, 6 * m->L * m->d, m->w_f, m->b_f, dsig, st));
+                                      m->mod_stride, 6 * m->L * m->d, m->w_f, m->b_f, dsig, st,
+                                      vout));
   m->launches += 1;
   return DC_OK;
 }
@@ -432,6 +434,11 @@ dc_status run_sampler(dc_model* m, float* lat, const dc_cond* cond, const dc_sch
                       cudaStream_t st, dc_run_stats* stats, float* trace,
                       void* r_trace = nullptr) {
   const int B = cond->B, K = sc->K, N = m->N, C = m->C;
+  // guidance: every scene s runs two branches -- internal scene s with its
+  // trajectory and internal scene B + s with the null trajectory -- each with
+  // its own cache; the plan and the drift check stay per scene
+  const bool cfg = sc->cfg_scale != 0.0;
+  const int Bi = cfg ? 2 * B : B;
   const dc_anchor_responses* anc = sc->anchors;
   const double eps = anc ? anc->eps : 1e-6;
   const int W = K + 1;
@@ -478,8 +485,9 @@ dc_status run_sampler(dc_model* m, float* lat, const dc_cond* cond, const dc_sch
   }
   const long long launches0 = m->launches;
 
-  // inputs of the conditioning: poses and sigmas
-  std::vector<double> poses((size_t)B * m->P * 3);
+  // inputs of the conditioning: poses (the null trajectory of the second
+  // branch is all zeros, so its pose features vanish) and sigmas
+  std::vector<double> poses((size_t)Bi * m->P * 3, 0.0);
   for (int s = 0; s < B; ++s)
     for (int t = 0; t < m->P; ++t) {
       const dc_pose& p = cond->traj[s].poses[t];
@@ -490,13 +498,13 @@ dc_status run_sampler(dc_model* m, float* lat, const dc_cond* cond, const dc_sch
                         cudaMemcpyHostToDevice, st));
   DC_CK(cudaMemcpyAsync(m->sig_d, sc->sigmas, (size_t)(K + 1) * sizeof(double),
                         cudaMemcpyHostToDevice, st));
-  DC_TRY(enqueue_conditioning<T>(m, B, K, st));
+  DC_TRY(enqueue_conditioning<T>(m, Bi, K, st));
 
   std::vector<SceneState> state(B);
   std::vector<unsigned char> reuse_now(B);
   for (int k = 1; k <= K; ++k) {
     const float dsig = (float)(sc->sigmas[k] - sc->sigmas[k - 1]);
-    const float* mod_k = m->mod + (size_t)(k - 1) * B * m->mod_stride;
+    const float* mod_k = m->mod + (size_t)(k - 1) * Bi * m->mod_stride;
     if (trace) {
       DC_CK(cudaMemcpyAsync(trace + (size_t)(k - 1) * B * N * C, lat, (size_t)B * N * C * 4,
                             cudaMemcpyDeviceToDevice, st));
@@ -557,11 +565,24 @@ dc_status run_sampler(dc_model* m, float* lat, const dc_cond* cond, const dc_sch
     }
     SlotMap cm{}, rm{};
     for (int s = 0; s < B; ++s) {
-      if (reuse_now[s]) rm.scene[rm.n++] = s;
-      else cm.scene[cm.n++] = s;
+      SlotMap& mp = reuse_now[s] ? rm : cm;
+      mp.scene[mp.n++] = s;
+      if (cfg) mp.scene[mp.n++] = B + s;
     }
-    DC_TRY(enqueue_compute<T>(m, lat, mod_k, cm, dsig, st));
-    DC_TRY(enqueue_reuse<T>(m, lat, mod_k, rm, dsig, st));
+    if (cfg) {
+      // both branches see x_k; their velocities are combined into x_{k+1}
+      const size_t xb = (size_t)B * N * C * 4;
+      DC_CK(cudaMemcpyAsync(m->cfg_x, lat, xb, cudaMemcpyDeviceToDevice, st));
+      DC_CK(cudaMemcpyAsync(m->cfg_x + (size_t)B * N * C, lat, xb, cudaMemcpyDeviceToDevice, st));
+      DC_TRY(enqueue_compute<T>(m, m->cfg_x, mod_k, cm, dsig, st, m->cfg_v));
+      DC_TRY(enqueue_reuse<T>(m, m->cfg_x, mod_k, rm, dsig, st, m->cfg_v));
+      DC_CK(dc::launch_cfg_combine(lat, m->cfg_v, B, (size_t)N * C, (float)sc->cfg_scale, dsig,
+                                   st));
+      m->launches += 1;
+    } else {
+      DC_TRY(enqueue_compute<T>(m, lat, mod_k, cm, dsig, st));
+      DC_TRY(enqueue_reuse<T>(m, lat, mod_k, rm, dsig, st));
+    }
     if (r_trace) {
       const size_t rb = (size_t)N * m->d * m->elt;
       DC_CK(cudaMemcpyAsync(static_cast<uint8_t*>(r_trace) + (size_t)(k - 1) * rb, m->r, rb,
@@ -599,6 +620,10 @@ dc_status check_call(dc_model* m, const dc_cond* cond, const dc_sched* sc) {
   }
   if (sc->K < 1 || sc->K > m->Kmax || !sc->sigmas) {
     dc::set_error("sched->K must be in [1, max_steps] with non-NULL sigmas");
+    return DC_ERR_INVALID_ARG;
+  }
+  if (!std::isfinite(sc->cfg_scale) || (sc->cfg_scale != 0.0 && 2 * cond->B > m->Bmax)) {
+    dc::set_error("cfg_scale must be finite, and guidance needs 2 B <= max_batch");
     return DC_ERR_INVALID_ARG;
   }
   for (int k = 0; k <= sc->K; ++k)
@@ -993,6 +1018,7 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
       {&m->o, B * N * d * m->elt}, {&m->m, B * N * m->md * m->elt},
       {&m->r, B * N * d * m->elt}, {(void**)&m->xj, B * N * m->C * 4},
       {(void**)&m->lat_stage, B * N * m->C * 4},
+      {(void**)&m->cfg_x, B * N * m->C * 4}, {(void**)&m->cfg_v, B * N * m->C * 4},
       {(void**)&m->mod, K * B * m->mod_stride * 4}, {(void**)&m->silu_c, K * B * d * 4},
       {(void**)&m->temb_f, K * 256 * 4}, {(void**)&m->temb_h, K * d * 4},
       {(void**)&m->temb, K * d * 4}, {(void**)&m->pose_f, B * 3 * m->P * 4},

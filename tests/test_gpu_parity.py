@@ -558,3 +558,61 @@ def test_measured_responses_end_to_end(dc):
     record("measured_responses_end_to_end", dict(tau=tau, tau_ref=tau_ref,
                                                   rel_x=rel(lat.cpu().numpy(), ref["x"])))
     assert rel(lat.cpu().numpy(), ref["x"]) <= 1e-4
+
+
+# ------------------------------------------------ guidance branches (Sec. 3.2)
+
+@pytest.mark.parametrize("g", [1.0, 3.0])
+def test_guidance_branches_fp32_controller(dc, g):
+    """Separate guidance branches through dc_denoise with the calibrated
+    controller (two scenes, so four branch evaluations per step) against
+    the oracle: plans, checks, and latents within 1e-4."""
+    base = WORKLOADS["c1"]
+    w, om, sig, anc, tabs, tau = _calibrated(base)
+    wl = base.with_(batch=2)
+    K, H = wl.steps, wl.h_max
+    x1 = gen.latents(wl)
+    trajs = [gen.unicycle(2.0, 0.0, wl.n_poses), gen.unicycle(5.0, 0.15, wl.n_poses)]
+    ref = Ctl.denoise(om, x1, trajs, sig, anc, tabs, tau, K, H, cfg_scale=g)
+    model = dc.Model(wl, gen.flat_blob(wl, w), max_batch=4)
+    lat = torch.tensor(x1, device="cuda")
+    st = dc.denoise(model, lat, list(trajs),
+                    dc.SchedArgs(K, sig, dc.AnchorArgs(K, H, anc, tabs), tau, cfg_scale=g))
+    torch.cuda.synchronize()
+    got = lat.cpu().numpy()
+    with pytest.raises(dc.DCError):  # four branches do not fit max_batch = 2 + 1
+        small = dc.Model(wl, gen.flat_blob(wl, w), max_batch=3)
+        try:
+            dc.denoise(small, lat[:2], list(trajs),
+                       dc.SchedArgs(K, sig, dc.AnchorArgs(K, H, anc, tabs), tau, cfg_scale=g))
+        finally:
+            small.close()
+    model.close()
+    for s in range(2):
+        assert st["planned"][s].tolist()[1:] == ref["plans"][s]["actions"][1:]
+        assert st["executed"][s].tolist()[1:] == ref["executed"][s][1:]
+    record(f"guidance_fp32_g{g}", dict(rel=rel(got, ref["x"])))
+    assert rel(got, ref["x"]) <= 1e-4
+    assert rel(got - x1, ref["x"] - x1) <= 1e-3
+
+
+def test_guidance_branches_bf16_forced(dc):
+    """bf16 model, forced schedule with reuses, guidance 4: both branch caches."""
+    wl = WORKLOADS["c2"].with_(n_blocks=2, frames=2, rows=8, cols=8, steps=6, batch=2, n_poses=5)
+    K = wl.steps
+    w = gen.weights(wl)
+    om = Ctl.build(wl, w)
+    sig = gen.sigmas(K)
+    x1 = gen.latents(wl)
+    trajs = [gen.unicycle(3.0, 0.1, wl.n_poses), gen.unicycle(9.0, -0.2, wl.n_poses)]
+    forced = np.array([[0, 1, 2, 2, 1, 2, 1], [0, 1, 1, 2, 2, 1, 2]], np.uint8)
+    ref = Ctl.denoise(om, x1, trajs, sig, dict(valid=0, L0=0, T0=0, L1=0, T1=0), None, 0.0, K,
+                      wl.h_max, forced=forced.tolist(), cfg_scale=4.0)
+    model = dc.Model(wl, gen.flat_blob(wl, w), max_batch=4)
+    lat = torch.tensor(np.asarray(x1, np.float32), device="cuda")
+    dc.denoise(model, lat, list(trajs),
+               dc.SchedArgs(K, sig, no_anchors(dc, K, wl.h_max), 0.0, forced=forced, cfg_scale=4.0))
+    torch.cuda.synchronize()
+    got = lat.cpu().numpy()
+    model.close()
+    check_bf16(got, ref["x"], x1, name="guidance_bf16")
