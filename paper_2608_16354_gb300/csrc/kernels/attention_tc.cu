@@ -3,12 +3,13 @@
 //
 // One CTA per (slot, head, NQ x 128 queries); keys stream in tiles of 128.
 //   warp 0        TMA: the NQ query tiles once; K_j and V_j into two rings of
-//                 their own (kStages stages each)
-//   warp 1        owns TMEM and issues, in a fixed order, for key tile j:
+//                 their own (kKStages and kVStages stages)
+//   warps 1..NQ   one MMA-issuing warp per query tile t (warp 1 also owns
+//                 TMEM); for key tile j it issues
 //                   S_{t,j}    = Q_t K_j^T   (M=128, N=128, K=dh; Q, K from shared memory)
 //                   O_t       += P_{t,j-1} V_{j-1}  (M=128, N=64 per MMA, K=128;
 //                                P from TMEM, V from shared memory)
-//   warps 2, 3    idle (they complete the control warpgroup)
+//   other warps of the control warpgroup are idle
 //   warps 4..     one softmax warpgroup per query tile, one query row per
 //                 thread.
 // TMEM per query tile t: O_t (dh columns), S_t (128), P_t (64: 128 bf16 keys).
@@ -21,11 +22,15 @@
 // `ref` that only moves when the row's max exceeds it by more than 8 (log2
 // units); when it moves, the row of O_t (and the row sum) is rescaled by
 // exp2(ref_old - ref_new) once PV_{t,j-1} has landed and before P_{t,j} is
-// released.  Every exponential runs on MUFU (ex2.approx): moving a share of
-// them to a polynomial on the FMA pipe, as done on other parts, measured
-// slower here (the softmax is bound by issue slots, not by MUFU).  V is consumed
-// as an MN-major operand straight from its [keys][dh] layout.  Keys beyond N
-// are masked (last tile only).  Every mbarrier wait is bounded.
+// released.  On a full key tile the exponentials run against the current
+// reference while the row max is taken alongside (ALU and MUFU in parallel);
+// the rare row whose max moves the reference recomputes its P.  Every
+// exponential runs on MUFU (ex2.approx): moving a share of them to a
+// polynomial on the FMA pipe measured slower here (MUFU is about half busy;
+// the loop is bound by the latency of the S -> softmax -> P -> PV chain, not
+// by one unit).  V is consumed as an MN-major operand straight from its
+// [keys][dh] layout.  Keys beyond N are masked (last tile only).  Every
+// mbarrier wait is bounded.
 #include <math.h>
 
 #include "common.cuh"
@@ -36,17 +41,19 @@ namespace dc {
 namespace {
 
 constexpr float kRefSlack = 8.0f;  // move the reference max only beyond this (log2 units)
-constexpr int kStages = 3;         // K and V ring depth
 
 template <int DHP, int NQ>
 struct AttCfg {
   static constexpr int kAtoms = DHP / 64;             // 64-element swizzle atoms along dh
+  // ring depths (key, value): deeper rings measured no faster at dh 64
+  static constexpr int kKStages = 3;
+  static constexpr int kVStages = 3;
   static constexpr int kTileBytes = kAtoms * 16384;   // 128 rows x DHP bf16
   static constexpr int kOffQ = 0;                              // NQ tiles
-  static constexpr int kOffK = kOffQ + NQ * kTileBytes;        // kStages stages
-  static constexpr int kOffV = kOffK + kStages * kTileBytes;   // kStages stages
-  static constexpr int kOffBar = kOffV + kStages * kTileBytes;
-  static constexpr int kSmem = 1024 + kOffBar + 256;
+  static constexpr int kOffK = kOffQ + NQ * kTileBytes;        // kKStages stages
+  static constexpr int kOffV = kOffK + kKStages * kTileBytes;  // kVStages stages
+  static constexpr int kOffBar = kOffV + kVStages * kTileBytes;
+  static constexpr int kSmem = 1024 + kOffBar + 512;
   static constexpr int kThreads = 128 + NQ * 128;   // control warpgroup + softmax
   // two query tiles: the control warpgroup gives registers to the softmax
   // warpgroups (128 x 72 + 256 x 216 = 384 x 168, the launch allocation)
@@ -63,11 +70,11 @@ struct AttCfg {
   static_assert(kSmem <= 232448, "shared memory budget");
 };
 
-template <int NQ>
+template <int NQ, int kKStages, int kVStages>
 struct __align__(8) AttBars {
   uint64_t q_full;
-  uint64_t k_full[kStages], k_empty[kStages];   // key ring: loader <-> S MMAs
-  uint64_t v_full[kStages], v_empty[kStages];   // value ring: loader <-> PV MMAs
+  uint64_t k_full[kKStages], k_empty[kKStages];  // key ring: loader <-> S MMAs
+  uint64_t v_full[kVStages], v_empty[kVStages];  // value ring: loader <-> PV MMAs
   uint64_t s_full[NQ];    // MMA -> softmax: S_{t,j} ready
   uint64_t s_free[NQ];    // softmax -> MMA: S_{t,j} read into registers
   uint64_t p_full[NQ];    // softmax -> MMA: P_{t,j} in TMEM (and O_t rescaled)
@@ -171,6 +178,25 @@ __device__ __forceinline__ float chunk_max(const uint32_t (&raw)[32], int c, int
   return fmaxf(m0, m1);
 }
 
+// One unmasked 32-column chunk against the current reference, as p_chunk,
+// with the raw chunk max folded in on the ALU pipe (four chains) while MUFU
+// runs the exponentials.
+__device__ __forceinline__ void p_chunk_max(const uint32_t (&v)[32], float scale_log2,
+                                            float neg_ref, float2 (&rs)[2], uint32_t* pk,
+                                            float (&m)[4]) {
+  const float2 sc = make_float2(scale_log2, scale_log2);
+  const float2 nr = make_float2(neg_ref, neg_ref);
+#pragma unroll
+  for (int e = 0; e < 32; e += 2) {
+    const float a = __uint_as_float(v[e]), b = __uint_as_float(v[e + 1]);
+    const float2 x = ffma2(make_float2(a, b), sc, nr);
+    const float2 p = make_float2(ex2_mufu(x.x), ex2_mufu(x.y));
+    m[(e >> 1) & 3] = fmax3f(m[(e >> 1) & 3], a, b);
+    rs[(e >> 1) & 1] = fadd2(rs[(e >> 1) & 1], p);
+    pk[e >> 1] = pack2(p.x, p.y);
+  }
+}
+
 template <int DHP, int NQ>
 __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tm, int nslots, int heads, int N,
@@ -181,8 +207,10 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  AttBars<NQ>* bar = reinterpret_cast<AttBars<NQ>*>(smem + Cfg::kOffBar);
-  static_assert(sizeof(AttBars<NQ>) <= 256, "barrier block exceeds its reserve");
+  constexpr int kKStages = Cfg::kKStages, kVStages = Cfg::kVStages;
+  using Bars = AttBars<NQ, kKStages, kVStages>;
+  Bars* bar = reinterpret_cast<Bars*>(smem + Cfg::kOffBar);
+  static_assert(sizeof(Bars) <= 512, "barrier block exceeds its reserve");
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int bh = blockIdx.y;
@@ -197,9 +225,11 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
     // read once, so that the whole CTA takes the same decision below
     bar->abort = *(volatile int*)err;
     mbar_init(&bar->q_full, 1);
-    for (int b = 0; b < kStages; ++b) {
+    for (int b = 0; b < kKStages; ++b) {
       mbar_init(&bar->k_full[b], 1);
       mbar_init(&bar->k_empty[b], NQ);  // every query tile's MMA warp releases it
+    }
+    for (int b = 0; b < kVStages; ++b) {
       mbar_init(&bar->v_full[b], 1);
       mbar_init(&bar->v_empty[b], NQ);
     }
@@ -242,8 +272,9 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
       // issued, so later key tiles stream in while the PV products on V_j
       // are still pending.
       bool ok = true;
-      int last_k[kStages], last_v[kStages];
-      for (int b = 0; b < kStages; ++b) last_k[b] = last_v[b] = -1;
+      int last_k[kKStages], last_v[kVStages];
+      for (int b = 0; b < kKStages; ++b) last_k[b] = -1;
+      for (int b = 0; b < kVStages; ++b) last_v[b] = -1;
       if (elect_one()) {
         mbar_arrive_expect_tx(&bar->q_full, NQ * Cfg::kTileBytes);
         for (int t = 0; t < NQ; ++t)
@@ -257,8 +288,8 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
       while (ok && nv < n_kv) {
         bool progressed = false;
         if (nk < n_kv) {
-          const int b = nk % kStages;
-          const uint32_t u = (uint32_t)(nk / kStages);
+          const int b = nk % kKStages;
+          const uint32_t u = (uint32_t)(nk / kKStages);
           int ready = 0;
           if (lane == 0) ready = mbar_test(&bar->k_empty[b], (u & 1) ^ 1);
           if (__shfl_sync(0xffffffffu, ready, 0)) {
@@ -275,8 +306,8 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
           }
         }
         if (nv < nk) {
-          const int b = nv % kStages;
-          const uint32_t u = (uint32_t)(nv / kStages);
+          const int b = nv % kVStages;
+          const uint32_t u = (uint32_t)(nv / kVStages);
           int ready = 0;
           if (lane == 0) ready = mbar_test(&bar->v_empty[b], (u & 1) ^ 1);
           if (__shfl_sync(0xffffffffu, ready, 0)) {
@@ -309,10 +340,10 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
       }
       // every copy in flight lands before the CTA can exit
       mbar_wait_warp(&bar->q_full, 0, err, kDevTimeoutTma);
-      for (int b = 0; b < kStages; ++b) {
+      for (int b = 0; b < kKStages; ++b)
         if (last_k[b] >= 0) mbar_wait_warp(&bar->k_full[b], (uint32_t)last_k[b], err, kDevTimeoutTma);
+      for (int b = 0; b < kVStages; ++b)
         if (last_v[b] >= 0) mbar_wait_warp(&bar->v_full[b], (uint32_t)last_v[b], err, kDevTimeoutTma);
-      }
     } else if (warp >= 1 && warp <= NQ) {
       // ------------------------------------------------------------ MMA
       // One warp per query tile t, fixed order with blocking waits.  Round j
@@ -332,8 +363,8 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
       const uint64_t dV = sw128_mnmajor_desc(smem_u32(smem + Cfg::kOffV));
       for (int j = 0; j <= n_kv && ok; ++j) {
         if (j < n_kv) {
-          const int kb = j % kStages;
-          ok = mbar_wait_warp(&bar->k_full[kb], (uint32_t)(j / kStages) & 1, err, kDevTimeoutMma) &&
+          const int kb = j % kKStages;
+          ok = mbar_wait_warp(&bar->k_full[kb], (uint32_t)(j / kKStages) & 1, err, kDevTimeoutMma) &&
                mbar_wait_warp(&bar->s_free[t], ((uint32_t)j & 1) ^ 1, err, kDevTimeoutMma);
           if (!ok) break;
           tc_fence_after();
@@ -352,8 +383,8 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
         }
         if (j >= 1) {
           const int jp = j - 1;
-          const int vb = jp % kStages;
-          ok = mbar_wait_warp(&bar->v_full[vb], (uint32_t)(jp / kStages) & 1, err, kDevTimeoutMma) &&
+          const int vb = jp % kVStages;
+          ok = mbar_wait_warp(&bar->v_full[vb], (uint32_t)(jp / kVStages) & 1, err, kDevTimeoutMma) &&
                mbar_wait_warp(&bar->p_full[t], (uint32_t)jp & 1, err, kDevTimeoutMma);
           if (!ok) break;
           tc_fence_after();
@@ -396,67 +427,91 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
     const uint32_t tP = tmem + Cfg::kColP + t * 64 + lane_off;
     float ref = -INFINITY, l = 0.f;
     bool ok = true;
-    for (int j = 0; j < n_kv && ok; ++j) {
-      if (!mbar_wait_warp(&bar->s_full[t], (uint32_t)j & 1, err, kDevTimeoutEpi)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-      uint32_t s0[32], s1[32], s2[32], s3[32];
-      tmem_ld32_async(tS + 0, s0);
-      tmem_ld32_async(tS + 32, s1);
-      tmem_ld32_async(tS + 64, s2);
-      tmem_ld32_async(tS + 96, s3);
-      tmem_ld_wait_regs(s0);
-      tmem_ld_wait_regs(s1);
-      tmem_ld_wait_regs(s2);
-      tmem_ld_wait_regs(s3);
-      // S is in registers: hand S_t back to the MMA warp
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bar->s_free[t]);
-
-      const int valid = min(128, N - j * 128);
-      float mx;
-      if (valid == 128) {
-        mx = chunk_max<false>(s0, 0, valid, -INFINITY);
-        mx = chunk_max<false>(s1, 1, valid, mx);
-        mx = chunk_max<false>(s2, 2, valid, mx);
-        mx = chunk_max<false>(s3, 3, valid, mx);
-      } else {
-        mx = chunk_max<true>(s0, 0, valid, -INFINITY);
-        mx = chunk_max<true>(s1, 1, valid, mx);
-        mx = chunk_max<true>(s2, 2, valid, mx);
-        mx = chunk_max<true>(s3, 3, valid, mx);
-      }
-      const float tm = mx * scale_log2;
+    // (Making the two query tiles take turns on MUFU through named barriers
+    // measured slower: the tiles' own S -> P -> PV chains set the pace.)
+    for (int j = 0; j < n_kv; ++j) {
+      ok = ok && mbar_wait_warp(&bar->s_full[t], (uint32_t)j & 1, err, kDevTimeoutEpi);
+      if (!ok) break;
       float c = 1.f;
-      if (j == 0) {
-        ref = tm;
-      } else if (tm > ref + kRefSlack) {
-        c = ex2_mufu(ref - tm);
-        ref = tm;
-      }
       uint32_t pk[64];
-      float2 rs2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-      const float neg_ref = -ref;
-      if (valid == 128) {
-        p_chunk<false>(s0, 0, valid, scale_log2, neg_ref, rs2, pk + 0);
-        p_chunk<false>(s1, 1, valid, scale_log2, neg_ref, rs2, pk + 16);
-        p_chunk<false>(s2, 2, valid, scale_log2, neg_ref, rs2, pk + 32);
-        p_chunk<false>(s3, 3, valid, scale_log2, neg_ref, rs2, pk + 48);
-      } else {
-        p_chunk<true>(s0, 0, valid, scale_log2, neg_ref, rs2, pk + 0);
-        p_chunk<true>(s1, 1, valid, scale_log2, neg_ref, rs2, pk + 16);
-        p_chunk<true>(s2, 2, valid, scale_log2, neg_ref, rs2, pk + 32);
-        p_chunk<true>(s3, 3, valid, scale_log2, neg_ref, rs2, pk + 48);
+      {
+        uint32_t s0[32], s1[32], s2[32], s3[32];
+        tc_fence_after();
+        tmem_ld32_async(tS + 0, s0);
+        tmem_ld32_async(tS + 32, s1);
+        tmem_ld32_async(tS + 64, s2);
+        tmem_ld32_async(tS + 96, s3);
+        tmem_ld_wait_regs(s0);
+        tmem_ld_wait_regs(s1);
+        tmem_ld_wait_regs(s2);
+        tmem_ld_wait_regs(s3);
+        // S is in registers: hand S_t back to the MMA warp
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&bar->s_free[t]);
+        const int valid = min(128, N - j * 128);
+        float2 rs2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+        if (j > 0 && valid == 128) {
+          // Speculate that the reference stays: exponentials against the
+          // current reference with the row max computed alongside, so the max
+          // is off the critical path.  A row whose max exceeds the reference by
+          // more than the slack (rare once the first tiles are in) moves it and
+          // recomputes its P and row sum from the S values still in registers;
+          // every row ends with exactly the values of the max-first order.
+          float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+          p_chunk_max(s0, scale_log2, -ref, rs2, pk + 0, m4);
+          p_chunk_max(s1, scale_log2, -ref, rs2, pk + 16, m4);
+          p_chunk_max(s2, scale_log2, -ref, rs2, pk + 32, m4);
+          p_chunk_max(s3, scale_log2, -ref, rs2, pk + 48, m4);
+          const float tm = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * scale_log2;
+          if (tm > ref + kRefSlack) {
+            c = ex2_mufu(ref - tm);
+            ref = tm;
+            rs2[0] = make_float2(0.f, 0.f);
+            rs2[1] = make_float2(0.f, 0.f);
+            p_chunk<false>(s0, 0, 128, scale_log2, -ref, rs2, pk + 0);
+            p_chunk<false>(s1, 1, 128, scale_log2, -ref, rs2, pk + 16);
+            p_chunk<false>(s2, 2, 128, scale_log2, -ref, rs2, pk + 32);
+            p_chunk<false>(s3, 3, 128, scale_log2, -ref, rs2, pk + 48);
+          }
+        } else {
+          float mx;
+          if (valid == 128) {
+            mx = chunk_max<false>(s0, 0, valid, -INFINITY);
+            mx = chunk_max<false>(s1, 1, valid, mx);
+            mx = chunk_max<false>(s2, 2, valid, mx);
+            mx = chunk_max<false>(s3, 3, valid, mx);
+          } else {
+            mx = chunk_max<true>(s0, 0, valid, -INFINITY);
+            mx = chunk_max<true>(s1, 1, valid, mx);
+            mx = chunk_max<true>(s2, 2, valid, mx);
+            mx = chunk_max<true>(s3, 3, valid, mx);
+          }
+          const float tm = mx * scale_log2;
+          if (j == 0) {
+            ref = tm;
+          } else if (tm > ref + kRefSlack) {
+            c = ex2_mufu(ref - tm);
+            ref = tm;
+          }
+          const float neg_ref = -ref;
+          if (valid == 128) {
+            p_chunk<false>(s0, 0, valid, scale_log2, neg_ref, rs2, pk + 0);
+            p_chunk<false>(s1, 1, valid, scale_log2, neg_ref, rs2, pk + 16);
+            p_chunk<false>(s2, 2, valid, scale_log2, neg_ref, rs2, pk + 32);
+            p_chunk<false>(s3, 3, valid, scale_log2, neg_ref, rs2, pk + 48);
+          } else {
+            p_chunk<true>(s0, 0, valid, scale_log2, neg_ref, rs2, pk + 0);
+            p_chunk<true>(s1, 1, valid, scale_log2, neg_ref, rs2, pk + 16);
+            p_chunk<true>(s2, 2, valid, scale_log2, neg_ref, rs2, pk + 32);
+            p_chunk<true>(s3, 3, valid, scale_log2, neg_ref, rs2, pk + 48);
+          }
+        }
+        l = l * c + ((rs2[0].x + rs2[0].y) + (rs2[1].x + rs2[1].y));
       }
-      l = l * c + ((rs2[0].x + rs2[0].y) + (rs2[1].x + rs2[1].y));
       // P_t and O_t are free once PV_{t,j-1} has landed
-      if (!mbar_wait_warp(&bar->p_free[t], ((uint32_t)j & 1) ^ 1, err, kDevTimeoutEpi)) {
-        ok = false;
-        break;
-      }
+      ok = mbar_wait_warp(&bar->p_free[t], ((uint32_t)j & 1) ^ 1, err, kDevTimeoutEpi);
+      if (!ok) break;
       tc_fence_after();
       if (__any_sync(0xffffffffu, c != 1.f)) {
         // the reference moved for some row of this warp: rescale the warp's
