@@ -271,6 +271,60 @@ dc_status dc_denoise(dc_model* m, float* latents, const dc_cond* cond, const dc_
 dc_status dc_denoise_host(dc_model* m, float* host_latents, const dc_cond* cond,
                           const dc_sched* sched, void* stream, dc_run_stats* stats);
 
+/* ------------------------------------------------ sampler-state snapshots
+ * A snapshot is the whole state of a sampler call after k_done of its K
+ * steps (Sec. 3.2 controller + Eq. 1 cache): the latents x_{k_done+1}, every
+ * scene's refresh latent x_j and cached r (both guidance branches), the
+ * plan of the remaining steps after any replans, the charge C, the last
+ * refresh j and cache age of each scene, and the call's record so far.
+ * Resuming from it (dc_denoise_steps) continues the call exactly: the final
+ * latents and record equal the uninterrupted call's bit for bit.  Use:
+ * preempting a long call, or moving it to another model instance or box.
+ * Layout (caller-owned host memory, native byte order):
+ *   header, 128 bytes: char magic[8] "DCSNAP01"; uint32 version (1);
+ *     int32 B, K, cfg (0 or 1), k_done, dtype, n_tokens, d_model, channels;
+ *     uint32 element bytes of r; uint64 digest; uint64 total bytes;
+ *     int64 backbone_calls; 56 zero bytes
+ *   B scene records of 48 bytes: double charge, D; int32 j, age, supported,
+ *     n_compute, n_reuse, n_veto, n_replan, 0
+ *   uint8 planned, plan, executed, checked: [B][K+1] each, each padded to
+ *     a multiple of 8 bytes
+ *   double d_obs, d_bar: [B][K+1] each
+ *   at the next multiple of 256: float latents [B][N][C], float x_j [B][N][C]
+ *   at the next multiple of 256: r [B_i][N][d] in the model dtype
+ *     (B_i = 2B with guidance, else B)
+ * digest: FNV-1a (64-bit) of the call's inputs (trajectories, sigmas, tau,
+ * veto, cfg_scale, and the forced actions or the anchor responses). */
+
+/* Bytes of a snapshot of B scenes and K steps for a model of this shape
+ * (cfg: 1 with guidance); 0 for an invalid argument.  Host only. */
+size_t dc_snapshot_bytes(const dc_model_desc* desc, int B, int K, int cfg);
+
+typedef struct {
+  int B, K, cfg, k_done, dtype, n_tokens, d_model, channels;
+  unsigned long long digest;
+  long long backbone_calls;
+} dc_snapshot_desc;
+
+/* Validate a snapshot's header and size (magic, version, field ranges,
+ * bytes == the size its shape implies) and describe it.  Host only;
+ * DC_ERR_INVALID_ARG on any mismatch. */
+dc_status dc_snapshot_info(const void* snap, size_t bytes, dc_snapshot_desc* out);
+
+/* dc_denoise over steps k0+1 .. k_stop only.  k0 = 0 when resume is NULL
+ * (latents holds x_1); otherwise k0 = the snapshot's k_done and latents is
+ * overwritten with its x_{k0+1} (the snapshot must come from a call with the
+ * same inputs -- its digest is checked -- on a model of the same dtype and
+ * shape, possibly another instance).  k0 < k_stop <= K.  save: NULL, or a
+ * host buffer of dc_snapshot_bytes(...) bytes that receives the state after
+ * step k_stop (the stream is synchronised before return).  stats: as for
+ * dc_denoise, covering steps 1..k_stop (restored from the snapshot for steps
+ * up to k0); launches counts this call's kernels only.  dc_denoise is
+ * dc_denoise_steps with k_stop = K and no snapshots. */
+dc_status dc_denoise_steps(dc_model* m, float* latents, const dc_cond* cond, const dc_sched* sched,
+                           int k_stop, const void* resume, size_t resume_bytes, void* save,
+                           size_t save_bytes, void* stream, dc_run_stats* stats);
+
 /* Eq. 5 along one full trace: run all K steps as full evaluations from
  * `noise` (DEVICE fp32 [N][C], not modified) under `traj`, and write
  * d_out[j*(H_max+1)+h] = ||u_{j+h} - u_j|| / (||u_{j+h}|| + eps) for

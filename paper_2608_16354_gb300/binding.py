@@ -81,6 +81,12 @@ class RunStats(C.Structure):
                 ("backbone_calls", C.c_longlong), ("launches", C.c_longlong)]
 
 
+class SnapshotDesc(C.Structure):
+    _fields_ = [("B", C.c_int), ("K", C.c_int), ("cfg", C.c_int), ("k_done", C.c_int),
+                ("dtype", C.c_int), ("n_tokens", C.c_int), ("d_model", C.c_int),
+                ("channels", C.c_int), ("digest", C.c_ulonglong), ("backbone_calls", C.c_longlong)]
+
+
 _lib = None
 
 
@@ -109,6 +115,10 @@ def lib():
         "dc_denoise": (st, [C.c_void_p, C.c_void_p, P(Cond), P(Sched), C.c_void_p, P(RunStats)]),
         "dc_denoise_host": (st, [C.c_void_p, P(C.c_float), P(Cond), P(Sched), C.c_void_p,
                                  P(RunStats)]),
+        "dc_denoise_steps": (st, [C.c_void_p, C.c_void_p, P(Cond), P(Sched), C.c_int, C.c_void_p,
+                                  C.c_size_t, C.c_void_p, C.c_size_t, C.c_void_p, P(RunStats)]),
+        "dc_snapshot_bytes": (C.c_size_t, [P(ModelDesc), C.c_int, C.c_int, C.c_int]),
+        "dc_snapshot_info": (st, [C.c_void_p, C.c_size_t, P(SnapshotDesc)]),
         "dc_legal_mask": (st, [C.c_int, C.c_int, C.c_int, C.c_int, C.c_int, P(C.c_ubyte)]),
         "dc_anchor_drift": (st, [C.c_void_p, C.c_void_p, P(Trajectory), C.c_int, P(C.c_double),
                                  C.c_int, C.c_double, P(C.c_double), C.c_void_p]),
@@ -350,6 +360,41 @@ def denoise(model: Model, latents, trajs, sched: SchedArgs, stream=None, stats=T
                             C.byref(sched.s), _stream_handle(stream),
                             C.byref(st.s) if st else None))
     return st.as_dict() if st else None
+
+
+def snapshot_bytes(desc: ModelDesc, B, K, cfg=False):
+    """dc_snapshot_bytes (host only); 0 for an invalid argument."""
+    return lib().dc_snapshot_bytes(C.byref(desc), int(B), int(K), int(bool(cfg)))
+
+
+def snapshot_info(snap):
+    """dc_snapshot_info on a host uint8 array: the validated header fields."""
+    buf = np.ascontiguousarray(snap, np.uint8)
+    out = SnapshotDesc()
+    _check(lib().dc_snapshot_info(C.c_void_p(buf.ctypes.data), buf.size, C.byref(out)))
+    return {f: getattr(out, f) for f, _ in SnapshotDesc._fields_}
+
+
+def denoise_steps(model: Model, latents, trajs, sched: SchedArgs, k_stop, resume=None,
+                  save=False, stream=None, stats=True):
+    """dc_denoise_steps on a CUDA fp32 tensor [B, N, C] (updated in place).
+    resume: a snapshot (host uint8 array) or None; save: return the state
+    after step k_stop as a new host uint8 array.  Returns (stats, snapshot)."""
+    B = latents.shape[0]
+    ta = TrajectoryArgs(trajs)
+    cond = Cond(B, ta.arr)
+    st = StatsArgs(B, sched.s.K) if stats else None
+    rin = None if resume is None else np.ascontiguousarray(resume, np.uint8)
+    out = None
+    if save:
+        n = snapshot_bytes(model.desc, B, sched.s.K, sched.s.cfg_scale != 0.0)
+        out = np.empty(n, np.uint8)
+    _check(lib().dc_denoise_steps(
+        model.h, C.c_void_p(latents.data_ptr()), C.byref(cond), C.byref(sched.s), int(k_stop),
+        C.c_void_p(rin.ctypes.data) if rin is not None else None, rin.size if rin is not None else 0,
+        C.c_void_p(out.ctypes.data) if out is not None else None, out.size if out is not None else 0,
+        _stream_handle(stream), C.byref(st.s) if st else None))
+    return (st.as_dict() if st else None), out
 
 
 def denoise_host(model: Model, host_latents, trajs, sched: SchedArgs, stream=None, stats=True):

@@ -24,6 +24,7 @@
 #include "drivecache.h"
 #include "kernels/kernels.h"
 #include "plan/planner.h"
+#include "runtime/snapshot.h"
 
 using dc::SlotMap;
 
@@ -426,13 +427,42 @@ struct SceneState {
   int j = 0, age = 0;
 };
 
+// The call's record, always kept (the caller's dc_run_stats and snapshots
+// are filled from it).
+struct Record {
+  std::vector<unsigned char> planned, executed, checked;  // [B][K+1]
+  std::vector<double> d_obs, d_bar;                       // [B][K+1]
+  std::vector<int> n_compute, n_reuse, n_veto, n_replan, supported;
+  std::vector<double> D;
+  long long backbone_calls = 0;
+  void init(int B, size_t W) {
+    planned.assign((size_t)B * W, 0);
+    executed.assign((size_t)B * W, 0);
+    checked.assign((size_t)B * W, 0);
+    d_obs.assign((size_t)B * W, NAN);
+    d_bar.assign((size_t)B * W, NAN);
+    n_compute.assign(B, 0); n_reuse.assign(B, 0); n_veto.assign(B, 0); n_replan.assign(B, 0);
+    supported.assign(B, 0);
+    D.assign(B, 0.0);
+  }
+};
+
+// Snapshot requests of one call: run steps k0+1 .. k_stop, resuming from
+// `in` (validated, digest checked) when non-null, saving into `out`.
+struct SnapIO {
+  int k_stop = 0;
+  const uint8_t* in = nullptr;
+  uint8_t* out = nullptr;
+  uint64_t digest = 0;
+};
+
 // The sampler.  trace (optional, device [K][B][N][C]) receives x_k before
 // step k; r_trace (optional, device [K][N][d] of the cache type) receives
 // scene 0's cached r after step k.
 template <typename T>
 dc_status run_sampler(dc_model* m, float* lat, const dc_cond* cond, const dc_sched* sc,
                       cudaStream_t st, dc_run_stats* stats, float* trace,
-                      void* r_trace = nullptr) {
+                      void* r_trace = nullptr, const SnapIO* io = nullptr) {
   const int B = cond->B, K = sc->K, N = m->N, C = m->C;
   // guidance: every scene s runs two branches -- internal scene s with its
   // trajectory and internal scene B + s with the null trajectory -- each with
@@ -442,10 +472,13 @@ dc_status run_sampler(dc_model* m, float* lat, const dc_cond* cond, const dc_sch
   const dc_anchor_responses* anc = sc->anchors;
   const double eps = anc ? anc->eps : 1e-6;
   const int W = K + 1;
+  const int k_stop = io ? io->k_stop : K;
+  const dc::SnapLayout lay = dc::snap_layout(B, K, cfg ? 1 : 0, N, m->d, C, m->elt);
   std::vector<unsigned char> acts((size_t)B * W, dc::kCompute);
   std::vector<dc::SceneTables> tabs(B);
-  std::vector<int> supported(B, 0);
-  std::vector<double> Dv(B, 0.0);
+  std::vector<SceneState> state(B);
+  Record rec;
+  rec.init(B, W);
   const bool forced = sc->forced != nullptr;
   for (int s = 0; s < B; ++s) {
     unsigned char* a = &acts[(size_t)s * W];
@@ -460,28 +493,47 @@ dc_status run_sampler(dc_model* m, float* lat, const dc_cond* cond, const dc_sch
     double L, Th, D, cost;
     int n_reuse;
     dc::motion_stats(pt.poses, pt.n_poses, &L, &Th);
-    supported[s] = dc::plan_scene(L, Th, *anc, sc->tau, a, &n_reuse, &cost, &D, &tabs[s]);
-    Dv[s] = D;
+    rec.supported[s] = dc::plan_scene(L, Th, *anc, sc->tau, a, &n_reuse, &cost, &D, &tabs[s]);
+    rec.D[s] = D;
   }
+  rec.planned = acts;
   // the fixed-interval baseline runs its pattern with no charge and no checks
   const bool unchecked = !forced && anc->variant == DC_VAR_FIXED_INTERVAL;
-  if (stats) {
-    if (stats->planned) std::memcpy(stats->planned, acts.data(), acts.size());
+
+  int k0 = 0;
+  if (io && io->in) {
+    // resume: the controller state and the record come from the snapshot
+    // (the scene tables above are a pure function of the same inputs)
+    const uint8_t* in = io->in;
+    dc::SnapHeader h;
+    std::memcpy(&h, in, sizeof(h));
+    k0 = h.k_done;
+    rec.backbone_calls = h.backbone_calls;
     for (int s = 0; s < B; ++s) {
-      if (stats->supported) stats->supported[s] = supported[s];
-      if (stats->D) stats->D[s] = Dv[s];
-      for (int k = 0; k <= K; ++k) {
-        if (stats->d_obs) stats->d_obs[(size_t)s * W + k] = NAN;
-        if (stats->d_bar) stats->d_bar[(size_t)s * W + k] = NAN;
-        if (stats->checked) stats->checked[(size_t)s * W + k] = 0;
-        if (stats->executed) stats->executed[(size_t)s * W + k] = 0;
-      }
-      if (stats->n_compute) stats->n_compute[s] = 0;
-      if (stats->n_reuse) stats->n_reuse[s] = 0;
-      if (stats->n_veto) stats->n_veto[s] = 0;
-      if (stats->n_replan) stats->n_replan[s] = 0;
+      dc::SnapScene r;
+      std::memcpy(&r, in + lay.scene + (size_t)s * sizeof(r), sizeof(r));
+      state[s].C = r.charge;
+      state[s].j = r.j;
+      state[s].age = r.age;
+      rec.D[s] = r.D;
+      rec.supported[s] = r.supported;
+      rec.n_compute[s] = r.n_compute;
+      rec.n_reuse[s] = r.n_reuse;
+      rec.n_veto[s] = r.n_veto;
+      rec.n_replan[s] = r.n_replan;
     }
-    stats->backbone_calls = 0;
+    const size_t bw = (size_t)B * W;
+    std::memcpy(rec.planned.data(), in + lay.planned, bw);
+    std::memcpy(acts.data(), in + lay.plan, bw);
+    std::memcpy(rec.executed.data(), in + lay.executed, bw);
+    std::memcpy(rec.checked.data(), in + lay.checked, bw);
+    std::memcpy(rec.d_obs.data(), in + lay.d_obs, bw * sizeof(double));
+    std::memcpy(rec.d_bar.data(), in + lay.d_bar, bw * sizeof(double));
+    const size_t xb = (size_t)B * N * C * sizeof(float);
+    DC_CK(cudaMemcpyAsync(lat, in + lay.lat, xb, cudaMemcpyHostToDevice, st));
+    DC_CK(cudaMemcpyAsync(m->xj, in + lay.xj, xb, cudaMemcpyHostToDevice, st));
+    DC_CK(cudaMemcpyAsync(m->r, in + lay.r, (size_t)Bi * N * m->d * m->elt,
+                          cudaMemcpyHostToDevice, st));
   }
   const long long launches0 = m->launches;
 
@@ -500,9 +552,8 @@ dc_status run_sampler(dc_model* m, float* lat, const dc_cond* cond, const dc_sch
                         cudaMemcpyHostToDevice, st));
   DC_TRY(enqueue_conditioning<T>(m, Bi, K, st));
 
-  std::vector<SceneState> state(B);
   std::vector<unsigned char> reuse_now(B);
-  for (int k = 1; k <= K; ++k) {
+  for (int k = k0 + 1; k <= k_stop; ++k) {
     const float dsig = (float)(sc->sigmas[k] - sc->sigmas[k - 1]);
     const float* mod_k = m->mod + (size_t)(k - 1) * Bi * m->mod_stride;
     if (trace) {
@@ -545,18 +596,16 @@ dc_status run_sampler(dc_model* m, float* lat, const dc_cond* cond, const dc_sch
         const double dbar = tabs[s].at_d(j, h);
         const double c = tabs[s].at_c(j, h);
         const bool ok = d_obs <= dbar + eps && S.C + c <= sc->tau;
-        if (stats) {
-          if (stats->d_obs) stats->d_obs[(size_t)s * W + k] = d_obs;
-          if (stats->d_bar) stats->d_bar[(size_t)s * W + k] = dbar;
-          if (stats->checked) stats->checked[(size_t)s * W + k] = ok ? 1 : 2;
-        }
+        rec.d_obs[(size_t)s * W + k] = d_obs;
+        rec.d_bar[(size_t)s * W + k] = dbar;
+        rec.checked[(size_t)s * W + k] = ok ? 1 : 2;
         if (ok) {
           reuse_now[s] = 1;
           S.C = S.C + c;
         } else {
-          if (stats && stats->n_veto) stats->n_veto[s]++;
+          rec.n_veto[s]++;
           if (anc->variant != DC_VAR_FIXED_PLACEMENT) {  // the fixed pattern is kept
-            if (stats && stats->n_replan) stats->n_replan[s]++;
+            rec.n_replan[s]++;
             double cost;
             dc::plan_suffix(tabs[s], anc->legal, k, sc->tau - S.C, &acts[(size_t)s * W], &cost);
           }
@@ -595,18 +644,66 @@ dc_status run_sampler(dc_model* m, float* lat, const dc_cond* cond, const dc_sch
         state[s].j = k;
         state[s].age = 0;
       }
-      if (stats) {
-        if (stats->executed) stats->executed[(size_t)s * W + k] = reuse_now[s] ? dc::kReuse : dc::kCompute;
-        if (reuse_now[s] && stats->n_reuse) stats->n_reuse[s]++;
-        if (!reuse_now[s] && stats->n_compute) stats->n_compute[s]++;
-      }
+      rec.executed[(size_t)s * W + k] = reuse_now[s] ? dc::kReuse : dc::kCompute;
+      if (reuse_now[s]) rec.n_reuse[s]++;
+      else rec.n_compute[s]++;
     }
-    if (stats) stats->backbone_calls += cm.n;
+    rec.backbone_calls += cm.n;
   }
-  DC_TRY(check_device_error(m, st));
+  if (io && io->out) {
+    // save: host state now, device payload after the stream drains
+    uint8_t* out = io->out;
+    dc::SnapHeader h{};
+    std::memcpy(h.magic, dc::kSnapMagic, sizeof(h.magic));
+    h.version = dc::kSnapVersion;
+    h.B = B; h.K = K; h.cfg = cfg ? 1 : 0; h.k_done = k_stop;
+    h.dtype = m->bf16 ? DC_DTYPE_BF16 : DC_DTYPE_F32;
+    h.N = N; h.d = m->d; h.C = C; h.elt = (uint32_t)m->elt;
+    h.digest = io->digest;
+    h.bytes = lay.total;
+    h.backbone_calls = rec.backbone_calls;
+    std::memset(out, 0, lay.lat);
+    std::memcpy(out, &h, sizeof(h));
+    for (int s = 0; s < B; ++s) {
+      dc::SnapScene r{};
+      r.charge = state[s].C; r.D = rec.D[s];
+      r.j = state[s].j; r.age = state[s].age; r.supported = rec.supported[s];
+      r.n_compute = rec.n_compute[s]; r.n_reuse = rec.n_reuse[s];
+      r.n_veto = rec.n_veto[s]; r.n_replan = rec.n_replan[s];
+      std::memcpy(out + lay.scene + (size_t)s * sizeof(r), &r, sizeof(r));
+    }
+    const size_t bw = (size_t)B * W;
+    std::memcpy(out + lay.planned, rec.planned.data(), bw);
+    std::memcpy(out + lay.plan, acts.data(), bw);
+    std::memcpy(out + lay.executed, rec.executed.data(), bw);
+    std::memcpy(out + lay.checked, rec.checked.data(), bw);
+    std::memcpy(out + lay.d_obs, rec.d_obs.data(), bw * sizeof(double));
+    std::memcpy(out + lay.d_bar, rec.d_bar.data(), bw * sizeof(double));
+    const size_t xb = (size_t)B * N * C * sizeof(float);
+    std::memset(out + lay.lat + 2 * xb, 0, lay.r - (lay.lat + 2 * xb));
+    DC_CK(cudaMemcpyAsync(out + lay.lat, lat, xb, cudaMemcpyDeviceToHost, st));
+    DC_CK(cudaMemcpyAsync(out + lay.xj, m->xj, xb, cudaMemcpyDeviceToHost, st));
+    DC_CK(cudaMemcpyAsync(out + lay.r, m->r, (size_t)Bi * N * m->d * m->elt,
+                          cudaMemcpyDeviceToHost, st));
+  }
+  DC_TRY(check_device_error(m, st));  // synchronises the stream
   if (stats) {
-    for (int s = 0; s < B; ++s)
+    const size_t bw = (size_t)B * W;
+    if (stats->planned) std::memcpy(stats->planned, rec.planned.data(), bw);
+    if (stats->executed) std::memcpy(stats->executed, rec.executed.data(), bw);
+    if (stats->checked) std::memcpy(stats->checked, rec.checked.data(), bw);
+    if (stats->d_obs) std::memcpy(stats->d_obs, rec.d_obs.data(), bw * sizeof(double));
+    if (stats->d_bar) std::memcpy(stats->d_bar, rec.d_bar.data(), bw * sizeof(double));
+    for (int s = 0; s < B; ++s) {
+      if (stats->n_compute) stats->n_compute[s] = rec.n_compute[s];
+      if (stats->n_reuse) stats->n_reuse[s] = rec.n_reuse[s];
+      if (stats->n_veto) stats->n_veto[s] = rec.n_veto[s];
+      if (stats->n_replan) stats->n_replan[s] = rec.n_replan[s];
+      if (stats->supported) stats->supported[s] = rec.supported[s];
+      if (stats->D) stats->D[s] = rec.D[s];
       if (stats->charge) stats->charge[s] = state[s].C;
+    }
+    stats->backbone_calls = rec.backbone_calls;
     stats->launches = m->launches - launches0;
   }
   return DC_OK;
@@ -1130,6 +1227,56 @@ dc_status dc_denoise(dc_model* m, float* latents, const dc_cond* cond, const dc_
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   if (m->bf16) return run_sampler<__nv_bfloat16>(m, latents, cond, sched, st, stats, nullptr);
   return run_sampler<float>(m, latents, cond, sched, st, stats, nullptr);
+}
+
+dc_status dc_denoise_steps(dc_model* m, float* latents, const dc_cond* cond, const dc_sched* sched,
+                           int k_stop, const void* resume, size_t resume_bytes, void* save,
+                           size_t save_bytes, void* stream, dc_run_stats* stats) {
+  DC_TRY(check_call(m, cond, sched));
+  if (!latents) { dc::set_error("latents is NULL"); return DC_ERR_INVALID_ARG; }
+  const int cfg = sched->cfg_scale != 0.0 ? 1 : 0;
+  const dc::SnapLayout lay = dc::snap_layout(cond->B, sched->K, cfg, m->N, m->d, m->C, m->elt);
+  SnapIO io;
+  io.k_stop = k_stop;
+  io.digest = dc::call_digest(cond, sched);
+  int k0 = 0;
+  if (resume) {
+    dc::SnapHeader h;
+    DC_TRY(dc::read_header(resume, resume_bytes, &h));
+    const int dtype = m->bf16 ? DC_DTYPE_BF16 : DC_DTYPE_F32;
+    if (h.B != cond->B || h.K != sched->K || h.cfg != cfg || h.dtype != dtype || h.N != m->N ||
+        h.d != m->d || h.C != m->C) {
+      dc::set_error("snapshot shape (B, K, guidance, dtype, N, d, C) does not match this call");
+      return DC_ERR_INVALID_ARG;
+    }
+    if (h.digest != io.digest) {
+      dc::set_error("snapshot was taken from a call with other inputs (digest mismatch)");
+      return DC_ERR_INVALID_ARG;
+    }
+    k0 = h.k_done;
+    io.in = static_cast<const uint8_t*>(resume);
+  }
+  if (k_stop <= k0 || k_stop > sched->K) {
+    dc::set_error("k_stop must satisfy k_done < k_stop <= K (k_done = " + std::to_string(k0) + ")");
+    return DC_ERR_INVALID_ARG;
+  }
+  if (save) {
+    if (save_bytes != lay.total) {
+      dc::set_error("save buffer must be dc_snapshot_bytes(...) = " + std::to_string(lay.total) +
+                    " bytes");
+      return DC_ERR_INVALID_ARG;
+    }
+    if (resume && static_cast<const uint8_t*>(save) < static_cast<const uint8_t*>(resume) + resume_bytes &&
+        static_cast<const uint8_t*>(resume) < static_cast<const uint8_t*>(save) + save_bytes) {
+      dc::set_error("save and resume buffers overlap");
+      return DC_ERR_INVALID_ARG;
+    }
+    io.out = static_cast<uint8_t*>(save);
+  }
+  DC_CK(cudaSetDevice(m->device));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (m->bf16) return run_sampler<__nv_bfloat16>(m, latents, cond, sched, st, stats, nullptr, nullptr, &io);
+  return run_sampler<float>(m, latents, cond, sched, st, stats, nullptr, nullptr, &io);
 }
 
 dc_status dc_denoise_host(dc_model* m, float* host_latents, const dc_cond* cond,
