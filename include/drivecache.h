@@ -162,6 +162,21 @@ dc_status dc_replan(const dc_anchor_responses* anc, double D, int k_refresh, dou
 dc_status dc_calibrate_budget(const dc_trajectory* clips, int n, const dc_anchor_responses* anc,
                               int target, int T, double* tau, int* reached);
 
+/* Distributed budget calibration (Sec. 3.2): the tau rule above split into
+ * a per-clip part, which any host can run on its share of the calibration
+ * clips, and a combining part over the gathered curves.
+ * dc_cost_curve writes m_out[n] = min_h J_T(n, h) for n = 0..T-1 (+infinity
+ * where n reuses are infeasible) from the clip's own tables; an unsupported
+ * clip gets an all-infinite curve and *supported = 0 (supported may be NULL).
+ * DC_VAR_FIXED_INTERVAL has no curve (DC_ERR_INVALID_ARG: its budget is the
+ * reuse count).  dc_budget_from_curves applies the tau rule to n curves
+ * (row-major [n][T]): for the same clips, in any order, it returns exactly
+ * what dc_calibrate_budget returns. */
+dc_status dc_cost_curve(const dc_trajectory* clip, const dc_anchor_responses* anc, int T,
+                        double* m_out, int* supported);
+dc_status dc_budget_from_curves(const double* curves, int n, int T, int target, double* tau,
+                                int* reached);
+
 /* Sec. 3.2 model-specific legality as the L(k, h) mask of Eq. 10: writes
  * out[k*(H_max+1)+h] = 1 iff reusing at step k with cache age h (refresh at
  * j = k - h) is allowed, for k = 0..K, h = 0..H_max (caller-owned

@@ -108,6 +108,10 @@ def lib():
         "dc_replan": (st, [P(AnchorResponses), C.c_double, C.c_int, C.c_double, P(Schedule)]),
         "dc_calibrate_budget": (st, [P(Trajectory), C.c_int, P(AnchorResponses), C.c_int,
                                      C.c_int, P(C.c_double), P(C.c_int)]),
+        "dc_cost_curve": (st, [P(Trajectory), P(AnchorResponses), C.c_int, P(C.c_double),
+                               P(C.c_int)]),
+        "dc_budget_from_curves": (st, [P(C.c_double), C.c_int, C.c_int, C.c_int,
+                                       P(C.c_double), P(C.c_int)]),
         "dc_model_weight_count": (C.c_size_t, [P(ModelDesc)]),
         "dc_model_create": (st, [P(ModelDesc), P(C.c_float), C.c_size_t, C.c_int,
                                  P(C.c_void_p)]),
@@ -255,6 +259,25 @@ def calibrate_budget(clip_poses, anchors: AnchorArgs, target, T):
     reached = C.c_int()
     _check(lib().dc_calibrate_budget(t.arr, len(t.bufs), anchors.ptr(), int(target), int(T),
                                      C.byref(tau), C.byref(reached)))
+    return tau.value, reached.value
+
+
+def cost_curve(poses, anchors: AnchorArgs, T):
+    """dc_cost_curve: (curve [T] with inf where infeasible, supported)."""
+    t = TrajectoryArgs([poses])
+    out = np.empty(int(T), np.float64)
+    sup = C.c_int()
+    _check(lib().dc_cost_curve(t.ptr(), anchors.ptr(), int(T), _dptr(out), C.byref(sup)))
+    return out, sup.value
+
+
+def budget_from_curves(curves, target):
+    """dc_budget_from_curves on a [n, T] array: (tau, reached)."""
+    c = np.ascontiguousarray(curves, np.float64)
+    tau = C.c_double()
+    reached = C.c_int()
+    _check(lib().dc_budget_from_curves(_dptr(c), c.shape[0], c.shape[1], int(target),
+                                       C.byref(tau), C.byref(reached)))
     return tau.value, reached.value
 
 

@@ -43,6 +43,41 @@ double median_of(std::vector<double> v) {
   return (v[n / 2 - 1] + v[n / 2]) / 2.0;
 }
 
+// Sec. 3.2 tau rule on the cost curves of the calibration clips (entry n =
+// min_h J_T(n, h), +inf where infeasible; an empty or all-infinite curve is a
+// clip that counts zero reuses): the smallest finite curve value whose
+// median B* reaches `target`, else the largest (*reached = 0); 0 without
+// candidates.  The result does not depend on the order of the clips.
+void budget_from_curves(const std::vector<std::vector<double>>& curves, int target, double* tau,
+                        int* reached) {
+  const int n = (int)curves.size();
+  std::set<double> cands;
+  for (const auto& c : curves)
+    for (double v : c)
+      if (v < kInf) cands.insert(v);
+  if (cands.empty()) {
+    *tau = 0.0;
+    if (reached) *reached = 0;
+    return;
+  }
+  std::vector<double> counts(n);
+  for (double c : cands) {
+    for (int i = 0; i < n; ++i) {
+      int b = 0;
+      for (size_t m = 0; m < curves[i].size(); ++m)
+        if (curves[i][m] < kInf && curves[i][m] <= c) b = (int)m;
+      counts[i] = (double)b;
+    }
+    if (median_of(counts) >= (double)target) {
+      *tau = c;
+      if (reached) *reached = 1;
+      return;
+    }
+  }
+  *tau = *cands.rbegin();
+  if (reached) *reached = 0;
+}
+
 void zscores(const double* v, int n, std::vector<double>* z) {
   double s = 0.0;
   for (int i = 0; i < n; ++i) s = s + v[i];
@@ -469,41 +504,61 @@ dc_status dc_calibrate_budget(const dc_trajectory* clips, int n, const dc_anchor
     return DC_OK;
   }
   std::vector<std::vector<double>> curves(n);
-  std::vector<char> has(n, 0);
-  std::set<double> cands;
   for (int i = 0; i < n; ++i) {
     double L, Th, D;
     dc::motion_stats(clips[i].poses, clips[i].n_poses, &L, &Th);
-    if (!dc::scene_intensity(L, Th, *anc, &D)) continue;
+    if (!dc::scene_intensity(L, Th, *anc, &D)) continue;  // counts as zero reuses
     dc::SceneTables t;
     dc::scene_tables(*anc, D, &t);
     dc::cost_curve(t, anc->legal, &curves[i]);
-    has[i] = 1;
-    for (double v : curves[i])
-      if (v < kInf) cands.insert(v);
   }
-  if (cands.empty()) {
-    *tau = 0.0;
-    if (reached) *reached = 0;
-    return DC_OK;
+  budget_from_curves(curves, target, tau, reached);
+  return DC_OK;
+}
+
+dc_status dc_cost_curve(const dc_trajectory* clip, const dc_anchor_responses* anc, int T,
+                        double* m_out, int* supported) {
+  dc_status s = dc::check_anchors(anc);
+  if (s != DC_OK) return s;
+  if (!clip || !m_out || T != anc->K) {
+    dc::set_error("dc_cost_curve: NULL clip/m_out or T != anchors.K");
+    return DC_ERR_INVALID_ARG;
   }
-  std::vector<double> counts(n);
-  for (double c : cands) {
-    for (int i = 0; i < n; ++i) {
-      int b = 0;
-      if (has[i])
-        for (size_t m = 0; m < curves[i].size(); ++m)
-          if (curves[i][m] < kInf && curves[i][m] <= c) b = (int)m;
-      counts[i] = (double)b;
-    }
-    if (median_of(counts) >= (double)target) {
-      *tau = c;
-      if (reached) *reached = 1;
-      return DC_OK;
-    }
+  if (anc->variant == DC_VAR_FIXED_INTERVAL) {
+    dc::set_error("dc_cost_curve: the fixed-interval variant has no cost curve (its budget is the reuse count)");
+    return DC_ERR_INVALID_ARG;
   }
-  *tau = *cands.rbegin();
-  if (reached) *reached = 0;
+  if ((s = check_traj(clip)) != DC_OK) return s;
+  for (int m = 0; m < T; ++m) m_out[m] = kInf;
+  double L, Th, D;
+  dc::motion_stats(clip->poses, clip->n_poses, &L, &Th);
+  const int sup = dc::scene_intensity(L, Th, *anc, &D);
+  if (supported) *supported = sup;
+  if (!sup) return DC_OK;
+  dc::SceneTables t;
+  dc::scene_tables(*anc, D, &t);
+  std::vector<double> c;
+  dc::cost_curve(t, anc->legal, &c);
+  for (size_t m = 0; m < c.size() && m < (size_t)T; ++m) m_out[m] = c[m];
+  return DC_OK;
+}
+
+dc_status dc_budget_from_curves(const double* curves, int n, int T, int target, double* tau,
+                                int* reached) {
+  if (!curves || n < 1 || T < 1 || target < 0 || !tau) {
+    dc::set_error("dc_budget_from_curves: NULL curves/tau, n < 1, T < 1 or target < 0");
+    return DC_ERR_INVALID_ARG;
+  }
+  std::vector<std::vector<double>> c(n);
+  for (int i = 0; i < n; ++i) {
+    c[i].assign(curves + (size_t)i * T, curves + (size_t)(i + 1) * T);
+    for (double v : c[i])
+      if (std::isnan(v) || v < 0.0) {
+        dc::set_error("dc_budget_from_curves: curve entries must be >= 0 or +infinity");
+        return DC_ERR_INVALID_ARG;
+      }
+  }
+  budget_from_curves(c, target, tau, reached);
   return DC_OK;
 }
 
