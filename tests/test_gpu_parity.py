@@ -408,6 +408,35 @@ def test_attention_kernel_growing_logits(dc, dh, N, heads, slots):
         assert rel(got[s], ref) <= 1e-2, rel(got[s], ref)
 
 
+@pytest.mark.parametrize("dh,N,heads,slots", [(64, 300, 40, 4), (128, 300, 30, 4)])
+def test_attention_kernel_many_items_per_cta(dc, dh, N, heads, slots):
+    """More (slot, head, query block) work items than SMs, so the launch runs
+    in several waves and every SM processes two or more items: each item must
+    start from a fresh running max and row sum and write only its own rows.
+    Growing key norms move the running max inside every item; the last query
+    block and key tile of each item are ragged."""
+    from oracle.dit import attention_core
+    rng = np.random.default_rng(7 * dh + N)
+    qkv = rng.standard_normal((3, slots, heads, N, dh)).astype(np.float32)
+    qkv[0] *= 2.0
+    qkv[1] *= np.linspace(1.0, 4.0, N, dtype=np.float32)[None, None, :, None]
+    # a different scale per (slot, head), so that an item reading another
+    # item's state or rows would show
+    qkv[0] *= rng.uniform(0.3, 1.5, (slots, heads))[:, :, None, None].astype(np.float32)
+    t = torch.tensor(qkv, device="cuda").to(torch.bfloat16)
+    ref_in = t.float().cpu().numpy()
+    out = torch.full((slots, N, heads * dh), float("nan"), device="cuda", dtype=torch.bfloat16)
+    dc.attention(t, slots, heads, N, dh, out)
+    torch.cuda.synchronize()
+    got = out.float().cpu().numpy()
+    assert np.isfinite(got).all()
+    for s in range(slots):
+        ref = attention_core(ref_in[0, s], ref_in[1, s], ref_in[2, s])
+        ref = ref.transpose(1, 0, 2).reshape(N, heads * dh)
+        record(f"attn_bf16_items_dh{dh}_N{N}", dict(rel=rel(got[s], ref)))
+        assert rel(got[s], ref) <= 1e-2, rel(got[s], ref)
+
+
 @pytest.mark.parametrize("dh,N", [(16, 128), (16, 77), (64, 50)])
 def test_attention_kernel_fp32(dc, dh, N):
     from oracle.dit import attention_core
