@@ -4,17 +4,22 @@
 //   weights, both K-major bf16), fp32 accumulation in TMEM, followed by one
 //   of the fused DiT epilogues (QKV scatter, GELU, gated residual).
 //
-// Design: persistent CTAs (one per SM) in clusters of two, 128 x 192 output
-// tiles, K in steps of 64 (one 128-byte swizzle atom per row).  The two CTAs
-// of a cluster work on vertically adjacent tiles with the same W columns:
-// each loads its own A tile and half of the W tile, multicast into both, so
-// every CTA pulls 28 KB instead of 40 KB per K step from L2 (the loads, not
-// the tensor core, bound these GEMMs).  Warp 0 streams the tiles with TMA
-// into a shared-memory ring whose stages are released by both CTAs' MMAs;
-// warp 1 owns the TMEM allocation and one elected lane issues tcgen05.mma
-// (M=128, N=192, K=16) into one of two TMEM accumulators; warps 2-9 drain the
-// other accumulator with tcgen05.ld and run the epilogue, so the epilogue of
-// tile i overlaps the MMAs of tile i+1.
+// Design: persistent CTAs (one per SM) in clusters of two that share one
+// M = 256 pair MMA (tcgen05.mma.cta_group::2): the pair owns a 256 x 192
+// output tile, each CTA holds its 128 rows of A and half of the W tile (96
+// rows) in its own shared memory at the same offsets, rank 0 issues the MMAs
+// and each CTA receives its 128 rows of the accumulator in its own TMEM.  A
+// CTA so pulls 28 KB per 64-deep K step instead of 40 KB, which buys six
+// ring stages (four for the residual kernels) within shared memory -- the
+// loads, whose latency reaches several thousand cycles under full load, not
+// the tensor core bound these GEMMs.  Rank 1's copies complete on rank 0's
+// full barriers; the MMA commits release the stages and hand the
+// accumulators to the epilogues of both CTAs (multicast), and both CTAs'
+// epilogue warps free an accumulator on rank 0.  Warp 0 streams the tiles
+// with TMA; warp 1 of rank 0 issues the MMAs into one of two TMEM
+// accumulators (warp 1 of each CTA takes part in the pair TMEM allocation);
+// warps 2-9 drain the other accumulator with tcgen05.ld and run the
+// epilogue, so the epilogue of tile i overlaps the MMAs of tile i+1.
 // N = 192 divides every projection width of the configured models (3d, d,
 // 4d for d = 384, 1152, 3072).
 //
@@ -37,31 +42,34 @@ namespace {
 
 constexpr int kBM = 128, kBN = 192, kBK = 64;
 constexpr int kABytes = kBM * kBK * 2;        // 16 KB
-constexpr int kBBytes = kBN * kBK * 2;        // 24 KB
-constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kBBytes = kBN * kBK * 2;        // 24 KB: the pair's W tile
+constexpr int kBHalf = kBBytes / 2;            // 12 KB: this CTA's half (96 rows)
+constexpr int kStageBytes = kABytes + kBHalf;  // 28 KB per CTA and K step
 constexpr int kTmemCols = 512;                // two 192-column accumulators at 0 / 256
 constexpr int kThreads = 320;                 // 10 warps
 constexpr int kEpiWarps = 8;
 constexpr int kEpiThreads = kEpiWarps * 32;
-constexpr uint32_t kIdesc = idesc_bf16_f32(kBM, kBN);
+constexpr uint32_t kIdesc = idesc_bf16_f32(2 * kBM, kBN);  // one M = 256 MMA over the pair
 
 template <int MODE>
 struct GemmCfg {
-  static constexpr int kStages = MODE == kEpiResid ? 3 : 4;
+  static constexpr int kStages = MODE == kEpiResid ? 4 : 6;
   // epilogue staging tile: residual 6 boxes of [128 rows][32 fp32], GELU and
   // QKV 3 boxes of [128 rows][64 bf16]; 16 KB per box, 128-byte swizzle
   static constexpr int kOutBytes = MODE == kEpiResid ? 6 * 16384 : 3 * 16384;
   static constexpr int kOffA = 0;
   static constexpr int kOffB = kOffA + kStages * kABytes;
-  static constexpr int kOffOut = kOffB + kStages * kBBytes;
+  static constexpr int kOffOut = kOffB + kStages * kBHalf;
   static constexpr int kOffVec = kOffOut + kOutBytes;            // bias + two gate rows
   static constexpr int kOffBar = kOffVec + 3 * kBN * 4;
   static constexpr int kSmem = 1024 + kOffBar + 256;
+  static_assert(kStages <= 6, "barrier arrays hold six stages");
+  static_assert(kSmem <= 232448, "shared memory budget");
 };
 
 struct __align__(8) Barriers {
-  uint64_t full[4];
-  uint64_t empty[4];
+  uint64_t full[6];   // rank 0: both CTAs' loads of a stage landed
+  uint64_t empty[6];  // each CTA: the pair MMAs have read its stage
   uint64_t tmem_full[2];
   uint64_t tmem_empty[2];
   uint64_t hin_full;
@@ -109,12 +117,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     // read once, so that the whole CTA takes the same decision below
     bar->abort = *(volatile int*)err;
     for (int s = 0; s < kStages; ++s) {
-      mbar_init(&bar->full[s], 1);
-      mbar_init(&bar->empty[s], 2);  // released by the MMAs of both CTAs
+      mbar_init(&bar->full[s], 2);   // one expect_tx arrival from each CTA's producer
+      mbar_init(&bar->empty[s], 1);  // the pair MMAs' commit, multicast to both CTAs
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bar->tmem_full[b], 1);
-      mbar_init(&bar->tmem_empty[b], kEpiWarps);
+      mbar_init(&bar->tmem_empty[b], 2 * kEpiWarps);  // used on rank 0: both CTAs' epilogues
     }
     mbar_init(&bar->hin_full, 1);
     mbar_init(&bar->drain, 1);
@@ -125,8 +133,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     if (MODE == kEpiResid) tma_prefetch_desc(&tmCin);
   }
   if (warp == 1) {
-    tmem_alloc(&bar->tmem_base, kTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(&bar->tmem_base, kTmemCols);
+    tmem_relinquish_pair();
   }
   // the peer's barriers are initialised before any multicast or remote arrive
   tc_fence_before();
@@ -152,30 +160,47 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const int m0 = m0_of(pt);
       const int n0 = n0_of(pt);
       for (int kb = 0; kb < KB; ++kb) {
-        // the stage is free once both CTAs' MMAs have read it (the W half
-        // goes into both)
+        // the stage is free once the pair MMAs have read it; both CTAs'
+        // copies are counted on rank 0's full barrier
         if (!mbar_wait_warp(&bar->empty[stage], phase ^ 1, err, kDevTimeoutTma)) { ok = false; break; }
         const int la = (2 * issued) & 7;
-        if (lane == la) mbar_arrive_expect_tx(&bar->full[stage], kStageBytes);
-        __syncwarp();
-        if (lane == la) tma_load_2d(sA + (size_t)stage * kABytes, &tmA, &bar->full[stage], kb * kBK, m0);
-        if (lane == la + 1)
-          tma_load_2d_mc(sB + (size_t)stage * kBBytes + rank * (kBBytes / 2), &tmB, &bar->full[stage],
-                         kb * kBK, n0 + rank * (kBN / 2), (uint16_t)0x3);
+        if (rank == 0) {
+          if (lane == la) mbar_arrive_expect_tx(&bar->full[stage], kStageBytes);
+          __syncwarp();
+          if (lane == la) tma_load_2d(sA + (size_t)stage * kABytes, &tmA, &bar->full[stage], kb * kBK, m0);
+          if (lane == la + 1)
+            tma_load_2d(sB + (size_t)stage * kBHalf, &tmB, &bar->full[stage], kb * kBK, n0);
+        } else {
+          const uint32_t fb = cluster_addr(&bar->full[stage], 0);
+          if (lane == la) mbar_arrive_expect_tx_cluster(fb, kStageBytes);
+          __syncwarp();
+          if (lane == la) tma_load_2d_pair(sA + (size_t)stage * kABytes, &tmA, fb, kb * kBK, m0);
+          if (lane == la + 1)
+            tma_load_2d_pair(sB + (size_t)stage * kBHalf, &tmB, fb, kb * kBK, n0 + kBN / 2);
+        }
         __syncwarp();
         ++issued;
         last_phase[stage] = (int)phase;
         if (++stage == kStages) { stage = 0; phase ^= 1; }
       }
     }
-    // do not leave the CTA with copies still landing in shared memory
-    for (int s = 0; s < kStages; ++s)
-      if (last_phase[s] >= 0) mbar_wait_warp(&bar->full[s], (uint32_t)last_phase[s], err, kDevTimeoutTma);
+    // do not leave the pair with copies still landing in shared memory: rank
+    // 0's full barriers count both CTAs' copies, and rank 1 stays until rank
+    // 0 has passed here (final cluster barrier)
+    if (rank == 0)
+      for (int s = 0; s < kStages; ++s)
+        if (last_phase[s] >= 0) mbar_wait_warp(&bar->full[s], (uint32_t)last_phase[s], err, kDevTimeoutTma);
+  } else if (warp == 1 && rank != 0) {
+    // rank 1 issues nothing; its shared memory and TMEM are in use by rank
+    // 0's pair MMAs until they drain
+    mbar_wait_warp(&bar->drain, 0, err, kDevTimeoutMma);
   } else if (warp == 1) {
-    // -------------------------------------------------- MMA issuer
+    // -------------------------------------------------- MMA issuer (rank 0)
     // The whole warp runs the loop with uniform descriptors; one elected lane
     // (the same one throughout: tcgen05.commit tracks the issuing thread)
-    // issues the MMAs and commits.
+    // issues the pair MMAs (M = 256: rows of A and half of the W columns from
+    // each CTA's shared memory at the same offsets, 128 rows of D in each
+    // CTA's TMEM) and commits.
     int stage = 0;
     uint32_t phase = 0;
     bool ok = true;
@@ -196,22 +221,23 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         if (elect_one()) {
 #pragma unroll
           for (int kk = 0; kk < kBK / 16; ++kk) {
-            tc_mma_f16(d_tmem, dA + ((uint32_t)(stage * kABytes + kk * 32) >> 4),
-                       dB + ((uint32_t)(stage * kBBytes + kk * 32) >> 4), kIdesc,
-                       (kb | kk) != 0 ? 1u : 0u);
+            tc_mma_f16_pair(d_tmem, dA + ((uint32_t)(stage * kABytes + kk * 32) >> 4),
+                            dB + ((uint32_t)(stage * kBHalf + kk * 32) >> 4), kIdesc,
+                            (kb | kk) != 0 ? 1u : 0u);
           }
-          tc_commit_mc(&bar->empty[stage], (uint16_t)0x3);  // release it in both CTAs
+          tc_commit_pair_mc(&bar->empty[stage], (uint16_t)0x3);  // release it in both CTAs
         }
         __syncwarp();
         if (++stage == kStages) { stage = 0; phase ^= 1; }
       }
       if (ok) {
-        if (elect_one()) tc_commit(&bar->tmem_full[b]);
+        if (elect_one()) tc_commit_pair_mc(&bar->tmem_full[b], (uint16_t)0x3);
         __syncwarp();
       }
     }
-    // every MMA this warp issued has completed once `drain` flips
-    if (elect_one()) tc_commit(&bar->drain);
+    // every pair MMA this warp issued has completed once `drain` flips (in
+    // both CTAs)
+    if (elect_one()) tc_commit_pair_mc(&bar->drain, (uint16_t)0x3);
     __syncwarp();
     mbar_wait_warp(&bar->drain, 0, err, kDevTimeoutMma);
   } else {
@@ -269,7 +295,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         tmem_ld_wait();
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&bar->tmem_empty[b]);
+        // the accumulator is in registers (wait::ld): rank 0 may reuse it
+        if (lane == 0) mbar_arrive_cluster_relaxed(cluster_addr(&bar->tmem_empty[b], 0));
       }
 
       // stage bias (and gate rows) of this tile once the previous tile is done
@@ -437,7 +464,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, kTmemCols);
+    tmem_dealloc_pair(tmem_base, kTmemCols);
   }
   // no CTA leaves while its peer may still multicast into it or arrive on
   // its barriers
