@@ -1,5 +1,6 @@
 // Full spatiotemporal attention on the 5th-generation tensor cores (sm_103a):
-// o = softmax(q k^T / sqrt(dh)) v for head dims 64 and 128.
+// o = softmax(q k^T / sqrt(dh)) v for head dims 64, 72 and 128 (72 runs in
+// the 128-column layout: S over 5 K steps of 16, O over 80 columns).
 //
 // One CTA per (slot, head, NQ x 128 queries); keys stream in tiles of 128.
 //   warp 0        TMA: the NQ query tiles once; K_j and V_j into two rings of
@@ -197,13 +198,23 @@ __device__ __forceinline__ void p_chunk_max(const uint32_t (&v)[32], float scale
   }
 }
 
-template <int DHP, int NQ>
+// DH: the head dimension; DHP: its storage in shared memory and TMEM (64 or
+// 128 columns, 64-element swizzle atoms).  DH < DHP (72 in 128) computes S
+// over ceil(DH / 16) K steps of 16 and O over DH rounded up to 16 columns;
+// the query/key/value rows hold round16(DH) elements, the rest of each
+// 64-element atom is the zero fill of the TMA loads.
+template <int DHP, int NQ, int DH = DHP>
 __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tm, int nslots, int heads, int N,
                    __nv_bfloat16* __restrict__ o, float scale_log2, int* err) {
   using Cfg = AttCfg<DHP, NQ>;
   constexpr uint32_t kIdS = idesc_bf16_f32(128, 128);
   constexpr uint32_t kIdPV = idesc_bf16_f32(128, 64) | (1u << 16);  // B (= V) MN-major
+  static_assert(DH % 8 == 0 && DH <= DHP && DH > DHP - 64, "head dim within the last atom");
+  constexpr int kDHR = (DH + 15) / 16 * 16;         // O columns computed
+  constexpr int kKSteps = kDHR / 16;                // K steps of the S products
+  constexpr int kLastN = kDHR - 64 * (Cfg::kAtoms - 1);  // N of the last atom's PV product
+  constexpr uint32_t kIdPVLast = idesc_bf16_f32(128, kLastN) | (1u << 16);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -370,7 +381,7 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
           tc_fence_after();
           if (elect_one()) {
 #pragma unroll
-            for (int kk = 0; kk < DHP / 16; ++kk) {
+            for (int kk = 0; kk < kKSteps; ++kk) {
               const uint32_t off = (kk >> 2) * 16384 + (kk & 3) * 32;
               tc_mma_f16(tmem + Cfg::kColS + t * 128, dQ + (off >> 4),
                          dK + ((uint32_t)(kb * Cfg::kTileBytes + off) >> 4), kIdS,
@@ -396,7 +407,8 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
                 tc_mma_f16_ta(tmem + Cfg::kColO + t * DHP + a * 64,
                               tmem + Cfg::kColP + t * 64 + kk * 8,
                               dV + ((uint32_t)(vb * Cfg::kTileBytes + a * 16384 + kk * 2048) >> 4),
-                              kIdPV, (jp > 0 || kk > 0) ? 1u : 0u);
+                              a == Cfg::kAtoms - 1 ? kIdPVLast : kIdPV,
+                              (jp > 0 || kk > 0) ? 1u : 0u);
             }
             tc_commit(&bar->p_free[t]);
             tc_commit(&bar->v_empty[vb]);
@@ -517,7 +529,7 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
         // the reference moved for some row of this warp: rescale the warp's
         // 32 rows of O_t (c = 1 elsewhere) before PV_{t,j} accumulates
 #pragma unroll
-        for (int ch = 0; ch < DHP / 32; ++ch) {
+        for (int ch = 0; ch < (kDHR + 31) / 32; ++ch) {
           uint32_t r[32];
           tmem_ld32_async(tO + ch * 32, r);
           tmem_ld_wait_regs(r);
@@ -540,15 +552,15 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
     if (ok) {
       tc_fence_after();
       const float inv = 1.f / l;
-      __nv_bfloat16* dst = o + ((size_t)slot * N + qrow) * ((size_t)heads * DHP) + head * DHP;
+      __nv_bfloat16* dst = o + ((size_t)slot * N + qrow) * ((size_t)heads * DH) + head * DH;
 #pragma unroll
-      for (int ch = 0; ch < DHP / 32; ++ch) {
+      for (int ch = 0; ch < (DH + 31) / 32; ++ch) {
         uint32_t r[32];
         tmem_ld32_async(tO + ch * 32, r);
         tmem_ld_wait_regs(r);
         if (qrow < N) {
 #pragma unroll
-          for (int e = 0; e < 32; e += 8) {
+          for (int e = 0; e < 32 && ch * 32 + e < DH; e += 8) {
             uint4 w;
             w.x = pack2(__uint_as_float(r[e]) * inv, __uint_as_float(r[e + 1]) * inv);
             w.y = pack2(__uint_as_float(r[e + 2]) * inv, __uint_as_float(r[e + 3]) * inv);
@@ -564,39 +576,40 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
   }
 }
 
-template <int DHP, int NQ>
+template <int DHP, int NQ, int DH = DHP>
 cudaError_t launch_tc(const CUtensorMap& tm, int nslots, int heads, int N, __nv_bfloat16* o,
                       int* err, cudaStream_t st) {
   using Cfg = AttCfg<DHP, NQ>;
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<DHP, NQ>,
+    cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<DHP, NQ, DH>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmem);
     if (e != cudaSuccess) return e;
     // setmaxnreg.inc waits until the CTA's launch allocation can serve it:
     // never launch a build whose allocation is not the one the split assumes
     cudaFuncAttributes fa;
-    e = cudaFuncGetAttributes(&fa, attn_tc_kernel<DHP, NQ>);
+    e = cudaFuncGetAttributes(&fa, attn_tc_kernel<DHP, NQ, DH>);
     if (e != cudaSuccess) return e;
     if (Cfg::kSplitRegs && fa.numRegs != Cfg::kRegsLaunch) return cudaErrorInvalidConfiguration;
     configured = true;
   }
   dim3 grid((N + 128 * NQ - 1) / (128 * NQ), nslots * heads);
-  const float scale_log2 = 1.4426950408889634f / sqrtf((float)DHP);
-  attn_tc_kernel<DHP, NQ><<<grid, Cfg::kThreads, Cfg::kSmem, st>>>(tm, nslots, heads, N, o,
+  const float scale_log2 = 1.4426950408889634f / sqrtf((float)DH);
+  attn_tc_kernel<DHP, NQ, DH><<<grid, Cfg::kThreads, Cfg::kSmem, st>>>(tm, nslots, heads, N, o,
                                                                    scale_log2, err);
   return cudaGetLastError();
 }
 
 }  // namespace
 
-bool attention_tc_supported(int dh) { return dh == 64 || dh == 128; }
+bool attention_tc_supported(int dh) { return dh == 64 || dh == 72 || dh == 128; }
 
 cudaError_t launch_attention_tc(const CUtensorMap& tm, int nslots, int heads, int N, int dh,
                                 __nv_bfloat16* o, int* err, cudaStream_t st) {
   if (nslots <= 0) return cudaSuccess;
   if (dh == 64) return launch_tc<64, 2>(tm, nslots, heads, N, o, err, st);
   if (dh == 128) return launch_tc<128, 1>(tm, nslots, heads, N, o, err, st);
+  if (dh == 72) return launch_tc<128, 1, 72>(tm, nslots, heads, N, o, err, st);
   return cudaErrorInvalidValue;
 }
 

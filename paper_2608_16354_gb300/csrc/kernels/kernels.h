@@ -51,9 +51,10 @@ cudaError_t launch_attention_bf16(const __nv_bfloat16* qkv, int slots, int heads
                                   int dhp, __nv_bfloat16* o, cudaStream_t st);
 cudaError_t launch_attention_f32(const float* qkv, int slots, int heads, int N, int dh, int dhp,
                                  float* o, cudaStream_t st);
-// tcgen05 attention (dh = dhp = 64 or 128): tm is a 2-D bf16 map over the
-// q/k/v buffer viewed as [3 * slots * heads * N][dhp], box 64 x 128, 128-byte
-// swizzle; err receives a code if a bounded wait gives up
+// tcgen05 attention (dh 64, 72 or 128; dhp = dh rounded up to 16, pad
+// columns zero): tm is a 2-D bf16 map over the q/k/v buffer viewed as
+// [3 * slots * heads * N][dhp], box 64 x 128, 128-byte swizzle; o is
+// [slots][N][heads * dh]; err receives a code if a bounded wait gives up
 bool attention_tc_supported(int dh);
 cudaError_t launch_attention_tc(const CUtensorMap& tm, int nslots, int heads, int N, int dh,
                                 __nv_bfloat16* o, int* err, cudaStream_t st);

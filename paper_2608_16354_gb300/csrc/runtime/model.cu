@@ -316,7 +316,8 @@ dc_status enqueue_compute(dc_model* m, float* lat, const float* mod_k, const Slo
     dc::EpiArgs e1 = ep;
     e1.N = 3 * d; e1.bias = w.b_qkv; e1.out = qkv;
     // q/k/v tiles go out by TMA through the attention's map when dh = 64 or 128
-    e1.qkv_tma = dc::attention_tc_supported(m->dh) ? 1 : 0;
+    // head blocks of whole 64-column swizzle atoms go out by TMA
+    e1.qkv_tma = dc::attention_tc_supported(m->dh) && m->dh % 64 == 0 ? 1 : 0;
     dc::EpiArgs e2 = ep;
     e2.N = d; e2.bias = w.b_o; e2.h = m->h; e2.h_in = h_in; e2.gate_off = base + 2 * d;
     dc::EpiArgs e3 = ep;

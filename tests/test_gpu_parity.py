@@ -383,7 +383,16 @@ def test_attention_kernel_sharp_softmax(dc, dh, N, heads, slots):
         assert rel(got[s], ref) <= 1e-2, rel(got[s], ref)
 
 
-@pytest.mark.parametrize("dh,N,heads,slots", [(64, 700, 2, 2), (128, 517, 1, 2)])
+def _pad16(qkv):
+    """q/k/v planes with the head dim padded with zeros to a multiple of 16
+    (the layout the bf16 attention entry point takes)."""
+    dh = qkv.shape[-1]
+    out = np.zeros(qkv.shape[:-1] + ((dh + 15) // 16 * 16,), np.float32)
+    out[..., :dh] = qkv
+    return out
+
+
+@pytest.mark.parametrize("dh,N,heads,slots", [(64, 700, 2, 2), (128, 517, 1, 2), (72, 600, 2, 2)])
 def test_attention_kernel_growing_logits(dc, dh, N, heads, slots):
     """Key norms ramp up 1 -> 5 along the sequence, so each row's running max
     keeps rising tile after tile: the running reference moves (and the
@@ -395,8 +404,8 @@ def test_attention_kernel_growing_logits(dc, dh, N, heads, slots):
     qkv[...] = rng.standard_normal((3, slots, heads, N, dh))
     qkv[0] *= 2.0
     qkv[1] *= np.linspace(1.0, 5.0, N, dtype=np.float32)[None, None, :, None]
-    t = torch.tensor(qkv, device="cuda").to(torch.bfloat16)
-    ref_in = t.float().cpu().numpy()
+    t = torch.tensor(_pad16(qkv), device="cuda").to(torch.bfloat16)
+    ref_in = t.float().cpu().numpy()[..., :dh]
     out = torch.zeros((slots, N, heads * dh), device="cuda", dtype=torch.bfloat16)
     dc.attention(t, slots, heads, N, dh, out)
     torch.cuda.synchronize()
@@ -408,7 +417,7 @@ def test_attention_kernel_growing_logits(dc, dh, N, heads, slots):
         assert rel(got[s], ref) <= 1e-2, rel(got[s], ref)
 
 
-@pytest.mark.parametrize("dh,N,heads,slots", [(64, 300, 40, 4), (128, 300, 30, 4)])
+@pytest.mark.parametrize("dh,N,heads,slots", [(64, 300, 40, 4), (128, 300, 30, 4), (72, 300, 32, 4)])
 def test_attention_kernel_many_items_per_cta(dc, dh, N, heads, slots):
     """More (slot, head, query block) work items than SMs, so the launch runs
     in several waves and every SM processes two or more items: each item must
@@ -423,8 +432,8 @@ def test_attention_kernel_many_items_per_cta(dc, dh, N, heads, slots):
     # a different scale per (slot, head), so that an item reading another
     # item's state or rows would show
     qkv[0] *= rng.uniform(0.3, 1.5, (slots, heads))[:, :, None, None].astype(np.float32)
-    t = torch.tensor(qkv, device="cuda").to(torch.bfloat16)
-    ref_in = t.float().cpu().numpy()
+    t = torch.tensor(_pad16(qkv), device="cuda").to(torch.bfloat16)
+    ref_in = t.float().cpu().numpy()[..., :dh]
     out = torch.full((slots, N, heads * dh), float("nan"), device="cuda", dtype=torch.bfloat16)
     dc.attention(t, slots, heads, N, dh, out)
     torch.cuda.synchronize()
