@@ -392,11 +392,11 @@ def main():
         one_call()
     ref_exec = None
     clocks = Clocks(local)
-    dc.profile(model, True)
     barrier()
     torch.cuda.synchronize()
     clocks.start()
-    # the timed region is the profiler range (ncu --profile-from-start off)
+    # the timed region is the profiler range (ncu --profile-from-start off);
+    # no per-kernel events inside it (they add about 6 % to a step)
     torch.cuda.profiler.start()
     ms_list, launches, calls = [], 0, 0
     for _ in range(args.steps):
@@ -412,6 +412,12 @@ def main():
     torch.cuda.profiler.stop()
     barrier()
     clk = clocks.stop()
+    # the same steps once more with CUDA events around every launch (on the
+    # call's stream): per-kernel device times for the roofline and the table
+    dc.profile(model, True)
+    for _ in range(args.steps):
+        _, st = one_call()
+        assert np.array_equal(ref_exec, st["executed"]), "schedule changed between steps"
     dc.profile(model, False)
     prof = dc.profile_read(model)
     total_ms = sum(ms_list)
@@ -495,7 +501,9 @@ def main():
                 "h2d_bytes_per_step": int(x1.numel() * 4), "d2h_bytes_per_step": int(x1.numel() * 4)},
         "roofline": {"kernel": dom, "bound": "tensor" if tensor else "hbm", "achieved": achieved,
                      "peak": peak, "unit": unit, "frac": achieved / peak, "traffic": traffic,
-                     "peak_source": f"{pk_src} ({'bf16 sustained' if tensor else 'HBM copy'})"},
+                     "peak_source": f"{pk_src} ({'bf16 sustained' if tensor else 'HBM copy'})",
+                     "timing": "CUDA events around every launch, over a repetition of the timed "
+                               "steps right after them (the same schedule)"},
         "kernels": kernels,
         "clocks": clk,
     }
