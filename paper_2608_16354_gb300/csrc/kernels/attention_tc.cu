@@ -261,6 +261,9 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  // the prologue above overlaps the previous kernel; q/k/v are read below
+  pdl_trigger();
+  pdl_wait();
   const uint32_t tmem = bar->tmem_base;
   if (bar->abort != 0) {
     // a bounded wait of an earlier launch gave up: do nothing (the host
@@ -595,9 +598,8 @@ cudaError_t launch_tc(const CUtensorMap& tm, int nslots, int heads, int N, __nv_
   }
   dim3 grid((N + 128 * NQ - 1) / (128 * NQ), nslots * heads);
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)DH);
-  attn_tc_kernel<DHP, NQ, DH><<<grid, Cfg::kThreads, Cfg::kSmem, st>>>(tm, nslots, heads, N, o,
-                                                                   scale_log2, err);
-  return cudaGetLastError();
+  return launch_pdl(attn_tc_kernel<DHP, NQ, DH>, grid, dim3(Cfg::kThreads), Cfg::kSmem, st, tm,
+                    nslots, heads, N, o, scale_log2, err);
 }
 
 }  // namespace

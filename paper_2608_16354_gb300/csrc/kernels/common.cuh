@@ -390,6 +390,34 @@ __device__ __forceinline__ uint64_t sw128_kmajor_desc(uint32_t start) {
 }
 
 // Instruction descriptor, kind::f16: bf16 A and B (K-major), fp32 D, M x N.
+// ------------------------------------------- programmatic dependent launch
+// A kernel launched with launch_pdl may start while the previous kernel of
+// its stream is still finishing.  pdl_wait() blocks until that kernel has
+// completed and its memory is visible (a no-op for an ordinary launch);
+// pdl_trigger() lets the next kernel launch once every CTA of this one has
+// passed it.  Work before pdl_wait() must not read what the previous kernel
+// writes.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t st, Args... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr{};
+  attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr.val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 // ------------------------------------------------ CTA pairs (cta_group::2)
 // A pair of CTAs (cluster ranks 0 and 1) shares one M=256 MMA: rank 0 issues
 // it, each CTA holds its 128 rows of A and half of the B columns in its own

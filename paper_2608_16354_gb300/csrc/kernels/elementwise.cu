@@ -96,6 +96,8 @@ template <typename T, int C>
 __global__ void embed_kernel(const float* __restrict__ x, const float* __restrict__ w_eT,
                              const float* __restrict__ b_e, const T* __restrict__ pos, SlotMap map,
                              int N, int d, float* __restrict__ u) {
+  pdl_trigger();
+  pdl_wait();
   const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int d4 = d >> 2;
   const size_t total = (size_t)map.n * N * d4;
@@ -185,6 +187,8 @@ template <typename T, int NV>
 __global__ void ln_mod_kernel(const float* __restrict__ h, int rows, int N, int d,
                               const float* __restrict__ mod, int mod_stride, int shift_off,
                               int scale_off, SlotMap map, T* __restrict__ a) {
+  pdl_trigger();
+  pdl_wait();
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (row >= rows) return;
@@ -261,6 +265,8 @@ __global__ void final_compute_kernel(const float* __restrict__ hL, const float* 
                                      const float* __restrict__ mod, int mod_stride, int fin_off,
                                      const float* __restrict__ w_f, const float* __restrict__ b_f,
                                      float dsig, float* __restrict__ vout) {
+  pdl_trigger();
+  pdl_wait();
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;  // slot * N + tok
   const int lane = threadIdx.x & 31;
   if (row >= map.n * N) return;
@@ -307,6 +313,8 @@ __global__ void final_reuse_kernel(float* __restrict__ x, const T* __restrict__ 
                                    const float* __restrict__ mod, int mod_stride, int fin_off,
                                    const float* __restrict__ w_f, const float* __restrict__ b_f,
                                    float dsig, float* __restrict__ vout) {
+  pdl_trigger();
+  pdl_wait();
   const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (row >= map.n * N) return;
@@ -506,14 +514,13 @@ cudaError_t launch_embed(const float* x, const float* w_eT, const float* b_e, co
   if (map.n <= 0) return cudaSuccess;
   const size_t n = (size_t)map.n * N * (d / 4);
   const unsigned blocks = (unsigned)((n + 255) / 256);
-  if (C == 16) {
-    embed_kernel<T, 16><<<blocks, 256, 0, st>>>(x, w_eT, b_e, pos, map, N, d, u);
-  } else if (C == 4) {
-    embed_kernel<T, 4><<<blocks, 256, 0, st>>>(x, w_eT, b_e, pos, map, N, d, u);
-  } else {
-    return cudaErrorInvalidValue;
-  }
-  return cudaGetLastError();
+  if (C == 16)
+    return launch_pdl(embed_kernel<T, 16>, dim3(blocks), dim3(256), 0, st, x, w_eT, b_e, pos, map,
+                      N, d, u);
+  if (C == 4)
+    return launch_pdl(embed_kernel<T, 4>, dim3(blocks), dim3(256), 0, st, x, w_eT, b_e, pos, map,
+                      N, d, u);
+  return cudaErrorInvalidValue;
 }
 template cudaError_t launch_embed<float>(const float*, const float*, const float*, const float*,
                                          const SlotMap&, int, int, int, float*, cudaStream_t);
@@ -527,8 +534,9 @@ cudaError_t launch_ln_mod(const float* h, int rows, int N, int d, const float* m
   if (rows <= 0) return cudaSuccess;
   const int threads = 256;
   const int blocks = (int)(((size_t)rows * 32 + threads - 1) / threads);
-  DC_NV_SWITCH(nv_for(d), (ln_mod_kernel<T, NV><<<blocks, threads, 0, st>>>(
-                              h, rows, N, d, mod, mod_stride, shift_off, scale_off, map, a)));
+  DC_NV_SWITCH(nv_for(d), return launch_pdl(ln_mod_kernel<T, NV>, dim3(blocks), dim3(threads), 0,
+                                             st, h, rows, N, d, mod, mod_stride, shift_off,
+                                             scale_off, map, a));
   return cudaGetLastError();
 }
 template cudaError_t launch_ln_mod<float>(const float*, int, int, int, const float*, int, int, int,
@@ -547,13 +555,13 @@ cudaError_t launch_final_compute(const float* hL, const float* u, float* x, floa
   const int threads = 256;
   const int blocks = (int)(((size_t)rows * 32 + threads - 1) / threads);
   if (C == 16) {
-    DC_NV_SWITCH(nv_for(d), (final_compute_kernel<T, NV, 16><<<blocks, threads, 0, st>>>(
-                                hL, u, x, xj, r, map, N, d, mod, mod_stride, fin_off, w_f, b_f, dsig,
-                                vout)));
+    DC_NV_SWITCH(nv_for(d), return launch_pdl(final_compute_kernel<T, NV, 16>, dim3(blocks),
+                                               dim3(threads), 0, st, hL, u, x, xj, r, map, N, d,
+                                               mod, mod_stride, fin_off, w_f, b_f, dsig, vout));
   } else if (C == 4) {
-    DC_NV_SWITCH(nv_for(d), (final_compute_kernel<T, NV, 4><<<blocks, threads, 0, st>>>(
-                                hL, u, x, xj, r, map, N, d, mod, mod_stride, fin_off, w_f, b_f, dsig,
-                                vout)));
+    DC_NV_SWITCH(nv_for(d), return launch_pdl(final_compute_kernel<T, NV, 4>, dim3(blocks),
+                                               dim3(threads), 0, st, hL, u, x, xj, r, map, N, d,
+                                               mod, mod_stride, fin_off, w_f, b_f, dsig, vout));
   } else {
     return cudaErrorInvalidValue;
   }
@@ -578,13 +586,13 @@ cudaError_t launch_final_reuse(float* x, const T* r, const float* w_e, const flo
   const int threads = 256;
   const int blocks = (int)(((size_t)rows * 32 + threads - 1) / threads);
   if (C == 16) {
-    DC_NV_SWITCH(nv_for(d), (final_reuse_kernel<T, NV, 16><<<blocks, threads, 0, st>>>(
-                                x, r, w_e, b_e, pos, map, N, d, mod, mod_stride, fin_off, w_f, b_f, dsig,
-                                vout)));
+    DC_NV_SWITCH(nv_for(d), return launch_pdl(final_reuse_kernel<T, NV, 16>, dim3(blocks),
+                                               dim3(threads), 0, st, x, r, w_e, b_e, pos, map, N,
+                                               d, mod, mod_stride, fin_off, w_f, b_f, dsig, vout));
   } else if (C == 4) {
-    DC_NV_SWITCH(nv_for(d), (final_reuse_kernel<T, NV, 4><<<blocks, threads, 0, st>>>(
-                                x, r, w_e, b_e, pos, map, N, d, mod, mod_stride, fin_off, w_f, b_f, dsig,
-                                vout)));
+    DC_NV_SWITCH(nv_for(d), return launch_pdl(final_reuse_kernel<T, NV, 4>, dim3(blocks),
+                                               dim3(threads), 0, st, x, r, w_e, b_e, pos, map, N,
+                                               d, mod, mod_stride, fin_off, w_f, b_f, dsig, vout));
   } else {
     return cudaErrorInvalidValue;
   }

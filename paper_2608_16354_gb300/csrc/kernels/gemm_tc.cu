@@ -140,6 +140,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   tc_fence_before();
   cluster_sync();
   tc_fence_after();
+  // the prologue above overlaps the previous kernel; its outputs are read below
+  pdl_trigger();
+  pdl_wait();
   const uint32_t tmem_base = bar->tmem_base;
   // a bounded wait of an earlier launch gave up: do nothing (the host reports
   // DC_ERR_DEVICE_TIMEOUT at its next check), but still meet the peer at the
@@ -486,9 +489,8 @@ cudaError_t launch_mode(const CUtensorMap& tmA, const CUtensorMap& tmB, const CU
   // clusters of two CTAs over pairs of m tiles (the grid is even)
   const int pair_tiles = ((M + kBM - 1) / kBM + 1) / 2 * (N / kBN);
   const int grid = 2 * (pair_tiles < n_sms / 2 ? pair_tiles : n_sms / 2);
-  gemm_bf16_tc_kernel<MODE><<<grid, kThreads, Cfg::kSmem, st>>>(tmA, tmB, tmCin, tmCout, M, N, K,
-                                                                ep, map, err);
-  return cudaGetLastError();
+  return launch_pdl(gemm_bf16_tc_kernel<MODE>, dim3(grid), dim3(kThreads), Cfg::kSmem, st, tmA,
+                    tmB, tmCin, tmCout, M, N, K, ep, map, err);
 }
 
 }  // namespace
