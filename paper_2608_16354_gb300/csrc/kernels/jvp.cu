@@ -173,105 +173,231 @@ __global__ void embed_f32_kernel(const float* __restrict__ x, const float* __res
 
 // Attention over all tokens of the one primal scene, and (TAN) its tangent
 // for T perturbations: qkv [N][3d] primal rows ([q | k | v], heads
-// contiguous), dqkv [T][N][3d].  Four threads per query row, each owning
-// DH/4 of the head dimensions; keys in tiles of 16 with an online softmax
+// contiguous), dqkv [T][N][3d].  Keys stream in tiles with an online softmax
 // (running max m, sum l) and, for the tangent, the running sums
 //   b = sum w ds,  Cv = sum w ds v,  Dv = sum w dv   (w = exp(s - m))
-// so that do = (Cv - (b / l) A + Dv) / l with A = sum w v.
+// so that do = (Cv - (b / l) A + Dv) / l with A = sum w v.  A block of 128 threads
+// takes BQ = 16 RQ query rows of one head (RQ = 4, or 2 at head dim 128) and
+// streams the keys in tiles of 32.  Thread t owns rows rg RQ .. rg RQ + RQ-1
+// (rg = t / 8) and, with g = t % 8:
+//   phase 1  s and ds of its rows against keys 4g .. 4g+3 of the tile
+//            (RQ x 4 register block; q, dq, k, dk read as float4 from
+//            transposed tiles in shared memory);
+//   phase 2  the online softmax of its rows, the tile's row max and sums
+//            reduced over the 8 lanes g that share the rows; w and w ds go
+//            to shared memory;
+//   phase 3  A, Cv, Dv of its rows for head dimensions g DH/8 .. (g+1) DH/8-1
+//            (RQ x DH/8 register block over the tile's 32 keys).
+// The lanes that share rows sit in one warp, so the running max m, sum l and
+// b = sum w ds live in registers of the same thread in all three phases.
 template <int DH, bool TAN>
-__global__ void __launch_bounds__(128) attn_f32_jvp_kernel(const float* __restrict__ qkv,
-                                                           const float* __restrict__ dqkv, int N,
-                                                           int d, float scale,
-                                                           float* __restrict__ o,
-                                                           float* __restrict__ dout) {
-  constexpr int D4 = DH / 4, KT = 16;
-  __shared__ float sK[KT][DH], sV[KT][DH], sdK[TAN ? KT : 1][DH], sdV[TAN ? KT : 1][DH];
-  const int g = threadIdx.x & 3, qi = threadIdx.x >> 2;
+struct JvpTile {
+  static constexpr int RQ = DH >= 128 ? 2 : 4, BQ = 16 * RQ, BK = 32, DG = DH / 8;
+  // shared memory (floats): q^T, dq^T [DH][BQ]; k^T, dk^T [DH][BK]; v, dv
+  // [BK][DH]; w, w ds [BK][BQ]
+  static constexpr int kQ = DH * BQ, kK = DH * BK, kW = BK * BQ;
+  static constexpr int kFloats = (TAN ? 2 : 1) * (kQ + 2 * kK) + (TAN ? 2 : 1) * kW;
+  static constexpr size_t kBytes = (size_t)kFloats * 4;
+};
+
+template <int DH, bool TAN>
+__global__ void __launch_bounds__(128) attn_f32_jvp_tiled_kernel(
+    const float* __restrict__ qkv, const float* __restrict__ dqkv, int N, int d, float scale,
+    float* __restrict__ o, float* __restrict__ dout) {
+  using Tl = JvpTile<DH, TAN>;
+  constexpr int RQ = Tl::RQ, BQ = Tl::BQ, BK = Tl::BK, DG = Tl::DG;
+  extern __shared__ float4 jvp_smem4[];
+  float* sm = reinterpret_cast<float*>(jvp_smem4);
+  float* sQ = sm;                                  // [DH][BQ]
+  float* sK = sQ + Tl::kQ;                         // [DH][BK]
+  float* sV = sK + Tl::kK;                         // [BK][DH]
+  float* sdQ = sV + Tl::kK;                        // (TAN) [DH][BQ]
+  float* sdK = sdQ + (TAN ? Tl::kQ : 0);           // (TAN) [DH][BK]
+  float* sdV = sdK + (TAN ? Tl::kK : 0);           // (TAN) [BK][DH]
+  float* sW = sdV + (TAN ? Tl::kK : 0);            // [BK][BQ]
+  float* sWd = sW + Tl::kW;                        // (TAN) [BK][BQ]
+  const int tid = threadIdx.x, rg = tid >> 3, g = tid & 7;
   const int head = blockIdx.y, t = blockIdx.z;
-  const int n = blockIdx.x * 32 + qi;
-  const bool live = n < N;
+  const int q0 = blockIdx.x * BQ;
   const size_t ld = (size_t)3 * d;
   const float* dbase = TAN ? dqkv + (size_t)t * N * ld : nullptr;
-  float q[D4], dq[D4], A[D4], Cv[D4], Dv[D4];
-#pragma unroll
-  for (int e = 0; e < D4; ++e) {
-    const int col = head * DH + g * D4 + e;
-    q[e] = live ? qkv[(size_t)n * ld + col] : 0.f;
-    dq[e] = (TAN && live) ? dbase[(size_t)n * ld + col] : 0.f;
-    A[e] = Cv[e] = Dv[e] = 0.f;
+  constexpr int D4 = DH / 4;
+  // queries of the block, transposed (row index fastest across threads, so
+  // the transposed stores hit distinct banks)
+  for (int i = tid; i < BQ * D4; i += 128) {
+    const int r = i % BQ, e4 = i / BQ, n = q0 + r;
+    const bool in = n < N;
+    const size_t at = (size_t)n * ld + head * DH + 4 * e4;
+    const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+    const float4 a = in ? *reinterpret_cast<const float4*>(qkv + at) : z;
+    sQ[(4 * e4 + 0) * BQ + r] = a.x; sQ[(4 * e4 + 1) * BQ + r] = a.y;
+    sQ[(4 * e4 + 2) * BQ + r] = a.z; sQ[(4 * e4 + 3) * BQ + r] = a.w;
+    if (TAN) {
+      const float4 da = in ? *reinterpret_cast<const float4*>(dbase + at) : z;
+      sdQ[(4 * e4 + 0) * BQ + r] = da.x; sdQ[(4 * e4 + 1) * BQ + r] = da.y;
+      sdQ[(4 * e4 + 2) * BQ + r] = da.z; sdQ[(4 * e4 + 3) * BQ + r] = da.w;
+    }
   }
-  float m = -INFINITY, l = 0.f, b = 0.f;
-  for (int k0 = 0; k0 < N; k0 += KT) {
-    __syncthreads();
-    for (int i = threadIdx.x; i < KT * DH; i += 128) {
-      const int kk = i / DH, e = i % DH, key = k0 + kk;
+  float A[RQ][DG], Cv[RQ][DG], Dv[RQ][DG];
+#pragma unroll
+  for (int r = 0; r < RQ; ++r)
+#pragma unroll
+    for (int e = 0; e < DG; ++e) A[r][e] = Cv[r][e] = Dv[r][e] = 0.f;
+  float m[RQ], l[RQ], b[RQ];
+#pragma unroll
+  for (int r = 0; r < RQ; ++r) { m[r] = -INFINITY; l[r] = 0.f; b[r] = 0.f; }
+
+  for (int k0 = 0; k0 < N; k0 += BK) {
+    __syncthreads();  // the previous tile's k, v, w are consumed
+    const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int i = tid; i < BK * D4; i += 128) {
+      // k, dk transposed: key index fastest across threads
+      const int j = i % BK, e4 = i / BK, key = k0 + j;
       const bool in = key < N;
-      sK[kk][e] = in ? qkv[(size_t)key * ld + d + head * DH + e] : 0.f;
-      sV[kk][e] = in ? qkv[(size_t)key * ld + 2 * d + head * DH + e] : 0.f;
+      const size_t at = (size_t)key * ld + d + head * DH + 4 * e4;
+      const float4 a = in ? *reinterpret_cast<const float4*>(qkv + at) : z;
+      sK[(4 * e4 + 0) * BK + j] = a.x; sK[(4 * e4 + 1) * BK + j] = a.y;
+      sK[(4 * e4 + 2) * BK + j] = a.z; sK[(4 * e4 + 3) * BK + j] = a.w;
       if (TAN) {
-        sdK[kk][e] = in ? dbase[(size_t)key * ld + d + head * DH + e] : 0.f;
-        sdV[kk][e] = in ? dbase[(size_t)key * ld + 2 * d + head * DH + e] : 0.f;
+        const float4 da = in ? *reinterpret_cast<const float4*>(dbase + at) : z;
+        sdK[(4 * e4 + 0) * BK + j] = da.x; sdK[(4 * e4 + 1) * BK + j] = da.y;
+        sdK[(4 * e4 + 2) * BK + j] = da.z; sdK[(4 * e4 + 3) * BK + j] = da.w;
       }
+    }
+    for (int i = tid; i < BK * D4; i += 128) {
+      // v, dv as rows: head dimension fastest
+      const int e4 = i % D4, j = i / D4, key = k0 + j;
+      const bool in = key < N;
+      const size_t at = (size_t)key * ld + 2 * (size_t)d + head * DH + 4 * e4;
+      *reinterpret_cast<float4*>(sV + j * DH + 4 * e4) =
+          in ? *reinterpret_cast<const float4*>(qkv + at) : z;
+      if (TAN)
+        *reinterpret_cast<float4*>(sdV + j * DH + 4 * e4) =
+            in ? *reinterpret_cast<const float4*>(dbase + at) : z;
     }
     __syncthreads();
-    float s[KT], ds[KT];
-    float tmax = -INFINITY;
+    // phase 1: s, ds for rows rg RQ + r and keys 4 g + c
+    float s[RQ][4], ds[RQ][4];
 #pragma unroll
-    for (int kk = 0; kk < KT; ++kk) {
-      float a = 0.f, da = 0.f;
+    for (int r = 0; r < RQ; ++r)
 #pragma unroll
-      for (int e = 0; e < D4; ++e) {
-        a = fmaf(q[e], sK[kk][g * D4 + e], a);
-        if (TAN) da = fmaf(dq[e], sK[kk][g * D4 + e], fmaf(q[e], sdK[kk][g * D4 + e], da));
-      }
-      a += __shfl_xor_sync(0xffffffffu, a, 1);
-      a += __shfl_xor_sync(0xffffffffu, a, 2);
-      if (TAN) {
-        da += __shfl_xor_sync(0xffffffffu, da, 1);
-        da += __shfl_xor_sync(0xffffffffu, da, 2);
-      }
-      const bool in = k0 + kk < N;
-      s[kk] = in ? a * scale : -INFINITY;
-      ds[kk] = da * scale;
-      tmax = fmaxf(tmax, s[kk]);
-    }
-    const float mn = fmaxf(m, tmax);
-    const float c = m == -INFINITY ? 0.f : expf(m - mn);
-    l *= c;
-    b *= c;
-#pragma unroll
-    for (int e = 0; e < D4; ++e) {
-      A[e] *= c;
-      Cv[e] *= c;
-      Dv[e] *= c;
-    }
-#pragma unroll
-    for (int kk = 0; kk < KT; ++kk) {
-      const float w = expf(s[kk] - mn);  // 0 for masked keys
-      l += w;
-      if (TAN) b = fmaf(w, ds[kk], b);
-#pragma unroll
-      for (int e = 0; e < D4; ++e) {
-        const float v = sV[kk][g * D4 + e];
-        A[e] = fmaf(w, v, A[e]);
+      for (int c = 0; c < 4; ++c) s[r][c] = ds[r][c] = 0.f;
+#pragma unroll 4
+    for (int e = 0; e < DH; ++e) {
+      float qv[RQ], dqv[RQ];
+      if constexpr (RQ == 4) {
+        const float4 a = *reinterpret_cast<const float4*>(sQ + e * BQ + rg * 4);
+        qv[0] = a.x; qv[1] = a.y; qv[2] = a.z; qv[3] = a.w;
         if (TAN) {
-          Cv[e] = fmaf(w * ds[kk], v, Cv[e]);
-          Dv[e] = fmaf(w, sdV[kk][g * D4 + e], Dv[e]);
+          const float4 da = *reinterpret_cast<const float4*>(sdQ + e * BQ + rg * 4);
+          dqv[0] = da.x; dqv[1] = da.y; dqv[2] = da.z; dqv[3] = da.w;
+        }
+      } else {
+        const float2 a = *reinterpret_cast<const float2*>(sQ + e * BQ + rg * 2);
+        qv[0] = a.x; qv[1] = a.y;
+        if (TAN) {
+          const float2 da = *reinterpret_cast<const float2*>(sdQ + e * BQ + rg * 2);
+          dqv[0] = da.x; dqv[1] = da.y;
+        }
+      }
+      const float4 kv = *reinterpret_cast<const float4*>(sK + e * BK + g * 4);
+      const float kk[4] = {kv.x, kv.y, kv.z, kv.w};
+      float dkk[4] = {0.f, 0.f, 0.f, 0.f};
+      if (TAN) {
+        const float4 dk = *reinterpret_cast<const float4*>(sdK + e * BK + g * 4);
+        dkk[0] = dk.x; dkk[1] = dk.y; dkk[2] = dk.z; dkk[3] = dk.w;
+      }
+#pragma unroll
+      for (int r = 0; r < RQ; ++r)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          s[r][c] = fmaf(qv[r], kk[c], s[r][c]);
+          if (TAN) ds[r][c] = fmaf(dqv[r], kk[c], fmaf(qv[r], dkk[c], ds[r][c]));
+        }
+    }
+    // phase 2: online softmax over the tile's 32 keys of each row
+#pragma unroll
+    for (int r = 0; r < RQ; ++r) {
+      float tmax = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const bool in = k0 + g * 4 + c < N;
+        s[r][c] = in ? s[r][c] * scale : -INFINITY;
+        ds[r][c] *= scale;
+        tmax = fmaxf(tmax, s[r][c]);
+      }
+      tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 1));
+      tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 2));
+      tmax = fmaxf(tmax, __shfl_xor_sync(0xffffffffu, tmax, 4));
+      const float mn = fmaxf(m[r], tmax);
+      const float cf = m[r] == -INFINITY ? 0.f : expf(m[r] - mn);
+      float ls = 0.f, bs = 0.f;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const float w = expf(s[r][c] - mn);  // 0 for masked keys
+        ls += w;
+        sW[(g * 4 + c) * BQ + rg * RQ + r] = w;
+        if (TAN) {
+          bs = fmaf(w, ds[r][c], bs);
+          sWd[(g * 4 + c) * BQ + rg * RQ + r] = w * ds[r][c];
+        }
+      }
+      ls += __shfl_xor_sync(0xffffffffu, ls, 1);
+      ls += __shfl_xor_sync(0xffffffffu, ls, 2);
+      ls += __shfl_xor_sync(0xffffffffu, ls, 4);
+      l[r] = l[r] * cf + ls;
+      if (TAN) {
+        bs += __shfl_xor_sync(0xffffffffu, bs, 1);
+        bs += __shfl_xor_sync(0xffffffffu, bs, 2);
+        bs += __shfl_xor_sync(0xffffffffu, bs, 4);
+        b[r] = b[r] * cf + bs;
+      }
+      m[r] = mn;
+#pragma unroll
+      for (int e = 0; e < DG; ++e) {
+        A[r][e] *= cf;
+        if (TAN) { Cv[r][e] *= cf; Dv[r][e] *= cf; }
+      }
+    }
+    __syncwarp();  // w of the 8 lanes g is in shared memory (one warp owns these rows)
+    // phase 3: accumulate over the tile's keys
+#pragma unroll 2
+    for (int j = 0; j < BK; ++j) {
+      float wv[RQ], wdv[RQ];
+#pragma unroll
+      for (int r = 0; r < RQ; ++r) {
+        wv[r] = sW[j * BQ + rg * RQ + r];
+        if (TAN) wdv[r] = sWd[j * BQ + rg * RQ + r];
+      }
+#pragma unroll
+      for (int e = 0; e < DG; ++e) {
+        const float v = sV[j * DH + g * DG + e];
+        const float dv = TAN ? sdV[j * DH + g * DG + e] : 0.f;
+#pragma unroll
+        for (int r = 0; r < RQ; ++r) {
+          A[r][e] = fmaf(wv[r], v, A[r][e]);
+          if (TAN) {
+            Cv[r][e] = fmaf(wdv[r], v, Cv[r][e]);
+            Dv[r][e] = fmaf(wv[r], dv, Dv[r][e]);
+          }
         }
       }
     }
-    m = mn;
   }
-  if (!live) return;
-  const float inv = 1.0f / l;
-  const float beta = b * inv;
 #pragma unroll
-  for (int e = 0; e < D4; ++e) {
-    const int col = head * DH + g * D4 + e;
-    if (TAN)
-      dout[((size_t)t * N + n) * d + col] = (Cv[e] - beta * A[e] + Dv[e]) * inv;
-    else
-      o[(size_t)n * d + col] = A[e] * inv;
+  for (int r = 0; r < RQ; ++r) {
+    const int n = q0 + rg * RQ + r;
+    if (n >= N) continue;
+    const float inv = 1.0f / l[r];
+    const float beta = b[r] * inv;
+#pragma unroll
+    for (int e = 0; e < DG; ++e) {
+      const int col = head * DH + g * DG + e;
+      if (TAN)
+        dout[((size_t)t * N + n) * d + col] = (Cv[r][e] - beta * A[r][e] + Dv[r][e]) * inv;
+      else
+        o[(size_t)n * d + col] = A[r][e] * inv;
+    }
   }
 }
 
@@ -343,6 +469,24 @@ template cudaError_t launch_embed_f32<__nv_bfloat16>(const float*, const float*,
                                                      const __nv_bfloat16*, int, int, int, int,
                                                      float*, cudaStream_t);
 
+namespace {
+template <int DH, bool TAN>
+cudaError_t launch_jvp_tiled(const float* qkv, const float* dqkv, int N, int d, int heads, int T,
+                             float scale, float* o, float* dout, cudaStream_t st) {
+  using Tl = JvpTile<DH, TAN>;
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(attn_f32_jvp_tiled_kernel<DH, TAN>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Tl::kBytes);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  dim3 grid((N + Tl::BQ - 1) / Tl::BQ, heads, T);
+  attn_f32_jvp_tiled_kernel<DH, TAN><<<grid, 128, Tl::kBytes, st>>>(qkv, dqkv, N, d, scale, o, dout);
+  return cudaGetLastError();
+}
+}  // namespace
+
 bool attention_f32_jvp_supported(int dh) {
   return dh == 8 || dh == 16 || dh == 32 || dh == 64 || dh == 72 || dh == 128;
 }
@@ -352,14 +496,10 @@ cudaError_t launch_attention_f32_jvp(const float* qkv, const float* dqkv, int N,
   if (N <= 0) return cudaSuccess;
   const float scale = 1.0f / sqrtf((float)dh);
   const bool tan = dqkv != nullptr;
-  dim3 grid((N + 31) / 32, heads, tan ? T : 1);
-#define DC_ATT_JVP(DHV)                                                                     \
-  if (dh == DHV) {                                                                          \
-    if (tan)                                                                                \
-      attn_f32_jvp_kernel<DHV, true><<<grid, 128, 0, st>>>(qkv, dqkv, N, d, scale, o, dout); \
-    else                                                                                    \
-      attn_f32_jvp_kernel<DHV, false><<<grid, 128, 0, st>>>(qkv, dqkv, N, d, scale, o, dout); \
-    return cudaGetLastError();                                                              \
+#define DC_ATT_JVP(DHV)                                                                      \
+  if (dh == DHV) {                                                                           \
+    if (tan) return launch_jvp_tiled<DHV, true>(qkv, dqkv, N, d, heads, T, scale, o, dout, st); \
+    return launch_jvp_tiled<DHV, false>(qkv, dqkv, N, d, heads, 1, scale, o, dout, st);       \
   }
   DC_ATT_JVP(8)
   DC_ATT_JVP(16)
