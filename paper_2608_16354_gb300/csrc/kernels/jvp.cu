@@ -186,8 +186,9 @@ __global__ void embed_f32_kernel(const float* __restrict__ x, const float* __res
 //   phase 2  the online softmax of its rows, the tile's row max and sums
 //            reduced over the 8 lanes g that share the rows; w and w ds go
 //            to shared memory;
-//   phase 3  A, Cv, Dv of its rows for head dimensions g DH/8 .. (g+1) DH/8-1
-//            (RQ x DH/8 register block over the tile's 32 keys).
+//   phase 3  A, Cv, Dv of its rows for head dimensions g, g + 8, g + 16, ...
+//            (RQ x DH/8 register block over the tile's 32 keys; the eight
+//            lanes g read eight consecutive banks of a value row).
 // The lanes that share rows sit in one warp, so the running max m, sum l and
 // b = sum w ds live in registers of the same thread in all three phases.
 template <int DH, bool TAN>
@@ -371,8 +372,8 @@ __global__ void __launch_bounds__(128) attn_f32_jvp_tiled_kernel(
       }
 #pragma unroll
       for (int e = 0; e < DG; ++e) {
-        const float v = sV[j * DH + g * DG + e];
-        const float dv = TAN ? sdV[j * DH + g * DG + e] : 0.f;
+        const float v = sV[j * DH + g + 8 * e];
+        const float dv = TAN ? sdV[j * DH + g + 8 * e] : 0.f;
 #pragma unroll
         for (int r = 0; r < RQ; ++r) {
           A[r][e] = fmaf(wv[r], v, A[r][e]);
@@ -392,7 +393,7 @@ __global__ void __launch_bounds__(128) attn_f32_jvp_tiled_kernel(
     const float beta = b[r] * inv;
 #pragma unroll
     for (int e = 0; e < DG; ++e) {
-      const int col = head * DH + g * DG + e;
+      const int col = head * DH + g + 8 * e;
       if (TAN)
         dout[((size_t)t * N + n) * d + col] = (Cv[r][e] - beta * A[r][e] + Dv[r][e]) * inv;
       else
