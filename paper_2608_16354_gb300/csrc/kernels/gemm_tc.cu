@@ -51,12 +51,15 @@ constexpr int kEpiWarps = 8;
 constexpr int kEpiThreads = kEpiWarps * 32;
 constexpr uint32_t kIdesc = idesc_bf16_f32(2 * kBM, kBN);  // one M = 256 MMA over the pair
 
-template <int MODE>
+// HALF (residual mode, long K): the fp32 residual tile is staged and
+// written in two 96-column halves, which frees 48 KB of shared memory for two
+// more ring stages.
+template <int MODE, bool HALF = false>
 struct GemmCfg {
-  static constexpr int kStages = MODE == kEpiResid ? 4 : 6;
+  static constexpr int kStages = MODE == kEpiResid && !HALF ? 4 : 6;
   // epilogue staging tile: residual 6 boxes of [128 rows][32 fp32], GELU and
   // QKV 3 boxes of [128 rows][64 bf16]; 16 KB per box, 128-byte swizzle
-  static constexpr int kOutBytes = MODE == kEpiResid ? 6 * 16384 : 3 * 16384;
+  static constexpr int kOutBytes = MODE == kEpiResid && !HALF ? 6 * 16384 : 3 * 16384;
   static constexpr int kOffA = 0;
   static constexpr int kOffB = kOffA + kStages * kABytes;
   static constexpr int kOffOut = kOffB + kStages * kBHalf;
@@ -82,15 +85,16 @@ struct __align__(8) Barriers {
 // with 128-byte swizzle (the layout TMA produces and consumes)
 __device__ __forceinline__ int sw128_off(int r, int c) { return r * 128 + ((c ^ (r & 7)) << 4); }
 
-template <int MODE>
+template <int MODE, bool HALF = false>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     gemm_bf16_tc_kernel(const __grid_constant__ CUtensorMap tmA,
                         const __grid_constant__ CUtensorMap tmB,
                         const __grid_constant__ CUtensorMap tmCin,
                         const __grid_constant__ CUtensorMap tmCout, int M, int N, int K,
                         EpiArgs ep, SlotMap map, int* err) {
-  using Cfg = GemmCfg<MODE>;
+  using Cfg = GemmCfg<MODE, HALF>;
   constexpr int kStages = Cfg::kStages;
+  constexpr int kHinBoxes = HALF ? 3 : 6;  // residual boxes staged at a time
   extern __shared__ uint8_t smem_raw[];
   const uint32_t base = smem_u32(smem_raw);
   uint8_t* smem = smem_raw + ((1024 - (base & 1023)) & 1023);
@@ -250,11 +254,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     const int et = threadIdx.x - 64;    // epilogue thread 0..255
     const bool copy_warp = warp == 2;   // issues the tile's bulk copies, one box per lane
     const int r = q * 32 + lane;        // row of the tile owned by this thread
-    int hin_loads = 0;                  // residual tiles requested so far
+    int hin_loads = 0, hin_used = 0;    // residual stagings requested / consumed
     if (MODE == kEpiResid && copy_warp && pair < n_pt) {
       if (lane == 0) mbar_arrive_expect_tx(&bar->hin_full, Cfg::kOutBytes);
       __syncwarp();
-      if (lane < 6)
+      if (lane < kHinBoxes)
         tma_load_2d(sOut + lane * 16384, &tmCin, &bar->hin_full, n0_of(pair) + 32 * lane, m0_of(pair));
       hin_loads = 1;
     }
@@ -322,55 +326,72 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         // rows spanning more than two slots (tokens per scene < 128) take the
         // gate from global memory per row
         const bool two_slots = slot_b - slot_a <= 1;
-        const bool hin_ok = mbar_wait_warp(&bar->hin_full, (uint32_t)t & 1, err, kDevTimeoutEpi);
         const int row = m0 + r;
         const float* gsel = vec + (row < split ? kBN : 2 * kBN);
         const float* grow = nullptr;
         if (!two_slots && row < M)
           grow = ep.mod + (size_t)map.scene[row / ep.n_tok] * ep.mod_stride + ep.gate_off + n0;
+        // h = h_in + gate (acc + b) on this thread's 96 columns, in the staged
+        // boxes whose first column is `base`
+        auto apply = [&](int base) {
 #pragma unroll
-        for (int c = 0; c < 3 && hin_ok; ++c) {
-          const int col0 = half * 96 + c * 32;  // tile column of this 32-column chunk
-          uint8_t* box = sOut + (col0 >> 5) * 16384;
+          for (int c = 0; c < 3; ++c) {
+            const int col0 = half * 96 + c * 32;  // tile column of this 32-column chunk
+            uint8_t* box = sOut + ((col0 - base) >> 5) * 16384;
 #pragma unroll
-          for (int ch = 0; ch < 8; ++ch) {
-            float4* p = reinterpret_cast<float4*>(box + sw128_off(r, ch));
-            float4 h = *p;
-            const int j = col0 + ch * 4;
-            float g0, g1, g2, g3;
-            if (two_slots) {
-              g0 = gsel[j]; g1 = gsel[j + 1]; g2 = gsel[j + 2]; g3 = gsel[j + 3];
-            } else if (grow) {
-              g0 = grow[j]; g1 = grow[j + 1]; g2 = grow[j + 2]; g3 = grow[j + 3];
-            } else {
-              g0 = g1 = g2 = g3 = 0.f;
+            for (int ch = 0; ch < 8; ++ch) {
+              float4* p = reinterpret_cast<float4*>(box + sw128_off(r, ch));
+              float4 h = *p;
+              const int j = col0 + ch * 4;
+              float g0, g1, g2, g3;
+              if (two_slots) {
+                g0 = gsel[j]; g1 = gsel[j + 1]; g2 = gsel[j + 2]; g3 = gsel[j + 3];
+              } else if (grow) {
+                g0 = grow[j]; g1 = grow[j + 1]; g2 = grow[j + 2]; g3 = grow[j + 3];
+              } else {
+                g0 = g1 = g2 = g3 = 0.f;
+              }
+              h.x += g0 * (acc[c][ch * 4 + 0] + vec[j + 0]);
+              h.y += g1 * (acc[c][ch * 4 + 1] + vec[j + 1]);
+              h.z += g2 * (acc[c][ch * 4 + 2] + vec[j + 2]);
+              h.w += g3 * (acc[c][ch * 4 + 3] + vec[j + 3]);
+              *p = h;
             }
-            h.x += g0 * (acc[c][ch * 4 + 0] + vec[j + 0]);
-            h.y += g1 * (acc[c][ch * 4 + 1] + vec[j + 1]);
-            h.z += g2 * (acc[c][ch * 4 + 2] + vec[j + 2]);
-            h.w += g3 * (acc[c][ch * 4 + 3] + vec[j + 3]);
-            *p = h;
+          }
+        };
+        const int next = pt + n_pairs;
+        bool failed = false;  // the same for all epilogue threads (named_bar_or)
+#pragma unroll 1
+        for (int pass = 0; pass < (HALF ? 2 : 1); ++pass) {
+          // pass p stages columns 96 p .. (all 192 without HALF)
+          const bool hin_ok = mbar_wait_warp(&bar->hin_full, HALF ? (uint32_t)pass : (uint32_t)t & 1,
+                                             err, kDevTimeoutEpi);
+          if (hin_ok) ++hin_used;
+          if (hin_ok && (!HALF || half == pass)) apply(HALF ? 96 * pass : 0);
+          fence_proxy_async();
+          failed = named_bar_or(1, kEpiThreads, !hin_ok);
+          if (failed) break;
+          if (copy_warp) {
+            const int c0 = HALF ? 96 * pass : 0;
+            if (live && lane < kHinBoxes) {
+              tma_store_2d(&tmCout, sOut + lane * 16384, n0 + c0 + 32 * lane, m0);
+              bulk_commit();
+              bulk_wait_read0();
+            }
+            __syncwarp();  // every box has been read out before the next staging lands
+            // next staging: the second half of this tile, else the next tile
+            const bool second = HALF && pass == 0;
+            if (second || next < n_pt) {
+              if (lane == 0) mbar_arrive_expect_tx(&bar->hin_full, Cfg::kOutBytes);
+              __syncwarp();
+              if (lane < kHinBoxes)
+                tma_load_2d(sOut + lane * 16384, &tmCin, &bar->hin_full,
+                            (second ? n0 + 96 : n0_of(next)) + 32 * lane, second ? m0 : m0_of(next));
+              ++hin_loads;
+            }
           }
         }
-        fence_proxy_async();
-        if (named_bar_or(1, kEpiThreads, !hin_ok)) { ok = false; break; }
-        if (copy_warp) {
-          if (live && lane < 6) {
-            tma_store_2d(&tmCout, sOut + lane * 16384, n0 + 32 * lane, m0);
-            bulk_commit();
-            bulk_wait_read0();
-          }
-          __syncwarp();  // every box has been read out before the next tile lands
-          const int next = pt + n_pairs;
-          if (next < n_pt) {
-            if (lane == 0) mbar_arrive_expect_tx(&bar->hin_full, Cfg::kOutBytes);
-            __syncwarp();
-            if (lane < 6)
-              tma_load_2d(sOut + lane * 16384, &tmCin, &bar->hin_full, n0_of(next) + 32 * lane,
-                          m0_of(next));
-            ++hin_loads;
-          }
-        }
+        if (failed) { ok = false; break; }
       } else if constexpr (MODE == kEpiGELU) {
 #pragma unroll
         for (int c = 0; c < 3; ++c) {
@@ -458,7 +479,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     if (copy_warp) {
       if (lane < 6) bulk_wait0();
       // a residual prefetch that was never consumed (aborted run) must land first
-      if (MODE == kEpiResid && lane == 0 && !ok && hin_loads > t)
+      if (MODE == kEpiResid && lane == 0 && !ok && hin_loads > hin_used)
         mbar_wait(&bar->hin_full, (uint32_t)(hin_loads - 1) & 1, err, kDevTimeoutEpi);
     }
   }
@@ -474,14 +495,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   cluster_sync();
 }
 
-template <int MODE>
+template <int MODE, bool HALF = false>
 cudaError_t launch_mode(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmCin,
                         const CUtensorMap& tmCout, int M, int N, int K, const EpiArgs& ep,
                         const SlotMap& map, int* err, int n_sms, cudaStream_t st) {
-  using Cfg = GemmCfg<MODE>;
+  using Cfg = GemmCfg<MODE, HALF>;
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_bf16_tc_kernel<MODE>,
+    cudaError_t e = cudaFuncSetAttribute(gemm_bf16_tc_kernel<MODE, HALF>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmem);
     if (e != cudaSuccess) return e;
     configured = true;
@@ -489,7 +510,7 @@ cudaError_t launch_mode(const CUtensorMap& tmA, const CUtensorMap& tmB, const CU
   // clusters of two CTAs over pairs of m tiles (the grid is even)
   const int pair_tiles = ((M + kBM - 1) / kBM + 1) / 2 * (N / kBN);
   const int grid = 2 * (pair_tiles < n_sms / 2 ? pair_tiles : n_sms / 2);
-  return launch_pdl(gemm_bf16_tc_kernel<MODE>, dim3(grid), dim3(kThreads), Cfg::kSmem, st, tmA,
+  return launch_pdl(gemm_bf16_tc_kernel<MODE, HALF>, dim3(grid), dim3(kThreads), Cfg::kSmem, st, tmA,
                     tmB, tmCin, tmCout, M, N, K, ep, map, err);
 }
 
@@ -507,6 +528,9 @@ cudaError_t launch_gemm_tc(int mode, const CUtensorMap& tmA, const CUtensorMap& 
     case kEpiGELU:
       return launch_mode<kEpiGELU>(tmA, tmB, tmCin, tmCout, M, N, K, ep, map, err, n_sms, st);
     case kEpiResid:
+      // long K: more ring stages, residual tile in two halves
+      if (K >= 1024)
+        return launch_mode<kEpiResid, true>(tmA, tmB, tmCin, tmCout, M, N, K, ep, map, err, n_sms, st);
       return launch_mode<kEpiResid>(tmA, tmB, tmCin, tmCout, M, N, K, ep, map, err, n_sms, st);
   }
   return cudaErrorInvalidValue;
