@@ -11,6 +11,43 @@
 
 namespace dc {
 
+// Packed fp32x2 arithmetic (one instruction for two lanes of work).
+__device__ __forceinline__ float2 f2_fma(float2 a, float2 b, float2 c) {
+  float2 r;
+  asm("{\n .reg .b64 a, b, c, d;\n mov.b64 a, {%2, %3};\n mov.b64 b, {%4, %5};\n"
+      " mov.b64 c, {%6, %7};\n fma.rn.f32x2 d, a, b, c;\n mov.b64 {%0, %1}, d;\n}\n"
+      : "=f"(r.x), "=f"(r.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+  return r;
+}
+__device__ __forceinline__ float2 f2_mul(float2 a, float2 b) {
+  float2 r;
+  asm("{\n .reg .b64 a, b, d;\n mov.b64 a, {%2, %3};\n mov.b64 b, {%4, %5};\n"
+      " mul.rn.f32x2 d, a, b;\n mov.b64 {%0, %1}, d;\n}\n"
+      : "=f"(r.x), "=f"(r.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return r;
+}
+__device__ __forceinline__ float2 f2_add(float2 a, float2 b) {
+  float2 r;
+  asm("{\n .reg .b64 a, b, d;\n mov.b64 a, {%2, %3};\n mov.b64 b, {%4, %5};\n"
+      " add.rn.f32x2 d, a, b;\n mov.b64 {%0, %1}, d;\n}\n"
+      : "=f"(r.x), "=f"(r.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return r;
+}
+
+// gelu_tanh of a pair: x/2 (1 + tanh(x (k0 + k0 c x^2))), packed except the
+// two hardware tanh
+__device__ __forceinline__ float2 gelu_tanh_pair(float2 x) {
+  const float k0 = 0.7978845608028654f, k1 = 0.7978845608028654f * 0.044715f;
+  const float2 x2 = f2_mul(x, x);
+  const float2 z = f2_mul(x, f2_fma(x2, make_float2(k1, k1), make_float2(k0, k0)));
+  const float2 th = make_float2(tanh_approx(z.x), tanh_approx(z.y));
+  const float2 hx = f2_mul(x, make_float2(0.5f, 0.5f));
+  return f2_fma(hx, th, hx);
+}
+
 enum { kEpiQKV = 0, kEpiGELU = 1, kEpiResid = 2 };
 
 struct EpiArgs {

@@ -401,7 +401,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             uint4 w;
             float v[8];
 #pragma unroll
-            for (int i = 0; i < 8; ++i) v[i] = gelu_tanh_bf16(acc[c][g * 8 + i] + vec[j + i]);
+            for (int i = 0; i < 8; i += 2) {
+              const float2 x = f2_add(make_float2(acc[c][g * 8 + i], acc[c][g * 8 + i + 1]),
+                                      make_float2(vec[j + i], vec[j + i + 1]));
+              const float2 y = gelu_tanh_pair(x);
+              v[i] = y.x;
+              v[i + 1] = y.y;
+            }
             __nv_bfloat162 p0 = __floats2bfloat162_rn(v[0], v[1]);
             __nv_bfloat162 p1 = __floats2bfloat162_rn(v[2], v[3]);
             __nv_bfloat162 p2 = __floats2bfloat162_rn(v[4], v[5]);
