@@ -35,6 +35,8 @@ import time
 import numpy as np
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
+# diagnostics written during a run (clock samples); DC_DIAG_DIR overrides
+DIAG_DIR = os.environ.get("DC_DIAG_DIR", os.path.join(ROOT, "diagnostics"))
 sys.path.insert(0, ROOT)
 
 from synth import WORKLOADS, gen  # noqa: E402
@@ -75,7 +77,7 @@ class Clocks:
     def __init__(self, index):
         self.index = index
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{index}.csv")
+        self.path = os.path.join(DIAG_DIR, f"clocks_rank{index}.csv")
 
     def start(self):
         try:

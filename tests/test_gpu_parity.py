@@ -31,10 +31,12 @@ def dc():
 
 
 def record(name, value):
-    """Append a measured error to gpurun_out/parity_errors.jsonl (diagnostic)."""
+    """Append a measured error to parity_errors.jsonl in the diagnostics folder
+    ($DC_DIAG_DIR, default diagnostics/ at the repository root)."""
     import json
     import os
-    d = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "gpurun_out")
+    d = os.environ.get("DC_DIAG_DIR") or os.path.join(
+        os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "diagnostics")
     os.makedirs(d, exist_ok=True)
     with open(os.path.join(d, "parity_errors.jsonl"), "a") as f:
         f.write(json.dumps({"case": name, **value}) + "\n")
