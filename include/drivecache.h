@@ -312,7 +312,10 @@ dc_status dc_denoise_host(dc_model* m, float* host_latents, const dc_cond* cond,
  * veto, cfg_scale, and the forced actions or the anchor responses). */
 
 /* Bytes of a snapshot of B scenes and K steps for a model of this shape
- * (cfg: 1 with guidance); 0 for an invalid argument.  Host only. */
+ * (cfg: 1 with guidance); 0 for an invalid argument.  Shapes are bounded so
+ * that no section size overflows: B <= 65536, K <= 100000, n_tokens <= 2^26,
+ * d_model and channels <= 65536; a header outside these bounds is rejected by
+ * dc_snapshot_info and dc_denoise_steps.  Host only. */
 size_t dc_snapshot_bytes(const dc_model_desc* desc, int B, int K, int cfg);
 
 typedef struct {

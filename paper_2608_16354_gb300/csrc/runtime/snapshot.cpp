@@ -93,8 +93,11 @@ dc_status read_header(const void* snap, size_t bytes, SnapHeader* h) {
     set_error("snapshot version " + std::to_string(h->version) + " is not supported");
     return DC_ERR_INVALID_ARG;
   }
-  if (h->B < 1 || h->K < 1 || (h->cfg != 0 && h->cfg != 1) || h->k_done < 1 || h->k_done > h->K ||
-      h->N < 1 || h->d < 1 || h->C < 1 || (h->dtype != DC_DTYPE_F32 && h->dtype != DC_DTYPE_BF16) ||
+  // shape bounds keep every section size far from size_t overflow
+  if (h->B < 1 || h->B > (1 << 16) || h->K < 1 || h->K > 100000 || (h->cfg != 0 && h->cfg != 1) ||
+      h->k_done < 1 || h->k_done > h->K || h->N < 1 || h->N > (1 << 26) || h->d < 1 ||
+      h->d > (1 << 16) || h->C < 1 || h->C > (1 << 16) ||
+      (h->dtype != DC_DTYPE_F32 && h->dtype != DC_DTYPE_BF16) ||
       h->elt != (h->dtype == DC_DTYPE_BF16 ? 2u : 4u) || h->backbone_calls < 0) {
     set_error("snapshot header fields out of range");
     return DC_ERR_INVALID_ARG;
@@ -113,8 +116,9 @@ dc_status read_header(const void* snap, size_t bytes, SnapHeader* h) {
 extern "C" {
 
 size_t dc_snapshot_bytes(const dc_model_desc* desc, int B, int K, int cfg) {
-  if (!desc || B < 1 || K < 1 || (cfg != 0 && cfg != 1) || desc->n_tokens < 1 ||
-      desc->d_model < 1 || desc->channels < 1 ||
+  if (!desc || B < 1 || B > (1 << 16) || K < 1 || K > 100000 || (cfg != 0 && cfg != 1) ||
+      desc->n_tokens < 1 || desc->n_tokens > (1 << 26) || desc->d_model < 1 ||
+      desc->d_model > (1 << 16) || desc->channels < 1 || desc->channels > (1 << 16) ||
       (desc->dtype != DC_DTYPE_F32 && desc->dtype != DC_DTYPE_BF16))
     return 0;
   const size_t elt = desc->dtype == DC_DTYPE_BF16 ? 2 : 4;

@@ -80,6 +80,19 @@ def test_snapshot_info_rejects_malformed_headers(dc, bad):
         dc.snapshot_info(_blob(**bad))
 
 
+def test_snapshot_shapes_beyond_bounds_are_rejected(dc):
+    """Shapes whose section sizes could overflow are refused by both calls."""
+    m = _desc(dc)
+    assert dc.snapshot_bytes(m, 1 << 17, 25) == 0
+    assert dc.snapshot_bytes(m, 4, 200000) == 0
+    m.n_tokens = 1 << 27
+    assert dc.snapshot_bytes(m, 4, 25) == 0
+    h = _header(B=1 << 20, K=4, cfg=0, k_done=2, dtype=DTYPE_F32, N=1 << 30, d=1 << 20, C=1 << 20,
+                total=0)
+    with pytest.raises(dc.DCError):
+        dc.snapshot_info(np.frombuffer(h, np.uint8).copy())
+
+
 def test_snapshot_info_rejects_wrong_sizes(dc):
     good = _blob()
     with pytest.raises(dc.DCError):
