@@ -193,9 +193,14 @@ dc_status dc_legal_mask(int K, int H_max, int expert_boundary, int segment_len,
 /* ------------------------------------------------------------------ model */
 
 /* Shape of the synthetic DiT.  n_tokens = views x frames x rows x cols
- * (patch 1); head_dim = d_model / n_heads must be 16, 64, 72 or 128 for
- * bf16 and d_model % 4 == 0 for f32.  max_batch / max_steps bound the
- * per-call workspace allocated by dc_model_create. */
+ * (patch 1); channels 4 or 16; d_model <= 3072 and head_dim = d_model /
+ * n_heads.  bf16: d_model and mlp_ratio * d_model multiples of 192 and
+ * head_dim 64, 72 or 128; f32: d_model % 8 == 0 and head_dim 8, 16, 32 or
+ * 64.  max_batch (internal scenes per call, two per scene with guidance,
+ * <= 64) and max_steps bound the per-call workspace allocated by
+ * dc_model_create.  Index bounds: n_blocks <= 4096, mlp_ratio <= 16,
+ * n_tokens <= 2^22, max_batch * n_tokens <= 2^25, n_poses <= 65536,
+ * max_steps <= 100000. */
 typedef struct {
   int dtype;       /* DC_DTYPE_F32 or DC_DTYPE_BF16 */
   int n_blocks, d_model, n_heads, mlp_ratio, channels, n_tokens, n_poses;
@@ -204,7 +209,8 @@ typedef struct {
 
 typedef struct dc_model dc_model;
 
-/* Number of floats dc_model_create expects in host_weights. */
+/* Number of floats dc_model_create expects in host_weights; 0 when desc is
+ * NULL or describes a shape dc_model_create rejects.  Host only. */
 size_t dc_model_weight_count(const dc_model_desc* desc);
 
 /* Create a model on `device` (the caller's current CUDA device when < 0).

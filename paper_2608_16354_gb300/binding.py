@@ -304,7 +304,7 @@ class Model:
         self.wl = wl
         blob = np.ascontiguousarray(weights_blob, np.float32)
         n = lib().dc_model_weight_count(C.byref(d))
-        if n != blob.size:
+        if n and n != blob.size:  # n == 0: dc_model_create reports the invalid shape
             raise ValueError(f"weight blob has {blob.size} floats, model expects {n}")
         h = C.c_void_p()
         _check(lib().dc_model_create(C.byref(d), blob.ctypes.data_as(C.POINTER(C.c_float)),

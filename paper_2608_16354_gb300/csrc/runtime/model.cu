@@ -204,6 +204,16 @@ dc_status check_desc(const dc_model_desc* d) {
     dc::set_error("model shape fields must be positive and d_model divisible by n_heads");
     return DC_ERR_INVALID_ARG;
   }
+  // index bounds: every row index (max_batch * n_tokens rows, 32 threads a
+  // row in the row kernels) and step index stays far inside int
+  if (d->n_blocks > 4096 || d->mlp_ratio > 16 || d->n_tokens > (1 << 22) ||
+      (long long)d->max_batch * d->n_tokens > (1LL << 25) || d->n_poses > 65536 ||
+      d->max_steps > 100000) {
+    dc::set_error("model shape beyond the index bounds (n_blocks <= 4096, mlp_ratio <= 16, "
+                  "n_tokens <= 2^22, max_batch * n_tokens <= 2^25, n_poses <= 65536, "
+                  "max_steps <= 100000)");
+    return DC_ERR_UNSUPPORTED;
+  }
   if (d->max_batch > dc::kMaxBatch) {
     dc::set_error("max_batch above " + std::to_string(dc::kMaxBatch));
     return DC_ERR_UNSUPPORTED;
@@ -1016,7 +1026,7 @@ dc_status anchor_response_impl(dc_model* m, const float* noise, const dc_traject
 extern "C" {
 
 size_t dc_model_weight_count(const dc_model_desc* desc) {
-  if (!desc) return 0;
+  if (check_desc(desc) != DC_OK) return 0;
   WeightLayout w;
   weight_layout(*desc, &w);
   return w.total;
