@@ -416,7 +416,8 @@ dc_status dc_cache_copy(dc_model* m, int scene, void* dst, size_t bytes, void* s
  * planes) with dhp = head_dim rounded up to a multiple of 16 for bf16 (pad
  * columns must be zero) and dhp = head_dim for fp32; out: DEVICE
  * [slots][n_tokens][heads * head_dim].  dtype DC_DTYPE_BF16 supports
- * head_dim 64, 72, 128 (and 16); DC_DTYPE_F32 supports 8, 16, 32, 64. */
+ * head_dim 64, 72, 128 (and 16); DC_DTYPE_F32 supports 8, 16, 32, 64.
+ * slots * heads <= 2^15 and n_tokens <= 2^22 (DC_ERR_UNSUPPORTED beyond). */
 dc_status dc_attention(int dtype, const void* qkv, int slots, int heads, int n_tokens,
                        int head_dim, void* out, void* stream);
 

@@ -1461,6 +1461,11 @@ dc_status dc_attention(int dtype, const void* qkv, int slots, int heads, int n_t
     dc::set_error("dc_attention: NULL pointer or non-positive size");
     return DC_ERR_INVALID_ARG;
   }
+  // keeps the work-item count (slot, head, 128-query tile) inside int
+  if ((long long)slots * heads > (1 << 15) || n_tokens > (1 << 22)) {
+    dc::set_error("dc_attention: slots * heads above 2^15 or n_tokens above 2^22");
+    return DC_ERR_UNSUPPORTED;
+  }
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   if (dtype == DC_DTYPE_BF16) {
     if (!(head_dim == 16 || head_dim == 64 || head_dim == 72 || head_dim == 128)) {
@@ -1469,18 +1474,28 @@ dc_status dc_attention(int dtype, const void* qkv, int slots, int heads, int n_t
     }
     const int dhp = ((head_dim + 15) / 16) * 16;
     if (dc::attention_tc_supported(head_dim)) {
-      // the tensor-core kernel: a TMA map over the caller's buffer and a
-      // library-owned error word; the call waits for the kernel to report
-      static int* err_d = nullptr;
-      if (!err_d) DC_CK(cudaMalloc(&err_d, sizeof(int)));
-      DC_CK(cudaMemsetAsync(err_d, 0, sizeof(int), st));
+      // the tensor-core kernel: a TMA map over the caller's buffer and an
+      // error word of this call's own (stream-ordered allocation, so calls
+      // from several threads, streams or devices never share one); the call
+      // waits for the kernel to report
       CUtensorMap tm;
       DC_TRY(make_map(&tm, qkv, dhp, (uint64_t)3 * slots * heads * n_tokens, 128));
-      DC_CK(dc::launch_attention_tc(tm, slots, heads, n_tokens, head_dim,
-                                    static_cast<__nv_bfloat16*>(out), err_d, st));
+      int* err_d = nullptr;
+      DC_CK(cudaMallocAsync(reinterpret_cast<void**>(&err_d), sizeof(int), st));
+      cudaError_t e = cudaMemsetAsync(err_d, 0, sizeof(int), st);
+      if (e == cudaSuccess)
+        e = dc::launch_attention_tc(tm, slots, heads, n_tokens, head_dim,
+                                    static_cast<__nv_bfloat16*>(out), err_d, st);
       int err = 0;
-      DC_CK(cudaMemcpyAsync(&err, err_d, sizeof(int), cudaMemcpyDeviceToHost, st));
-      DC_CK(cudaStreamSynchronize(st));
+      if (e == cudaSuccess)
+        e = cudaMemcpyAsync(&err, err_d, sizeof(int), cudaMemcpyDeviceToHost, st);
+      const cudaError_t ef = cudaFreeAsync(err_d, st);
+      if (e == cudaSuccess) e = ef;
+      if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+      if (e != cudaSuccess) {
+        dc::set_error(std::string("dc_attention: ") + cudaGetErrorString(e));
+        return DC_ERR_CUDA;
+      }
       if (err) {
         dc::set_error("dc_attention: a bounded device wait gave up");
         return DC_ERR_DEVICE_TIMEOUT;

@@ -75,3 +75,20 @@ def test_weight_blob_size_is_checked_before_any_device_call(dc):
     h = dc.C.c_void_p()
     assert dc.lib().dc_model_create(dc.C.byref(m), blob, n - 1, 0, dc.C.byref(h)) == INVALID_ARG
     assert "expected" in dc.lib().dc_last_error().decode()
+
+
+@pytest.mark.parametrize("args,status", [
+    ((DTYPE_BF16, 0, 1, 1, 128, 64), INVALID_ARG),           # NULL qkv
+    ((DTYPE_BF16, 16, 0, 1, 128, 64), INVALID_ARG),          # no slots
+    ((DTYPE_BF16, 16, 1, 1, 128, 0), INVALID_ARG),           # head_dim 0
+    ((DTYPE_BF16, 16, 256, 129, 128, 64), UNSUPPORTED),      # slots * heads > 2^15
+    ((DTYPE_BF16, 16, 1, 1, (1 << 22) + 1, 64), UNSUPPORTED),
+    ((DTYPE_BF16, 16, 1, 1, 128, 32), UNSUPPORTED),          # no bf16 kernel for dim 32
+    ((DTYPE_F32, 16, 1, 1, 128, 128), UNSUPPORTED),          # no fp32 kernel for dim 128
+    ((7, 16, 1, 1, 128, 64), INVALID_ARG)])                  # unknown dtype
+def test_attention_arguments_checked_before_any_device_call(dc, args, status):
+    dtype, qkv, slots, heads, n, dh = args
+    # the pointers are never dereferenced: every case fails its checks first
+    got = dc.lib().dc_attention(dtype, dc.C.c_void_p(qkv or None), slots, heads, n, dh,
+                                dc.C.c_void_p(16), None)
+    assert got == status, dc.lib().dc_last_error().decode()
