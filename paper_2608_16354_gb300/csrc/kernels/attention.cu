@@ -232,13 +232,12 @@ cudaError_t launch_dhp(const __nv_bfloat16* qkv, int slots, int heads, int N, in
                        __nv_bfloat16* o, cudaStream_t st) {
   constexpr int LD = DHP + 8;
   const size_t smem = (size_t)(kQ + 4 * kKV) * LD * sizeof(__nv_bfloat16);
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(attn_bf16_kernel<DHP>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  static std::atomic<unsigned long long> configured{0};
+  cudaError_t e = configure_once_per_device(configured, [&] {
+    return cudaFuncSetAttribute(attn_bf16_kernel<DHP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)smem);
+  });
+  if (e != cudaSuccess) return e;
   dim3 grid((N + kQ - 1) / kQ, slots * heads);
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)dh);
   attn_bf16_kernel<DHP><<<grid, kWarps * 32, smem, st>>>(qkv, slots, heads, N, dh, o, scale_log2);

@@ -583,19 +583,20 @@ template <int DHP, int NQ, int DH = DHP>
 cudaError_t launch_tc(const CUtensorMap& tm, int nslots, int heads, int N, __nv_bfloat16* o,
                       int* err, cudaStream_t st) {
   using Cfg = AttCfg<DHP, NQ>;
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<DHP, NQ, DH>,
+  static std::atomic<unsigned long long> configured{0};
+  const cudaError_t e = configure_once_per_device(configured, [] {
+    cudaError_t r = cudaFuncSetAttribute(attn_tc_kernel<DHP, NQ, DH>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmem);
-    if (e != cudaSuccess) return e;
+    if (r != cudaSuccess) return r;
     // setmaxnreg.inc waits until the CTA's launch allocation can serve it:
     // never launch a build whose allocation is not the one the split assumes
     cudaFuncAttributes fa;
-    e = cudaFuncGetAttributes(&fa, attn_tc_kernel<DHP, NQ, DH>);
-    if (e != cudaSuccess) return e;
+    r = cudaFuncGetAttributes(&fa, attn_tc_kernel<DHP, NQ, DH>);
+    if (r != cudaSuccess) return r;
     if (Cfg::kSplitRegs && fa.numRegs != Cfg::kRegsLaunch) return cudaErrorInvalidConfiguration;
-    configured = true;
-  }
+    return cudaSuccess;
+  });
+  if (e != cudaSuccess) return e;
   dim3 grid((N + 128 * NQ - 1) / (128 * NQ), nslots * heads);
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)DH);
   return launch_pdl(attn_tc_kernel<DHP, NQ, DH>, grid, dim3(Cfg::kThreads), Cfg::kSmem, st, tm,

@@ -13,6 +13,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 namespace dc {
 
 constexpr int kMaxBatch = 64;  // scenes per call (slot maps travel by value)
@@ -389,7 +391,6 @@ __device__ __forceinline__ uint64_t sw128_kmajor_desc(uint32_t start) {
   return d;
 }
 
-// Instruction descriptor, kind::f16: bf16 A and B (K-major), fp32 D, M x N.
 // ------------------------------------------- programmatic dependent launch
 // A kernel launched with launch_pdl may start while the previous kernel of
 // its stream is still finishing.  pdl_wait() blocks until that kernel has
@@ -416,6 +417,24 @@ inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, s
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
+// One-time launch configuration per device: kernel attributes such as the
+// dynamic shared-memory limit apply to the current device only, so
+// `configure` runs before the first launch on each device (one bit of `done`
+// per device ordinal; ordinals >= 64 configure before every launch).  Two
+// threads may both configure a device; setting an attribute twice is
+// harmless.
+template <typename F>
+inline cudaError_t configure_once_per_device(std::atomic<unsigned long long>& done, F configure) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const unsigned long long bit = dev < 64 ? 1ull << dev : 0ull;
+  if (bit && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+  e = configure();
+  if (e == cudaSuccess && bit) done.fetch_or(bit, std::memory_order_release);
+  return e;
 }
 
 // ------------------------------------------------ CTA pairs (cta_group::2)
@@ -488,6 +507,7 @@ __device__ __forceinline__ void tc_commit_pair_mc(uint64_t* bar, uint16_t mask) 
       : "memory");
 }
 
+// Instruction descriptor, kind::f16: bf16 A and B (K-major), fp32 D, M x N.
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
   return (1u << 4)                       // D format: f32
          | (1u << 7)                     // A format: bf16

@@ -506,13 +506,12 @@ cudaError_t launch_mode(const CUtensorMap& tmA, const CUtensorMap& tmB, const CU
                         const CUtensorMap& tmCout, int M, int N, int K, const EpiArgs& ep,
                         const SlotMap& map, int* err, int n_sms, cudaStream_t st) {
   using Cfg = GemmCfg<MODE, HALF>;
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_bf16_tc_kernel<MODE, HALF>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmem);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  static std::atomic<unsigned long long> configured{0};
+  const cudaError_t e = configure_once_per_device(configured, [] {
+    return cudaFuncSetAttribute(gemm_bf16_tc_kernel<MODE, HALF>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmem);
+  });
+  if (e != cudaSuccess) return e;
   // clusters of two CTAs over pairs of m tiles (the grid is even)
   const int pair_tiles = ((M + kBM - 1) / kBM + 1) / 2 * (N / kBN);
   const int grid = 2 * (pair_tiles < n_sms / 2 ? pair_tiles : n_sms / 2);

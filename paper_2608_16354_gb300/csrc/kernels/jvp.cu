@@ -475,13 +475,12 @@ template <int DH, bool TAN>
 cudaError_t launch_jvp_tiled(const float* qkv, const float* dqkv, int N, int d, int heads, int T,
                              float scale, float* o, float* dout, cudaStream_t st) {
   using Tl = JvpTile<DH, TAN>;
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(attn_f32_jvp_tiled_kernel<DH, TAN>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Tl::kBytes);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  static std::atomic<unsigned long long> configured{0};
+  const cudaError_t e = configure_once_per_device(configured, [] {
+    return cudaFuncSetAttribute(attn_f32_jvp_tiled_kernel<DH, TAN>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Tl::kBytes);
+  });
+  if (e != cudaSuccess) return e;
   dim3 grid((N + Tl::BQ - 1) / Tl::BQ, heads, T);
   attn_f32_jvp_tiled_kernel<DH, TAN><<<grid, 128, Tl::kBytes, st>>>(qkv, dqkv, N, d, scale, o, dout);
   return cudaGetLastError();
