@@ -42,34 +42,65 @@ __global__ void temb_features_kernel(const double* __restrict__ sig, int K, floa
   out[(size_t)k * 256 + 128 + i] = (float)sin(t * f);
 }
 
+// Y[R][O] = act(X)[R][I] W[O][I]^T + b, fp32 accumulation.  A CTA computes a
+// 64-row x 128-output tile: 32-deep slices of X and W are staged k-major in
+// shared memory and each thread accumulates 8 rows x 4 outputs (outputs
+// lane + 32 c, so that stores are coalesced), summing over i in order.
+constexpr int kRlRows = 64, kRlCols = 128, kRlK = 32;
+
 template <typename TW>
-__global__ void rows_linear_kernel(const float* __restrict__ X, int R, int I,
-                                   const TW* __restrict__ W, const float* __restrict__ b, int O,
-                                   float* __restrict__ Y, int in_silu) {
-  const int o = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  if (o >= O) return;
-  const TW* w = W + (size_t)o * I;
-  constexpr int RT = 8;
-  for (int r0 = 0; r0 < R; r0 += RT) {
-    float acc[RT];
+__global__ void __launch_bounds__(256) rows_linear_kernel(const float* __restrict__ X, int R, int I,
+                                                          const TW* __restrict__ W,
+                                                          const float* __restrict__ b, int O,
+                                                          float* __restrict__ Y, int in_silu) {
+  // row strides: 68 keeps the float4 reads aligned, 129 spreads the
+  // transposing stores over the banks
+  __shared__ __align__(16) float xs[kRlK][kRlRows + 4];
+  __shared__ float ws[kRlK][kRlCols + 1];
+  const int tid = threadIdx.x, lane = tid & 31, ty = tid >> 5;
+  const int o0 = blockIdx.x * kRlCols, r0 = blockIdx.y * kRlRows;
+  float acc[8][4];
 #pragma unroll
-    for (int j = 0; j < RT; ++j) acc[j] = 0.f;
-    for (int i = lane; i < I; i += 32) {
-      const float wv = to_f(w[i]);
+  for (int j = 0; j < 8; ++j)
 #pragma unroll
-      for (int j = 0; j < RT; ++j) {
-        if (r0 + j < R) {
-          float xv = X[(size_t)(r0 + j) * I + i];
-          if (in_silu) xv = silu(xv);
-          acc[j] += xv * wv;
-        }
-      }
+    for (int c = 0; c < 4; ++c) acc[j][c] = 0.f;
+  for (int k0 = 0; k0 < I; k0 += kRlK) {
+    const int kk = tid & (kRlK - 1), k = k0 + kk;
+#pragma unroll
+    for (int e = 0; e < kRlRows * kRlK / 256; ++e) {
+      const int row = (tid >> 5) + 8 * e, r = r0 + row;
+      float v = r < R && k < I ? X[(size_t)r * I + k] : 0.f;
+      if (in_silu && r < R && k < I) v = silu(v);
+      xs[kk][row] = v;
     }
 #pragma unroll
-    for (int j = 0; j < RT; ++j) {
-      const float v = warp_sum(acc[j]);
-      if (lane == 0 && r0 + j < R) Y[(size_t)(r0 + j) * O + o] = v + b[o];
+    for (int e = 0; e < kRlCols * kRlK / 256; ++e) {
+      const int col = (tid >> 5) + 8 * e, o = o0 + col;
+      ws[kk][col] = o < O && k < I ? to_f(W[(size_t)o * I + k]) : 0.f;
+    }
+    __syncthreads();
+#pragma unroll 4
+    for (int q = 0; q < kRlK; ++q) {
+      const float4 xa = *reinterpret_cast<const float4*>(&xs[q][ty * 8]);
+      const float4 xb = *reinterpret_cast<const float4*>(&xs[q][ty * 8 + 4]);
+      const float xv[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const float wv = ws[q][lane + 32 * c];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[j][c] = fmaf(xv[j], wv, acc[j][c]);
+      }
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const int r = r0 + ty * 8 + j;
+    if (r >= R) break;
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+      const int o = o0 + lane + 32 * c;
+      if (o < O) Y[(size_t)r * O + o] = acc[j][c] + b[o];
     }
   }
 }
@@ -90,8 +121,11 @@ __global__ void cond_combine_kernel(const float* __restrict__ temb, const float*
 template <typename T>
 __device__ __forceinline__ float4 load4(const T* src);
 
-// u = x W_e^T + b_e + pos, one thread per 4 consecutive outputs; W_e is read
-// transposed ([C][d]) so that the threads of a warp load contiguous float4.
+// u = x W_e^T + b_e + pos: a thread computes 4 consecutive outputs of
+// kEmbedRows consecutive tokens, so that its W_e columns (read transposed,
+// [C][d], contiguous float4 across the warp) are loaded once for all of them.
+constexpr int kEmbedRows = 4;
+
 template <typename T, int C>
 __global__ void embed_kernel(const float* __restrict__ x, const float* __restrict__ w_eT,
                              const float* __restrict__ b_e, const T* __restrict__ pos, SlotMap map,
@@ -100,27 +134,36 @@ __global__ void embed_kernel(const float* __restrict__ x, const float* __restric
   pdl_wait();
   const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int d4 = d >> 2;
-  const size_t total = (size_t)map.n * N * d4;
-  if (i >= total) return;
+  const size_t rows = (size_t)map.n * N;
+  const size_t groups = (rows + kEmbedRows - 1) / kEmbedRows;
+  if (i >= groups * d4) return;
   const int e4 = (int)(i % d4);
-  const size_t row = i / d4;  // slot * N + tok
-  const int slot = (int)(row / N), tok = (int)(row - (size_t)slot * N);
-  const float4* xr = reinterpret_cast<const float4*>(x + ((size_t)map.scene[slot] * N + tok) * C);
-  float xv[C];
+  const size_t g = i / d4;
+  float4 w[C];
 #pragma unroll
-  for (int c = 0; c < C / 4; ++c) {
-    const float4 t = __ldg(xr + c);
-    xv[4 * c] = t.x; xv[4 * c + 1] = t.y; xv[4 * c + 2] = t.z; xv[4 * c + 3] = t.w;
-  }
+  for (int c = 0; c < C; ++c) w[c] = __ldg(reinterpret_cast<const float4*>(w_eT + (size_t)c * d) + e4);
   const float4 bv = __ldg(reinterpret_cast<const float4*>(b_e) + e4);
-  const float4 pv = load4<T>(pos + (size_t)tok * d + 4 * e4);
-  float4 acc = make_float4(bv.x + pv.x, bv.y + pv.y, bv.z + pv.z, bv.w + pv.w);
 #pragma unroll
-  for (int c = 0; c < C; ++c) {
-    const float4 w = __ldg(reinterpret_cast<const float4*>(w_eT + (size_t)c * d) + e4);
-    acc.x += w.x * xv[c]; acc.y += w.y * xv[c]; acc.z += w.z * xv[c]; acc.w += w.w * xv[c];
+  for (int t = 0; t < kEmbedRows; ++t) {
+    const size_t row = g * kEmbedRows + t;  // slot * N + tok
+    if (row >= rows) break;
+    const int slot = (int)(row / N), tok = (int)(row - (size_t)slot * N);
+    const float4* xr = reinterpret_cast<const float4*>(x + ((size_t)map.scene[slot] * N + tok) * C);
+    float xv[C];
+#pragma unroll
+    for (int c = 0; c < C / 4; ++c) {
+      const float4 v = __ldg(xr + c);
+      xv[4 * c] = v.x; xv[4 * c + 1] = v.y; xv[4 * c + 2] = v.z; xv[4 * c + 3] = v.w;
+    }
+    const float4 pv = load4<T>(pos + (size_t)tok * d + 4 * e4);
+    float4 acc = make_float4(bv.x + pv.x, bv.y + pv.y, bv.z + pv.z, bv.w + pv.w);
+#pragma unroll
+    for (int c = 0; c < C; ++c) {
+      acc.x += w[c].x * xv[c]; acc.y += w[c].y * xv[c];
+      acc.z += w[c].z * xv[c]; acc.w += w[c].w * xv[c];
+    }
+    reinterpret_cast<float4*>(u)[row * d4 + e4] = acc;
   }
-  reinterpret_cast<float4*>(u)[i] = acc;
 }
 
 // --------------------------------------------------------------- LN + mod
@@ -491,9 +534,9 @@ cudaError_t launch_temb_features(const double* sigmas, int K, float* out, cudaSt
 template <typename TW>
 cudaError_t launch_rows_linear(const float* X, int R, int I, const TW* W, const float* b, int O,
                                float* Y, int in_silu, cudaStream_t st) {
-  const int threads = 256;
-  const int blocks = (int)(((size_t)O * 32 + threads - 1) / threads);
-  rows_linear_kernel<TW><<<blocks, threads, 0, st>>>(X, R, I, W, b, O, Y, in_silu);
+  if (R <= 0 || O <= 0) return cudaSuccess;
+  const dim3 grid((unsigned)((O + kRlCols - 1) / kRlCols), (unsigned)((R + kRlRows - 1) / kRlRows));
+  rows_linear_kernel<TW><<<grid, 256, 0, st>>>(X, R, I, W, b, O, Y, in_silu);
   return cudaGetLastError();
 }
 template cudaError_t launch_rows_linear<float>(const float*, int, int, const float*, const float*,
@@ -512,8 +555,8 @@ template <typename T>
 cudaError_t launch_embed(const float* x, const float* w_eT, const float* b_e, const T* pos,
                          const SlotMap& map, int N, int C, int d, float* u, cudaStream_t st) {
   if (map.n <= 0) return cudaSuccess;
-  const size_t n = (size_t)map.n * N * (d / 4);
-  const unsigned blocks = (unsigned)((n + 255) / 256);
+  const size_t groups = ((size_t)map.n * N + kEmbedRows - 1) / kEmbedRows;
+  const unsigned blocks = (unsigned)((groups * (d / 4) + 255) / 256);
   if (C == 16)
     return launch_pdl(embed_kernel<T, 16>, dim3(blocks), dim3(256), 0, st, x, w_eT, b_e, pos, map,
                       N, d, u);
