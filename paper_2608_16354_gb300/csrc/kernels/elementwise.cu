@@ -259,26 +259,52 @@ __global__ void ln_mod_kernel(const float* __restrict__ h, int rows, int N, int 
 
 // ---------------------------------------------------- interface + Euler
 
-// v[c] = sum_e a_e w_f[c][e] + b_f[c] for the modulated, normalised row held
-// in registers; returns v[c] on every lane.
+// v_c = sum_e a_e w_f[c][e] + b_f[c] for the modulated, normalised row held
+// in registers; lane c < C returns v_c.  The C per-lane partial sums are
+// reduced and scattered over the xor butterfly 16, 8, 4, 2, 1 (C - 1 + 5 -
+// log2 C shuffles instead of 5 C): at each offset a lane keeps the half of its
+// values selected by its lane bit and adds its partner's copy of that half,
+// so every sum pairs the same operands in the same order as warp_sum and is
+// bitwise the value warp_sum gives.  Lane l ends with channel l / (32 / C).
 template <int NV, int C>
-__device__ __forceinline__ void head_dot(const float4 (&a)[NV], int d, int d4, int lane,
-                                         const float* __restrict__ w_f,
-                                         const float* __restrict__ b_f, float (&v)[C]) {
+__device__ __forceinline__ float head_dot(const float4 (&a)[NV], int d, int d4, int lane,
+                                          const float* __restrict__ w_f,
+                                          const float* __restrict__ b_f) {
+  static_assert(C >= 1 && C <= 32 && (C & (C - 1)) == 0, "C must be a power of two <= 32");
+  float s[C];
 #pragma unroll
   for (int c = 0; c < C; ++c) {
     const float4* w = reinterpret_cast<const float4*>(w_f + (size_t)c * d);
-    float s = 0.f;
+    float t = 0.f;
 #pragma unroll
     for (int j = 0; j < NV; ++j) {
       const int i = lane + 32 * j;
       if (i < d4) {
         const float4 ww = __ldg(w + i);
-        s += (a[j].x * ww.x + a[j].y * ww.y) + (a[j].z * ww.z + a[j].w * ww.w);
+        t += (a[j].x * ww.x + a[j].y * ww.y) + (a[j].z * ww.z + a[j].w * ww.w);
       }
     }
-    v[c] = warp_sum(s) + b_f[c];
+    s[c] = t;
   }
+#pragma unroll
+  for (int step = 0; step < 5; ++step) {
+    const int off = 16 >> step;
+    const int n = C >> step;  // values this lane still holds
+    if (n >= 2) {
+      const bool upper = (lane & off) != 0;
+#pragma unroll
+      for (int k = 0; k < n / 2; ++k) {
+        const float send = upper ? s[k] : s[k + n / 2];
+        const float keep = upper ? s[k + n / 2] : s[k];
+        s[k] = keep + __shfl_xor_sync(0xffffffffu, send, off);
+      }
+    } else {
+      s[0] += __shfl_xor_sync(0xffffffffu, s[0], off);
+    }
+  }
+  constexpr int kSpan = 32 / C;  // lanes holding the same channel
+  const float v = s[0] + b_f[(lane / kSpan) & (C - 1)];
+  return __shfl_sync(0xffffffffu, v, (lane * kSpan) & 31);
 }
 
 template <int NV>
@@ -334,13 +360,8 @@ __global__ void final_compute_kernel(const float* __restrict__ hL, const float* 
   float mu, rs;
   row_stats<NV>(hv, d, d4, lane, &mu, &rs);
   modulate<NV>(hv, mu, rs, mod + (size_t)scene * mod_stride, fin_off, fin_off + d, d4, lane);
-  float v[C];
-  head_dot<NV, C>(hv, d, d4, lane, w_f, b_f, v);
+  const float vc = head_dot<NV, C>(hv, d, d4, lane, w_f, b_f);
   if (lane < C) {
-    float vc = v[0];
-#pragma unroll
-    for (int c = 1; c < C; ++c)
-      if (lane == c) vc = v[c];
     const size_t xi = ((size_t)scene * N + tok) * C + lane;
     const float xo = x[xi];
     xj[xi] = xo;
@@ -393,14 +414,9 @@ __global__ void final_reuse_kernel(float* __restrict__ x, const T* __restrict__ 
   float mu, rs;
   row_stats<NV>(hv, d, d4, lane, &mu, &rs);
   modulate<NV>(hv, mu, rs, mod + (size_t)scene * mod_stride, fin_off, fin_off + d, d4, lane);
-  float v[C];
-  head_dot<NV, C>(hv, d, d4, lane, w_f, b_f, v);
+  const float vc = head_dot<NV, C>(hv, d, d4, lane, w_f, b_f);
   __syncwarp();
   if (lane < C) {
-    float vc = v[0];
-#pragma unroll
-    for (int c = 1; c < C; ++c)
-      if (lane == c) vc = v[c];
     float xo = xv[0];
 #pragma unroll
     for (int c = 1; c < C; ++c)
