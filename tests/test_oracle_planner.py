@@ -368,3 +368,132 @@ def test_dp_hand_worked_golden():
         acts, n, cost = P.plan_suffix(g["c_hat"], g["K"], g["H"], 1, case["tau"])
         s = "".join("C" if acts[k] == C else "R" for k in range(1, g["K"] + 1))
         assert (n, cost, s) == (case["n_reuse"], case["cost"], case["actions"])
+
+
+# ------------------------------------- tie-breaks, drift and the controller
+
+def test_median_matches_numpy():
+    """Sec. 3.1 and the tau rule use the median; of an even count it is the
+    mean of the two middle values, as numpy.median."""
+    rng = random.Random(21)
+    for n in range(1, 14):
+        v = [rng.randint(-6, 6) / 4.0 for _ in range(n)]
+        assert P._median(v) == float(np.median(v))
+
+
+@pytest.mark.parametrize("seed", range(24))
+def test_dp_ties_match_brute_force(seed):
+    """Coarse costs (0, 1/8, 1/4; all zero for every fourth seed) make many
+    schedules tie in count and cost, so the deterministic tie-break of Sec.
+    3.2 (latest refresh: smallest terminal age, smallest age at every
+    refresh) decides the schedule."""
+    rng = random.Random(900 + seed)
+    K = rng.randint(3, 10)
+    H = rng.randint(1, min(4, K))
+    c = [[0.0] * (H + 1) for _ in range(K)]
+    for j in range(1, K):
+        for h in range(1, H + 1):
+            c[j][h] = 0.0 if seed % 4 == 0 else rng.choice((0.0, 0.125, 0.25))
+    for tau in (0.0, 0.125, 0.5, math.inf):
+        acts, n, cost = P.plan_suffix(c, K, H, 1, tau)
+        bacts, bn, bcost = _brute_plan(c, K, H, 1, tau, _legal_all(H))
+        assert (n, cost) == (bn, bcost)
+        assert [acts[k] for k in range(1, K + 1)] == [bacts[k] for k in range(1, K + 1)]
+
+
+def test_drift_closed_forms():
+    """Eq. 12 (and Eq. 5): ||u_now - u_ref|| / (||u_now|| + eps) over the
+    whole per-scene tensor."""
+    rng = np.random.default_rng(3)
+    u = rng.standard_normal((7, 5))
+    n = math.sqrt(float(np.sum(u * u)))
+    z = np.zeros_like(u)
+    assert P.drift(u, u) == 0.0
+    assert math.isclose(P.drift(2.0 * u, u), n / (2.0 * n + P.EPS), rel_tol=1e-13)
+    assert math.isclose(P.drift(u, 2.0 * u), n / (n + P.EPS), rel_tol=1e-13)
+    assert math.isclose(P.drift(u, z), n / (n + P.EPS), rel_tol=1e-13)
+    assert math.isclose(P.drift(z, u), n / P.EPS, rel_tol=1e-13)
+
+
+def test_acceptance_needs_both_conditions():
+    """Sec. 3.2: a planned reuse is accepted only when d_obs <= d_bar + eps
+    and C_k + c_hat <= tau, both bounds inclusive."""
+    e = P.EPS
+    assert P.accept_reuse(0.5, 0.5, 0.25, 0.5, 0.75)
+    assert P.accept_reuse(0.5 + e, 0.5, 0.0, 0.0, 0.0)
+    assert not P.accept_reuse(0.5 + 3 * e, 0.5, 0.0, 0.0, 1.0)
+    assert not P.accept_reuse(0.0, 0.5, 0.25, 0.5625, 0.75)
+    assert not P.accept_reuse(0.0, 0.5, 0.25, 0.5, 0.625)
+
+
+def _replay(c, dbar, K, H, tau, full_budget=False):
+    """Sec. 3.2 step by step with brute-force planning: a planned reuse is
+    checked (drift: d_bar >= 0 accepts, d_bar < 0 refuses; charge:
+    C + c_hat <= tau); a refusal computes the step and replans steps k..K
+    under tau - C (under tau itself with full_budget, the mistake the
+    scripted scene must expose)."""
+    legal = _legal_all(H)
+    plan, _, _ = _brute_plan(c, K, H, 1, tau, legal)
+    acts = dict(plan)
+    charge, j, age = 0.0, 1, 0
+    executed, checks = [C], []
+    for k in range(2, K + 1):
+        if acts[k] == R:
+            h = age + 1
+            ok = dbar[j][h] >= 0.0 and charge + c[j][h] <= tau
+            checks.append((k, ok))
+            if ok:
+                charge += c[j][h]
+                age += 1
+                executed.append(R)
+                continue
+            sub, _, _ = _brute_plan(c, K, H, k, tau if full_budget else tau - charge, legal)
+            acts.update(sub)
+        executed.append(C)
+        j, age = k, 0
+    return executed, checks, charge, plan
+
+
+def test_controller_replans_the_suffix_with_the_remaining_budget():
+    """A scripted scene on the tiny model: q0 = q1 and d0 = d1, so the scene's
+    tables do not depend on its motion; the drift threshold accepts every
+    check except the one at the (j, h) of the plan's second reuse.  The
+    executed schedule, the sequence of checks and the charge equal the
+    brute-force replay, which replans under tau - C_k after the refusal."""
+    from oracle import controller as Ctl
+    from synth import WORKLOADS
+    wl = WORKLOADS["c1"]
+    K, H = wl.steps, wl.h_max
+    model = Ctl.build(wl, gen.weights(wl))
+    anc = dict(L0=0.0, T0=0.0, L1=1e6, T1=1e6, valid=1)
+    tr = gen.scene_trajectories(wl)
+    for seed in range(200):
+        rng = random.Random(4000 + seed)
+        c = [[0.0] * (H + 1) for _ in range(K)]
+        q = [[0.0] * (H + 1) for _ in range(K)]
+        for j in range(1, K):
+            for h in range(1, H + 1):
+                c[j][h] = rng.randint(1, 16) / 256.0
+                q[j][h] = q[j][h - 1] + c[j][h]
+        tau = rng.randint(8, 40) / 256.0
+        plan, _, _ = _brute_plan(c, K, H, 1, tau, _legal_all(H))
+        reuses = [k for k in range(2, K + 1) if plan[k] == R]
+        if len(reuses) < 3:
+            continue
+        dtab = [[1e9] * (H + 1) for _ in range(K)]
+        k2 = reuses[1]
+        j2 = max(k for k in range(1, k2) if plan[k] == C)
+        dtab[j2][k2 - j2] = -1.0
+        executed, checks, charge, _ = _replay(c, dtab, K, H, tau)
+        if _replay(c, dtab, K, H, tau, full_budget=True)[:2] != (executed, checks):
+            break  # the remaining budget changes this scene's suffix
+    else:
+        pytest.fail("no scripted scene separates the remaining budget from tau")
+    tables = dict(q0=q, q1=q, d0=dtab, d1=dtab)
+    out = Ctl.denoise(model, gen.latents(wl), tr, gen.sigmas(K), anc, tables, tau, K, H)
+    assert out["plans"][0]["actions"][1:] == [plan[k] for k in range(1, K + 1)]
+    assert out["executed"][0][1:] == executed
+    assert [(e["k"], e["accept"]) for e in out["log"][0]] == checks
+    assert out["stats"][0]["charge"] == charge
+    assert any(not ok for _, ok in checks) and sum(ok for _, ok in checks) >= 1
+
