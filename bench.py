@@ -174,9 +174,16 @@ def cpu_threads():
         return os.cpu_count()
 
 
+def workload_config(wl, B, K, tau, world, l2):
+    """The `config` object of both arms' lines."""
+    return {"workload": wl.name, "batch": B, "steps": K, "tokens": wl.n_tokens,
+            "d_model": wl.d_model, "blocks": wl.n_blocks, "heads": wl.n_heads,
+            "rho_tar": wl.rho_tar, "tau": tau, "parallelism": f"replicas{world}", "l2": l2}
+
+
 def planned_mix(wl):
     """Compute/reuse scene-step counts of the planned schedules (oracle
-    planner; drift vetoes ignored) for the reference arm."""
+    planner; drift vetoes ignored) and tau, for the reference arm."""
     from oracle import planner as P
     K, H = wl.steps, wl.h_max
     clips = gen.calibration_trajectories(wl)
@@ -187,13 +194,13 @@ def planned_mix(wl):
     tabs = dict(q0=q0, q1=q1, d0=z, d1=z)
     tau, _ = P.calibrate_budget(list(clips), anc, tabs, wl.target(), K, H)
     nr = sum(P.plan_scene(t, anc, tabs, tau, K, H)["n_reuse"] for t in gen.scene_trajectories(wl))
-    return wl.batch * K - nr, nr
+    return wl.batch * K - nr, nr, tau
 
 
 def run_reference(args, wl, rank, world):
     if rank != 0:
         return
-    nc, nr = planned_mix(wl)
+    nc, nr, tau = planned_mix(wl)
     times, rates = [], []
     for i in range(args.warmup + args.steps):
         t0 = time.perf_counter()
@@ -210,8 +217,8 @@ def run_reference(args, wl, rank, world):
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1000.0 * wl.batch * wl.steps / rate, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": wl.name, "batch": wl.batch, "steps": wl.steps,
-                       "tokens": wl.n_tokens},
+            "config": workload_config(wl, wl.batch, wl.steps, tau, world,
+                                      "host run: no GPU L2 to flush"),
             "cpu_baseline": {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": rate, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -485,10 +492,7 @@ def main():
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32", "data": "synthetic",
-        "config": {"workload": wl.name, "batch": B, "steps": K, "tokens": wl.n_tokens,
-                   "d_model": wl.d_model, "blocks": wl.n_blocks, "heads": wl.n_heads,
-                   "rho_tar": wl.rho_tar, "tau": tau, "parallelism": f"replicas{world}",
-                   "l2": "flushed between steps (512 MB write)"},
+        "config": workload_config(wl, B, K, tau, world, "flushed between steps (512 MB write)"),
         "videos_per_s": world * B / (ms_step / 1000.0),
         "full_compute_steps_per_s": world * B * K / (full_ms / 1000.0),
         "speedup_vs_full_compute": full_ms / ms_step,
