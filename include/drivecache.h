@@ -22,6 +22,15 @@
  *    message for the last failure on the calling thread.
  *  - Host planner calls (dc_motion_stats .. dc_calibrate_budget) are pure
  *    fp64 host code with no device dependency and are thread-safe.
+ *  - A dc_model serves one call at a time: its workspace (activations,
+ *    caches, profile counters) is shared by every call that takes the model,
+ *    so such calls must not overlap, from several threads or on several
+ *    streams.  Distinct models (on one device or several) are independent.
+ *  - Calls whose results are device arrays (dc_drift_sums,
+ *    dc_drift_sums_noalloc, dc_cache_copy, and dc_attention outside its
+ *    tensor-core head dims) are asynchronous on their stream; calls that
+ *    return host results, or that check a device error word, synchronise
+ *    their stream before they return.
  */
 #ifndef DRIVECACHE_H
 #define DRIVECACHE_H
