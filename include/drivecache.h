@@ -361,7 +361,8 @@ dc_status dc_denoise_steps(dc_model* m, float* latents, const dc_cond* cond, con
 /* Eq. 5 along one full trace: run all K steps as full evaluations from
  * `noise` (DEVICE fp32 [N][C], not modified) under `traj`, and write
  * d_out[j*(H_max+1)+h] = ||u_{j+h} - u_j|| / (||u_{j+h}|| + eps) for
- * j = 1..K-1, h = 1..min(H_max, K-j) (other entries 0).  Host d_out. */
+ * j = 1..K-1, h = 1..min(H_max, K-j) (other entries 0).  Host d_out,
+ * [K][H_max+1] doubles; 1 <= K <= max_steps, 1 <= H_max <= 4096. */
 dc_status dc_anchor_drift(dc_model* m, const float* noise, const dc_trajectory* traj, int K,
                           const double* sigmas, int H_max, double eps, double* d_out, void* stream);
 
@@ -379,7 +380,8 @@ dc_status dc_anchor_drift(dc_model* m, const float* noise, const dc_trajectory* 
  * the calibration cost is O(K^2 H_max) tangent passes, batched per trace
  * point.  Device workspace is allocated and freed inside the call (about
  * 8 GB at most for the tangents plus the stored activations); the call
- * synchronises `stream`.  head_dim must be 8, 16, 32, 64, 72 or 128. */
+ * synchronises `stream`.  head_dim must be 8, 16, 32, 64, 72 or 128;
+ * 1 <= K <= max_steps, 1 <= H_max <= 4096. */
 dc_status dc_anchor_response(dc_model* m, const float* noise, const dc_trajectory* traj, int K,
                              const double* sigmas, int H_max, double eps, double* q_out,
                              void* stream);

@@ -1310,8 +1310,9 @@ dc_status dc_anchor_drift(dc_model* m, const float* noise, const dc_trajectory* 
                           const double* sigmas, int H_max, double eps, double* d_out,
                           void* stream) {
   if (!m || !noise || !traj || !sigmas || !d_out || K < 1 || K > m->Kmax || H_max < 1 ||
-      !(eps > 0.0)) {
-    dc::set_error("dc_anchor_drift: NULL argument, K outside [1, max_steps], H_max < 1 or eps <= 0");
+      H_max > 4096 || !(eps > 0.0)) {
+    dc::set_error("dc_anchor_drift: NULL argument, K outside [1, max_steps], H_max outside "
+                  "[1, 4096] or eps <= 0");
     return DC_ERR_INVALID_ARG;
   }
   DC_CK(cudaSetDevice(m->device));
@@ -1383,8 +1384,9 @@ dc_status dc_anchor_response(dc_model* m, const float* noise, const dc_trajector
                              const double* sigmas, int H_max, double eps, double* q_out,
                              void* stream) {
   if (!m || !noise || !traj || !sigmas || !q_out || K < 1 || K > m->Kmax || H_max < 1 ||
-      !(eps > 0.0)) {
-    dc::set_error("dc_anchor_response: NULL argument, K outside [1, max_steps], H_max < 1 or eps <= 0");
+      H_max > 4096 || !(eps > 0.0)) {
+    dc::set_error("dc_anchor_response: NULL argument, K outside [1, max_steps], H_max outside "
+                  "[1, 4096] or eps <= 0");
     return DC_ERR_INVALID_ARG;
   }
   if (!dc::attention_f32_jvp_supported(m->dh)) {
