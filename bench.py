@@ -165,6 +165,24 @@ def oracle_rate(wl, n_compute, n_reuse, blocks=1):
     return (n_compute + n_reuse) / total, t_compute, t_reuse, (t3 - t0) + t_reuse
 
 
+def host_cpu():
+    """Architecture, logical cores and model of the host CPU (for the oracle
+    baseline lines)."""
+    import platform
+    model = ""
+    try:
+        with open("/proc/cpuinfo") as fh:
+            info = fh.read().splitlines()
+        for key in ("model name", "CPU part"):
+            vals = [l.split(":", 1)[1].strip() for l in info if l.startswith(key) and ":" in l]
+            if vals:
+                model = vals[0] if key == "model name" else f"CPU part {vals[0]}"
+                break
+    except OSError:
+        pass
+    return f"{platform.machine()}, {os.cpu_count()} logical cores" + (f", {model}" if model else "")
+
+
 def cpu_threads():
     try:
         import threadpoolctl
@@ -219,7 +237,7 @@ def run_reference(args, wl, rank, world):
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": workload_config(wl, wl.batch, wl.steps, tau, world,
                                       "host run: no GPU L2 to flush"),
-            "cpu_baseline": {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "cpu_baseline": {"value": rate, "unit": UNIT, "cores": cores, "cpu": host_cpu(), "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": rate, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -340,7 +358,7 @@ def run_calibration(args, wl):
         blk = oracle_block_jvp_seconds(wl)
         # every pass runs L block tangents; the primal points cost about as much again
         est = blk * wl.n_blocks * (passes + K)
-        line["cpu_baseline"] = {"value": est, "unit": "s", "cores": cpu_threads(), "kind": "oracle",
+        line["cpu_baseline"] = {"value": est, "unit": "s", "cores": cpu_threads(), "cpu": host_cpu(), "kind": "oracle",
                                 "sample": (f"one block tangent at full size ({blk:.2f} s, fp64 NumPy), "
                                            f"scaled by {wl.n_blocks} blocks x ({passes} tangent passes "
                                            f"+ {K} primal points)")}
@@ -516,7 +534,7 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         rate, tc, tr, spent = oracle_rate(wl, n_comp, n_reuse)
         line["cpu_baseline"] = {
-            "value": rate, "unit": UNIT, "cores": cpu_threads(), "kind": "oracle",
+            "value": rate, "unit": UNIT, "cores": cpu_threads(), "cpu": host_cpu(), "kind": "oracle",
             "sample": (f"one block of one compute scene-step ({tc:.2f} s when scaled to "
                        f"L={wl.n_blocks}) and one reuse scene-step ({tr:.3f} s), fp64 NumPy, "
                        f"weighted by this run's executed mix ({n_comp} compute / {n_reuse} reuse)")}
