@@ -281,3 +281,36 @@ def test_legal_mask_arguments(dc):
         dc.legal_mask(0, 4)
     with pytest.raises(dc.DCError):
         dc.legal_mask(10, 4, expert_boundary=-1)
+
+
+@pytest.mark.parametrize("seed", range(24))
+def test_plan_and_replan_ties_bit_exact(dc, seed):
+    """Coarse costs (0, 1/8, 1/4; all zero for every fourth seed) leave many
+    schedules with equal count and cost: the library's tie-break (smallest
+    terminal age, smallest age at every refresh) must pick the oracle's
+    schedule, which the oracle's pins tie to brute force."""
+    rng = random.Random(3000 + seed)
+    K = rng.randint(2, 30)
+    H = rng.randint(1, 5)
+    t = np.zeros((K, H + 1))
+    for j in range(1, K):
+        for h in range(1, H + 1):
+            t[j, h] = 0.0 if seed % 4 == 0 else rng.choice((0.0, 0.125, 0.25))
+    tabs = dict(q0=t, q1=t, d0=t, d1=t)
+    anc = dict(L0=0.0, T0=0.0, L1=50.0, T1=2.0, valid=1)
+    A = dc.AnchorArgs(K, H, anc, tabs)
+    st = P.scene_tables(tabs, 0.5, K, H)
+    for k0 in sorted({1, rng.randint(1, K), K}):
+        for rem in (0.0, 0.125, 0.5, math.inf):
+            prefix = [0] + [P.COMPUTE] * K
+            got = dc.replan(A, 0.5, k0, rem, prefix)
+            acts, n, cost = P.plan_suffix(st["c"], K, H, k0, rem)
+            exp = prefix[:k0] + [acts[k] for k in range(k0, K + 1)]
+            assert got["actions"] == exp and got["cost"] == cost
+            assert got["n_reuse"] == sum(1 for a in exp[1:] if a == P.REUSE)
+    poses = gen.unicycle(10.0, 0.2, 29, 0.1)
+    for tau in (0.0, 0.25, math.inf):
+        got = dc.plan(poses, A, tau, K)
+        ref = P.plan_scene(poses, anc, tabs, tau, K, H)
+        assert (got["actions"][1:], got["n_reuse"], got["cost"]) == \
+            (ref["actions"][1:], ref["n_reuse"], ref["cost"])
