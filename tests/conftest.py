@@ -11,6 +11,9 @@ if ROOT not in sys.path:
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (sm_103a) and the built library")
     config.addinivalue_line("markers", "slow: long CPU test")
+    # torch's own forward-mode helpers (the oracle's JVP pins) call a deprecated API
+    config.addinivalue_line("filterwarnings",
+                            "ignore:`torch.jit.script` is deprecated:DeprecationWarning")
 
 
 def gpu_available():
