@@ -399,8 +399,8 @@ dc_status dc_drift_sums(dc_model* m, const float* x_now, const float* x_ref, int
  * run (for example a planning loop whose memory budget is fixed at start-up,
  * or a host process that may not call cudaMalloc after initialisation,
  * since cudaMalloc can synchronise the device and can fail).  The paper has
- * no counterpart; this is a deployment variant of the Eq. 12 sums.
- * Same inputs, outputs and result as dc_drift_sums (x_now, x_ref: DEVICE
+ * no counterpart.  It returns the same sums as dc_drift_sums, from the
+ * same inputs into the same outputs (x_now, x_ref: DEVICE
  * fp32 [B][N][C]; out: DEVICE fp32 [2B]), but the reduction scratch is a
  * fixed 32 KiB array in device memory that every GPU loading this library
  * holds until the process exits; no device memory is allocated or freed.
@@ -410,7 +410,10 @@ dc_status dc_drift_sums(dc_model* m, const float* x_now, const float* x_ref, int
  * first call before capturing the stream into a graph.  All calls share the
  * one array: calls that can overlap on the GPU (different streams without
  * ordering) race on it and must be serialised by the caller.  Every scratch
- * entry a call reads is written earlier in the same call. */
+ * entry a call reads is written earlier in the same call.  The cached
+ * address does not survive a cudaDeviceReset, which also invalidates every
+ * model on the device: destroy models before a reset, create them again
+ * after it. */
 dc_status dc_drift_sums_noalloc(dc_model* m, const float* x_now, const float* x_ref, int B,
                                 float* out, void* stream);
 

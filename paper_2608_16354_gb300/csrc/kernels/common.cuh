@@ -173,18 +173,6 @@ __device__ __forceinline__ void tma_load_2d(void* smem_dst, const CUtensorMap* m
       : "memory");
 }
 
-// Tiled 2-D load multicast to every CTA of the cluster in `mask`: the box
-// lands at the same shared-memory offset in each, and each destination CTA's
-// mbarrier at `bar`'s offset receives the byte count.
-__device__ __forceinline__ void tma_load_2d_mc(void* smem_dst, const CUtensorMap* map, uint64_t* bar,
-                                               int x, int y, uint16_t mask) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster"
-      " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(smem_u32(smem_dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_u32(bar)), "h"(mask)
-      : "memory");
-}
-
 // Rank of this CTA in its cluster, and a full cluster barrier (all threads of
 // every CTA; release/acquire orders shared-memory writes such as barrier
 // initialisation before the peers' remote operations).

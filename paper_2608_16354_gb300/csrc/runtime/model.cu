@@ -1547,7 +1547,11 @@ float* g_scratch_addr[kScratchDevices] = {};
 
 // Device address of the scratch array on `dev` (which must be current).  The
 // array's name is only a host-side stand-in; the address is looked up once
-// per device and cached.
+// per device and cached for the life of the process.  A cudaDeviceReset
+// unloads the module and so invalidates the cached address -- and, with it,
+// every model on that device, whose weights it frees as well: models must be
+// destroyed before a reset and created again after it, and no call may use
+// this entry point across a reset.
 dc_status scratch_address(int dev, float** out) {
   std::lock_guard<std::mutex> lock(g_scratch_mu);
   if (dev < 0 || dev >= kScratchDevices) {
@@ -1593,8 +1597,11 @@ extern "C" dc_status dc_drift_sums_noalloc(dc_model* m, const float* x_now, cons
     it.ref[i] = x_ref + i * NC;
   }
   // every partial the final pass reads is written by the first pass of the
-  // same call, so nothing in the scratch needs clearing
-  DC_CK(dc::launch_drift(it, m->gram, m->gp, m->gs, m->N, m->C, scratch, out,
-                         static_cast<cudaStream_t>(stream)));
+  // same call, so nothing in the scratch needs clearing; the two launches are
+  // counted (and timed under dc_profile) like those of dc_drift_sums
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  DC_LAUNCH(DC_PROF_DRIFT, 4.0 * it.n * m->N * m->C * m->C, 8.0 * it.n * m->N * m->C,
+            dc::launch_drift(it, m->gram, m->gp, m->gs, m->N, m->C, scratch, out, st));
+  m->launches += 2;
   return DC_OK;
 }

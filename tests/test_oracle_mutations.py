@@ -24,6 +24,7 @@ LEGAL = "tests/test_oracle_legality.py"
 VARIANTS = "tests/test_oracle_variants.py"
 RESPONSE = "tests/test_oracle_response.py"
 GUIDANCE = "tests/test_oracle_guidance.py"
+DRIFT = "tests/test_oracle_drift_trace.py"
 
 # (name, file under oracle/, text, replacement, pin test files)
 MUTANTS = [
@@ -83,6 +84,14 @@ MUTANTS = [
     ("replan ignores the spent charge", "controller.py",
      'P.plan_suffix(tabs["c"], K, H, k, tau - S["C"], legal)',
      'P.plan_suffix(tabs["c"], K, H, k, tau, legal)', [PLANNER]),
+    ("anchor drift normalised by the earlier input", "controller.py",
+     "d[j][l] = P.drift(us[j + l], us[j], eps)", "d[j][l] = P.drift(us[j], us[j + l], eps)",
+     [DRIFT]),
+    ("anchor drift one step early", "controller.py",
+     "d[j][l] = P.drift(us[j + l], us[j], eps)", "d[j][l] = P.drift(us[j + l - 1], us[j], eps)",
+     [DRIFT]),
+    ("checked drift normalised by the refresh input", "controller.py",
+     'd_obs = P.drift(u_k, S["u_ref"], eps)', 'd_obs = P.drift(S["u_ref"], u_k, eps)', [DRIFT]),
     ("refresh does not reset the cache age", "controller.py",
      'S["j"], S["age"], S["r"], S["u_ref"] = k, 0, r, u',
      'S["j"], S["r"], S["u_ref"] = k, r, u', [DIT]),
@@ -152,7 +161,7 @@ def _copy_tree(dst, mutant=None):
     shutil.copytree(os.path.join(ROOT, "tests", "golden"), os.path.join(dst, "tests", "golden"))
     for f in ("conftest.py", "test_oracle_planner.py", "test_oracle_dit.py",
               "test_oracle_legality.py", "test_oracle_variants.py", "test_oracle_response.py",
-              "test_oracle_guidance.py"):
+              "test_oracle_guidance.py", "test_oracle_drift_trace.py"):
         shutil.copy(os.path.join(ROOT, "tests", f), os.path.join(dst, "tests", f))
     if mutant is not None:
         _, fname, old, new, _ = mutant
