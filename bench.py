@@ -18,7 +18,7 @@ videos/s, the all-compute throughput and the speedup, per-kernel device
 times, the roofline of the dominant kernel, an end-to-end number through
 dc_denoise_host (host latents in and out) and the CPU oracle baseline.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c2]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c5]
   python bench.py --impl reference ...   (times the CPU oracle instead)
 """
 
@@ -52,7 +52,7 @@ def parse():
     p.add_argument("--steps", type=int, default=5)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    p.add_argument("--workload", default="c2", choices=sorted(WORKLOADS))
+    p.add_argument("--workload", default="c5", choices=sorted(WORKLOADS))
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--calibration", action="store_true",
                    help="time the joint run responses (Eq. 6-7) of one anchor instead")
@@ -138,31 +138,117 @@ def calibrate(dc, model, wl, torch, dev):
 
 # ------------------------------------------------------------ cpu baseline
 
-def oracle_rate(wl, n_compute, n_reuse, blocks=1):
-    """Time the CPU oracle on a bounded sample of the workload and convert to
-    scene-steps/s for the given mix of compute and reuse scene-steps: one
-    compute scene-step is timed on `blocks` blocks and scaled to L blocks
-    (plus the embedding, conditioning and interface, timed in full); one
-    reuse scene-step is timed in full."""
+PROFILE_CALLS = 2  # calls repeated with per-launch events after the timed region
+SAMPLE_PARTS = 24  # the oracle sample takes 1 / SAMPLE_PARTS of the token rows
+
+
+_SETUP = {}
+
+
+def _oracle_sample_setup(wl):
+    """Inputs of the oracle sample (not timed): a one-block model of the
+    workload's widths, a scene's latent and poses, its modulation, one head's
+    keys and values for all N tokens, and a cached feature for R rows."""
+    if wl.name in _SETUP:
+        return _SETUP[wl.name]
     from oracle import dit as O
-    w = gen.weights(wl.with_(n_blocks=blocks))
-    m = O.Model(wl.with_(n_blocks=blocks), w)
-    x = gen.latents(wl, batch=1)[0]
-    tr = gen.scene_trajectories(wl, batch=1)[0]
-    t0 = time.perf_counter()
+    one = wl.with_(n_blocks=1, batch=1)
+    m = O.Model(one, gen.weights(one))
+    N, d, H = wl.n_tokens, wl.d_model, wl.n_heads
+    R = -(-N // SAMPLE_PARTS)
+    x = gen.latents(one)[0]
+    tr = gen.scene_trajectories(one)[0]
     blk, fmod = m.mods(0.5, tr)
-    u = O.embed(m.w, x)
+    wb = O.block_weights(m.w, 0)
+    a_all = O.layer_norm(O.embed(m.w, x)) * (1.0 + blk[0]["scale1"]) + blk[0]["shift1"]
+    dh = d // H
+    kw = np.concatenate([wb["w_qkv"][d:d + dh], wb["w_qkv"][2 * d:2 * d + dh]])
+    kv = O.linear(a_all, kw, np.zeros(2 * dh))
+    r_cache = 0.1 * np.random.default_rng(0).standard_normal((R, d))
+    _SETUP.clear()
+    _SETUP[wl.name] = (m, x, tr, blk, fmod, kv[:, :dh].copy(), kv[:, dh:].copy(), r_cache)
+    return _SETUP[wl.name]
+
+
+def oracle_step_seconds(wl):
+    """Time the CPU oracle on a bounded sample of one compute and one reuse
+    scene-step and scale each to the whole step.
+
+    Every op of a scene-step except attention acts row by row on the tokens
+    (embedding, LayerNorm, projections, MLP, head, Euler), and attention is
+    separable by query row and head.  So the sample is R = ceil(N / 24) token
+    rows through every row-wise op of one block, plus one head's attention
+    core for those R queries against all N keys; a block's time is the
+    row-wise time x N / R plus the attention time x heads x N / R, and a
+    compute step is L blocks plus the embedding, head and Euler update
+    (row-sampled the same way) plus the step's conditioning (the adaLN table
+    of one block timed, scaled to the 6 L + 2 rows of the table).  A reuse
+    step is the conditioning plus the embedding, head and Euler update.
+    Returns (t_compute, t_reuse, seconds spent inside the sample)."""
+    from oracle import dit as O
+    m, x, tr, blk, fmod, k1, v1, r_cache = _oracle_sample_setup(wl)
+    wb = O.block_weights(m.w, 0)
+    N, d, H = wl.n_tokens, wl.d_model, wl.n_heads
+    dh = d // H
+    R = -(-N // SAMPLE_PARTS)
+    scale = N / R
+    rows = np.arange(R)
+
+    t0 = time.perf_counter()
+    O.modulation(m.w, O.conditioning(m.w, 0.5, tr), 1, d)
     t1 = time.perf_counter()
-    h = O.backbone(m.w, u, blk, m.heads)
+    u = O.linear(x[rows], m.w["w_embed"], m.w["b_embed"]) + m.w["pos"][rows]  # embed, R rows
     t2 = time.perf_counter()
-    O.head(m.w, h, fmod)
+    # one block, row-wise part on R rows
+    mod = blk[0]
+    a = O.layer_norm(u) * (1.0 + mod["scale1"]) + mod["shift1"]
+    qkv = O.linear(a, wb["w_qkv"], wb["b_qkv"])
     t3 = time.perf_counter()
-    t_compute = (t1 - t0) + (t2 - t1) * wl.n_blocks / blocks + (t3 - t2)
+    o1 = O.attention_core(qkv[None, :, :dh], k1[None], v1[None])
     t4 = time.perf_counter()
-    m.reuse_step(x, h - u, 0.5, tr)
-    t_reuse = time.perf_counter() - t4
-    total = n_compute * t_compute + n_reuse * t_reuse
-    return (n_compute + n_reuse) / total, t_compute, t_reuse, (t3 - t0) + t_reuse
+    o = np.repeat(o1[0], H, axis=1)
+    h = u + mod["gate1"] * O.linear(o, wb["w_o"], wb["b_o"])
+    a = O.layer_norm(h) * (1.0 + mod["scale2"]) + mod["shift2"]
+    h = h + mod["gate2"] * O.linear(O.gelu_tanh(O.linear(a, wb["w_1"], wb["b_1"])), wb["w_2"], wb["b_2"])
+    t5 = time.perf_counter()
+    v = O.head(m.w, h, fmod)
+    O.euler(x[rows], v, 0.5, 0.48)
+    t6 = time.perf_counter()
+    v = O.head(m.w, u + r_cache, fmod)
+    O.euler(x[rows], v, 0.5, 0.48)
+    t7 = time.perf_counter()
+    t_cond = (t1 - t0) * (6 * wl.n_blocks + 2) / 8.0
+    t_rowwise = (t3 - t2) + (t5 - t4)
+    t_block = t_rowwise * scale + (t4 - t3) * H * scale
+    t_compute = t_cond + (t2 - t1) * scale + wl.n_blocks * t_block + (t6 - t5) * scale
+    t_reuse = t_cond + ((t2 - t1) + (t7 - t6)) * scale
+    return t_compute, t_reuse, t7 - t0
+
+
+def oracle_rate(wl, n_compute, n_reuse, min_seconds=0.0):
+    """Oracle scene-steps/s for the given mix of compute and reuse
+    scene-steps, from oracle_step_seconds; the sample is repeated until
+    min_seconds of oracle work have run and the median estimate is kept."""
+    tcs, trs, spent = [], [], 0.0
+    while True:
+        tc, tr, sp = oracle_step_seconds(wl)
+        tcs.append(tc)
+        trs.append(tr)
+        spent += sp
+        if spent >= min_seconds:
+            break
+    tc, tr = statistics.median(tcs), statistics.median(trs)
+    total = n_compute * tc + n_reuse * tr
+    return (n_compute + n_reuse) / total, tc, tr, spent, len(tcs)
+
+
+def sample_text(wl, tc, tr, reps):
+    R = -(-wl.n_tokens // SAMPLE_PARTS)
+    return (f"scaled, not timed in full: {R} of {wl.n_tokens} token rows through every row-wise op "
+            f"of one block, the embedding, head and Euler update, plus one of {wl.n_heads} heads' "
+            f"attention for those rows against all keys, scaled to the whole step and to "
+            f"L={wl.n_blocks} blocks (compute scene-step {tc:.2f} s, reuse scene-step {tr:.3f} s; "
+            f"median of {reps} samples), fp64 NumPy")
 
 
 def host_cpu():
@@ -222,15 +308,14 @@ def run_reference(args, wl, rank, world):
     times, rates = [], []
     for i in range(args.warmup + args.steps):
         t0 = time.perf_counter()
-        rate, tc, tr, _ = oracle_rate(wl, nc, nr)
+        rate, tc, tr, _, _ = oracle_rate(wl, nc, nr)
         if i >= args.warmup:
             times.append(time.perf_counter() - t0)
             rates.append(rate)
     rate = statistics.median(rates)
     cores = cpu_threads()
-    sample = (f"per step: one block of one compute scene-step scaled to L={wl.n_blocks} blocks "
-              f"plus one reuse scene-step, fp64 NumPy, weighted by the planned mix "
-              f"({nc} compute / {nr} reuse scene-steps per call)")
+    sample = ("per step: " + sample_text(wl, tc, tr, 1) +
+              f", weighted by the planned mix ({nc} compute / {nr} reuse scene-steps per call)")
     line = {"impl": "reference", "metric": METRIC, "value": rate, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1000.0 * wl.batch * wl.steps / rate, "higher_is_better": True,
@@ -441,8 +526,9 @@ def main():
     clk = clocks.stop()
     # the same steps once more with CUDA events around every launch (on the
     # call's stream): per-kernel device times for the roofline and the table
+    prof_calls = min(args.steps, PROFILE_CALLS)
     dc.profile(model, True)
-    for _ in range(args.steps):
+    for _ in range(prof_calls):
         _, st = one_call()
         assert np.array_equal(ref_exec, st["executed"]), "schedule changed between steps"
     dc.profile(model, False)
@@ -458,8 +544,7 @@ def main():
     # all-compute reference (no cache) for the speedup
     forced = np.full((B, K + 1), dc.COMPUTE, np.uint8)
     full_s = dc.SchedArgs(K, sig, A, tau, forced=forced)
-    one_call(full_s)
-    full_ms = statistics.median([one_call(full_s)[0] for _ in range(2)])
+    full_ms = one_call(full_s)[0]
 
     # end to end through the C ABI with host buffers (pinned)
     host = torch.empty(x1.shape, dtype=torch.float32).pin_memory()
@@ -500,9 +585,9 @@ def main():
         tinfo = json.load(open(tpath))
         same_src = tinfo.get("source_sha256", {}).get(dom) == kernel_source_hash(dom)
         if tinfo.get("workload") == wl.name and dom in tinfo.get("per_unit_bytes", {}) and same_src:
-            units = n_comp * args.steps * wl.n_blocks / n_launch
+            units = n_comp * prof_calls * wl.n_blocks / n_launch
             traffic = tinfo["per_unit_bytes"][dom] * units
-    kernels = {k: {"ms_per_call": v["ms"] / args.steps, "launches_per_call": v["launches"] / args.steps,
+    kernels = {k: {"ms_per_call": v["ms"] / prof_calls, "launches_per_call": v["launches"] / prof_calls,
                    "tflops": (v["flops"] / (v["ms"] / 1000.0) / 1e12) if v["ms"] > 0 and v["flops"] else None,
                    "gbs": (v["bytes"] / (v["ms"] / 1000.0) / 1e9) if v["ms"] > 0 else None}
                for k, v in prof.items() if v["launches"]}
@@ -526,18 +611,17 @@ def main():
         "roofline": {"kernel": dom, "bound": "tensor" if tensor else "hbm", "achieved": achieved,
                      "peak": peak, "unit": unit, "frac": achieved / peak, "traffic": traffic,
                      "peak_source": f"{pk_src} ({'bf16 sustained' if tensor else 'HBM copy'})",
-                     "timing": "CUDA events around every launch, over a repetition of the timed "
-                               "steps right after them (the same schedule)"},
+                     "timing": f"CUDA events around every launch, over a repetition of {prof_calls} "
+                               "of the timed steps right after them (the same schedule)"},
         "kernels": kernels,
         "clocks": clk,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        rate, tc, tr, spent = oracle_rate(wl, n_comp, n_reuse)
+        rate, tc, tr, spent, reps = oracle_rate(wl, n_comp, n_reuse, min_seconds=10.0)
         line["cpu_baseline"] = {
             "value": rate, "unit": UNIT, "cores": cpu_threads(), "cpu": host_cpu(), "kind": "oracle",
-            "sample": (f"one block of one compute scene-step ({tc:.2f} s when scaled to "
-                       f"L={wl.n_blocks}) and one reuse scene-step ({tr:.3f} s), fp64 NumPy, "
-                       f"weighted by this run's executed mix ({n_comp} compute / {n_reuse} reuse)")}
+            "sample": (sample_text(wl, tc, tr, reps) + f", {spent:.1f} s of oracle work, weighted by "
+                       f"this run's executed mix ({n_comp} compute / {n_reuse} reuse)")}
     if rank == 0:
         print(json.dumps(line), flush=True)
     model.close()

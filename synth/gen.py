@@ -77,34 +77,68 @@ def _tensor_id(name: str) -> int:
     return h
 
 
+class _Weights(dict):
+    """Weight dict whose tensors are views, in weight_specs order, into one
+    flat fp32 array (`blob`), so that flat_blob need not copy them."""
+    blob = None
+    views = ()
+
+
+def _draw(seed, key, shape, std, bf16, out):
+    a = (_rng(seed, _tensor_id(key)).standard_normal(shape) * std).astype(np.float32)
+    if bf16:
+        a = round_to_bf16(a)
+    out[...] = a
+
+
 def weights(wl: Workload, seed: int = None, std: float = 0.02) -> dict:
-    """Random-init weights: matrices N(0, std), biases zero."""
+    """Random-init weights: matrices N(0, std), biases zero.  Every matrix
+    (and every block's slice of the ada table) has its own stream, so the
+    tensors are drawn in parallel threads with the same values as drawn one
+    after another."""
+    import os
+    from concurrent.futures import ThreadPoolExecutor
     seed = wl.seed if seed is None else seed
-    out = {}
-    for name, shape, kind in weight_specs(wl):
+    specs = weight_specs(wl)
+    total = sum(int(np.prod(shape)) for _, shape, _ in specs)
+    blob = np.empty(total, np.float32)
+    out = _Weights()
+    out.blob = blob
+    bf16 = wl.dtype == "bf16"
+    jobs, o = [], 0
+    for name, shape, kind in specs:
+        n = int(np.prod(shape))
+        view = blob[o:o + n].reshape(shape)
+        o += n
+        out[name] = view
         if kind == "b":
-            a = np.zeros(shape, np.float32)
-        else:
+            view[...] = 0.0
+        elif name == "w_ada":
             # the ada table is drawn row-block by row-block so that it does not
             # depend on L for the blocks that two workloads share
-            if name == "w_ada":
-                d = wl.d_model
-                parts = [(_rng(seed, _tensor_id(f"w_ada.blk{l}")).standard_normal((6 * d, d)) * std)
-                         for l in range(wl.n_blocks)]
-                parts.append(_rng(seed, _tensor_id("w_ada.final")).standard_normal((2 * d, d)) * std)
-                a = np.concatenate(parts, 0).astype(np.float32)
-            else:
-                a = (_rng(seed, _tensor_id(name)).standard_normal(shape) * std).astype(np.float32)
-        if wl.dtype == "bf16":
-            a = round_to_bf16(a)
-        out[name] = a
+            d = wl.d_model
+            for l in range(wl.n_blocks):
+                jobs.append((f"w_ada.blk{l}", (6 * d, d), view[6 * d * l:6 * d * (l + 1)]))
+            jobs.append(("w_ada.final", (2 * d, d), view[6 * d * wl.n_blocks:]))
+        else:
+            jobs.append((name, shape, view))
+    out.views = tuple(out[n] for n, _, _ in specs)
+    big = sum(int(np.prod(sh)) for _, sh, _ in jobs) > (1 << 22)
+    workers = min(32, os.cpu_count() or 1) if big else 1
+    with ThreadPoolExecutor(workers) as ex:
+        for f in [ex.submit(_draw, seed, k, sh, std, bf16, v) for k, sh, v in jobs]:
+            f.result()
     return out
 
 
 def flat_blob(wl: Workload, w: dict) -> np.ndarray:
-    """Concatenate the tensors in weight_specs order into one fp32 array."""
-    return np.concatenate([np.ascontiguousarray(w[n], np.float32).ravel()
-                           for n, _, _ in weight_specs(wl)])
+    """The tensors in weight_specs order as one fp32 array (no copy when w
+    is weights()'s own, unmodified dict)."""
+    names = [n for n, _, _ in weight_specs(wl)]
+    if isinstance(w, _Weights) and w.blob is not None and len(w.views) == len(names) and \
+            all(w[n] is v for n, v in zip(names, w.views)):
+        return w.blob
+    return np.concatenate([np.ascontiguousarray(w[n], np.float32).ravel() for n in names])
 
 
 # ------------------------------------------------------------------- latents
