@@ -304,16 +304,17 @@ dc_status dc_denoise_host(dc_model* m, float* host_latents, const dc_cond* cond,
 /* ------------------------------------------------ sampler-state snapshots
  * A snapshot is the whole state of a sampler call after k_done of its K
  * steps (Sec. 3.2 controller + Eq. 1 cache): the latents x_{k_done+1}, every
- * scene's refresh latent x_j and cached r (both guidance branches), the
+ * scene's refresh latent x_j and cache row c = r + b_e + pos (both guidance
+ * branches), the
  * plan of the remaining steps after any replans, the charge C, the last
  * refresh j and cache age of each scene, and the call's record so far.
  * Resuming from it (dc_denoise_steps) continues the call exactly: the final
  * latents and record equal the uninterrupted call's bit for bit.  Use:
  * preempting a long call, or moving it to another model instance or box.
  * Layout (caller-owned host memory, native byte order):
- *   header, 128 bytes: char magic[8] "DCSNAP01"; uint32 version (1);
+ *   header, 128 bytes: char magic[8] "DCSNAP01"; uint32 version (2);
  *     int32 B, K, cfg (0 or 1), k_done, dtype, n_tokens, d_model, channels;
- *     uint32 element bytes of r; uint64 digest; uint64 total bytes;
+ *     uint32 element bytes of c; uint64 digest; uint64 total bytes;
  *     int64 backbone_calls; 56 zero bytes
  *   B scene records of 48 bytes: double charge, D; int32 j, age, supported,
  *     n_compute, n_reuse, n_veto, n_replan, 0
@@ -321,7 +322,7 @@ dc_status dc_denoise_host(dc_model* m, float* host_latents, const dc_cond* cond,
  *     a multiple of 8 bytes
  *   double d_obs, d_bar: [B][K+1] each
  *   at the next multiple of 256: float latents [B][N][C], float x_j [B][N][C]
- *   at the next multiple of 256: r [B_i][N][d] in the model dtype
+ *   at the next multiple of 256: c [B_i][N][d] in the model dtype
  *     (B_i = 2B with guidance, else B)
  * digest: FNV-1a (64-bit) of the call's inputs (trajectories, sigmas, tau,
  * veto, cfg_scale, and the forced actions or the anchor responses). */
@@ -417,11 +418,13 @@ dc_status dc_drift_sums(dc_model* m, const float* x_now, const float* x_ref, int
 dc_status dc_drift_sums_noalloc(dc_model* m, const float* x_now, const float* x_ref, int B,
                                 float* out, void* stream);
 
-/* Copy the cached backbone output r_j (Eq. 1: r = h_L - u of the scene's
+/* Write the cached backbone output r_j (Eq. 1: r = h_L - u of the scene's
  * last full evaluation) of `scene` (0 <= scene < max_batch) into DEVICE
- * memory dst.  The cache holds [N][d] elements of the model dtype (fp32 or
- * bf16); `bytes` must equal N * d * sizeof(element).  Asynchronous on
- * `stream`.  Intended for inspection and tests. */
+ * memory dst, [N][d] elements of the model dtype (fp32 or bf16); `bytes`
+ * must equal N * d * sizeof(element).  The cache itself holds c = h_L -
+ * x W_e^T = r + b_e + pos (so that a reuse step rebuilds u + r from the
+ * latent alone); this call returns c - b_e - pos, rounded to the model
+ * dtype.  Asynchronous on `stream`.  Intended for inspection and tests. */
 dc_status dc_cache_copy(dc_model* m, int scene, void* dst, size_t bytes, void* stream);
 
 /* The attention kernel of the block stack on caller-provided operands:

@@ -327,8 +327,29 @@ __device__ __forceinline__ void modulate(float4 (&v)[NV], float mu, float rs, co
   }
 }
 
+// Rows of the interface on the SIMT path (fp32 models, or C != 16).  The
+// cache row of a compute step is c = h_L - x W_e^T (the block-stack residual
+// plus b_e + pos), so a reuse step forms h = x W_e^T + c.
+template <int NV, int C>
+__device__ __forceinline__ void embed_latent(const float (&xv)[C], const float* __restrict__ w_eT,
+                                             int d, int d4, int lane, float4 (&o)[NV]) {
+#pragma unroll
+  for (int j = 0; j < NV; ++j) {
+    const int i = lane + 32 * j;
+    float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (i < d4) {
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const float4 w = __ldg(reinterpret_cast<const float4*>(w_eT + (size_t)c * d) + i);
+        a.x += w.x * xv[c]; a.y += w.y * xv[c]; a.z += w.z * xv[c]; a.w += w.w * xv[c];
+      }
+    }
+    o[j] = a;
+  }
+}
+
 template <typename T, int NV, int C>
-__global__ void final_compute_kernel(const float* __restrict__ hL, const float* __restrict__ u,
+__global__ void final_compute_kernel(const float* __restrict__ hL, const float* __restrict__ w_eT,
                                      float* __restrict__ x, float* __restrict__ xj,
                                      T* __restrict__ r, SlotMap map, int N, int d,
                                      const float* __restrict__ mod, int mod_stride, int fin_off,
@@ -344,26 +365,34 @@ __global__ void final_compute_kernel(const float* __restrict__ hL, const float* 
   const int d4 = d >> 2;
   float4 hv[NV];
   load_row<NV>(hL + (size_t)row * d, d4, lane, hv);
-  // cache the reusable backbone output r = h_L - u
+  const float* xr = x + ((size_t)scene * N + tok) * C;
+  float xv[C];
+#pragma unroll
+  for (int c = 0; c < C; ++c) xv[c] = xr[c];
+  // cache the reusable backbone output c = h_L - x W_e^T
   {
-    const float4* up = reinterpret_cast<const float4*>(u + (size_t)row * d);
+    float4 ue[NV];
+    embed_latent<NV, C>(xv, w_eT, d, d4, lane, ue);
     T* rd = r + ((size_t)scene * N + tok) * d;
 #pragma unroll
     for (int j = 0; j < NV; ++j) {
       const int i = lane + 32 * j;
-      if (i < d4) {
-        const float4 uu = up[i];
-        store4<T>(rd + 4 * i, hv[j].x - uu.x, hv[j].y - uu.y, hv[j].z - uu.z, hv[j].w - uu.w);
-      }
+      if (i < d4)
+        store4<T>(rd + 4 * i, hv[j].x - ue[j].x, hv[j].y - ue[j].y, hv[j].z - ue[j].z,
+                  hv[j].w - ue[j].w);
     }
   }
   float mu, rs;
   row_stats<NV>(hv, d, d4, lane, &mu, &rs);
   modulate<NV>(hv, mu, rs, mod + (size_t)scene * mod_stride, fin_off, fin_off + d, d4, lane);
   const float vc = head_dot<NV, C>(hv, d, d4, lane, w_f, b_f);
+  __syncwarp();
   if (lane < C) {
+    float xo = xv[0];
+#pragma unroll
+    for (int c = 1; c < C; ++c)
+      if (lane == c) xo = xv[c];
     const size_t xi = ((size_t)scene * N + tok) * C + lane;
-    const float xo = x[xi];
     xj[xi] = xo;
     if (vout) vout[xi] = vc;  // the caller combines velocities (guidance)
     else x[xi] = xo + dsig * vc;
@@ -372,8 +401,7 @@ __global__ void final_compute_kernel(const float* __restrict__ hL, const float* 
 
 template <typename T, int NV, int C>
 __global__ void final_reuse_kernel(float* __restrict__ x, const T* __restrict__ r,
-                                   const float* __restrict__ w_eT, const float* __restrict__ b_e,
-                                   const T* __restrict__ pos, SlotMap map, int N, int d,
+                                   const float* __restrict__ w_eT, SlotMap map, int N, int d,
                                    const float* __restrict__ mod, int mod_stride, int fin_off,
                                    const float* __restrict__ w_f, const float* __restrict__ b_f,
                                    float dsig, float* __restrict__ vout) {
@@ -390,25 +418,14 @@ __global__ void final_reuse_kernel(float* __restrict__ x, const T* __restrict__ 
 #pragma unroll
   for (int c = 0; c < C; ++c) xv[c] = xr[c];
   const T* rr = r + ((size_t)scene * N + tok) * d;
-  const T* pr = pos + (size_t)tok * d;
   float4 hv[NV];
+  embed_latent<NV, C>(xv, w_eT, d, d4, lane, hv);
 #pragma unroll
   for (int j = 0; j < NV; ++j) {
     const int i = lane + 32 * j;
     if (i < d4) {
       const float4 rv = load4<T>(rr + 4 * i);
-      const float4 pv = load4<T>(pr + 4 * i);
-      const float4 bv = __ldg(reinterpret_cast<const float4*>(b_e) + i);
-      float4 o = make_float4(bv.x + pv.x + rv.x, bv.y + pv.y + rv.y, bv.z + pv.z + rv.z,
-                             bv.w + pv.w + rv.w);
-#pragma unroll
-      for (int c = 0; c < C; ++c) {
-        const float4 w = __ldg(reinterpret_cast<const float4*>(w_eT + (size_t)c * d) + i);
-        o.x += w.x * xv[c]; o.y += w.y * xv[c]; o.z += w.z * xv[c]; o.w += w.w * xv[c];
-      }
-      hv[j] = o;
-    } else {
-      hv[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+      hv[j].x += rv.x; hv[j].y += rv.y; hv[j].z += rv.z; hv[j].w += rv.w;
     }
   }
   float mu, rs;
@@ -425,6 +442,17 @@ __global__ void final_reuse_kernel(float* __restrict__ x, const T* __restrict__ 
     if (vout) vout[xi] = vc;
     else x[xi] = xo + dsig * vc;
   }
+}
+
+// The model's r_j = c_j - b_e - pos_t from the cache row c_j (inspection):
+// out [N][d] of the cache type.
+template <typename T>
+__global__ void cache_to_residual_kernel(const T* __restrict__ c, const float* __restrict__ b_e,
+                                         const T* __restrict__ pos, int N, int d, T* __restrict__ out) {
+  const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (size_t)N * d) return;
+  const int e = (int)(i % d);
+  out[i] = from_f<T>(to_f<T>(c[i]) - b_e[e] - to_f<T>(pos[i]));
 }
 
 // Guidance: x_s += dsig (v_u + g (v_c - v_u)) with v_c = v[s], v_u = v[B + s].
@@ -605,7 +633,7 @@ template cudaError_t launch_ln_mod<__nv_bfloat16>(const float*, int, int, int, c
                                                   cudaStream_t);
 
 template <typename T>
-cudaError_t launch_final_compute(const float* hL, const float* u, float* x, float* xj, T* r,
+cudaError_t launch_final_compute(const float* hL, const float* w_eT, float* x, float* xj, T* r,
                                  const SlotMap& map, int N, int C, int d, const float* mod,
                                  int mod_stride, int fin_off, const float* w_f, const float* b_f,
                                  float dsig, cudaStream_t st, float* vout) {
@@ -615,11 +643,11 @@ cudaError_t launch_final_compute(const float* hL, const float* u, float* x, floa
   const int blocks = (int)(((size_t)rows * 32 + threads - 1) / threads);
   if (C == 16) {
     DC_NV_SWITCH(nv_for(d), return launch_pdl(final_compute_kernel<T, NV, 16>, dim3(blocks),
-                                               dim3(threads), 0, st, hL, u, x, xj, r, map, N, d,
+                                               dim3(threads), 0, st, hL, w_eT, x, xj, r, map, N, d,
                                                mod, mod_stride, fin_off, w_f, b_f, dsig, vout));
   } else if (C == 4) {
     DC_NV_SWITCH(nv_for(d), return launch_pdl(final_compute_kernel<T, NV, 4>, dim3(blocks),
-                                               dim3(threads), 0, st, hL, u, x, xj, r, map, N, d,
+                                               dim3(threads), 0, st, hL, w_eT, x, xj, r, map, N, d,
                                                mod, mod_stride, fin_off, w_f, b_f, dsig, vout));
   } else {
     return cudaErrorInvalidValue;
@@ -636,36 +664,48 @@ template cudaError_t launch_final_compute<__nv_bfloat16>(const float*, const flo
                                                          const float*, float, cudaStream_t, float*);
 
 template <typename T>
-cudaError_t launch_final_reuse(float* x, const T* r, const float* w_e, const float* b_e,
-                               const T* pos, const SlotMap& map, int N, int C, int d,
-                               const float* mod, int mod_stride, int fin_off, const float* w_f,
-                               const float* b_f, float dsig, cudaStream_t st, float* vout) {
+cudaError_t launch_final_reuse(float* x, const T* r, const float* w_eT, const SlotMap& map, int N,
+                               int C, int d, const float* mod, int mod_stride, int fin_off,
+                               const float* w_f, const float* b_f, float dsig, cudaStream_t st,
+                               float* vout) {
   if (map.n <= 0) return cudaSuccess;
   const int rows = map.n * N;
   const int threads = 256;
   const int blocks = (int)(((size_t)rows * 32 + threads - 1) / threads);
   if (C == 16) {
     DC_NV_SWITCH(nv_for(d), return launch_pdl(final_reuse_kernel<T, NV, 16>, dim3(blocks),
-                                               dim3(threads), 0, st, x, r, w_e, b_e, pos, map, N,
-                                               d, mod, mod_stride, fin_off, w_f, b_f, dsig, vout));
+                                               dim3(threads), 0, st, x, r, w_eT, map, N, d, mod,
+                                               mod_stride, fin_off, w_f, b_f, dsig, vout));
   } else if (C == 4) {
     DC_NV_SWITCH(nv_for(d), return launch_pdl(final_reuse_kernel<T, NV, 4>, dim3(blocks),
-                                               dim3(threads), 0, st, x, r, w_e, b_e, pos, map, N,
-                                               d, mod, mod_stride, fin_off, w_f, b_f, dsig, vout));
+                                               dim3(threads), 0, st, x, r, w_eT, map, N, d, mod,
+                                               mod_stride, fin_off, w_f, b_f, dsig, vout));
   } else {
     return cudaErrorInvalidValue;
   }
   return cudaGetLastError();
 }
-template cudaError_t launch_final_reuse<float>(float*, const float*, const float*, const float*,
-                                               const float*, const SlotMap&, int, int, int,
-                                               const float*, int, int, const float*, const float*,
-                                               float, cudaStream_t, float*);
+template cudaError_t launch_final_reuse<float>(float*, const float*, const float*, const SlotMap&,
+                                               int, int, int, const float*, int, int, const float*,
+                                               const float*, float, cudaStream_t, float*);
 template cudaError_t launch_final_reuse<__nv_bfloat16>(float*, const __nv_bfloat16*, const float*,
-                                                       const float*, const __nv_bfloat16*,
                                                        const SlotMap&, int, int, int, const float*,
                                                        int, int, const float*, const float*, float,
                                                        cudaStream_t, float*);
+
+template <typename T>
+cudaError_t launch_cache_to_residual(const T* c, const float* b_e, const T* pos, int N, int d, T* out,
+                                     cudaStream_t st) {
+  const size_t n = (size_t)N * d;
+  if (n == 0) return cudaSuccess;
+  cache_to_residual_kernel<T><<<(unsigned)((n + 255) / 256), 256, 0, st>>>(c, b_e, pos, N, d, out);
+  return cudaGetLastError();
+}
+template cudaError_t launch_cache_to_residual<float>(const float*, const float*, const float*, int,
+                                                     int, float*, cudaStream_t);
+template cudaError_t launch_cache_to_residual<__nv_bfloat16>(const __nv_bfloat16*, const float*,
+                                                             const __nv_bfloat16*, int, int,
+                                                             __nv_bfloat16*, cudaStream_t);
 
 cudaError_t launch_cfg_combine(float* x, const float* v, int B, size_t per_scene, float g,
                                float dsig, cudaStream_t st) {

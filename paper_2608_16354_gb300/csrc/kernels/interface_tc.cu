@@ -1,0 +1,498 @@
+// Interface + Euler kernels of the bf16 path on the tensor cores (Eq. 1: the
+// interface H_k on compute and on reuse steps, with the cache write of the
+// compute step).
+//
+// The cache holds, per scene, c = h_L - x W_e^T (bf16 [N][d]) from the
+// scene's last full evaluation: the block-stack residual r = h_L - u plus
+// the part b_e + pos of the embedding that does not depend on the latent,
+// so a reuse step rebuilds u_k + r_j = x_k W_e^T + c_j from the latent alone
+// and reads nothing else of size N x d.
+//
+// The head is linear in the LayerNorm output, so with a_e = (h_e - mu) rs
+// (1 + s_e) + sh_e and W'[c][e] = (1 + s_e) W_f[c][e]:
+//   v_c = rs (P_c - mu S'_c) + beta_c,  P_c = sum_e h_e W'[c][e],
+//   S'_c = sum_e W'[c][e],               beta_c = sum_e sh_e W_f[c][e] + b_f[c],
+// and the LayerNorm moments come from sum_e h_e and sum_e h_e^2 of the same
+// pass, so one read of each row suffices.  S', beta and W' (as bf16 hi + lo
+// halves, W' = hi + lo to 2^-16) are per (step, scene) tables built once per
+// call.  On a reuse step h = x W_e^T + c gives
+//   P_c      = (x G_s)_c + Q_c,  Q_c = sum_e c_e W'[c][e],  G_s = W_e^T diag(1 + s) W_f^T [C][C]
+//   sum h    = x . w_sum + sum c,                           w_sum = sum_e W_e^T[:, e]
+//   sum h^2  = x^T G x + 2 x . A + sum c^2,  A = W_e c,     G = W_e^T W_e
+// so the contractions over d read only c: [A | Q] = c [W_e^T | W'hi | W'lo],
+// 48 columns, on the tensor cores (mma.sync m16n8k16, bf16 in, fp32 out).
+// On a compute step P = h [W'hi | W'lo] with h split into bf16 hi + lo
+// halves (hi W'hi + lo W'hi + hi W'lo), and c = h - x W_e^T is written.
+//
+// Layout trick: the order of the contraction index inside a 32-column block
+// is free as long as both operands use it, so each thread loads 8
+// consecutive columns of a row (16 B of bf16, 32 B of fp32) and those land
+// exactly in its A fragment of the block's two 16-deep steps; the B
+// fragments are then 16-byte loads of 8 consecutive columns of a W row.
+//
+// A CTA (4 warps) takes 32 tokens of one scene (reuse; 16 on compute
+// steps); each warp takes every 4th 32-column block of d for all of the
+// CTA's tokens, and the partial sums of the four warps are added in shared
+// memory in a fixed order (deterministic).  C = 16 channels.
+#include "common.cuh"
+#include "kernels.h"
+
+namespace dc {
+
+namespace {
+
+constexpr int kHC = 16;          // latent channels the tensor-core interface supports
+constexpr int kHeadTab = 2 * kHC + kHC * kHC;  // S', beta, G_s per (step, scene)
+
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                               uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+      "{%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// 16-byte loads: streamed data (read once) bypasses L1; tables stay cached
+__device__ __forceinline__ uint4 ld_stream16(const void* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+__device__ __forceinline__ uint4 ld_tab16(const void* p) {
+  uint4 v;
+  asm volatile("ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+               : "l"(p));
+  return v;
+}
+__device__ __forceinline__ float4 ld_stream_f4(const float* p) {
+  float4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "l"(p));
+  return v;
+}
+__device__ __forceinline__ void st_stream16(void* p, uint4 v) {
+  asm volatile("st.global.cs.v4.u32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x), "r"(v.y),
+               "r"(v.z), "r"(v.w)
+               : "memory");
+}
+
+__device__ __forceinline__ uint32_t pack_bf2(float lo_elem, float hi_elem) {
+  __nv_bfloat162 t = __floats2bfloat162_rn(lo_elem, hi_elem);
+  return *reinterpret_cast<uint32_t*>(&t);
+}
+__device__ __forceinline__ float2 unpack_bf2(uint32_t w) {
+  __nv_bfloat162 t = *reinterpret_cast<__nv_bfloat162*>(&w);
+  return __bfloat1622float2(t);
+}
+// v = hi + lo with hi = bf16(v), lo = bf16(v - hi), for a pair of values
+__device__ __forceinline__ void split_pair(float a, float b, uint32_t* hi, uint32_t* lo) {
+  const __nv_bfloat16 ha = __float2bfloat16_rn(a), hb = __float2bfloat16_rn(b);
+  __nv_bfloat162 h2;
+  h2.x = ha;
+  h2.y = hb;
+  *hi = *reinterpret_cast<uint32_t*>(&h2);
+  *lo = pack_bf2(a - __bfloat162float(ha), b - __bfloat162float(hb));
+}
+
+// ------------------------------------------------ per (step, scene) tables
+
+// One CTA per (step, scene) item: W' = (1 + scale) W_f as bf16 hi and lo
+// halves [32][d] (rows 0-15 hi, 16-31 lo), and S', beta, G_s (fp32).
+__global__ void __launch_bounds__(256) head_tables_kernel(
+    const float* __restrict__ mod, int mod_stride, int fin_off, int d,
+    const float* __restrict__ w_f, const float* __restrict__ b_f, const float* __restrict__ w_eT,
+    __nv_bfloat16* __restrict__ wp, float* __restrict__ tab) {
+  const int item = blockIdx.x;
+  const float* sh = mod + (size_t)item * mod_stride + fin_off;
+  const float* sc = sh + d;
+  __nv_bfloat16* w = wp + (size_t)item * 2 * kHC * d;
+  for (int i = threadIdx.x; i < kHC * d; i += blockDim.x) {
+    const int c = i / d, e = i - c * d;
+    const float v = (1.f + sc[e]) * w_f[i];
+    const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+    w[(size_t)c * d + e] = hi;
+    w[(size_t)(kHC + c) * d + e] = __float2bfloat16_rn(v - __bfloat162float(hi));
+  }
+  float* t = tab + (size_t)item * kHeadTab;
+  const int a = threadIdx.x >> 4, c = threadIdx.x & 15;  // G_s[a][c]
+  float g = 0.f;
+  for (int e = 0; e < d; ++e) g = fmaf(w_eT[(size_t)a * d + e] * (1.f + sc[e]), w_f[(size_t)c * d + e], g);
+  t[2 * kHC + a * kHC + c] = g;
+  if (threadIdx.x < 2 * kHC) {
+    const int cc = threadIdx.x & 15;
+    float s = 0.f;
+    if (threadIdx.x < kHC) {
+      for (int e = 0; e < d; ++e) s = fmaf(1.f + sc[e], w_f[(size_t)cc * d + e], s);
+      t[cc] = s;
+    } else {
+      for (int e = 0; e < d; ++e) s = fmaf(sh[e], w_f[(size_t)cc * d + e], s);
+      t[kHC + cc] = s + b_f[cc];
+    }
+  }
+}
+
+// ---------------------------------------------------------------- reuse step
+
+constexpr int kReuseTok = 32;  // tokens per CTA on reuse steps (two m16 tiles per warp)
+constexpr int kCmpTok = 16;    // tokens per CTA on compute steps (one m16 tile per warp)
+
+// Reuse step of the scenes in `map`: h = x W_e^T + c_j, v = head(h), x += dsig v
+// (or v to vout).  wp_k / tab_k: this step's tables, indexed by scene.
+__global__ void __launch_bounds__(128) head_reuse_kernel(
+    float* __restrict__ x, const __nv_bfloat16* __restrict__ cache, SlotMap map, int N, int d,
+    const __nv_bfloat16* __restrict__ w_eT_bf, const __nv_bfloat16* __restrict__ wp_k,
+    const float* __restrict__ tab_k, const float* __restrict__ wsum, const float* __restrict__ gram,
+    float dsig, float* __restrict__ vout) {
+  pdl_trigger();
+  pdl_wait();
+  __shared__ float part[4][kReuseTok][2 * kHC + 2];  // per warp: A, Q, sum c, sum c^2
+  __shared__ float stab[kHeadTab + kHC + kHC * kHC];  // S', beta, G_s | w_sum | G
+  const int slot = blockIdx.y, scene = map.scene[slot];
+  const int tok0 = blockIdx.x * kReuseTok;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, q = lane & 3;
+  for (int i = threadIdx.x; i < kHeadTab; i += blockDim.x) stab[i] = tab_k[(size_t)scene * kHeadTab + i];
+  if (threadIdx.x < kHC) stab[kHeadTab + threadIdx.x] = wsum[threadIdx.x];
+  for (int i = threadIdx.x; i < kHC * kHC; i += blockDim.x) stab[kHeadTab + kHC + i] = gram[i];
+
+  const __nv_bfloat16* cs = cache + (size_t)scene * N * d;
+  const __nv_bfloat16* wk = wp_k + (size_t)scene * 2 * kHC * d;
+  int row[2][2];
+  bool ok[2][2];
+#pragma unroll
+  for (int i = 0; i < 2; ++i)
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      row[i][h] = tok0 + 16 * i + 8 * h + g;
+      ok[i][h] = row[i][h] < N;
+    }
+  float D[2][6][4];
+#pragma unroll
+  for (int i = 0; i < 2; ++i)
+#pragma unroll
+    for (int j = 0; j < 6; ++j)
+#pragma unroll
+      for (int t = 0; t < 4; ++t) D[i][j][t] = 0.f;
+  float s1[2][2] = {{0.f, 0.f}, {0.f, 0.f}}, s2[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
+  const int nblk = d >> 5;
+#pragma unroll 2
+  for (int b = warp; b < nblk; b += 4) {
+    const int e = (b << 5) + (q << 3);
+    uint4 av[2][2];
+#pragma unroll
+    for (int i = 0; i < 2; ++i)
+#pragma unroll
+      for (int h = 0; h < 2; ++h)
+        av[i][h] = ok[i][h] ? ld_stream16(cs + (size_t)row[i][h] * d + e) : make_uint4(0u, 0u, 0u, 0u);
+    // B rows: W_e^T (channels 0-7, 8-15), W' hi (0-7, 8-15), W' lo (0-7, 8-15)
+    uint4 bw[6];
+    bw[0] = ld_tab16(w_eT_bf + (size_t)g * d + e);
+    bw[1] = ld_tab16(w_eT_bf + (size_t)(8 + g) * d + e);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) bw[2 + j] = ld_tab16(wk + (size_t)(8 * j + g) * d + e);
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const uint32_t w4[4] = {av[i][h].x, av[i][h].y, av[i][h].z, av[i][h].w};
+#pragma unroll
+        for (int p = 0; p < 4; ++p) {
+          const float2 f = unpack_bf2(w4[p]);
+          s1[i][h] += f.x + f.y;
+          s2[i][h] = fmaf(f.x, f.x, fmaf(f.y, f.y, s2[i][h]));
+        }
+      }
+#pragma unroll
+      for (int s = 0; s < 2; ++s) {
+        const uint32_t a0 = s ? av[i][0].z : av[i][0].x;  // row g, cols 4s + 0, 1
+        const uint32_t a1 = s ? av[i][1].z : av[i][1].x;  // row g + 8
+        const uint32_t a2 = s ? av[i][0].w : av[i][0].y;  // row g, cols 4s + 2, 3
+        const uint32_t a3 = s ? av[i][1].w : av[i][1].y;  // row g + 8
+#pragma unroll
+        for (int j = 0; j < 6; ++j)
+          mma_bf16_16816(D[i][j], a0, a1, a2, a3, s ? bw[j].z : bw[j].x, s ? bw[j].w : bw[j].y);
+      }
+    }
+  }
+  // lanes 4 g .. 4 g + 3 hold the same rows: add their column sums
+#pragma unroll
+  for (int i = 0; i < 2; ++i)
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      s1[i][h] += __shfl_xor_sync(0xffffffffu, s1[i][h], 1);
+      s1[i][h] += __shfl_xor_sync(0xffffffffu, s1[i][h], 2);
+      s2[i][h] += __shfl_xor_sync(0xffffffffu, s2[i][h], 1);
+      s2[i][h] += __shfl_xor_sync(0xffffffffu, s2[i][h], 2);
+    }
+#pragma unroll
+  for (int i = 0; i < 2; ++i)
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      float* pp = part[warp][16 * i + 8 * h + g];
+#pragma unroll
+      for (int j = 0; j < 2; ++j)
+#pragma unroll
+        for (int t = 0; t < 2; ++t) {
+          pp[8 * j + 2 * q + t] = D[i][j][2 * h + t];
+          pp[kHC + 8 * j + 2 * q + t] = D[i][2 + j][2 * h + t] + D[i][4 + j][2 * h + t];
+        }
+      if (q == 0) {
+        pp[2 * kHC] = s1[i][h];
+        pp[2 * kHC + 1] = s2[i][h];
+      }
+    }
+  __syncthreads();
+
+  // finish: 4 threads per token, 4 channels each
+  const int tt = threadIdx.x >> 2, cq = threadIdx.x & 3;
+  const int tok = tok0 + tt;
+  const bool live = tok < N;
+  float xv[kHC], vv[4];
+  if (live) {
+    const float4* xr = reinterpret_cast<const float4*>(x + ((size_t)scene * N + tok) * kHC);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float4 t4 = xr[k];
+      xv[4 * k] = t4.x; xv[4 * k + 1] = t4.y; xv[4 * k + 2] = t4.z; xv[4 * k + 3] = t4.w;
+    }
+    const float *S = stab, *beta = stab + kHC, *Gs = stab + 2 * kHC, *ws = stab + kHeadTab,
+                *G = stab + kHeadTab + kHC;
+    float sum1 = 0.f, sum2 = 0.f, xA = 0.f, xGx = 0.f;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+      sum1 += part[w][tt][2 * kHC];
+      sum2 += part[w][tt][2 * kHC + 1];
+    }
+#pragma unroll
+    for (int a = 0; a < kHC; ++a) {
+      const float A = ((part[0][tt][a] + part[1][tt][a]) + part[2][tt][a]) + part[3][tt][a];
+      xA = fmaf(xv[a], A, xA);
+      sum1 = fmaf(xv[a], ws[a], sum1);
+      float t = 0.f;
+#pragma unroll
+      for (int b2 = 0; b2 < kHC; ++b2) t = fmaf(G[a * kHC + b2], xv[b2], t);
+      xGx = fmaf(xv[a], t, xGx);
+    }
+    const float sq = xGx + 2.f * xA + sum2;
+    const float mu = sum1 / (float)d;
+    const float var = fmaxf(sq / (float)d - mu * mu, 0.f);
+    const float rs = rsqrtf(var + 1e-6f);
+#pragma unroll
+    for (int cc = 0; cc < 4; ++cc) {
+      const int c = 4 * cq + cc;
+      float P = ((part[0][tt][kHC + c] + part[1][tt][kHC + c]) + part[2][tt][kHC + c]) +
+                part[3][tt][kHC + c];
+#pragma unroll
+      for (int a = 0; a < kHC; ++a) P = fmaf(xv[a], Gs[a * kHC + c], P);
+      vv[cc] = fmaf(rs, P - mu * S[c], beta[c]);
+    }
+  }
+  const size_t xi = ((size_t)scene * N + tok) * kHC + 4 * cq;
+  const float4 xo = live ? *reinterpret_cast<const float4*>(x + xi) : make_float4(0.f, 0.f, 0.f, 0.f);
+  __syncwarp();  // every thread of the token has read its x row
+  if (live) {
+    if (vout) {
+      *reinterpret_cast<float4*>(vout + xi) = make_float4(vv[0], vv[1], vv[2], vv[3]);
+    } else {
+      *reinterpret_cast<float4*>(x + xi) =
+          make_float4(fmaf(dsig, vv[0], xo.x), fmaf(dsig, vv[1], xo.y), fmaf(dsig, vv[2], xo.z),
+                      fmaf(dsig, vv[3], xo.w));
+    }
+  }
+}
+
+// ------------------------------------------------------------- compute step
+
+// Compute step of the scenes in `map` (h_L rows packed by slot): the cache
+// row c = h_L - x W_e^T is written, v = head(h_L), x_j <- x, x += dsig v (or
+// v to vout).  x W_e^T is formed in fp32 from W_e^T [C][d] (16 FMAs per
+// element), the head on the tensor cores.
+__global__ void __launch_bounds__(128) head_compute_kernel(
+    const float* __restrict__ hL, float* __restrict__ x, float* __restrict__ xj,
+    __nv_bfloat16* __restrict__ cache, SlotMap map, int N, int d, const float* __restrict__ w_eT,
+    const __nv_bfloat16* __restrict__ wp_k, const float* __restrict__ tab_k, float dsig,
+    float* __restrict__ vout) {
+  pdl_trigger();
+  pdl_wait();
+  __shared__ float part[4][kCmpTok][kHC + 2];  // per warp: P, sum h, sum h^2
+  __shared__ float stab[2 * kHC];              // S', beta
+  const int slot = blockIdx.y, scene = map.scene[slot];
+  const int tok0 = blockIdx.x * kCmpTok;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, q = lane & 3;
+  if (threadIdx.x < 2 * kHC) stab[threadIdx.x] = tab_k[(size_t)scene * kHeadTab + threadIdx.x];
+  const __nv_bfloat16* wk = wp_k + (size_t)scene * 2 * kHC * d;
+  int row[2];
+  bool ok[2];
+  float xv[2][kHC];
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    row[h] = tok0 + 8 * h + g;
+    ok[h] = row[h] < N;
+    const float4* xr = reinterpret_cast<const float4*>(x + ((size_t)scene * N + row[h]) * kHC);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float4 t4 = ok[h] ? xr[k] : make_float4(0.f, 0.f, 0.f, 0.f);
+      xv[h][4 * k] = t4.x; xv[h][4 * k + 1] = t4.y; xv[h][4 * k + 2] = t4.z; xv[h][4 * k + 3] = t4.w;
+    }
+  }
+  float D[4][4];
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+#pragma unroll
+    for (int t = 0; t < 4; ++t) D[j][t] = 0.f;
+  float s1[2] = {0.f, 0.f}, s2[2] = {0.f, 0.f};
+  const int nblk = d >> 5;
+  for (int b = warp; b < nblk; b += 4) {
+    const int e = (b << 5) + (q << 3);
+    float hv[2][8];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const float* hr = hL + ((size_t)slot * N + row[h]) * d + e;
+      const float4 p0 = ok[h] ? ld_stream_f4(hr) : make_float4(0.f, 0.f, 0.f, 0.f);
+      const float4 p1 = ok[h] ? ld_stream_f4(hr + 4) : make_float4(0.f, 0.f, 0.f, 0.f);
+      hv[h][0] = p0.x; hv[h][1] = p0.y; hv[h][2] = p0.z; hv[h][3] = p0.w;
+      hv[h][4] = p1.x; hv[h][5] = p1.y; hv[h][6] = p1.z; hv[h][7] = p1.w;
+    }
+    uint4 bw[4];  // W' hi (channels 0-7, 8-15), W' lo (0-7, 8-15)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) bw[j] = ld_tab16(wk + (size_t)(8 * j + g) * d + e);
+    // the cache row: c = h - x W_e^T
+    float u[2][8];
+#pragma unroll
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+      for (int k = 0; k < 8; ++k) u[h][k] = 0.f;
+#pragma unroll
+    for (int c = 0; c < kHC; ++c) {
+      const float4 w0 = __ldg(reinterpret_cast<const float4*>(w_eT + (size_t)c * d + e));
+      const float4 w1 = __ldg(reinterpret_cast<const float4*>(w_eT + (size_t)c * d + e + 4));
+      const float wv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
+#pragma unroll
+      for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int k = 0; k < 8; ++k) u[h][k] = fmaf(xv[h][c], wv[k], u[h][k]);
+    }
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      if (ok[h]) {
+        uint4 cw;
+        cw.x = pack_bf2(hv[h][0] - u[h][0], hv[h][1] - u[h][1]);
+        cw.y = pack_bf2(hv[h][2] - u[h][2], hv[h][3] - u[h][3]);
+        cw.z = pack_bf2(hv[h][4] - u[h][4], hv[h][5] - u[h][5]);
+        cw.w = pack_bf2(hv[h][6] - u[h][6], hv[h][7] - u[h][7]);
+        st_stream16(cache + ((size_t)scene * N + row[h]) * d + e, cw);
+      }
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        s1[h] += hv[h][k];
+        s2[h] = fmaf(hv[h][k], hv[h][k], s2[h]);
+      }
+    }
+    uint32_t hi[2][4], lo[2][4];
+#pragma unroll
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+      for (int p = 0; p < 4; ++p) split_pair(hv[h][2 * p], hv[h][2 * p + 1], &hi[h][p], &lo[h][p]);
+#pragma unroll
+    for (int s = 0; s < 2; ++s) {
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const uint32_t b0 = s ? bw[j].z : bw[j].x, b1 = s ? bw[j].w : bw[j].y;
+        mma_bf16_16816(D[j], hi[0][2 * s], hi[1][2 * s], hi[0][2 * s + 1], hi[1][2 * s + 1], b0, b1);
+        if (j < 2)
+          mma_bf16_16816(D[j], lo[0][2 * s], lo[1][2 * s], lo[0][2 * s + 1], lo[1][2 * s + 1], b0, b1);
+      }
+    }
+  }
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    s1[h] += __shfl_xor_sync(0xffffffffu, s1[h], 1);
+    s1[h] += __shfl_xor_sync(0xffffffffu, s1[h], 2);
+    s2[h] += __shfl_xor_sync(0xffffffffu, s2[h], 1);
+    s2[h] += __shfl_xor_sync(0xffffffffu, s2[h], 2);
+    float* pp = part[warp][8 * h + g];
+#pragma unroll
+    for (int j = 0; j < 2; ++j)
+#pragma unroll
+      for (int t = 0; t < 2; ++t) pp[8 * j + 2 * q + t] = D[j][2 * h + t] + D[2 + j][2 * h + t];
+    if (q == 0) {
+      pp[kHC] = s1[h];
+      pp[kHC + 1] = s2[h];
+    }
+  }
+  __syncthreads();
+
+  // finish: 4 threads per token (64 threads), 4 channels each
+  if (threadIdx.x < 4 * kCmpTok) {
+    const int tt = threadIdx.x >> 2, cq = threadIdx.x & 3;
+    const int tok = tok0 + tt;
+    if (tok < N) {
+      float sum1 = 0.f, sum2 = 0.f;
+#pragma unroll
+      for (int w = 0; w < 4; ++w) {
+        sum1 += part[w][tt][kHC];
+        sum2 += part[w][tt][kHC + 1];
+      }
+      const float mu = sum1 / (float)d;
+      const float var = fmaxf(sum2 / (float)d - mu * mu, 0.f);
+      const float rs = rsqrtf(var + 1e-6f);
+      float vv[4];
+#pragma unroll
+      for (int cc = 0; cc < 4; ++cc) {
+        const int c = 4 * cq + cc;
+        const float P = ((part[0][tt][c] + part[1][tt][c]) + part[2][tt][c]) + part[3][tt][c];
+        vv[cc] = fmaf(rs, P - mu * stab[c], stab[kHC + c]);
+      }
+      const size_t xi = ((size_t)scene * N + tok) * kHC + 4 * cq;
+      const float4 xo = *reinterpret_cast<const float4*>(x + xi);
+      *reinterpret_cast<float4*>(xj + xi) = xo;
+      if (vout) {
+        *reinterpret_cast<float4*>(vout + xi) = make_float4(vv[0], vv[1], vv[2], vv[3]);
+      } else {
+        *reinterpret_cast<float4*>(x + xi) =
+            make_float4(fmaf(dsig, vv[0], xo.x), fmaf(dsig, vv[1], xo.y), fmaf(dsig, vv[2], xo.z),
+                        fmaf(dsig, vv[3], xo.w));
+      }
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_head_tables(const float* mod, int n_items, int mod_stride, int fin_off, int d,
+                               const float* w_f, const float* b_f, const float* w_eT,
+                               __nv_bfloat16* wp, float* tab, cudaStream_t st) {
+  if (n_items <= 0) return cudaSuccess;
+  head_tables_kernel<<<n_items, 256, 0, st>>>(mod, mod_stride, fin_off, d, w_f, b_f, w_eT, wp, tab);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_head_reuse(float* x, const __nv_bfloat16* cache, const SlotMap& map, int N, int d,
+                              const __nv_bfloat16* w_eT_bf, const __nv_bfloat16* wp_k,
+                              const float* tab_k, const float* wsum, const float* gram, float dsig,
+                              cudaStream_t st, float* vout) {
+  if (map.n <= 0) return cudaSuccess;
+  if (d % 32 != 0) return cudaErrorInvalidValue;
+  const dim3 grid((unsigned)((N + kReuseTok - 1) / kReuseTok), (unsigned)map.n);
+  return launch_pdl(head_reuse_kernel, grid, dim3(128), 0, st, x, cache, map, N, d, w_eT_bf, wp_k,
+                    tab_k, wsum, gram, dsig, vout);
+}
+
+cudaError_t launch_head_compute(const float* hL, float* x, float* xj, __nv_bfloat16* cache,
+                                const SlotMap& map, int N, int d, const float* w_eT,
+                                const __nv_bfloat16* wp_k, const float* tab_k, float dsig,
+                                cudaStream_t st, float* vout) {
+  if (map.n <= 0) return cudaSuccess;
+  if (d % 32 != 0) return cudaErrorInvalidValue;
+  const dim3 grid((unsigned)((N + kCmpTok - 1) / kCmpTok), (unsigned)map.n);
+  return launch_pdl(head_compute_kernel, grid, dim3(128), 0, st, hL, x, xj, cache, map, N, d, w_eT,
+                    wp_k, tab_k, dsig, vout);
+}
+
+int head_table_floats() { return kHeadTab; }
+
+}  // namespace dc

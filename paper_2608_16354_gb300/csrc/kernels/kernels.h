@@ -19,6 +19,15 @@ cudaError_t launch_temb_features(const double* sigmas, int K, float* out, cudaSt
 template <typename TW>
 cudaError_t launch_rows_linear(const float* X, int R, int I, const TW* W, const float* b, int O,
                                float* Y, int in_silu, cudaStream_t st);
+// adaLN table on the tensor cores (bf16 models, cond_tc.cu): xs = silu(temb[k]
+// + traj[s]) split into bf16 hi / lo rows per group of cond_tc_group_rows()
+// rows ([groups][2 x 64][d]), then Y[r][o] = xs_r . W[o] + b[o] for R = K B
+// rows against W [O][d] bf16 (tmW: box 64 x 128, tmX over xs: box 64 x 128)
+int cond_tc_group_rows();
+cudaError_t launch_cond_split(const float* temb, const float* traj, int K, int B, int d,
+                              __nv_bfloat16* xs, cudaStream_t st);
+cudaError_t launch_cond_gemm_tc(const CUtensorMap& tmW, const CUtensorMap& tmX, int R, int O, int d,
+                                const float* bias, float* Y, int* err, int n_sms, cudaStream_t st);
 // c[k][s] = temb[k] + traj[s]; out = silu(c)   ([K][B][d])
 cudaError_t launch_cond_combine(const float* temb, const float* traj, int K, int B, int d,
                                 float* silu_c, cudaStream_t st);
@@ -58,19 +67,44 @@ cudaError_t launch_attention_f32(const float* qkv, int slots, int heads, int N, 
 bool attention_tc_supported(int dh);
 cudaError_t launch_attention_tc(const CUtensorMap& tm, int nslots, int heads, int N, int dh,
                                 __nv_bfloat16* o, int* err, cudaStream_t st);
-// compute-step interface + Euler: v = head(h_L); x_j <- x; x += dsig v; r <- h_L - u
+// The cache row of a scene is c = h_L - x W_e^T of its last full evaluation
+// (the block-stack residual r = h_L - u plus b_e + pos), so a reuse step
+// forms u_k + r_j = x_k W_e^T + c_j.
+// SIMT interface (fp32 models and C = 4): compute step v = head(h_L),
+// x_j <- x, x += dsig v, c <- h_L - x W_e^T; reuse step h = x W_e^T + c_j,
+// v = head(h), x += dsig v  (w_eT = W_e^T [C][d] fp32)
 template <typename T>
-cudaError_t launch_final_compute(const float* hL, const float* u, float* x, float* xj, T* r,
+cudaError_t launch_final_compute(const float* hL, const float* w_eT, float* x, float* xj, T* r,
                                  const SlotMap& map, int N, int C, int d, const float* mod,
                                  int mod_stride, int fin_off, const float* w_f, const float* b_f,
                                  float dsig, cudaStream_t st, float* vout = nullptr);
-// reuse step: u = embed(x); h = u + r_j; v = head(h); x += dsig v  (w_eT = W_e^T [C][d])
 template <typename T>
-cudaError_t launch_final_reuse(float* x, const T* r, const float* w_eT, const float* b_e,
-                               const T* pos, const SlotMap& map, int N, int C, int d,
-                               const float* mod, int mod_stride, int fin_off, const float* w_f,
-                               const float* b_f, float dsig, cudaStream_t st,
+cudaError_t launch_final_reuse(float* x, const T* r, const float* w_eT, const SlotMap& map, int N,
+                               int C, int d, const float* mod, int mod_stride, int fin_off,
+                               const float* w_f, const float* b_f, float dsig, cudaStream_t st,
                                float* vout = nullptr);
+// r_j = c_j - b_e - pos (inspection of a cache row), out [N][d]
+template <typename T>
+cudaError_t launch_cache_to_residual(const T* c, const float* b_e, const T* pos, int N, int d, T* out,
+                                     cudaStream_t st);
+// Tensor-core interface of bf16 models with C = 16 (interface_tc.cu).  Per
+// (step, scene) item of the call's modulation table: W' = (1 + scale) W_f as
+// bf16 hi + lo rows [32][d], and S', beta, G_s (head_table_floats() fp32).
+int head_table_floats();
+cudaError_t launch_head_tables(const float* mod, int n_items, int mod_stride, int fin_off, int d,
+                               const float* w_f, const float* b_f, const float* w_eT,
+                               __nv_bfloat16* wp, float* tab, cudaStream_t st);
+// reuse step (wp_k, tab_k: the step's tables, indexed by scene; w_eT_bf:
+// W_e^T [16][d] bf16; wsum: row sums of W_e^T; gram: W_e^T W_e [16][16])
+cudaError_t launch_head_reuse(float* x, const __nv_bfloat16* cache, const SlotMap& map, int N, int d,
+                              const __nv_bfloat16* w_eT_bf, const __nv_bfloat16* wp_k,
+                              const float* tab_k, const float* wsum, const float* gram, float dsig,
+                              cudaStream_t st, float* vout = nullptr);
+// compute step: writes the cache rows, x_j <- x, x += dsig v
+cudaError_t launch_head_compute(const float* hL, float* x, float* xj, __nv_bfloat16* cache,
+                                const SlotMap& map, int N, int d, const float* w_eT,
+                                const __nv_bfloat16* wp_k, const float* tab_k, float dsig,
+                                cudaStream_t st, float* vout = nullptr);
 // vout != NULL (both): write the velocity v[scene][tok][c] instead of the
 // Euler update (x is left as it is; the compute step still sets x_j = x).
 // guidance: x_s += dsig (v_u + g (v_c - v_u)), v_c = v[s], v_u = v[B + s]

@@ -60,6 +60,12 @@ struct dc_model {
   float* drift_host = nullptr;  // pinned
   // derived tables: W_e^T [C][d] and the Gram tables of the drift sums
   float *w_eT = nullptr, *gram = nullptr, *gp = nullptr, *gs = nullptr;
+  // tensor-core interface (bf16 models, C = 16): W_e^T in bf16, its row
+  // sums, and per (step, scene) head tables of the call
+  bool head_tc = false;
+  __nv_bfloat16 *w_eT_bf = nullptr, *head_wp = nullptr, *cond_xs = nullptr;
+  CUtensorMap tm_ada, tm_xs;  // adaLN weight and the split activations (bf16 models)
+  float *wsum = nullptr, *head_tab = nullptr;
   CUtensorMap tm_a, tm_oact, tm_m, tm_qkv, tm_u32, tm_h32;
   long long launches = 0;
   // per-kernel profiling (dc_profile)
@@ -89,6 +95,12 @@ namespace {
   } while (0)
 
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+// row groups of the split activations of the tensor-core adaLN product
+size_t cond_groups(size_t rows) {
+  const size_t g = (size_t)dc::cond_tc_group_rows();
+  return (rows + g - 1) / g;
+}
 
 cudaEvent_t take_event(dc_model* m) {
   if (!m->ev_pool.empty()) {
@@ -277,9 +289,21 @@ dc_status enqueue_conditioning(dc_model* m, int B, int K, cudaStream_t st) {
   DC_CK(dc::launch_pose_features(m->poses_d, B, m->P, m->pose_f, st));
   DC_CK(dc::launch_rows_linear<float>(m->pose_f, B, 3 * m->P, m->w_traj, m->b_traj, d, m->traj, 0,
                                       st));
-  DC_CK(dc::launch_cond_combine(m->temb, m->traj, K, B, d, m->silu_c, st));
-  DC_CK(dc::launch_rows_linear<T>(m->silu_c, K * B, d, static_cast<const T*>(m->w_ada), m->b_ada,
-                                  m->mod_stride, m->mod, 0, st));
+  if (m->bf16) {
+    // the adaLN weight streamed once through the tensor cores
+    DC_CK(dc::launch_cond_split(m->temb, m->traj, K, B, d, m->cond_xs, st));
+    DC_CK(dc::launch_cond_gemm_tc(m->tm_ada, m->tm_xs, K * B, m->mod_stride, d, m->b_ada, m->mod,
+                                  m->err_d, m->n_sms, st));
+  } else {
+    DC_CK(dc::launch_cond_combine(m->temb, m->traj, K, B, d, m->silu_c, st));
+    DC_CK(dc::launch_rows_linear<T>(m->silu_c, K * B, d, static_cast<const T*>(m->w_ada), m->b_ada,
+                                    m->mod_stride, m->mod, 0, st));
+  }
+  if (m->head_tc) {
+    DC_CK(dc::launch_head_tables(m->mod, K * B, m->mod_stride, 6 * m->L * d, d, m->w_f, m->b_f,
+                                 m->w_eT, m->head_wp, m->head_tab, st));
+    m->launches += 1;
+  }
   // algorithmic bytes: the adaLN weight table read once + the table written
   DC_TRY(prof_stop(m, DC_PROF_CONDITION, st, ev, 2.0 * K * B * d * m->mod_stride,
                    (double)m->mod_stride * d * m->elt + 4.0 * K * B * m->mod_stride));
@@ -288,9 +312,17 @@ dc_status enqueue_conditioning(dc_model* m, int B, int K, cudaStream_t st) {
 }
 
 // One full backbone pass + interface + Euler for the scenes in `map`.
+// This step's head tables (tensor-core interface): items (k - 1) * Bi + scene.
+const __nv_bfloat16* head_wp_k(const dc_model* m, int k, int Bi) {
+  return m->head_wp + (size_t)(k - 1) * Bi * 32 * m->d;
+}
+const float* head_tab_k(const dc_model* m, int k, int Bi) {
+  return m->head_tab + (size_t)(k - 1) * Bi * dc::head_table_floats();
+}
+
 template <typename T>
 dc_status enqueue_compute(dc_model* m, float* lat, const float* mod_k, const SlotMap& map,
-                          float dsig, cudaStream_t st, float* vout = nullptr) {
+                          float dsig, int k, int Bi, cudaStream_t st, float* vout = nullptr) {
   const int N = m->N, d = m->d, nc = map.n, M = nc * N;
   if (nc == 0) return DC_OK;
   T* a = static_cast<T*>(m->a);
@@ -387,26 +419,40 @@ dc_status enqueue_compute(dc_model* m, float* lat, const float* mod_k, const Slo
     }
     m->launches += 7;
   }
-  DC_LAUNCH(DC_PROF_FINAL, 2.0 * M * d * m->C, 8.0 * Md + E * Md + 12.0 * M * m->C,
-            dc::launch_final_compute<T>(m->h, m->u, lat, m->xj, static_cast<T*>(m->r), map, N,
-                                        m->C, d, mod_k, m->mod_stride, 6 * m->L * d, m->w_f,
-                                        m->b_f, dsig, st, vout));
+  // algorithmic bytes: h_L read, the cache row written, x read, x and x_j written
+  if (m->head_tc && sizeof(T) == 2) {
+    DC_LAUNCH(DC_PROF_FINAL, 4.0 * M * d * m->C, 4.0 * Md + E * Md + 12.0 * M * m->C,
+              dc::launch_head_compute(m->h, lat, m->xj, reinterpret_cast<__nv_bfloat16*>(m->r), map,
+                                      N, d, m->w_eT, head_wp_k(m, k, Bi), head_tab_k(m, k, Bi), dsig,
+                                      st, vout));
+  } else {
+    DC_LAUNCH(DC_PROF_FINAL, 4.0 * M * d * m->C, 4.0 * Md + E * Md + 12.0 * M * m->C,
+              dc::launch_final_compute<T>(m->h, m->w_eT, lat, m->xj, static_cast<T*>(m->r), map, N,
+                                          m->C, d, mod_k, m->mod_stride, 6 * m->L * d, m->w_f,
+                                          m->b_f, dsig, st, vout));
+  }
   m->launches += 1;
   return DC_OK;
 }
 
 template <typename T>
 dc_status enqueue_reuse(dc_model* m, float* lat, const float* mod_k, const SlotMap& map, float dsig,
-                        cudaStream_t st, float* vout = nullptr) {
+                        int k, int Bi, cudaStream_t st, float* vout = nullptr) {
   if (map.n == 0) return DC_OK;
   const double M = (double)map.n * m->N;
-  // algorithmic bytes of a reuse scene-step: r_j (N d elements) + x_k read,
-  // x_{k+1} written and x_j read by the drift check (3 N C fp32)
-  DC_LAUNCH(DC_PROF_REUSE, 4.0 * M * m->d * m->C, M * ((double)m->d * m->elt + 12.0 * m->C),
-            dc::launch_final_reuse<T>(lat, static_cast<const T*>(m->r), m->w_eT, m->b_e,
-                                      static_cast<const T*>(m->pos), map, m->N, m->C, m->d, mod_k,
-                                      m->mod_stride, 6 * m->L * m->d, m->w_f, m->b_f, dsig, st,
-                                      vout));
+  // algorithmic bytes of a reuse scene-step: the cached row (N d elements) +
+  // x_k read, x_{k+1} written and x_j read by the drift check (3 N C fp32)
+  if (m->head_tc && sizeof(T) == 2) {
+    DC_LAUNCH(DC_PROF_REUSE, 2.0 * M * m->d * 3 * m->C, M * ((double)m->d * m->elt + 12.0 * m->C),
+              dc::launch_head_reuse(lat, reinterpret_cast<const __nv_bfloat16*>(m->r), map, m->N,
+                                    m->d, m->w_eT_bf, head_wp_k(m, k, Bi), head_tab_k(m, k, Bi),
+                                    m->wsum, m->gram, dsig, st, vout));
+  } else {
+    DC_LAUNCH(DC_PROF_REUSE, 4.0 * M * m->d * m->C, M * ((double)m->d * m->elt + 12.0 * m->C),
+              dc::launch_final_reuse<T>(lat, static_cast<const T*>(m->r), m->w_eT, map, m->N, m->C,
+                                        m->d, mod_k, m->mod_stride, 6 * m->L * m->d, m->w_f, m->b_f,
+                                        dsig, st, vout));
+  }
   m->launches += 1;
   return DC_OK;
 }
@@ -634,14 +680,14 @@ dc_status run_sampler(dc_model* m, float* lat, const dc_cond* cond, const dc_sch
       const size_t xb = (size_t)B * N * C * 4;
       DC_CK(cudaMemcpyAsync(m->cfg_x, lat, xb, cudaMemcpyDeviceToDevice, st));
       DC_CK(cudaMemcpyAsync(m->cfg_x + (size_t)B * N * C, lat, xb, cudaMemcpyDeviceToDevice, st));
-      DC_TRY(enqueue_compute<T>(m, m->cfg_x, mod_k, cm, dsig, st, m->cfg_v));
-      DC_TRY(enqueue_reuse<T>(m, m->cfg_x, mod_k, rm, dsig, st, m->cfg_v));
+      DC_TRY(enqueue_compute<T>(m, m->cfg_x, mod_k, cm, dsig, k, Bi, st, m->cfg_v));
+      DC_TRY(enqueue_reuse<T>(m, m->cfg_x, mod_k, rm, dsig, k, Bi, st, m->cfg_v));
       DC_CK(dc::launch_cfg_combine(lat, m->cfg_v, B, (size_t)N * C, (float)sc->cfg_scale, dsig,
                                    st));
       m->launches += 1;
     } else {
-      DC_TRY(enqueue_compute<T>(m, lat, mod_k, cm, dsig, st));
-      DC_TRY(enqueue_reuse<T>(m, lat, mod_k, rm, dsig, st));
+      DC_TRY(enqueue_compute<T>(m, lat, mod_k, cm, dsig, k, Bi, st));
+      DC_TRY(enqueue_reuse<T>(m, lat, mod_k, rm, dsig, k, Bi, st));
     }
     if (r_trace) {
       const size_t rb = (size_t)N * m->d * m->elt;
@@ -810,9 +856,10 @@ dc_status interface_f32(dc_model* m, ResponseWork<T>& w, const float* x, const T
                         const float* mod, float* v, cudaStream_t st) {
   const size_t Nd = (size_t)w.N * w.d;
   const float* fsh = mod + (size_t)6 * w.L * w.d;
+  // the cache row c = r + b_e + pos: u + r = x W_e^T + c
   DC_LAUNCH(DC_PROF_JVP_OTHER, 0.0, 0.0,
-              dc::launch_embed_f32<T>(x, m->w_eT, m->b_e, static_cast<const T*>(m->pos), w.N, w.N, w.C,
-                                w.d, w.hcur, st));
+              dc::launch_embed_f32<T>(x, m->w_eT, nullptr, static_cast<const T*>(nullptr), w.N, w.N,
+                                      w.C, w.d, w.hcur, st));
   DC_LAUNCH(DC_PROF_JVP_OTHER, 0.0, 0.0,
               dc::launch_add_cache<T>(w.hcur, r, w.hcur, Nd, st));
   DC_LAUNCH(DC_PROF_JVP_OTHER, 0.0, 0.0,
@@ -1118,6 +1165,7 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
   }
 
   // ---- workspace
+  m->head_tc = m->bf16 && m->C == 16;
   const size_t B = m->Bmax, N = m->N, d = m->d, K = m->Kmax;
   struct Buf { void** p; size_t bytes; };
   std::vector<Buf> bufs = {
@@ -1136,7 +1184,11 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
       {(void**)&m->poses_d, B * m->P * 3 * 8}, {(void**)&m->sig_d, (K + 1) * 8},
       {(void**)&m->err_d, 256}, {(void**)&m->w_eT, (size_t)m->C * d * 4},
       {(void**)&m->gram, (size_t)m->C * m->C * 4}, {(void**)&m->gp, N * m->C * 4},
-      {(void**)&m->gs, N * 4}};
+      {(void**)&m->gs, N * 4}, {(void**)&m->w_eT_bf, (size_t)m->C * d * 2},
+      {(void**)&m->wsum, (size_t)m->C * 4},
+      {(void**)&m->head_wp, m->head_tc ? K * B * 32 * d * 2 : 0},
+      {(void**)&m->head_tab, m->head_tc ? K * B * (size_t)dc::head_table_floats() * 4 : 0},
+      {(void**)&m->cond_xs, m->bf16 ? cond_groups(K * B) * 2 * dc::cond_tc_group_rows() * d * 2 : 0}};
   size_t wsb = 0;
   for (auto& b : bufs) wsb += align256(b.bytes);
   if (cudaMalloc(&m->ws, wsb) != cudaSuccess) {
@@ -1156,9 +1208,18 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
     const float* we = host_weights;                 // w_embed [d][C]
     const float* be = host_weights + (size_t)D * C;  // b_embed [d]
     const float* ps = be + D;                        // pos [N][d]
-    std::vector<float> weT((size_t)C * D), gram((size_t)C * C), gp(N * C), gs(N);
+    std::vector<float> weT((size_t)C * D), gram((size_t)C * C), gp(N * C), gs(N), wsum(C);
+    std::vector<uint16_t> weT_bf((size_t)C * D);
     for (int e = 0; e < D; ++e)
-      for (int c = 0; c < C; ++c) weT[(size_t)c * D + e] = we[(size_t)e * C + c];
+      for (int c = 0; c < C; ++c) {
+        weT[(size_t)c * D + e] = we[(size_t)e * C + c];
+        weT_bf[(size_t)c * D + e] = f2bf_host(we[(size_t)e * C + c]);
+      }
+    for (int c = 0; c < C; ++c) {
+      double acc = 0.0;
+      for (int e = 0; e < D; ++e) acc += (double)we[(size_t)e * C + c];
+      wsum[c] = (float)acc;
+    }
     for (int a = 0; a < C; ++a)
       for (int b = 0; b < C; ++b) {
         double acc = 0.0;
@@ -1187,7 +1248,9 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
     if (cudaMemcpy(m->w_eT, weT.data(), weT.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
         cudaMemcpy(m->gram, gram.data(), gram.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
         cudaMemcpy(m->gp, gp.data(), gp.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
-        cudaMemcpy(m->gs, gs.data(), gs.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess) {
+        cudaMemcpy(m->gs, gs.data(), gs.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaMemcpy(m->w_eT_bf, weT_bf.data(), weT_bf.size() * 2, cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaMemcpy(m->wsum, wsum.data(), wsum.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess) {
       dc::set_error("upload of the derived tables failed");
       return fail(DC_ERR_CUDA);
     }
@@ -1204,6 +1267,10 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
     if ((s = make_map(&m->tm_m, m->m, m->md, B * N, bm)) != DC_OK) return fail(s);
     if ((s = make_map(&m->tm_u32, m->u, d, B * N, bm, true)) != DC_OK) return fail(s);
     if ((s = make_map(&m->tm_h32, m->h, d, B * N, bm, true)) != DC_OK) return fail(s);
+    if ((s = make_map(&m->tm_ada, m->w_ada, d, m->mod_stride, 128)) != DC_OK) return fail(s);
+    if ((s = make_map(&m->tm_xs, m->cond_xs, d, cond_groups(K * B) * 2 * dc::cond_tc_group_rows(),
+                      128)) != DC_OK)
+      return fail(s);
     if (dc::attention_tc_supported(m->dh) &&
         (s = make_map(&m->tm_qkv, m->qkv, m->dhp, 3 * B * m->heads * N, 128)) != DC_OK)
       return fail(s);
@@ -1452,8 +1519,18 @@ dc_status dc_cache_copy(dc_model* m, int scene, void* dst, size_t bytes, void* s
     return DC_ERR_INVALID_ARG;
   }
   DC_CK(cudaSetDevice(m->device));
-  const uint8_t* src = static_cast<const uint8_t*>(m->r) + (size_t)scene * bytes;
-  DC_CK(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToDevice, static_cast<cudaStream_t>(stream)));
+  // the cache row is c = r + b_e + pos: return r
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t off = (size_t)scene * m->N * m->d;
+  if (m->bf16) {
+    DC_CK(dc::launch_cache_to_residual(static_cast<const __nv_bfloat16*>(m->r) + off, m->b_e,
+                                       static_cast<const __nv_bfloat16*>(m->pos), m->N, m->d,
+                                       static_cast<__nv_bfloat16*>(dst), st));
+  } else {
+    DC_CK(dc::launch_cache_to_residual(static_cast<const float*>(m->r) + off, m->b_e,
+                                       static_cast<const float*>(m->pos), m->N, m->d,
+                                       static_cast<float*>(dst), st));
+  }
   return DC_OK;
 }
 

@@ -12,7 +12,7 @@
 namespace dc {
 
 constexpr char kSnapMagic[8] = {'D', 'C', 'S', 'N', 'A', 'P', '0', '1'};
-constexpr uint32_t kSnapVersion = 1;
+constexpr uint32_t kSnapVersion = 2;  // 2: the cache section holds c = r + b_e + pos
 
 struct SnapHeader {
   char magic[8];

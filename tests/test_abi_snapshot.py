@@ -35,7 +35,7 @@ def _documented_size(B, K, cfg, N, d, C, elt):
 
 
 def _header(B, K, cfg, k_done, dtype, N, d, C, total, digest=0x0123456789ABCDEF, calls=7,
-            magic=b"DCSNAP01", version=1):
+            magic=b"DCSNAP01", version=2):
     elt = 2 if dtype == DTYPE_BF16 else 4
     h = magic + struct.pack("<I8iIQQq", version, B, K, cfg, k_done, dtype, N, d, C, elt, digest,
                             total, calls)
@@ -73,7 +73,7 @@ def test_snapshot_info_reads_documented_header(dc):
 
 
 @pytest.mark.parametrize("bad", [
-    dict(magic=b"DCSNAP02"), dict(version=2), dict(k_done=0), dict(k_done=7), dict(cfg=2),
+    dict(magic=b"DCSNAP02"), dict(version=1), dict(k_done=0), dict(k_done=7), dict(cfg=2),
     dict(B=0), dict(dtype=3), dict(calls=-1)])
 def test_snapshot_info_rejects_malformed_headers(dc, bad):
     with pytest.raises(dc.DCError):
