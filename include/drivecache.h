@@ -418,6 +418,19 @@ dc_status dc_drift_sums(dc_model* m, const float* x_now, const float* x_ref, int
 dc_status dc_drift_sums_noalloc(dc_model* m, const float* x_now, const float* x_ref, int B,
                                 float* out, void* stream);
 
+/* Test hook for the failure detection of the device kernels.  Every wait of
+ * the tensor-core kernels (TMA copies landing, MMAs completing, the stages of
+ * the warp-specialised pipelines handing work to each other) gives up after
+ * a limit, records a code in the model's error word, lets the rest of the
+ * launch drain and return, and makes later tensor-core launches of the model
+ * skip their work until the host has read the word: the call then returns
+ * DC_ERR_DEVICE_TIMEOUT and clears the word, and the next call runs normally.
+ * The limit is 2 s; this call sets it to `ns` nanoseconds for the waits on
+ * work in progress of the model's later launches (0 restores 2 s), so that a
+ * test can make them run out.  Waits that drain copies or MMAs a CTA has
+ * already issued keep the 2 s limit.  Synchronises the device. */
+dc_status dc_set_wait_limit(dc_model* m, unsigned int ns);
+
 /* Write the cached backbone output r_j (Eq. 1: r = h_L - u of the scene's
  * last full evaluation) of `scene` (0 <= scene < max_batch) into DEVICE
  * memory dst, [N][d] elements of the model dtype (fp32 or bf16); `bytes`

@@ -137,6 +137,7 @@ def lib():
         "dc_attention": (st, [C.c_int, C.c_void_p, C.c_int, C.c_int, C.c_int, C.c_int, C.c_void_p,
                               C.c_void_p]),
         "dc_profile": (st, [C.c_void_p, C.c_int]),
+        "dc_set_wait_limit": (st, [C.c_void_p, C.c_uint]),
         "dc_profile_read": (st, [C.c_void_p, P(C.c_double), P(C.c_longlong), P(C.c_double),
                                  P(C.c_double)]),
         "dc_status_string": (C.c_char_p, [C.c_int]),
@@ -483,6 +484,12 @@ def attention(qkv, slots, heads, n_tokens, head_dim, out, stream=None):
 PROF_NAMES = ["condition", "embed", "ln_mod", "gemm_qkv", "attention", "gemm_out", "gemm_mlp1",
               "gemm_mlp2", "final_compute", "reuse", "drift", "jvp_attention", "jvp_gemm",
               "jvp_other"]
+
+
+def set_wait_limit(model: Model, ns):
+    """dc_set_wait_limit: the limit (ns) of the device waits on work in
+    progress; 0 restores the default."""
+    _check(lib().dc_set_wait_limit(model.h, int(ns)))
 
 
 def profile(model: Model, enable):

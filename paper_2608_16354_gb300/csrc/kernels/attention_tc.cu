@@ -46,9 +46,14 @@ constexpr float kRefSlack = 8.0f;  // move the reference max only beyond this (l
 template <int DHP, int NQ>
 struct AttCfg {
   static constexpr int kAtoms = DHP / 64;             // 64-element swizzle atoms along dh
+  // Two 128-column query tiles (dh in the 128-column layout): O 2 x 128 and
+  // S 2 x 128 fill TMEM, so P_t is written over the first 64 columns of S_t
+  // once S_t is in registers, and S_{t,j+1} is issued after PV_{t,j} (the
+  // MMAs of one thread run in issue order).
+  static constexpr bool kAliasP = DHP == 128 && NQ == 2;
   // ring depths (key, value): deeper rings measured no faster at dh 64
-  static constexpr int kKStages = 3;
-  static constexpr int kVStages = 3;
+  static constexpr int kKStages = kAliasP ? 2 : 3;
+  static constexpr int kVStages = kAliasP ? 2 : 3;
   static constexpr int kTileBytes = kAtoms * 16384;   // 128 rows x DHP bf16
   static constexpr int kOffQ = 0;                              // NQ tiles
   static constexpr int kOffK = kOffQ + NQ * kTileBytes;        // kKStages stages
@@ -65,9 +70,11 @@ struct AttCfg {
   // TMEM columns
   static constexpr int kColO = 0;                     // O_t at t * DHP
   static constexpr int kColS = NQ * DHP;              // S_t at kColS + t * 128
-  static constexpr int kColP = kColS + NQ * 128;      // P_t at kColP + t * 64
+  static constexpr int kColP = kAliasP ? kColS : kColS + NQ * 128;  // P_t at kColP + t * kPStride
+  static constexpr int kPStride = kAliasP ? 128 : 64;
   static constexpr int kTmemCols = 512;
-  static_assert(kColP + NQ * 64 <= kTmemCols, "TMEM budget");
+  static_assert(kColS + NQ * 128 <= kTmemCols && kColP + (NQ - 1) * kPStride + 64 <= kTmemCols,
+                "TMEM budget");
   static_assert(kSmem <= 232448, "shared memory budget");
 };
 
@@ -353,11 +360,11 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
         }
       }
       // every copy in flight lands before the CTA can exit
-      mbar_wait_warp(&bar->q_full, 0, err, kDevTimeoutTma);
+      mbar_wait_warp(&bar->q_full, 0, err, kDevTimeoutTma, true);
       for (int b = 0; b < kKStages; ++b)
-        if (last_k[b] >= 0) mbar_wait_warp(&bar->k_full[b], (uint32_t)last_k[b], err, kDevTimeoutTma);
+        if (last_k[b] >= 0) mbar_wait_warp(&bar->k_full[b], (uint32_t)last_k[b], err, kDevTimeoutTma, true);
       for (int b = 0; b < kVStages; ++b)
-        if (last_v[b] >= 0) mbar_wait_warp(&bar->v_full[b], (uint32_t)last_v[b], err, kDevTimeoutTma);
+        if (last_v[b] >= 0) mbar_wait_warp(&bar->v_full[b], (uint32_t)last_v[b], err, kDevTimeoutTma, true);
     } else if (warp >= 1 && warp <= NQ) {
       // ------------------------------------------------------------ MMA
       // One warp per query tile t, fixed order with blocking waits.  Round j
@@ -375,53 +382,64 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
       const uint64_t dQ = sw128_kmajor_desc(smem_u32(smem + Cfg::kOffQ + t * Cfg::kTileBytes));
       const uint64_t dK = sw128_kmajor_desc(smem_u32(smem + Cfg::kOffK));
       const uint64_t dV = sw128_mnmajor_desc(smem_u32(smem + Cfg::kOffV));
-      for (int j = 0; j <= n_kv && ok; ++j) {
-        if (j < n_kv) {
-          const int kb = j % kKStages;
-          ok = mbar_wait_warp(&bar->k_full[kb], (uint32_t)(j / kKStages) & 1, err, kDevTimeoutMma) &&
-               mbar_wait_warp(&bar->s_free[t], ((uint32_t)j & 1) ^ 1, err, kDevTimeoutMma);
-          if (!ok) break;
-          tc_fence_after();
-          if (elect_one()) {
+      // S_{t,j} = Q_t K_j^T: needs K_j, and S_t no longer needed (read by the
+      // softmax; with P aliased onto S_t, PV_{t,j-1} issued before it)
+      auto issue_s = [&](int j) -> bool {
+        const int kb = j % kKStages;
+        bool good = mbar_wait_warp(&bar->k_full[kb], (uint32_t)(j / kKStages) & 1, err, kDevTimeoutMma);
+        if (!Cfg::kAliasP)
+          good = good && mbar_wait_warp(&bar->s_free[t], ((uint32_t)j & 1) ^ 1, err, kDevTimeoutMma);
+        if (!good) return false;
+        tc_fence_after();
+        if (elect_one()) {
 #pragma unroll
-            for (int kk = 0; kk < kKSteps; ++kk) {
-              const uint32_t off = (kk >> 2) * 16384 + (kk & 3) * 32;
-              tc_mma_f16(tmem + Cfg::kColS + t * 128, dQ + (off >> 4),
-                         dK + ((uint32_t)(kb * Cfg::kTileBytes + off) >> 4), kIdS,
-                         kk > 0 ? 1u : 0u);
-            }
-            tc_commit(&bar->s_full[t]);
-            tc_commit(&bar->k_empty[kb]);
+          for (int kk = 0; kk < kKSteps; ++kk) {
+            const uint32_t off = (kk >> 2) * 16384 + (kk & 3) * 32;
+            tc_mma_f16(tmem + Cfg::kColS + t * 128, dQ + (off >> 4),
+                       dK + ((uint32_t)(kb * Cfg::kTileBytes + off) >> 4), kIdS, kk > 0 ? 1u : 0u);
           }
-          __syncwarp();
+          tc_commit(&bar->s_full[t]);
+          tc_commit(&bar->k_empty[kb]);
         }
-        if (j >= 1) {
-          const int jp = j - 1;
-          const int vb = jp % kVStages;
-          ok = mbar_wait_warp(&bar->v_full[vb], (uint32_t)(jp / kVStages) & 1, err, kDevTimeoutMma) &&
-               mbar_wait_warp(&bar->p_full[t], (uint32_t)jp & 1, err, kDevTimeoutMma);
-          if (!ok) break;
-          tc_fence_after();
-          if (elect_one()) {
+        __syncwarp();
+        return true;
+      };
+      // O_t += P_{t,jp} V_jp: needs V_jp and P_{t,jp} in TMEM
+      auto issue_pv = [&](int jp) -> bool {
+        const int vb = jp % kVStages;
+        const bool good =
+            mbar_wait_warp(&bar->v_full[vb], (uint32_t)(jp / kVStages) & 1, err, kDevTimeoutMma) &&
+            mbar_wait_warp(&bar->p_full[t], (uint32_t)jp & 1, err, kDevTimeoutMma);
+        if (!good) return false;
+        tc_fence_after();
+        if (elect_one()) {
 #pragma unroll
-            for (int kk = 0; kk < 8; ++kk) {
+          for (int kk = 0; kk < 8; ++kk) {
 #pragma unroll
-              for (int a = 0; a < Cfg::kAtoms; ++a)
-                tc_mma_f16_ta(tmem + Cfg::kColO + t * DHP + a * 64,
-                              tmem + Cfg::kColP + t * 64 + kk * 8,
-                              dV + ((uint32_t)(vb * Cfg::kTileBytes + a * 16384 + kk * 2048) >> 4),
-                              a == Cfg::kAtoms - 1 ? kIdPVLast : kIdPV,
-                              (jp > 0 || kk > 0) ? 1u : 0u);
-            }
-            tc_commit(&bar->p_free[t]);
-            tc_commit(&bar->v_empty[vb]);
+            for (int a = 0; a < Cfg::kAtoms; ++a)
+              tc_mma_f16_ta(tmem + Cfg::kColO + t * DHP + a * 64,
+                            tmem + Cfg::kColP + t * Cfg::kPStride + kk * 8,
+                            dV + ((uint32_t)(vb * Cfg::kTileBytes + a * 16384 + kk * 2048) >> 4),
+                            a == Cfg::kAtoms - 1 ? kIdPVLast : kIdPV, (jp > 0 || kk > 0) ? 1u : 0u);
           }
-          __syncwarp();
+          tc_commit(&bar->p_free[t]);
+          tc_commit(&bar->v_empty[vb]);
+        }
+        __syncwarp();
+        return true;
+      };
+      for (int j = 0; j <= n_kv && ok; ++j) {
+        if (Cfg::kAliasP) {
+          if (j >= 1) ok = issue_pv(j - 1);
+          if (ok && j < n_kv) ok = issue_s(j);
+        } else {
+          if (j < n_kv) ok = issue_s(j);
+          if (ok && j >= 1) ok = issue_pv(j - 1);
         }
       }
       if (elect_one()) tc_commit(&bar->drain);
       __syncwarp();
-      mbar_wait_warp(&bar->drain, 0, err, kDevTimeoutMma);
+      mbar_wait_warp(&bar->drain, 0, err, kDevTimeoutMma, true);
     }
     tc_fence_before();
     named_bar(1, Cfg::kThreads);
@@ -439,7 +457,7 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     const uint32_t tO = tmem + Cfg::kColO + t * DHP + lane_off;
     const uint32_t tS = tmem + Cfg::kColS + t * 128 + lane_off;
-    const uint32_t tP = tmem + Cfg::kColP + t * 64 + lane_off;
+    const uint32_t tP = tmem + Cfg::kColP + t * Cfg::kPStride + lane_off;
     float ref = -INFINITY, l = 0.f;
     bool ok = true;
     // (Making the two query tiles take turns on MUFU through named barriers
@@ -460,10 +478,13 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
         tmem_ld_wait_regs(s1);
         tmem_ld_wait_regs(s2);
         tmem_ld_wait_regs(s3);
-        // S is in registers: hand S_t back to the MMA warp
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&bar->s_free[t]);
+        // S is in registers: hand S_t back to the MMA warp (with P aliased
+        // onto S_t, the hand-back is p_full below)
+        if (!Cfg::kAliasP) {
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&bar->s_free[t]);
+        }
         const int valid = min(128, N - j * 128);
         float2 rs2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
         if (j > 0 && valid == 128) {
@@ -611,8 +632,8 @@ cudaError_t launch_attention_tc(const CUtensorMap& tm, int nslots, int heads, in
                                 __nv_bfloat16* o, int* err, cudaStream_t st) {
   if (nslots <= 0) return cudaSuccess;
   if (dh == 64) return launch_tc<64, 2>(tm, nslots, heads, N, o, err, st);
-  if (dh == 128) return launch_tc<128, 1>(tm, nslots, heads, N, o, err, st);
-  if (dh == 72) return launch_tc<128, 1, 72>(tm, nslots, heads, N, o, err, st);
+  if (dh == 128) return launch_tc<128, 2>(tm, nslots, heads, N, o, err, st);
+  if (dh == 72) return launch_tc<128, 2, 72>(tm, nslots, heads, N, o, err, st);
   return cudaErrorInvalidValue;
 }
 

@@ -129,14 +129,28 @@ __device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// The error word of a launch is two ints: [0] the code of the first wait
+// that gave up (0 while none has), [1] a limit in ns for the waits on work in
+// progress (0: kWaitLimitNs; a test shortens it to make such waits run out).
+// Waits that drain copies or MMAs this CTA has already issued (`drain`)
+// always use kWaitLimitNs, so a CTA never leaves with its own copies in
+// flight.
+__device__ __forceinline__ unsigned long long wait_limit_ns(const int* err, bool drain) {
+  if (drain) return kWaitLimitNs;
+  const unsigned v = *reinterpret_cast<const volatile unsigned*>(err + 1);
+  return v != 0u ? (unsigned long long)v : kWaitLimitNs;
+}
+
 // Bounded wait for the phase with the given parity.  Returns false (and
 // records `code` in *err) if it gave up.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* err, int code) {
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* err, int code,
+                                          bool drain = false) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = global_ns();
+  const unsigned long long limit = wait_limit_ns(err, drain);
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
-    if (global_ns() - t0 > kWaitLimitNs) {
+    if (global_ns() - t0 > limit) {
       atomicCAS(err, 0, code);
       return false;
     }
@@ -157,8 +171,9 @@ __device__ __forceinline__ bool elect_one() {
 // Bounded wait by every lane of a warp with a warp-uniform outcome: if any
 // lane gave up, all lanes report failure (so warp-collective instructions
 // that follow are executed by all lanes or by none).
-__device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity, int* err, int code) {
-  const bool ok = mbar_wait(bar, parity, err, code);
+__device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity, int* err, int code,
+                                               bool drain = false) {
+  const bool ok = mbar_wait(bar, parity, err, code, drain);
   return __all_sync(0xffffffffu, ok);
 }
 

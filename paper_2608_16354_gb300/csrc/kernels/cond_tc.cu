@@ -133,7 +133,7 @@ __global__ void __launch_bounds__(kCThreads, 1)
     }
     // no copy may still be landing when the CTA leaves
     for (int s = 0; s < kCStages; ++s)
-      if (last_phase[s] >= 0) mbar_wait_warp(&bar->full[s], (uint32_t)last_phase[s], err, kDevTimeoutTma);
+      if (last_phase[s] >= 0) mbar_wait_warp(&bar->full[s], (uint32_t)last_phase[s], err, kDevTimeoutTma, true);
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     int stage = 0;
@@ -170,7 +170,7 @@ __global__ void __launch_bounds__(kCThreads, 1)
     // every MMA issued here has completed once `drain` flips
     if (elect_one()) tc_commit(&bar->drain);
     __syncwarp();
-    mbar_wait_warp(&bar->drain, 0, err, kDevTimeoutMma);
+    mbar_wait_warp(&bar->drain, 0, err, kDevTimeoutMma, true);
   } else {
     // -------------------------------------------------------------- epilogue
     const int q = warp & 3;  // TMEM lane quarter: weight rows 32 q .. 32 q + 31

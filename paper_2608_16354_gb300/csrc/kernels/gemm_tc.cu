@@ -196,11 +196,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     // 0 has passed here (final cluster barrier)
     if (rank == 0)
       for (int s = 0; s < kStages; ++s)
-        if (last_phase[s] >= 0) mbar_wait_warp(&bar->full[s], (uint32_t)last_phase[s], err, kDevTimeoutTma);
+        if (last_phase[s] >= 0) mbar_wait_warp(&bar->full[s], (uint32_t)last_phase[s], err, kDevTimeoutTma, true);
   } else if (warp == 1 && rank != 0) {
     // rank 1 issues nothing; its shared memory and TMEM are in use by rank
     // 0's pair MMAs until they drain
-    mbar_wait_warp(&bar->drain, 0, err, kDevTimeoutMma);
+    mbar_wait_warp(&bar->drain, 0, err, kDevTimeoutMma, true);
   } else if (warp == 1) {
     // -------------------------------------------------- MMA issuer (rank 0)
     // The whole warp runs the loop with uniform descriptors; one elected lane
@@ -246,7 +246,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     // both CTAs)
     if (elect_one()) tc_commit_pair_mc(&bar->drain, (uint16_t)0x3);
     __syncwarp();
-    mbar_wait_warp(&bar->drain, 0, err, kDevTimeoutMma);
+    mbar_wait_warp(&bar->drain, 0, err, kDevTimeoutMma, true);
   } else {
     // ---------------------------------------------------- epilogue warps
     const int q = warp & 3;             // TMEM lane quarter this warp may access
@@ -486,7 +486,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       if (lane < 6) bulk_wait0();
       // a residual prefetch that was never consumed (aborted run) must land first
       if (MODE == kEpiResid && lane == 0 && !ok && hin_loads > hin_used)
-        mbar_wait(&bar->hin_full, (uint32_t)(hin_loads - 1) & 1, err, kDevTimeoutEpi);
+        mbar_wait(&bar->hin_full, (uint32_t)(hin_loads - 1) & 1, err, kDevTimeoutEpi, true);
     }
   }
 

@@ -53,32 +53,25 @@ __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint3
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-// 16-byte loads: streamed data (read once) bypasses L1; tables stay cached
-__device__ __forceinline__ uint4 ld_stream16(const void* p) {
-  uint4 v;
-  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
-               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-               : "l"(p));
-  return v;
+// Streamed rows go through a per-warp ring in shared memory filled with
+// cp.async (16 bytes per thread and row, read back by the same thread), so
+// that several 32-column blocks are in flight per warp without holding them
+// in registers; tables are read through L1.
+constexpr int kRing = 4;  // blocks in flight per warp
+
+__device__ __forceinline__ void cp_async16(void* smem_dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem_dst)), "l"(src)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 __device__ __forceinline__ uint4 ld_tab16(const void* p) {
-  uint4 v;
-  asm volatile("ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%4];"
-               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-               : "l"(p));
-  return v;
-}
-__device__ __forceinline__ float4 ld_stream_f4(const float* p) {
-  float4 v;
-  asm volatile("ld.global.nc.L1::no_allocate.v4.f32 {%0, %1, %2, %3}, [%4];"
-               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-               : "l"(p));
-  return v;
-}
-__device__ __forceinline__ void st_stream16(void* p, uint4 v) {
-  asm volatile("st.global.cs.v4.u32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x), "r"(v.y),
-               "r"(v.z), "r"(v.w)
-               : "memory");
+  return __ldg(reinterpret_cast<const uint4*>(p));
 }
 
 __device__ __forceinline__ uint32_t pack_bf2(float lo_elem, float hi_elem) {
@@ -150,7 +143,12 @@ __global__ void __launch_bounds__(128) head_reuse_kernel(
     float dsig, float* __restrict__ vout) {
   pdl_trigger();
   pdl_wait();
-  __shared__ float part[4][kReuseTok][2 * kHC + 2];  // per warp: A, Q, sum c, sum c^2
+  // per warp: the cp.async ring (rows (m tile, half) x lanes); after the main
+  // loop the same memory holds the warps' partial sums (A, Q, sum c, sum c^2)
+  __shared__ uint4 ring[4][kRing][4][32];
+  static_assert(sizeof(float) * 4 * kReuseTok * (2 * kHC + 2) <= sizeof(uint4) * 4 * kRing * 4 * 32,
+                "partials exceed the ring");
+  auto part = reinterpret_cast<float (*)[kReuseTok][2 * kHC + 2]>(&ring[0][0][0][0]);
   __shared__ float stab[kHeadTab + kHC + kHC * kHC];  // S', beta, G_s | w_sum | G
   const int slot = blockIdx.y, scene = map.scene[slot];
   const int tok0 = blockIdx.x * kReuseTok;
@@ -179,45 +177,63 @@ __global__ void __launch_bounds__(128) head_reuse_kernel(
       for (int t = 0; t < 4; ++t) D[i][j][t] = 0.f;
   float s1[2][2] = {{0.f, 0.f}, {0.f, 0.f}}, s2[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
   const int nblk = d >> 5;
-#pragma unroll 2
-  for (int b = warp; b < nblk; b += 4) {
-    const int e = (b << 5) + (q << 3);
-    uint4 av[2][2];
+  const int nbw = warp < nblk ? (nblk - 1 - warp) / 4 + 1 : 0;  // blocks of this warp
+  // block i of this warp (columns 32 (warp + 4 i) ..) into ring stage i % kRing
+  auto fetch = [&](int i) {
+    if (i < nbw) {
+      const int e = ((warp + 4 * i) << 5) + (q << 3);
+      uint4* st = &ring[warp][i % kRing][0][lane];
 #pragma unroll
-    for (int i = 0; i < 2; ++i)
+      for (int k = 0; k < 4; ++k) {
+        const int ii = k >> 1, h = k & 1;
+        if (ok[ii][h]) cp_async16(st + 32 * k, cs + (size_t)row[ii][h] * d + e);
+        else st[32 * k] = make_uint4(0u, 0u, 0u, 0u);
+      }
+    }
+    cp_async_commit();  // an empty group past the end keeps the count uniform
+  };
 #pragma unroll
-      for (int h = 0; h < 2; ++h)
-        av[i][h] = ok[i][h] ? ld_stream16(cs + (size_t)row[i][h] * d + e) : make_uint4(0u, 0u, 0u, 0u);
+  for (int i = 0; i < kRing - 1; ++i) fetch(i);
+  for (int i = 0; i < nbw; ++i) {
+    fetch(i + kRing - 1);
+    const int e = ((warp + 4 * i) << 5) + (q << 3);
     // B rows: W_e^T (channels 0-7, 8-15), W' hi (0-7, 8-15), W' lo (0-7, 8-15)
     uint4 bw[6];
     bw[0] = ld_tab16(w_eT_bf + (size_t)g * d + e);
     bw[1] = ld_tab16(w_eT_bf + (size_t)(8 + g) * d + e);
 #pragma unroll
     for (int j = 0; j < 4; ++j) bw[2 + j] = ld_tab16(wk + (size_t)(8 * j + g) * d + e);
+    cp_async_wait<kRing - 1>();  // block i has landed (this thread's copies)
+    uint4 av[2][2];
+    const uint4* st = &ring[warp][i % kRing][0][lane];
 #pragma unroll
-    for (int i = 0; i < 2; ++i) {
+    for (int k = 0; k < 4; ++k) av[k >> 1][k & 1] = st[32 * k];
+#pragma unroll
+    for (int ii = 0; ii < 2; ++ii) {
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
-        const uint32_t w4[4] = {av[i][h].x, av[i][h].y, av[i][h].z, av[i][h].w};
+        const uint32_t w4[4] = {av[ii][h].x, av[ii][h].y, av[ii][h].z, av[ii][h].w};
 #pragma unroll
         for (int p = 0; p < 4; ++p) {
           const float2 f = unpack_bf2(w4[p]);
-          s1[i][h] += f.x + f.y;
-          s2[i][h] = fmaf(f.x, f.x, fmaf(f.y, f.y, s2[i][h]));
+          s1[ii][h] += f.x + f.y;
+          s2[ii][h] = fmaf(f.x, f.x, fmaf(f.y, f.y, s2[ii][h]));
         }
       }
 #pragma unroll
       for (int s = 0; s < 2; ++s) {
-        const uint32_t a0 = s ? av[i][0].z : av[i][0].x;  // row g, cols 4s + 0, 1
-        const uint32_t a1 = s ? av[i][1].z : av[i][1].x;  // row g + 8
-        const uint32_t a2 = s ? av[i][0].w : av[i][0].y;  // row g, cols 4s + 2, 3
-        const uint32_t a3 = s ? av[i][1].w : av[i][1].y;  // row g + 8
+        const uint32_t a0 = s ? av[ii][0].z : av[ii][0].x;  // row g, cols 4s + 0, 1
+        const uint32_t a1 = s ? av[ii][1].z : av[ii][1].x;  // row g + 8
+        const uint32_t a2 = s ? av[ii][0].w : av[ii][0].y;  // row g, cols 4s + 2, 3
+        const uint32_t a3 = s ? av[ii][1].w : av[ii][1].y;  // row g + 8
 #pragma unroll
         for (int j = 0; j < 6; ++j)
-          mma_bf16_16816(D[i][j], a0, a1, a2, a3, s ? bw[j].z : bw[j].x, s ? bw[j].w : bw[j].y);
+          mma_bf16_16816(D[ii][j], a0, a1, a2, a3, s ? bw[j].z : bw[j].x, s ? bw[j].w : bw[j].y);
       }
     }
   }
+  cp_async_wait<0>();
+  __syncthreads();  // every warp is done with its ring: the partials reuse it
   // lanes 4 g .. 4 g + 3 hold the same rows: add their column sums
 #pragma unroll
   for (int i = 0; i < 2; ++i)
@@ -319,6 +335,7 @@ __global__ void __launch_bounds__(128) head_compute_kernel(
   pdl_trigger();
   pdl_wait();
   __shared__ float part[4][kCmpTok][kHC + 2];  // per warp: P, sum h, sum h^2
+  __shared__ uint4 ring[4][kRing][4][32];       // per warp: (row half, 16-byte piece) x lanes
   __shared__ float stab[2 * kHC];              // S', beta
   const int slot = blockIdx.y, scene = map.scene[slot];
   const int tok0 = blockIdx.x * kCmpTok;
@@ -346,16 +363,38 @@ __global__ void __launch_bounds__(128) head_compute_kernel(
     for (int t = 0; t < 4; ++t) D[j][t] = 0.f;
   float s1[2] = {0.f, 0.f}, s2[2] = {0.f, 0.f};
   const int nblk = d >> 5;
-  for (int b = warp; b < nblk; b += 4) {
-    const int e = (b << 5) + (q << 3);
-    float hv[2][8];
+  const int nbw = warp < nblk ? (nblk - 1 - warp) / 4 + 1 : 0;  // blocks of this warp
+  // block i of this warp: rows g and g + 8, 8 fp32 columns each (two 16-byte
+  // copies per row) into ring stage i % kRing
+  auto fetch = [&](int i) {
+    if (i < nbw) {
+      const int e = ((warp + 4 * i) << 5) + (q << 3);
+      uint4* st = &ring[warp][i % kRing][0][lane];
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const float* hr = hL + ((size_t)slot * N + row[h]) * d + e;
-      const float4 p0 = ok[h] ? ld_stream_f4(hr) : make_float4(0.f, 0.f, 0.f, 0.f);
-      const float4 p1 = ok[h] ? ld_stream_f4(hr + 4) : make_float4(0.f, 0.f, 0.f, 0.f);
-      hv[h][0] = p0.x; hv[h][1] = p0.y; hv[h][2] = p0.z; hv[h][3] = p0.w;
-      hv[h][4] = p1.x; hv[h][5] = p1.y; hv[h][6] = p1.z; hv[h][7] = p1.w;
+      for (int k = 0; k < 4; ++k) {
+        const int h = k >> 1;
+        if (ok[h]) cp_async16(st + 32 * k, hL + ((size_t)slot * N + row[h]) * d + e + 4 * (k & 1));
+        else st[32 * k] = make_uint4(0u, 0u, 0u, 0u);
+      }
+    }
+    cp_async_commit();
+  };
+#pragma unroll
+  for (int i = 0; i < kRing - 1; ++i) fetch(i);
+  for (int i = 0; i < nbw; ++i) {
+    fetch(i + kRing - 1);
+    const int e = ((warp + 4 * i) << 5) + (q << 3);
+    cp_async_wait<kRing - 1>();
+    float hv[2][8];
+    {
+      const uint4* st = &ring[warp][i % kRing][0][lane];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const uint4 w = st[32 * k];
+        float* dst = &hv[k >> 1][4 * (k & 1)];
+        dst[0] = __uint_as_float(w.x); dst[1] = __uint_as_float(w.y);
+        dst[2] = __uint_as_float(w.z); dst[3] = __uint_as_float(w.w);
+      }
     }
     uint4 bw[4];  // W' hi (channels 0-7, 8-15), W' lo (0-7, 8-15)
 #pragma unroll
@@ -384,7 +423,7 @@ __global__ void __launch_bounds__(128) head_compute_kernel(
         cw.y = pack_bf2(hv[h][2] - u[h][2], hv[h][3] - u[h][3]);
         cw.z = pack_bf2(hv[h][4] - u[h][4], hv[h][5] - u[h][5]);
         cw.w = pack_bf2(hv[h][6] - u[h][6], hv[h][7] - u[h][7]);
-        st_stream16(cache + ((size_t)scene * N + row[h]) * d + e, cw);
+        __stcs(reinterpret_cast<uint4*>(cache + ((size_t)scene * N + row[h]) * d + e), cw);
       }
 #pragma unroll
       for (int k = 0; k < 8; ++k) {
@@ -408,6 +447,7 @@ __global__ void __launch_bounds__(128) head_compute_kernel(
       }
     }
   }
+  cp_async_wait<0>();
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
     s1[h] += __shfl_xor_sync(0xffffffffu, s1[h], 1);

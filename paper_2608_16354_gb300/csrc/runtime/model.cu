@@ -1488,6 +1488,14 @@ dc_status dc_drift_sums(dc_model* m, const float* x_now, const float* x_ref, int
   return m->bf16 ? enqueue_drift<__nv_bfloat16>(m, it, out, st) : enqueue_drift<float>(m, it, out, st);
 }
 
+dc_status dc_set_wait_limit(dc_model* m, unsigned int ns) {
+  if (!m) { dc::set_error("model is NULL"); return DC_ERR_INVALID_ARG; }
+  DC_CK(cudaSetDevice(m->device));
+  DC_CK(cudaDeviceSynchronize());  // no launch of this model is in flight
+  DC_CK(cudaMemcpy(m->err_d + 1, &ns, sizeof(ns), cudaMemcpyHostToDevice));
+  return DC_OK;
+}
+
 dc_status dc_profile(dc_model* m, int enable) {
   if (!m) { dc::set_error("model is NULL"); return DC_ERR_INVALID_ARG; }
   if (enable) {
@@ -1560,8 +1568,8 @@ dc_status dc_attention(int dtype, const void* qkv, int slots, int heads, int n_t
       CUtensorMap tm;
       DC_TRY(make_map(&tm, qkv, dhp, (uint64_t)3 * slots * heads * n_tokens, 128));
       int* err_d = nullptr;
-      DC_CK(cudaMallocAsync(reinterpret_cast<void**>(&err_d), sizeof(int), st));
-      cudaError_t e = cudaMemsetAsync(err_d, 0, sizeof(int), st);
+      DC_CK(cudaMallocAsync(reinterpret_cast<void**>(&err_d), 2 * sizeof(int), st));
+      cudaError_t e = cudaMemsetAsync(err_d, 0, 2 * sizeof(int), st);  // code, wait limit
       if (e == cudaSuccess)
         e = dc::launch_attention_tc(tm, slots, heads, n_tokens, head_dim,
                                     static_cast<__nv_bfloat16*>(out), err_d, st);
