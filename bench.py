@@ -54,6 +54,11 @@ def parse():
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--workload", default="c5", choices=sorted(WORKLOADS))
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--blocks", type=int, default=None,
+                   help="run the workload with this many DiT blocks (profiling captures; the "
+                        "per-launch shapes stay those of the workload)")
+    p.add_argument("--denoise-steps", type=int, default=None,
+                   help="denoising steps per call instead of the workload's (profiling captures)")
     p.add_argument("--calibration", action="store_true",
                    help="time the joint run responses (Eq. 6-7) of one anchor instead")
     return p.parse_args()
@@ -453,6 +458,10 @@ def run_calibration(args, wl):
 def main():
     args = parse()
     wl = WORKLOADS[args.workload]
+    if args.blocks is not None:
+        wl = wl.with_(n_blocks=args.blocks, name=f"{wl.name}-only{args.blocks}blocks")
+    if args.denoise_steps is not None:
+        wl = wl.with_(steps=args.denoise_steps, name=f"{wl.name}-only{args.denoise_steps}steps")
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))

@@ -90,6 +90,7 @@ struct __align__(8) AttBars {
   uint64_t drain;
   uint32_t tmem_base;
   int abort;              // the error word was set before this CTA started
+  uint32_t wlim;          // limit of the waits on work in progress (ns)
 };
 
 // Descriptor of an MN-major operand tile written by TMA with 128-byte swizzle
@@ -242,6 +243,7 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
   if (threadIdx.x == 0) {
     // read once, so that the whole CTA takes the same decision below
     bar->abort = *(volatile int*)err;
+    bar->wlim = work_wait_limit(err);
     mbar_init(&bar->q_full, 1);
     for (int b = 0; b < kKStages; ++b) {
       mbar_init(&bar->k_full[b], 1);
@@ -272,6 +274,7 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
   pdl_trigger();
   pdl_wait();
   const uint32_t tmem = bar->tmem_base;
+  const uint32_t wlim = bar->wlim;
   if (bar->abort != 0) {
     // a bounded wait of an earlier launch gave up: do nothing (the host
     // reports DC_ERR_DEVICE_TIMEOUT at its next check)
@@ -360,11 +363,11 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
         }
       }
       // every copy in flight lands before the CTA can exit
-      mbar_wait_warp(&bar->q_full, 0, err, kDevTimeoutTma, true);
+      mbar_wait_warp(&bar->q_full, 0, err, kDevTimeoutTma);
       for (int b = 0; b < kKStages; ++b)
-        if (last_k[b] >= 0) mbar_wait_warp(&bar->k_full[b], (uint32_t)last_k[b], err, kDevTimeoutTma, true);
+        if (last_k[b] >= 0) mbar_wait_warp(&bar->k_full[b], (uint32_t)last_k[b], err, kDevTimeoutTma);
       for (int b = 0; b < kVStages; ++b)
-        if (last_v[b] >= 0) mbar_wait_warp(&bar->v_full[b], (uint32_t)last_v[b], err, kDevTimeoutTma, true);
+        if (last_v[b] >= 0) mbar_wait_warp(&bar->v_full[b], (uint32_t)last_v[b], err, kDevTimeoutTma);
     } else if (warp >= 1 && warp <= NQ) {
       // ------------------------------------------------------------ MMA
       // One warp per query tile t, fixed order with blocking waits.  Round j
@@ -376,7 +379,7 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
       // elected lane (the same one throughout, as tcgen05.commit tracks the
       // issuing thread) issues.
       const int t = warp - 1;
-      bool ok = mbar_wait_warp(&bar->q_full, 0, err, kDevTimeoutMma);
+      bool ok = mbar_wait_warp(&bar->q_full, 0, err, kDevTimeoutMma, wlim);
       // descriptor + (byte offset >> 4) moves the start address (no carry:
       // shared-memory addresses are below 256 KB)
       const uint64_t dQ = sw128_kmajor_desc(smem_u32(smem + Cfg::kOffQ + t * Cfg::kTileBytes));
@@ -386,9 +389,9 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
       // softmax; with P aliased onto S_t, PV_{t,j-1} issued before it)
       auto issue_s = [&](int j) -> bool {
         const int kb = j % kKStages;
-        bool good = mbar_wait_warp(&bar->k_full[kb], (uint32_t)(j / kKStages) & 1, err, kDevTimeoutMma);
+        bool good = mbar_wait_warp(&bar->k_full[kb], (uint32_t)(j / kKStages) & 1, err, kDevTimeoutMma, wlim);
         if (!Cfg::kAliasP)
-          good = good && mbar_wait_warp(&bar->s_free[t], ((uint32_t)j & 1) ^ 1, err, kDevTimeoutMma);
+          good = good && mbar_wait_warp(&bar->s_free[t], ((uint32_t)j & 1) ^ 1, err, kDevTimeoutMma, wlim);
         if (!good) return false;
         tc_fence_after();
         if (elect_one()) {
@@ -408,8 +411,8 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
       auto issue_pv = [&](int jp) -> bool {
         const int vb = jp % kVStages;
         const bool good =
-            mbar_wait_warp(&bar->v_full[vb], (uint32_t)(jp / kVStages) & 1, err, kDevTimeoutMma) &&
-            mbar_wait_warp(&bar->p_full[t], (uint32_t)jp & 1, err, kDevTimeoutMma);
+            mbar_wait_warp(&bar->v_full[vb], (uint32_t)(jp / kVStages) & 1, err, kDevTimeoutMma, wlim) &&
+            mbar_wait_warp(&bar->p_full[t], (uint32_t)jp & 1, err, kDevTimeoutMma, wlim);
         if (!good) return false;
         tc_fence_after();
         if (elect_one()) {
@@ -439,7 +442,7 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
       }
       if (elect_one()) tc_commit(&bar->drain);
       __syncwarp();
-      mbar_wait_warp(&bar->drain, 0, err, kDevTimeoutMma, true);
+      mbar_wait_warp(&bar->drain, 0, err, kDevTimeoutMma);
     }
     tc_fence_before();
     named_bar(1, Cfg::kThreads);
@@ -463,7 +466,7 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
     // (Making the two query tiles take turns on MUFU through named barriers
     // measured slower: the tiles' own S -> P -> PV chains set the pace.)
     for (int j = 0; j < n_kv; ++j) {
-      ok = ok && mbar_wait_warp(&bar->s_full[t], (uint32_t)j & 1, err, kDevTimeoutEpi);
+      ok = ok && mbar_wait_warp_sl(&bar->s_full[t], (uint32_t)j & 1, err, kDevTimeoutEpi, &bar->wlim);
       if (!ok) break;
       float c = 1.f;
       uint32_t pk[64];
@@ -546,7 +549,7 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
         l = l * c + ((rs2[0].x + rs2[0].y) + (rs2[1].x + rs2[1].y));
       }
       // P_t and O_t are free once PV_{t,j-1} has landed
-      ok = mbar_wait_warp(&bar->p_free[t], ((uint32_t)j & 1) ^ 1, err, kDevTimeoutEpi);
+      ok = mbar_wait_warp_sl(&bar->p_free[t], ((uint32_t)j & 1) ^ 1, err, kDevTimeoutEpi, &bar->wlim);
       if (!ok) break;
       tc_fence_after();
       if (__any_sync(0xffffffffu, c != 1.f)) {
@@ -571,7 +574,7 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
       if (lane == 0) mbar_arrive(&bar->p_full[t]);
     }
     // the last PV product of this query tile completes O_t
-    if (ok) ok = mbar_wait_warp(&bar->p_free[t], (uint32_t)(n_kv - 1) & 1, err, kDevTimeoutEpi);
+    if (ok) ok = mbar_wait_warp_sl(&bar->p_free[t], (uint32_t)(n_kv - 1) & 1, err, kDevTimeoutEpi, &bar->wlim);
     const int qrow = q0 + t * 128 + row;
     if (ok) {
       tc_fence_after();

@@ -132,25 +132,23 @@ __device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
 // The error word of a launch is two ints: [0] the code of the first wait
 // that gave up (0 while none has), [1] a limit in ns for the waits on work in
 // progress (0: kWaitLimitNs; a test shortens it to make such waits run out).
-// Waits that drain copies or MMAs this CTA has already issued (`drain`)
-// always use kWaitLimitNs, so a CTA never leaves with its own copies in
-// flight.
-__device__ __forceinline__ unsigned long long wait_limit_ns(const int* err, bool drain) {
-  if (drain) return kWaitLimitNs;
+// A kernel reads the limit once at its start (work_wait_limit) and passes it
+// to those waits; waits that drain copies or MMAs the CTA has already issued
+// keep kWaitLimitNs, so a CTA never leaves with its own copies in flight.
+__device__ __forceinline__ uint32_t work_wait_limit(const int* err) {
   const unsigned v = *reinterpret_cast<const volatile unsigned*>(err + 1);
-  return v != 0u ? (unsigned long long)v : kWaitLimitNs;
+  return v != 0u ? v : (uint32_t)kWaitLimitNs;
 }
 
 // Bounded wait for the phase with the given parity.  Returns false (and
-// records `code` in *err) if it gave up.
+// records `code` in *err) if it gave up after `limit_ns`.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* err, int code,
-                                          bool drain = false) {
+                                          uint32_t limit_ns = (uint32_t)kWaitLimitNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = global_ns();
-  const unsigned long long limit = wait_limit_ns(err, drain);
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
-    if (global_ns() - t0 > limit) {
+    if (global_ns() - t0 > (unsigned long long)limit_ns) {
       atomicCAS(err, 0, code);
       return false;
     }
@@ -172,8 +170,17 @@ __device__ __forceinline__ bool elect_one() {
 // lane gave up, all lanes report failure (so warp-collective instructions
 // that follow are executed by all lanes or by none).
 __device__ __forceinline__ bool mbar_wait_warp(uint64_t* bar, uint32_t parity, int* err, int code,
-                                               bool drain = false) {
-  const bool ok = mbar_wait(bar, parity, err, code, drain);
+                                               uint32_t limit_ns = (uint32_t)kWaitLimitNs) {
+  const bool ok = mbar_wait(bar, parity, err, code, limit_ns);
+  return __all_sync(0xffffffffu, ok);
+}
+
+// As mbar_wait_warp, with the limit kept in shared memory and read only when
+// the first test fails (for code that has no register to spare for it).
+__device__ __forceinline__ bool mbar_wait_warp_sl(uint64_t* bar, uint32_t parity, int* err, int code,
+                                                  const uint32_t* limit_smem) {
+  bool ok = mbar_try_wait(bar, parity);
+  if (!ok) ok = mbar_wait(bar, parity, err, code, *reinterpret_cast<const volatile uint32_t*>(limit_smem));
   return __all_sync(0xffffffffu, ok);
 }
 

@@ -148,6 +148,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   pdl_trigger();
   pdl_wait();
   const uint32_t tmem_base = bar->tmem_base;
+  const uint32_t wlim = work_wait_limit(err);
   // a bounded wait of an earlier launch gave up: do nothing (the host reports
   // DC_ERR_DEVICE_TIMEOUT at its next check), but still meet the peer at the
   // final cluster barrier
@@ -169,7 +170,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       for (int kb = 0; kb < KB; ++kb) {
         // the stage is free once the pair MMAs have read it; both CTAs'
         // copies are counted on rank 0's full barrier
-        if (!mbar_wait_warp(&bar->empty[stage], phase ^ 1, err, kDevTimeoutTma)) { ok = false; break; }
+        if (!mbar_wait_warp(&bar->empty[stage], phase ^ 1, err, kDevTimeoutTma, wlim)) { ok = false; break; }
         const int la = (2 * issued) & 7;
         if (rank == 0) {
           if (lane == la) mbar_arrive_expect_tx(&bar->full[stage], kStageBytes);
@@ -196,11 +197,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     // 0 has passed here (final cluster barrier)
     if (rank == 0)
       for (int s = 0; s < kStages; ++s)
-        if (last_phase[s] >= 0) mbar_wait_warp(&bar->full[s], (uint32_t)last_phase[s], err, kDevTimeoutTma, true);
+        if (last_phase[s] >= 0) mbar_wait_warp(&bar->full[s], (uint32_t)last_phase[s], err, kDevTimeoutTma);
   } else if (warp == 1 && rank != 0) {
     // rank 1 issues nothing; its shared memory and TMEM are in use by rank
     // 0's pair MMAs until they drain
-    mbar_wait_warp(&bar->drain, 0, err, kDevTimeoutMma, true);
+    mbar_wait_warp(&bar->drain, 0, err, kDevTimeoutMma);
   } else if (warp == 1) {
     // -------------------------------------------------- MMA issuer (rank 0)
     // The whole warp runs the loop with uniform descriptors; one elected lane
@@ -219,11 +220,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     for (int pt = pair; pt < n_pt && ok; pt += n_pairs, ++t) {
       const int b = t & 1;
       const uint32_t use = (uint32_t)(t >> 1);
-      if (!mbar_wait_warp(&bar->tmem_empty[b], (use & 1) ^ 1, err, kDevTimeoutMma)) { ok = false; break; }
+      if (!mbar_wait_warp(&bar->tmem_empty[b], (use & 1) ^ 1, err, kDevTimeoutMma, wlim)) { ok = false; break; }
       tc_fence_after();
       const uint32_t d_tmem = tmem_base + (uint32_t)(b * 256);
       for (int kb = 0; kb < KB; ++kb) {
-        if (!mbar_wait_warp(&bar->full[stage], phase, err, kDevTimeoutMma)) { ok = false; break; }
+        if (!mbar_wait_warp(&bar->full[stage], phase, err, kDevTimeoutMma, wlim)) { ok = false; break; }
         tc_fence_after();
         if (elect_one()) {
 #pragma unroll
@@ -246,7 +247,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     // both CTAs)
     if (elect_one()) tc_commit_pair_mc(&bar->drain, (uint16_t)0x3);
     __syncwarp();
-    mbar_wait_warp(&bar->drain, 0, err, kDevTimeoutMma, true);
+    mbar_wait_warp(&bar->drain, 0, err, kDevTimeoutMma);
   } else {
     // ---------------------------------------------------- epilogue warps
     const int q = warp & 3;             // TMEM lane quarter this warp may access
@@ -284,7 +285,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const uint32_t use = (uint32_t)(t >> 1);
       // every wait outcome is made uniform (warp, then the 8 epilogue warps at
       // the named barrier) so that an abort is taken by all of them together
-      const bool acc_ok = mbar_wait_warp(&bar->tmem_full[b], use & 1, err, kDevTimeoutEpi);
+      const bool acc_ok = mbar_wait_warp(&bar->tmem_full[b], use & 1, err, kDevTimeoutEpi, wlim);
       const int m0 = m0_of(pt);
       const int n0 = n0_of(pt);
       // the second tile of the last pair may lie below M: it runs (its A rows
@@ -365,7 +366,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         for (int pass = 0; pass < (HALF ? 2 : 1); ++pass) {
           // pass p stages columns 96 p .. (all 192 without HALF)
           const bool hin_ok = mbar_wait_warp(&bar->hin_full, HALF ? (uint32_t)pass : (uint32_t)t & 1,
-                                             err, kDevTimeoutEpi);
+                                             err, kDevTimeoutEpi, wlim);
           if (hin_ok) ++hin_used;
           if (hin_ok && (!HALF || half == pass)) apply(HALF ? 96 * pass : 0);
           fence_proxy_async();
@@ -486,7 +487,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       if (lane < 6) bulk_wait0();
       // a residual prefetch that was never consumed (aborted run) must land first
       if (MODE == kEpiResid && lane == 0 && !ok && hin_loads > hin_used)
-        mbar_wait(&bar->hin_full, (uint32_t)(hin_loads - 1) & 1, err, kDevTimeoutEpi, true);
+        mbar_wait(&bar->hin_full, (uint32_t)(hin_loads - 1) & 1, err, kDevTimeoutEpi);
     }
   }
 

@@ -38,9 +38,12 @@ def rel(a, b):
 
 @pytest.mark.timeout(300)
 def test_bounded_waits_run_out_and_the_model_recovers(dc):
-    # d 384 / dh 64: tcgen05 GEMMs in clusters of two, the two-tile attention,
-    # the adaLN table; 2 scenes x 256 tokens, one compute and one reuse step
-    wl = WORKLOADS["c2"].with_(n_blocks=1, frames=1, rows=16, cols=16, batch=2, steps=2)
+    # d 3072 / dh 128, 2025 tokens, one block: the GEMMs run K loops of up to
+    # 12288 (tens of microseconds per tile), so their epilogue waits, and the
+    # attention's, outlast any wait limit of a few microseconds (an mbarrier
+    # try_wait itself may block for a while before it reports "not yet");
+    # one compute and one reuse step
+    wl = WORKLOADS["c5"].with_(n_blocks=1, frames=1, rows=45, cols=45, batch=1, steps=2)
     w = gen.weights(wl)
     K = wl.steps
     sig = gen.sigmas(K)
