@@ -34,6 +34,8 @@
 // steps); each warp takes every 4th 32-column block of d for all of the
 // CTA's tokens, and the partial sums of the four warps are added in shared
 // memory in a fixed order (deterministic).  C = 16 channels.
+#include <cstring>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -131,11 +133,20 @@ __global__ void __launch_bounds__(256) head_tables_kernel(
 
 // ---------------------------------------------------------------- reuse step
 
-constexpr int kReuseTok = 32;  // tokens per CTA on reuse steps (two m16 tiles per warp)
+constexpr int kReuseWarps = 4;                // one 16-token tile per warp
+constexpr int kReuseTok = 16 * kReuseWarps;   // tokens per CTA on reuse steps
+constexpr int kReuseStages = 12;              // 32-column blocks in flight per CTA
+constexpr int kBRows = 48;                    // B rows: W_e^T (16), W' hi (16), W' lo (16)
+// one stage: each warp's A block (16 rows x 64 B) and the shared B block (48 x 64 B)
+constexpr int kReuseStageBytes = kReuseWarps * 1024 + kBRows * 64;
+constexpr int kReuseSmem = kReuseStages * kReuseStageBytes;
 constexpr int kCmpTok = 16;    // tokens per CTA on compute steps (one m16 tile per warp)
 
 // Reuse step of the scenes in `map`: h = x W_e^T + c_j, v = head(h), x += dsig v
-// (or v to vout).  wp_k / tab_k: this step's tables, indexed by scene.
+// (or v to vout).  wp_k / tab_k: this step's tables, indexed by scene.  Each
+// warp takes 16 tokens over all of d; per 32-column block the CTA stages the
+// warps' cache rows and the 48 B rows (shared by the four warps) in a
+// kReuseStages-deep cp.async ring.
 __global__ void __launch_bounds__(128) head_reuse_kernel(
     float* __restrict__ x, const __nv_bfloat16* __restrict__ cache, SlotMap map, int N, int d,
     const __nv_bfloat16* __restrict__ w_eT_bf, const __nv_bfloat16* __restrict__ wp_k,
@@ -143,131 +154,122 @@ __global__ void __launch_bounds__(128) head_reuse_kernel(
     float dsig, float* __restrict__ vout) {
   pdl_trigger();
   pdl_wait();
-  // per warp: the cp.async ring (rows (m tile, half) x lanes); after the main
-  // loop the same memory holds the warps' partial sums (A, Q, sum c, sum c^2)
-  __shared__ uint4 ring[4][kRing][4][32];
-  static_assert(sizeof(float) * 4 * kReuseTok * (2 * kHC + 2) <= sizeof(uint4) * 4 * kRing * 4 * 32,
-                "partials exceed the ring");
-  auto part = reinterpret_cast<float (*)[kReuseTok][2 * kHC + 2]>(&ring[0][0][0][0]);
-  __shared__ float stab[kHeadTab + kHC + kHC * kHC];  // S', beta, G_s | w_sum | G
+  extern __shared__ __align__(16) uint8_t rsm[];
+  __shared__ float part[kReuseWarps][16][2 * kHC + 2];  // per token: A, Q, sum c, sum c^2
+  __shared__ float stab[kHeadTab + kHC + kHC * kHC];    // S', beta, G_s | w_sum | G
   const int slot = blockIdx.y, scene = map.scene[slot];
   const int tok0 = blockIdx.x * kReuseTok;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, q = lane & 3;
-  for (int i = threadIdx.x; i < kHeadTab; i += blockDim.x) stab[i] = tab_k[(size_t)scene * kHeadTab + i];
-  if (threadIdx.x < kHC) stab[kHeadTab + threadIdx.x] = wsum[threadIdx.x];
-  for (int i = threadIdx.x; i < kHC * kHC; i += blockDim.x) stab[kHeadTab + kHC + i] = gram[i];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, q = lane & 3;
+  for (int i = tid; i < kHeadTab; i += blockDim.x) stab[i] = tab_k[(size_t)scene * kHeadTab + i];
+  if (tid < kHC) stab[kHeadTab + tid] = wsum[tid];
+  for (int i = tid; i < kHC * kHC; i += blockDim.x) stab[kHeadTab + kHC + i] = gram[i];
 
   const __nv_bfloat16* cs = cache + (size_t)scene * N * d;
   const __nv_bfloat16* wk = wp_k + (size_t)scene * 2 * kHC * d;
-  int row[2][2];
-  bool ok[2][2];
+  int row[2];
+  bool ok[2];
 #pragma unroll
-  for (int i = 0; i < 2; ++i)
+  for (int h = 0; h < 2; ++h) {
+    row[h] = tok0 + 16 * warp + 8 * h + g;
+    ok[h] = row[h] < N;
+  }
+  // this thread's copies of block b into stage st: its own two cache pieces,
+  // and B pieces tid and tid + 128 (of 48 rows x 4 pieces)
+  auto fetch = [&](int b, int st) {
+    uint8_t* base = rsm + st * kReuseStageBytes;
+    const int e = (b << 5) + (q << 3);
+    uint4* a = reinterpret_cast<uint4*>(base + warp * 1024) + lane;
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-      row[i][h] = tok0 + 16 * i + 8 * h + g;
-      ok[i][h] = row[i][h] < N;
+      if (ok[h]) cp_async16(a + 32 * h, cs + (size_t)row[h] * d + e);
+      else a[32 * h] = make_uint4(0u, 0u, 0u, 0u);
     }
-  float D[2][6][4];
+    uint4* bb = reinterpret_cast<uint4*>(base + kReuseWarps * 1024);
 #pragma unroll
-  for (int i = 0; i < 2; ++i)
-#pragma unroll
-    for (int j = 0; j < 6; ++j)
-#pragma unroll
-      for (int t = 0; t < 4; ++t) D[i][j][t] = 0.f;
-  float s1[2][2] = {{0.f, 0.f}, {0.f, 0.f}}, s2[2][2] = {{0.f, 0.f}, {0.f, 0.f}};
-  const int nblk = d >> 5;
-  const int nbw = warp < nblk ? (nblk - 1 - warp) / 4 + 1 : 0;  // blocks of this warp
-  // block i of this warp (columns 32 (warp + 4 i) ..) into ring stage i % kRing
-  auto fetch = [&](int i) {
-    if (i < nbw) {
-      const int e = ((warp + 4 * i) << 5) + (q << 3);
-      uint4* st = &ring[warp][i % kRing][0][lane];
-#pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const int ii = k >> 1, h = k & 1;
-        if (ok[ii][h]) cp_async16(st + 32 * k, cs + (size_t)row[ii][h] * d + e);
-        else st[32 * k] = make_uint4(0u, 0u, 0u, 0u);
+    for (int k = 0; k < 2; ++k) {
+      const int c = tid + 128 * k;
+      if (c < kBRows * 4) {
+        const int r = c >> 2, piece = c & 3;
+        const __nv_bfloat16* src = r < kHC ? w_eT_bf + (size_t)r * d : wk + (size_t)(r - kHC) * d;
+        cp_async16(bb + c, src + (b << 5) + (piece << 3));
       }
     }
-    cp_async_commit();  // an empty group past the end keeps the count uniform
   };
+  float D[6][4];
 #pragma unroll
-  for (int i = 0; i < kRing - 1; ++i) fetch(i);
-  for (int i = 0; i < nbw; ++i) {
-    fetch(i + kRing - 1);
-    const int e = ((warp + 4 * i) << 5) + (q << 3);
-    // B rows: W_e^T (channels 0-7, 8-15), W' hi (0-7, 8-15), W' lo (0-7, 8-15)
+  for (int j = 0; j < 6; ++j)
+#pragma unroll
+    for (int t = 0; t < 4; ++t) D[j][t] = 0.f;
+  float s1[2] = {0.f, 0.f}, s2[2] = {0.f, 0.f};
+  const int nblk = d >> 5;
+#pragma unroll 1
+  for (int i = 0; i < kReuseStages - 1; ++i) {
+    if (i < nblk) fetch(i, i);
+    cp_async_commit();
+  }
+#pragma unroll 1
+  for (int b = 0; b < nblk; ++b) {
+    cp_async_wait<kReuseStages - 2>();  // this thread's copies of block b have landed
+    __syncthreads();                    // everyone's have, and block b - 1 is consumed
+    const int nb = b + kReuseStages - 1;
+    if (nb < nblk) fetch(nb, nb % kReuseStages);
+    cp_async_commit();
+    const uint8_t* base = rsm + (b % kReuseStages) * kReuseStageBytes;
+    const uint4* a = reinterpret_cast<const uint4*>(base + warp * 1024) + lane;
+    const uint4 av0 = a[0], av1 = a[32];
+    const uint4* bb = reinterpret_cast<const uint4*>(base + kReuseWarps * 1024);
     uint4 bw[6];
-    bw[0] = ld_tab16(w_eT_bf + (size_t)g * d + e);
-    bw[1] = ld_tab16(w_eT_bf + (size_t)(8 + g) * d + e);
 #pragma unroll
-    for (int j = 0; j < 4; ++j) bw[2 + j] = ld_tab16(wk + (size_t)(8 * j + g) * d + e);
-    cp_async_wait<kRing - 1>();  // block i has landed (this thread's copies)
-    uint4 av[2][2];
-    const uint4* st = &ring[warp][i % kRing][0][lane];
+    for (int j = 0; j < 6; ++j) bw[j] = bb[(8 * j + g) * 4 + q];
+    {
+      const uint32_t w8[8] = {av0.x, av0.y, av0.z, av0.w, av1.x, av1.y, av1.z, av1.w};
 #pragma unroll
-    for (int k = 0; k < 4; ++k) av[k >> 1][k & 1] = st[32 * k];
-#pragma unroll
-    for (int ii = 0; ii < 2; ++ii) {
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const uint32_t w4[4] = {av[ii][h].x, av[ii][h].y, av[ii][h].z, av[ii][h].w};
-#pragma unroll
-        for (int p = 0; p < 4; ++p) {
-          const float2 f = unpack_bf2(w4[p]);
-          s1[ii][h] += f.x + f.y;
-          s2[ii][h] = fmaf(f.x, f.x, fmaf(f.y, f.y, s2[ii][h]));
-        }
+      for (int p = 0; p < 8; ++p) {
+        const float2 f = unpack_bf2(w8[p]);
+        s1[p >> 2] += f.x + f.y;
+        s2[p >> 2] = fmaf(f.x, f.x, fmaf(f.y, f.y, s2[p >> 2]));
       }
+    }
 #pragma unroll
-      for (int s = 0; s < 2; ++s) {
-        const uint32_t a0 = s ? av[ii][0].z : av[ii][0].x;  // row g, cols 4s + 0, 1
-        const uint32_t a1 = s ? av[ii][1].z : av[ii][1].x;  // row g + 8
-        const uint32_t a2 = s ? av[ii][0].w : av[ii][0].y;  // row g, cols 4s + 2, 3
-        const uint32_t a3 = s ? av[ii][1].w : av[ii][1].y;  // row g + 8
+    for (int s = 0; s < 2; ++s) {
+      const uint32_t a0 = s ? av0.z : av0.x;  // row g, cols 4s + 0, 1
+      const uint32_t a1 = s ? av1.z : av1.x;  // row g + 8
+      const uint32_t a2 = s ? av0.w : av0.y;  // row g, cols 4s + 2, 3
+      const uint32_t a3 = s ? av1.w : av1.y;  // row g + 8
 #pragma unroll
-        for (int j = 0; j < 6; ++j)
-          mma_bf16_16816(D[ii][j], a0, a1, a2, a3, s ? bw[j].z : bw[j].x, s ? bw[j].w : bw[j].y);
-      }
+      for (int j = 0; j < 6; ++j)
+        mma_bf16_16816(D[j], a0, a1, a2, a3, s ? bw[j].z : bw[j].x, s ? bw[j].w : bw[j].y);
     }
   }
   cp_async_wait<0>();
-  __syncthreads();  // every warp is done with its ring: the partials reuse it
   // lanes 4 g .. 4 g + 3 hold the same rows: add their column sums
 #pragma unroll
-  for (int i = 0; i < 2; ++i)
+  for (int h = 0; h < 2; ++h) {
+    s1[h] += __shfl_xor_sync(0xffffffffu, s1[h], 1);
+    s1[h] += __shfl_xor_sync(0xffffffffu, s1[h], 2);
+    s2[h] += __shfl_xor_sync(0xffffffffu, s2[h], 1);
+    s2[h] += __shfl_xor_sync(0xffffffffu, s2[h], 2);
+    float* pp = part[warp][8 * h + g];
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      s1[i][h] += __shfl_xor_sync(0xffffffffu, s1[i][h], 1);
-      s1[i][h] += __shfl_xor_sync(0xffffffffu, s1[i][h], 2);
-      s2[i][h] += __shfl_xor_sync(0xffffffffu, s2[i][h], 1);
-      s2[i][h] += __shfl_xor_sync(0xffffffffu, s2[i][h], 2);
-    }
+    for (int j = 0; j < 2; ++j)
 #pragma unroll
-  for (int i = 0; i < 2; ++i)
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      float* pp = part[warp][16 * i + 8 * h + g];
-#pragma unroll
-      for (int j = 0; j < 2; ++j)
-#pragma unroll
-        for (int t = 0; t < 2; ++t) {
-          pp[8 * j + 2 * q + t] = D[i][j][2 * h + t];
-          pp[kHC + 8 * j + 2 * q + t] = D[i][2 + j][2 * h + t] + D[i][4 + j][2 * h + t];
-        }
-      if (q == 0) {
-        pp[2 * kHC] = s1[i][h];
-        pp[2 * kHC + 1] = s2[i][h];
+      for (int t = 0; t < 2; ++t) {
+        pp[8 * j + 2 * q + t] = D[j][2 * h + t];
+        pp[kHC + 8 * j + 2 * q + t] = D[2 + j][2 * h + t] + D[4 + j][2 * h + t];
       }
+    if (q == 0) {
+      pp[2 * kHC] = s1[h];
+      pp[2 * kHC + 1] = s2[h];
     }
-  __syncthreads();
+  }
+  __syncwarp();
 
-  // finish: 4 threads per token, 4 channels each
-  const int tt = threadIdx.x >> 2, cq = threadIdx.x & 3;
-  const int tok = tok0 + tt;
+  // finish: two lanes per token of this warp, 8 channels each
+  const int tt = lane >> 1, ch = lane & 1;
+  const int tok = tok0 + 16 * warp + tt;
   const bool live = tok < N;
-  float xv[kHC], vv[4];
+  const float* pt = part[warp][tt];
+  float xv[kHC], vv[8];
   if (live) {
     const float4* xr = reinterpret_cast<const float4*>(x + ((size_t)scene * N + tok) * kHC);
 #pragma unroll
@@ -277,46 +279,44 @@ __global__ void __launch_bounds__(128) head_reuse_kernel(
     }
     const float *S = stab, *beta = stab + kHC, *Gs = stab + 2 * kHC, *ws = stab + kHeadTab,
                 *G = stab + kHeadTab + kHC;
-    float sum1 = 0.f, sum2 = 0.f, xA = 0.f, xGx = 0.f;
-#pragma unroll
-    for (int w = 0; w < 4; ++w) {
-      sum1 += part[w][tt][2 * kHC];
-      sum2 += part[w][tt][2 * kHC + 1];
-    }
+    float sum1 = pt[2 * kHC], xA = 0.f, xGx = 0.f;
 #pragma unroll
     for (int a = 0; a < kHC; ++a) {
-      const float A = ((part[0][tt][a] + part[1][tt][a]) + part[2][tt][a]) + part[3][tt][a];
-      xA = fmaf(xv[a], A, xA);
+      xA = fmaf(xv[a], pt[a], xA);
       sum1 = fmaf(xv[a], ws[a], sum1);
       float t = 0.f;
 #pragma unroll
       for (int b2 = 0; b2 < kHC; ++b2) t = fmaf(G[a * kHC + b2], xv[b2], t);
       xGx = fmaf(xv[a], t, xGx);
     }
-    const float sq = xGx + 2.f * xA + sum2;
+    const float sq = xGx + 2.f * xA + pt[2 * kHC + 1];
     const float mu = sum1 / (float)d;
     const float var = fmaxf(sq / (float)d - mu * mu, 0.f);
     const float rs = rsqrtf(var + 1e-6f);
 #pragma unroll
-    for (int cc = 0; cc < 4; ++cc) {
-      const int c = 4 * cq + cc;
-      float P = ((part[0][tt][kHC + c] + part[1][tt][kHC + c]) + part[2][tt][kHC + c]) +
-                part[3][tt][kHC + c];
+    for (int cc = 0; cc < 8; ++cc) {
+      const int c = 8 * ch + cc;
+      float P = pt[kHC + c];
 #pragma unroll
       for (int a = 0; a < kHC; ++a) P = fmaf(xv[a], Gs[a * kHC + c], P);
       vv[cc] = fmaf(rs, P - mu * S[c], beta[c]);
     }
   }
-  const size_t xi = ((size_t)scene * N + tok) * kHC + 4 * cq;
-  const float4 xo = live ? *reinterpret_cast<const float4*>(x + xi) : make_float4(0.f, 0.f, 0.f, 0.f);
-  __syncwarp();  // every thread of the token has read its x row
+  const size_t xi = ((size_t)scene * N + tok) * kHC + 8 * ch;
+  const float4 xo0 = live ? *reinterpret_cast<const float4*>(x + xi) : make_float4(0.f, 0.f, 0.f, 0.f);
+  const float4 xo1 = live ? *reinterpret_cast<const float4*>(x + xi + 4) : make_float4(0.f, 0.f, 0.f, 0.f);
+  __syncwarp();  // both lanes of the token have read its x row
   if (live) {
     if (vout) {
       *reinterpret_cast<float4*>(vout + xi) = make_float4(vv[0], vv[1], vv[2], vv[3]);
+      *reinterpret_cast<float4*>(vout + xi + 4) = make_float4(vv[4], vv[5], vv[6], vv[7]);
     } else {
       *reinterpret_cast<float4*>(x + xi) =
-          make_float4(fmaf(dsig, vv[0], xo.x), fmaf(dsig, vv[1], xo.y), fmaf(dsig, vv[2], xo.z),
-                      fmaf(dsig, vv[3], xo.w));
+          make_float4(fmaf(dsig, vv[0], xo0.x), fmaf(dsig, vv[1], xo0.y), fmaf(dsig, vv[2], xo0.z),
+                      fmaf(dsig, vv[3], xo0.w));
+      *reinterpret_cast<float4*>(x + xi + 4) =
+          make_float4(fmaf(dsig, vv[4], xo1.x), fmaf(dsig, vv[5], xo1.y), fmaf(dsig, vv[6], xo1.z),
+                      fmaf(dsig, vv[7], xo1.w));
     }
   }
 }
@@ -329,9 +329,9 @@ __global__ void __launch_bounds__(128) head_reuse_kernel(
 // element), the head on the tensor cores.
 __global__ void __launch_bounds__(128) head_compute_kernel(
     const float* __restrict__ hL, float* __restrict__ x, float* __restrict__ xj,
-    __nv_bfloat16* __restrict__ cache, SlotMap map, int N, int d, const float* __restrict__ w_eT,
-    const __nv_bfloat16* __restrict__ wp_k, const float* __restrict__ tab_k, float dsig,
-    float* __restrict__ vout) {
+    __nv_bfloat16* __restrict__ cache, SlotMap map, int N, int d,
+    const __nv_bfloat16* __restrict__ we_frag, const __nv_bfloat16* __restrict__ wp_k,
+    const float* __restrict__ tab_k, float dsig, float* __restrict__ vout) {
   pdl_trigger();
   pdl_wait();
   __shared__ float part[4][kCmpTok][kHC + 2];  // per warp: P, sum h, sum h^2
@@ -344,17 +344,18 @@ __global__ void __launch_bounds__(128) head_compute_kernel(
   const __nv_bfloat16* wk = wp_k + (size_t)scene * 2 * kHC * d;
   int row[2];
   bool ok[2];
-  float xv[2][kHC];
+  // A fragments of x (tokens x channels, hi and lo halves): rows g and
+  // g + 8, channels 2q, 2q + 1 and 2q + 8, 2q + 9
+  uint32_t xa_hi[4], xa_lo[4];
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
     row[h] = tok0 + 8 * h + g;
     ok[h] = row[h] < N;
-    const float4* xr = reinterpret_cast<const float4*>(x + ((size_t)scene * N + row[h]) * kHC);
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const float4 t4 = ok[h] ? xr[k] : make_float4(0.f, 0.f, 0.f, 0.f);
-      xv[h][4 * k] = t4.x; xv[h][4 * k + 1] = t4.y; xv[h][4 * k + 2] = t4.z; xv[h][4 * k + 3] = t4.w;
-    }
+    const float* xr = x + ((size_t)scene * N + row[h]) * kHC;
+    const float2 p0 = ok[h] ? *reinterpret_cast<const float2*>(xr + 2 * q) : make_float2(0.f, 0.f);
+    const float2 p1 = ok[h] ? *reinterpret_cast<const float2*>(xr + 2 * q + 8) : make_float2(0.f, 0.f);
+    split_pair(p0.x, p0.y, &xa_hi[h], &xa_lo[h]);
+    split_pair(p1.x, p1.y, &xa_hi[2 + h], &xa_lo[2 + h]);
   }
   float D[4][4];
 #pragma unroll
@@ -399,21 +400,23 @@ __global__ void __launch_bounds__(128) head_compute_kernel(
     uint4 bw[4];  // W' hi (channels 0-7, 8-15), W' lo (0-7, 8-15)
 #pragma unroll
     for (int j = 0; j < 4; ++j) bw[j] = ld_tab16(wk + (size_t)(8 * j + g) * d + e);
-    // the cache row: c = h - x W_e^T
+    // the cache row c = h - x W_e^T: x W_e^T on the tensor cores (K = C = 16),
+    // with the B fragments of this block's W_e^T columns laid out so that the
+    // four 8-column products land on this thread's own 8 columns (product j:
+    // columns e + 2 j, e + 2 j + 1 of rows g and g + 8)
     float u[2][8];
+    {
+      const uint4* fp = reinterpret_cast<const uint4*>(we_frag) + ((size_t)((warp + 4 * i) * 32 + lane) << 1);
+      const uint4 f0 = __ldg(fp), f1 = __ldg(fp + 1);
+      const uint32_t fb[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
 #pragma unroll
-    for (int h = 0; h < 2; ++h)
-#pragma unroll
-      for (int k = 0; k < 8; ++k) u[h][k] = 0.f;
-#pragma unroll
-    for (int c = 0; c < kHC; ++c) {
-      const float4 w0 = __ldg(reinterpret_cast<const float4*>(w_eT + (size_t)c * d + e));
-      const float4 w1 = __ldg(reinterpret_cast<const float4*>(w_eT + (size_t)c * d + e + 4));
-      const float wv[8] = {w0.x, w0.y, w0.z, w0.w, w1.x, w1.y, w1.z, w1.w};
-#pragma unroll
-      for (int h = 0; h < 2; ++h)
-#pragma unroll
-        for (int k = 0; k < 8; ++k) u[h][k] = fmaf(xv[h][c], wv[k], u[h][k]);
+      for (int j = 0; j < 4; ++j) {
+        float du[4] = {0.f, 0.f, 0.f, 0.f};
+        mma_bf16_16816(du, xa_hi[0], xa_hi[1], xa_hi[2], xa_hi[3], fb[2 * j], fb[2 * j + 1]);
+        mma_bf16_16816(du, xa_lo[0], xa_lo[1], xa_lo[2], xa_lo[3], fb[2 * j], fb[2 * j + 1]);
+        u[0][2 * j] = du[0]; u[0][2 * j + 1] = du[1];
+        u[1][2 * j] = du[2]; u[1][2 * j + 1] = du[3];
+      }
     }
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
@@ -517,20 +520,47 @@ cudaError_t launch_head_reuse(float* x, const __nv_bfloat16* cache, const SlotMa
                               cudaStream_t st, float* vout) {
   if (map.n <= 0) return cudaSuccess;
   if (d % 32 != 0) return cudaErrorInvalidValue;
+  static std::atomic<unsigned long long> configured{0};
+  const cudaError_t e = configure_once_per_device(configured, [] {
+    return cudaFuncSetAttribute(head_reuse_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                kReuseSmem);
+  });
+  if (e != cudaSuccess) return e;
   const dim3 grid((unsigned)((N + kReuseTok - 1) / kReuseTok), (unsigned)map.n);
-  return launch_pdl(head_reuse_kernel, grid, dim3(128), 0, st, x, cache, map, N, d, w_eT_bf, wp_k,
-                    tab_k, wsum, gram, dsig, vout);
+  return launch_pdl(head_reuse_kernel, grid, dim3(128), kReuseSmem, st, x, cache, map, N, d,
+                    w_eT_bf, wp_k, tab_k, wsum, gram, dsig, vout);
 }
 
 cudaError_t launch_head_compute(const float* hL, float* x, float* xj, __nv_bfloat16* cache,
-                                const SlotMap& map, int N, int d, const float* w_eT,
+                                const SlotMap& map, int N, int d, const __nv_bfloat16* we_frag,
                                 const __nv_bfloat16* wp_k, const float* tab_k, float dsig,
                                 cudaStream_t st, float* vout) {
   if (map.n <= 0) return cudaSuccess;
   if (d % 32 != 0) return cudaErrorInvalidValue;
   const dim3 grid((unsigned)((N + kCmpTok - 1) / kCmpTok), (unsigned)map.n);
-  return launch_pdl(head_compute_kernel, grid, dim3(128), 0, st, hL, x, xj, cache, map, N, d, w_eT,
-                    wp_k, tab_k, dsig, vout);
+  return launch_pdl(head_compute_kernel, grid, dim3(128), 0, st, hL, x, xj, cache, map, N, d,
+                    we_frag, wp_k, tab_k, dsig, vout);
+}
+
+void head_we_fragments(const float* w_eT, int d, uint16_t* out) {
+  // [block][lane][product j][4]: W_e^T rows 2q, 2q + 1, 2q + 8, 2q + 9 at the
+  // column that feeds lane (g, q)'s 8-column product j of the block
+  const int nblk = d / 32;
+  for (int b = 0; b < nblk; ++b)
+    for (int lane = 0; lane < 32; ++lane) {
+      const int g = lane >> 2, q = lane & 3;
+      for (int j = 0; j < 4; ++j) {
+        const int col = 32 * b + 8 * (g >> 1) + 2 * j + (g & 1);
+        const int rows[4] = {2 * q, 2 * q + 1, 2 * q + 8, 2 * q + 9};
+        for (int k = 0; k < 4; ++k) {
+          float v = w_eT[(size_t)rows[k] * d + col];
+          uint32_t u;
+          std::memcpy(&u, &v, 4);
+          const uint32_t lsb = (u >> 16) & 1u;  // round to nearest even
+          out[(((size_t)b * 32 + lane) * 4 + j) * 4 + k] = (uint16_t)((u + 0x7FFFu + lsb) >> 16);
+        }
+      }
+    }
 }
 
 int head_table_floats() { return kHeadTab; }

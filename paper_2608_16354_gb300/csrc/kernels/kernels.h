@@ -100,11 +100,13 @@ cudaError_t launch_head_reuse(float* x, const __nv_bfloat16* cache, const SlotMa
                               const __nv_bfloat16* w_eT_bf, const __nv_bfloat16* wp_k,
                               const float* tab_k, const float* wsum, const float* gram, float dsig,
                               cudaStream_t st, float* vout = nullptr);
-// compute step: writes the cache rows, x_j <- x, x += dsig v
+// compute step: writes the cache rows, x_j <- x, x += dsig v; we_frag: W_e^T
+// (16 x d, bf16) in the fragment order head_we_fragments builds (host)
 cudaError_t launch_head_compute(const float* hL, float* x, float* xj, __nv_bfloat16* cache,
-                                const SlotMap& map, int N, int d, const float* w_eT,
+                                const SlotMap& map, int N, int d, const __nv_bfloat16* we_frag,
                                 const __nv_bfloat16* wp_k, const float* tab_k, float dsig,
                                 cudaStream_t st, float* vout = nullptr);
+void head_we_fragments(const float* w_eT, int d, uint16_t* out /* 16 d values */);
 // vout != NULL (both): write the velocity v[scene][tok][c] instead of the
 // Euler update (x is left as it is; the compute step still sets x_j = x).
 // guidance: x_s += dsig (v_u + g (v_c - v_u)), v_c = v[s], v_u = v[B + s]

@@ -63,7 +63,7 @@ struct dc_model {
   // tensor-core interface (bf16 models, C = 16): W_e^T in bf16, its row
   // sums, and per (step, scene) head tables of the call
   bool head_tc = false;
-  __nv_bfloat16 *w_eT_bf = nullptr, *head_wp = nullptr, *cond_xs = nullptr;
+  __nv_bfloat16 *w_eT_bf = nullptr, *head_wp = nullptr, *cond_xs = nullptr, *we_frag = nullptr;
   CUtensorMap tm_ada, tm_xs;  // adaLN weight and the split activations (bf16 models)
   float *wsum = nullptr, *head_tab = nullptr;
   CUtensorMap tm_a, tm_oact, tm_m, tm_qkv, tm_u32, tm_h32;
@@ -423,8 +423,8 @@ dc_status enqueue_compute(dc_model* m, float* lat, const float* mod_k, const Slo
   if (m->head_tc && sizeof(T) == 2) {
     DC_LAUNCH(DC_PROF_FINAL, 4.0 * M * d * m->C, 4.0 * Md + E * Md + 12.0 * M * m->C,
               dc::launch_head_compute(m->h, lat, m->xj, reinterpret_cast<__nv_bfloat16*>(m->r), map,
-                                      N, d, m->w_eT, head_wp_k(m, k, Bi), head_tab_k(m, k, Bi), dsig,
-                                      st, vout));
+                                      N, d, m->we_frag, head_wp_k(m, k, Bi), head_tab_k(m, k, Bi),
+                                      dsig, st, vout));
   } else {
     DC_LAUNCH(DC_PROF_FINAL, 4.0 * M * d * m->C, 4.0 * Md + E * Md + 12.0 * M * m->C,
               dc::launch_final_compute<T>(m->h, m->w_eT, lat, m->xj, static_cast<T*>(m->r), map, N,
@@ -1185,7 +1185,7 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
       {(void**)&m->err_d, 256}, {(void**)&m->w_eT, (size_t)m->C * d * 4},
       {(void**)&m->gram, (size_t)m->C * m->C * 4}, {(void**)&m->gp, N * m->C * 4},
       {(void**)&m->gs, N * 4}, {(void**)&m->w_eT_bf, (size_t)m->C * d * 2},
-      {(void**)&m->wsum, (size_t)m->C * 4},
+      {(void**)&m->wsum, (size_t)m->C * 4}, {(void**)&m->we_frag, (size_t)m->C * d * 2},
       {(void**)&m->head_wp, m->head_tc ? K * B * 32 * d * 2 : 0},
       {(void**)&m->head_tab, m->head_tc ? K * B * (size_t)dc::head_table_floats() * 4 : 0},
       {(void**)&m->cond_xs, m->bf16 ? cond_groups(K * B) * 2 * dc::cond_tc_group_rows() * d * 2 : 0}};
@@ -1220,6 +1220,8 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
       for (int e = 0; e < D; ++e) acc += (double)we[(size_t)e * C + c];
       wsum[c] = (float)acc;
     }
+    std::vector<uint16_t> we_frag(m->head_tc ? (size_t)C * D : 0);
+    if (m->head_tc) dc::head_we_fragments(weT.data(), D, we_frag.data());
     for (int a = 0; a < C; ++a)
       for (int b = 0; b < C; ++b) {
         double acc = 0.0;
@@ -1250,7 +1252,9 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
         cudaMemcpy(m->gp, gp.data(), gp.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
         cudaMemcpy(m->gs, gs.data(), gs.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
         cudaMemcpy(m->w_eT_bf, weT_bf.data(), weT_bf.size() * 2, cudaMemcpyHostToDevice) != cudaSuccess ||
-        cudaMemcpy(m->wsum, wsum.data(), wsum.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess) {
+        cudaMemcpy(m->wsum, wsum.data(), wsum.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
+        (m->head_tc && cudaMemcpy(m->we_frag, we_frag.data(), we_frag.size() * 2,
+                                  cudaMemcpyHostToDevice) != cudaSuccess)) {
       dc::set_error("upload of the derived tables failed");
       return fail(DC_ERR_CUDA);
     }
