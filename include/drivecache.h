@@ -459,7 +459,7 @@ dc_status dc_attention(int dtype, const void* qkv, int slots, int heads, int n_t
  * recording; dc_profile(m, 0) stops.  dc_profile_read fills DC_PROF_N
  * entries per array (any may be NULL). */
 enum {
-  DC_PROF_CONDITION = 0, /* timestep/trajectory MLPs + adaLN modulation table */
+  DC_PROF_CONDITION = 0, /* adaLN modulation table (activations split + product) */
   DC_PROF_EMBED,         /* u = x W_e^T + b_e + pos */
   DC_PROF_LN,            /* adaLN LayerNorm + modulation */
   DC_PROF_GEMM_QKV,      /* tcgen05 GEMM, QKV scatter epilogue */
@@ -473,6 +473,8 @@ enum {
   DC_PROF_JVP_ATTENTION, /* dc_anchor_response: attention and its tangent (fp32) */
   DC_PROF_JVP_GEMM,      /* dc_anchor_response: linear layers and their tangents (fp32) */
   DC_PROF_JVP_OTHER,     /* dc_anchor_response: LayerNorm, embedding, interface, updates */
+  DC_PROF_COND_MLP,      /* the rest of the conditioning: timestep/trajectory MLPs before the
+                            adaLN table and the per-step head tables after it */
   DC_PROF_N
 };
 dc_status dc_profile(dc_model* m, int enable);

@@ -483,7 +483,7 @@ def attention(qkv, slots, heads, n_tokens, head_dim, out, stream=None):
 
 PROF_NAMES = ["condition", "embed", "ln_mod", "gemm_qkv", "attention", "gemm_out", "gemm_mlp1",
               "gemm_mlp2", "final_compute", "reuse", "drift", "jvp_attention", "jvp_gemm",
-              "jvp_other"]
+              "jvp_other", "cond_mlp"]
 
 
 def set_wait_limit(model: Model, ns):

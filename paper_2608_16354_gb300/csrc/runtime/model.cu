@@ -289,6 +289,11 @@ dc_status enqueue_conditioning(dc_model* m, int B, int K, cudaStream_t st) {
   DC_CK(dc::launch_pose_features(m->poses_d, B, m->P, m->pose_f, st));
   DC_CK(dc::launch_rows_linear<float>(m->pose_f, B, 3 * m->P, m->w_traj, m->b_traj, d, m->traj, 0,
                                       st));
+  // algorithmic work: the small MLPs' weights read once
+  DC_TRY(prof_stop(m, DC_PROF_COND_MLP, st, ev,
+                   2.0 * K * (256.0 * d + (double)d * d) + 2.0 * B * 3.0 * m->P * d,
+                   4.0 * (256.0 * d + (double)d * d + 3.0 * m->P * d)));
+  DC_TRY(prof_start(m, st, &ev));
   if (m->bf16) {
     // the adaLN weight streamed once through the tensor cores
     DC_CK(dc::launch_cond_split(m->temb, m->traj, K, B, d, m->cond_xs, st));
@@ -299,19 +304,19 @@ dc_status enqueue_conditioning(dc_model* m, int B, int K, cudaStream_t st) {
     DC_CK(dc::launch_rows_linear<T>(m->silu_c, K * B, d, static_cast<const T*>(m->w_ada), m->b_ada,
                                     m->mod_stride, m->mod, 0, st));
   }
-  if (m->head_tc) {
-    DC_CK(dc::launch_head_tables(m->mod, K * B, m->mod_stride, 6 * m->L * d, d, m->w_f, m->b_f,
-                                 m->w_eT, m->head_wp, m->head_tab, st));
-    m->launches += 1;
-  }
   // algorithmic bytes: the adaLN weight table read once + the table written
   DC_TRY(prof_stop(m, DC_PROF_CONDITION, st, ev, 2.0 * K * B * d * m->mod_stride,
                    (double)m->mod_stride * d * m->elt + 4.0 * K * B * m->mod_stride));
   m->launches += 7;
+  if (m->head_tc) {
+    DC_LAUNCH(DC_PROF_COND_MLP, 2.0 * K * B * 18.0 * 16.0 * d, 4.0 * K * B * 64.0 * d,
+              dc::launch_head_tables(m->mod, K * B, m->mod_stride, 6 * m->L * d, d, m->w_f, m->b_f,
+                                     m->w_eT, m->head_wp, m->head_tab, st));
+    m->launches += 1;
+  }
   return DC_OK;
 }
 
-// One full backbone pass + interface + Euler for the scenes in `map`.
 // This step's head tables (tensor-core interface): items (k - 1) * Bi + scene.
 const __nv_bfloat16* head_wp_k(const dc_model* m, int k, int Bi) {
   return m->head_wp + (size_t)(k - 1) * Bi * 32 * m->d;
