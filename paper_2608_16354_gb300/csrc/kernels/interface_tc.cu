@@ -45,6 +45,7 @@ namespace {
 
 constexpr int kHC = 16;          // latent channels the tensor-core interface supports
 constexpr int kHeadTab = 2 * kHC + kHC * kHC;  // S', beta, G_s per (step, scene)
+constexpr int kBRows = 3 * kHC;  // B rows per (step, scene): W_e^T, W' hi, W' lo
 
 __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
                                                uint32_t a3, uint32_t b0, uint32_t b1) {
@@ -96,8 +97,9 @@ __device__ __forceinline__ void split_pair(float a, float b, uint32_t* hi, uint3
 
 // ------------------------------------------------ per (step, scene) tables
 
-// One CTA per (step, scene) item: W' = (1 + scale) W_f as bf16 hi and lo
-// halves [32][d] (rows 0-15 hi, 16-31 lo), and S', beta, G_s (fp32).
+// One CTA per (step, scene) item: the reuse step's B rows [48][d] in bf16 --
+// W_e^T (rows 0-15), W' = (1 + scale) W_f as hi (16-31) and lo (32-47)
+// halves -- and S', beta, G_s (fp32).
 __global__ void __launch_bounds__(256) head_tables_kernel(
     const float* __restrict__ mod, int mod_stride, int fin_off, int d,
     const float* __restrict__ w_f, const float* __restrict__ b_f, const float* __restrict__ w_eT,
@@ -105,13 +107,14 @@ __global__ void __launch_bounds__(256) head_tables_kernel(
   const int item = blockIdx.x;
   const float* sh = mod + (size_t)item * mod_stride + fin_off;
   const float* sc = sh + d;
-  __nv_bfloat16* w = wp + (size_t)item * 2 * kHC * d;
+  __nv_bfloat16* w = wp + (size_t)item * kBRows * d;
   for (int i = threadIdx.x; i < kHC * d; i += blockDim.x) {
     const int c = i / d, e = i - c * d;
     const float v = (1.f + sc[e]) * w_f[i];
     const __nv_bfloat16 hi = __float2bfloat16_rn(v);
-    w[(size_t)c * d + e] = hi;
-    w[(size_t)(kHC + c) * d + e] = __float2bfloat16_rn(v - __bfloat162float(hi));
+    w[(size_t)c * d + e] = __float2bfloat16_rn(w_eT[i]);
+    w[(size_t)(kHC + c) * d + e] = hi;
+    w[(size_t)(2 * kHC + c) * d + e] = __float2bfloat16_rn(v - __bfloat162float(hi));
   }
   float* t = tab + (size_t)item * kHeadTab;
   const int a = threadIdx.x >> 4, c = threadIdx.x & 15;  // G_s[a][c]
@@ -136,11 +139,9 @@ __global__ void __launch_bounds__(256) head_tables_kernel(
 constexpr int kReuseWarps = 4;                // one 16-token tile per warp
 constexpr int kReuseTok = 16 * kReuseWarps;   // tokens per CTA on reuse steps
 constexpr int kReuseStages = 12;              // 32-column blocks in flight per CTA
-constexpr int kBRows = 48;                    // B rows: W_e^T (16), W' hi (16), W' lo (16)
 // one stage: each warp's A block (16 rows x 64 B) and the shared B block (48 x 64 B)
 constexpr int kReuseStageBytes = kReuseWarps * 1024 + kBRows * 64;
 constexpr int kReuseSmem = kReuseStages * kReuseStageBytes;
-constexpr int kCmpTok = 16;    // tokens per CTA on compute steps (one m16 tile per warp)
 
 // Reuse step of the scenes in `map`: h = x W_e^T + c_j, v = head(h), x += dsig v
 // (or v to vout).  wp_k / tab_k: this step's tables, indexed by scene.  Each
@@ -149,9 +150,9 @@ constexpr int kCmpTok = 16;    // tokens per CTA on compute steps (one m16 tile 
 // kReuseStages-deep cp.async ring.
 __global__ void __launch_bounds__(128) head_reuse_kernel(
     float* __restrict__ x, const __nv_bfloat16* __restrict__ cache, SlotMap map, int N, int d,
-    const __nv_bfloat16* __restrict__ w_eT_bf, const __nv_bfloat16* __restrict__ wp_k,
-    const float* __restrict__ tab_k, const float* __restrict__ wsum, const float* __restrict__ gram,
-    float dsig, float* __restrict__ vout) {
+    const __nv_bfloat16* __restrict__ wp_k, const float* __restrict__ tab_k,
+    const float* __restrict__ wsum, const float* __restrict__ gram, float dsig,
+    float* __restrict__ vout) {
   pdl_trigger();
   pdl_wait();
   extern __shared__ __align__(16) uint8_t rsm[];
@@ -165,7 +166,7 @@ __global__ void __launch_bounds__(128) head_reuse_kernel(
   for (int i = tid; i < kHC * kHC; i += blockDim.x) stab[kHeadTab + kHC + i] = gram[i];
 
   const __nv_bfloat16* cs = cache + (size_t)scene * N * d;
-  const __nv_bfloat16* wk = wp_k + (size_t)scene * 2 * kHC * d;
+  const __nv_bfloat16* wk = wp_k + (size_t)scene * kBRows * d;
   int row[2];
   bool ok[2];
 #pragma unroll
@@ -188,11 +189,7 @@ __global__ void __launch_bounds__(128) head_reuse_kernel(
 #pragma unroll
     for (int k = 0; k < 2; ++k) {
       const int c = tid + 128 * k;
-      if (c < kBRows * 4) {
-        const int r = c >> 2, piece = c & 3;
-        const __nv_bfloat16* src = r < kHC ? w_eT_bf + (size_t)r * d : wk + (size_t)(r - kHC) * d;
-        cp_async16(bb + c, src + (b << 5) + (piece << 3));
-      }
+      if (c < kBRows * 4) cp_async16(bb + c, wk + (size_t)(c >> 2) * d + (b << 5) + ((c & 3) << 3));
     }
   };
   float D[6][4];
@@ -200,7 +197,11 @@ __global__ void __launch_bounds__(128) head_reuse_kernel(
   for (int j = 0; j < 6; ++j)
 #pragma unroll
     for (int t = 0; t < 4; ++t) D[j][t] = 0.f;
-  float s1[2] = {0.f, 0.f}, s2[2] = {0.f, 0.f};
+  // per-token sum c (a B column of ones) and sum c^2 (the diagonal of the
+  // tile's Gram matrix c c^T, whose B fragments are the A fragments' own
+  // rows: tokens 0-7 of the tile, then 8-15), on the tensor cores as well
+  float GS[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}}, S1[4] = {0.f, 0.f, 0.f, 0.f};
+  const uint32_t ones = g == 0 ? 0x3F803F80u : 0u;  // bf16 (1, 1) in column 0
   const int nblk = d >> 5;
 #pragma unroll 1
   for (int i = 0; i < kReuseStages - 1; ++i) {
@@ -221,15 +222,6 @@ __global__ void __launch_bounds__(128) head_reuse_kernel(
     uint4 bw[6];
 #pragma unroll
     for (int j = 0; j < 6; ++j) bw[j] = bb[(8 * j + g) * 4 + q];
-    {
-      const uint32_t w8[8] = {av0.x, av0.y, av0.z, av0.w, av1.x, av1.y, av1.z, av1.w};
-#pragma unroll
-      for (int p = 0; p < 8; ++p) {
-        const float2 f = unpack_bf2(w8[p]);
-        s1[p >> 2] += f.x + f.y;
-        s2[p >> 2] = fmaf(f.x, f.x, fmaf(f.y, f.y, s2[p >> 2]));
-      }
-    }
 #pragma unroll
     for (int s = 0; s < 2; ++s) {
       const uint32_t a0 = s ? av0.z : av0.x;  // row g, cols 4s + 0, 1
@@ -239,16 +231,14 @@ __global__ void __launch_bounds__(128) head_reuse_kernel(
 #pragma unroll
       for (int j = 0; j < 6; ++j)
         mma_bf16_16816(D[j], a0, a1, a2, a3, s ? bw[j].z : bw[j].x, s ? bw[j].w : bw[j].y);
+      mma_bf16_16816(GS[0], a0, a1, a2, a3, a0, a2);
+      mma_bf16_16816(GS[1], a0, a1, a2, a3, a1, a3);
+      mma_bf16_16816(S1, a0, a1, a2, a3, ones, ones);
     }
   }
   cp_async_wait<0>();
-  // lanes 4 g .. 4 g + 3 hold the same rows: add their column sums
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
-    s1[h] += __shfl_xor_sync(0xffffffffu, s1[h], 1);
-    s1[h] += __shfl_xor_sync(0xffffffffu, s1[h], 2);
-    s2[h] += __shfl_xor_sync(0xffffffffu, s2[h], 1);
-    s2[h] += __shfl_xor_sync(0xffffffffu, s2[h], 2);
     float* pp = part[warp][8 * h + g];
 #pragma unroll
     for (int j = 0; j < 2; ++j)
@@ -257,10 +247,10 @@ __global__ void __launch_bounds__(128) head_reuse_kernel(
         pp[8 * j + 2 * q + t] = D[j][2 * h + t];
         pp[kHC + 8 * j + 2 * q + t] = D[2 + j][2 * h + t] + D[4 + j][2 * h + t];
       }
-    if (q == 0) {
-      pp[2 * kHC] = s1[h];
-      pp[2 * kHC + 1] = s2[h];
-    }
+    // token 8 h + g: sum c in column 0 of the ones product (lane q = 0), sum
+    // c^2 on the diagonal of the Gram product of its half (lane q = g / 2)
+    if (q == 0) pp[2 * kHC] = S1[2 * h];
+    if (q == (g >> 1)) pp[2 * kHC + 1] = (g & 1) ? GS[h][2 * h + 1] : GS[h][2 * h];
   }
   __syncwarp();
 
@@ -323,10 +313,22 @@ __global__ void __launch_bounds__(128) head_reuse_kernel(
 
 // ------------------------------------------------------------- compute step
 
+constexpr int kCmpWarps = 4;                 // one 16-token tile per warp
+constexpr int kCmpTok = 16 * kCmpWarps;      // tokens per CTA on compute steps
+constexpr int kCmpStages = 8;                // 32-column blocks in flight per CTA
+// one stage: each warp's h_L block (16 rows x 128 B), the W' rows (32 x 64 B)
+// and the block's W_e^T fragments (32 lanes x 32 B)
+constexpr int kCmpStageBytes = kCmpWarps * 2048 + 2 * kHC * 64 + 1024;
+constexpr int kCmpSmem = kCmpStages * kCmpStageBytes;
+
 // Compute step of the scenes in `map` (h_L rows packed by slot): the cache
 // row c = h_L - x W_e^T is written, v = head(h_L), x_j <- x, x += dsig v (or
-// v to vout).  x W_e^T is formed in fp32 from W_e^T [C][d] (16 FMAs per
-// element), the head on the tensor cores.
+// v to vout).  Each warp takes 16 tokens over all of d; per 32-column block
+// the CTA stages the warps' h_L rows, the W' rows and the W_e^T fragments
+// (shared by the four warps) in a kCmpStages-deep cp.async ring.  x W_e^T
+// runs on the tensor cores with K = C = 16: the fragment-ordered W_e^T puts
+// its four 8-column products on the thread's own columns (product j:
+// columns e + 2 j, e + 2 j + 1 of rows g and g + 8).
 __global__ void __launch_bounds__(128) head_compute_kernel(
     const float* __restrict__ hL, float* __restrict__ x, float* __restrict__ xj,
     __nv_bfloat16* __restrict__ cache, SlotMap map, int N, int d,
@@ -334,14 +336,15 @@ __global__ void __launch_bounds__(128) head_compute_kernel(
     const float* __restrict__ tab_k, float dsig, float* __restrict__ vout) {
   pdl_trigger();
   pdl_wait();
-  __shared__ float part[4][kCmpTok][kHC + 2];  // per warp: P, sum h, sum h^2
-  __shared__ uint4 ring[4][kRing][4][32];       // per warp: (row half, 16-byte piece) x lanes
-  __shared__ float stab[2 * kHC];              // S', beta
+  extern __shared__ __align__(16) uint8_t csm[];
+  __shared__ float part[kCmpWarps][16][kHC + 2];  // per token: P, sum h, sum h^2
+  __shared__ float stab[2 * kHC];                 // S', beta
   const int slot = blockIdx.y, scene = map.scene[slot];
   const int tok0 = blockIdx.x * kCmpTok;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, q = lane & 3;
-  if (threadIdx.x < 2 * kHC) stab[threadIdx.x] = tab_k[(size_t)scene * kHeadTab + threadIdx.x];
-  const __nv_bfloat16* wk = wp_k + (size_t)scene * 2 * kHC * d;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, q = lane & 3;
+  if (tid < 2 * kHC) stab[tid] = tab_k[(size_t)scene * kHeadTab + tid];
+  const __nv_bfloat16* wk = wp_k + (size_t)scene * kBRows * d + (size_t)kHC * d;  // W' rows
+  const uint8_t* wf = reinterpret_cast<const uint8_t*>(we_frag);
   int row[2];
   bool ok[2];
   // A fragments of x (tokens x channels, hi and lo halves): rows g and
@@ -349,7 +352,7 @@ __global__ void __launch_bounds__(128) head_compute_kernel(
   uint32_t xa_hi[4], xa_lo[4];
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
-    row[h] = tok0 + 8 * h + g;
+    row[h] = tok0 + 16 * warp + 8 * h + g;
     ok[h] = row[h] < N;
     const float* xr = x + ((size_t)scene * N + row[h]) * kHC;
     const float2 p0 = ok[h] ? *reinterpret_cast<const float2*>(xr + 2 * q) : make_float2(0.f, 0.f);
@@ -357,6 +360,22 @@ __global__ void __launch_bounds__(128) head_compute_kernel(
     split_pair(p0.x, p0.y, &xa_hi[h], &xa_lo[h]);
     split_pair(p1.x, p1.y, &xa_hi[2 + h], &xa_lo[2 + h]);
   }
+  // this thread's copies of block b into stage st: its h_L pieces (rows g and
+  // g + 8, 8 fp32 each), W' piece tid (32 rows x 4), fragment piece tid < 64
+  auto fetch = [&](int b, int st) {
+    uint8_t* base = csm + st * kCmpStageBytes;
+    const int e = (b << 5) + (q << 3);
+    uint4* a = reinterpret_cast<uint4*>(base + warp * 2048) + lane;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int h = k >> 1;
+      if (ok[h]) cp_async16(a + 32 * k, hL + ((size_t)slot * N + row[h]) * d + e + 4 * (k & 1));
+      else a[32 * k] = make_uint4(0u, 0u, 0u, 0u);
+    }
+    uint4* bb = reinterpret_cast<uint4*>(base + kCmpWarps * 2048);
+    cp_async16(bb + tid, wk + (size_t)(tid >> 2) * d + (b << 5) + ((tid & 3) << 3));
+    if (tid < 64) cp_async16(bb + 128 + tid, wf + (size_t)b * 1024 + tid * 16);
+  };
   float D[4][4];
 #pragma unroll
   for (int j = 0; j < 4; ++j)
@@ -364,50 +383,39 @@ __global__ void __launch_bounds__(128) head_compute_kernel(
     for (int t = 0; t < 4; ++t) D[j][t] = 0.f;
   float s1[2] = {0.f, 0.f}, s2[2] = {0.f, 0.f};
   const int nblk = d >> 5;
-  const int nbw = warp < nblk ? (nblk - 1 - warp) / 4 + 1 : 0;  // blocks of this warp
-  // block i of this warp: rows g and g + 8, 8 fp32 columns each (two 16-byte
-  // copies per row) into ring stage i % kRing
-  auto fetch = [&](int i) {
-    if (i < nbw) {
-      const int e = ((warp + 4 * i) << 5) + (q << 3);
-      uint4* st = &ring[warp][i % kRing][0][lane];
-#pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const int h = k >> 1;
-        if (ok[h]) cp_async16(st + 32 * k, hL + ((size_t)slot * N + row[h]) * d + e + 4 * (k & 1));
-        else st[32 * k] = make_uint4(0u, 0u, 0u, 0u);
-      }
-    }
+#pragma unroll 1
+  for (int i = 0; i < kCmpStages - 1; ++i) {
+    if (i < nblk) fetch(i, i);
     cp_async_commit();
-  };
-#pragma unroll
-  for (int i = 0; i < kRing - 1; ++i) fetch(i);
-  for (int i = 0; i < nbw; ++i) {
-    fetch(i + kRing - 1);
-    const int e = ((warp + 4 * i) << 5) + (q << 3);
-    cp_async_wait<kRing - 1>();
+  }
+#pragma unroll 1
+  for (int b = 0; b < nblk; ++b) {
+    cp_async_wait<kCmpStages - 2>();
+    __syncthreads();
+    const int nb = b + kCmpStages - 1;
+    if (nb < nblk) fetch(nb, nb % kCmpStages);
+    cp_async_commit();
+    const uint8_t* base = csm + (b % kCmpStages) * kCmpStageBytes;
+    const int e = (b << 5) + (q << 3);
     float hv[2][8];
     {
-      const uint4* st = &ring[warp][i % kRing][0][lane];
+      const uint4* a = reinterpret_cast<const uint4*>(base + warp * 2048) + lane;
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
-        const uint4 w = st[32 * k];
+        const uint4 w = a[32 * k];
         float* dst = &hv[k >> 1][4 * (k & 1)];
         dst[0] = __uint_as_float(w.x); dst[1] = __uint_as_float(w.y);
         dst[2] = __uint_as_float(w.z); dst[3] = __uint_as_float(w.w);
       }
     }
+    const uint4* bb = reinterpret_cast<const uint4*>(base + kCmpWarps * 2048);
     uint4 bw[4];  // W' hi (channels 0-7, 8-15), W' lo (0-7, 8-15)
 #pragma unroll
-    for (int j = 0; j < 4; ++j) bw[j] = ld_tab16(wk + (size_t)(8 * j + g) * d + e);
-    // the cache row c = h - x W_e^T: x W_e^T on the tensor cores (K = C = 16),
-    // with the B fragments of this block's W_e^T columns laid out so that the
-    // four 8-column products land on this thread's own 8 columns (product j:
-    // columns e + 2 j, e + 2 j + 1 of rows g and g + 8)
+    for (int j = 0; j < 4; ++j) bw[j] = bb[(8 * j + g) * 4 + q];
+    // the cache row c = h - x W_e^T
     float u[2][8];
     {
-      const uint4* fp = reinterpret_cast<const uint4*>(we_frag) + ((size_t)((warp + 4 * i) * 32 + lane) << 1);
-      const uint4 f0 = __ldg(fp), f1 = __ldg(fp + 1);
+      const uint4 f0 = bb[128 + 2 * lane], f1 = bb[129 + 2 * lane];
       const uint32_t fb[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
@@ -467,39 +475,37 @@ __global__ void __launch_bounds__(128) head_compute_kernel(
       pp[kHC + 1] = s2[h];
     }
   }
-  __syncthreads();
+  __syncwarp();
 
-  // finish: 4 threads per token (64 threads), 4 channels each
-  if (threadIdx.x < 4 * kCmpTok) {
-    const int tt = threadIdx.x >> 2, cq = threadIdx.x & 3;
-    const int tok = tok0 + tt;
-    if (tok < N) {
-      float sum1 = 0.f, sum2 = 0.f;
+  // finish: two lanes per token of this warp, 8 channels each
+  const int tt = lane >> 1, ch = lane & 1;
+  const int tok = tok0 + 16 * warp + tt;
+  if (tok < N) {
+    const float* pt = part[warp][tt];
+    const float mu = pt[kHC] / (float)d;
+    const float var = fmaxf(pt[kHC + 1] / (float)d - mu * mu, 0.f);
+    const float rs = rsqrtf(var + 1e-6f);
+    float vv[8];
 #pragma unroll
-      for (int w = 0; w < 4; ++w) {
-        sum1 += part[w][tt][kHC];
-        sum2 += part[w][tt][kHC + 1];
-      }
-      const float mu = sum1 / (float)d;
-      const float var = fmaxf(sum2 / (float)d - mu * mu, 0.f);
-      const float rs = rsqrtf(var + 1e-6f);
-      float vv[4];
-#pragma unroll
-      for (int cc = 0; cc < 4; ++cc) {
-        const int c = 4 * cq + cc;
-        const float P = ((part[0][tt][c] + part[1][tt][c]) + part[2][tt][c]) + part[3][tt][c];
-        vv[cc] = fmaf(rs, P - mu * stab[c], stab[kHC + c]);
-      }
-      const size_t xi = ((size_t)scene * N + tok) * kHC + 4 * cq;
-      const float4 xo = *reinterpret_cast<const float4*>(x + xi);
-      *reinterpret_cast<float4*>(xj + xi) = xo;
-      if (vout) {
-        *reinterpret_cast<float4*>(vout + xi) = make_float4(vv[0], vv[1], vv[2], vv[3]);
-      } else {
-        *reinterpret_cast<float4*>(x + xi) =
-            make_float4(fmaf(dsig, vv[0], xo.x), fmaf(dsig, vv[1], xo.y), fmaf(dsig, vv[2], xo.z),
-                        fmaf(dsig, vv[3], xo.w));
-      }
+    for (int cc = 0; cc < 8; ++cc) {
+      const int c = 8 * ch + cc;
+      vv[cc] = fmaf(rs, pt[c] - mu * stab[c], stab[kHC + c]);
+    }
+    const size_t xi = ((size_t)scene * N + tok) * kHC + 8 * ch;
+    const float4 xo0 = *reinterpret_cast<const float4*>(x + xi);
+    const float4 xo1 = *reinterpret_cast<const float4*>(x + xi + 4);
+    *reinterpret_cast<float4*>(xj + xi) = xo0;
+    *reinterpret_cast<float4*>(xj + xi + 4) = xo1;
+    if (vout) {
+      *reinterpret_cast<float4*>(vout + xi) = make_float4(vv[0], vv[1], vv[2], vv[3]);
+      *reinterpret_cast<float4*>(vout + xi + 4) = make_float4(vv[4], vv[5], vv[6], vv[7]);
+    } else {
+      *reinterpret_cast<float4*>(x + xi) =
+          make_float4(fmaf(dsig, vv[0], xo0.x), fmaf(dsig, vv[1], xo0.y), fmaf(dsig, vv[2], xo0.z),
+                      fmaf(dsig, vv[3], xo0.w));
+      *reinterpret_cast<float4*>(x + xi + 4) =
+          make_float4(fmaf(dsig, vv[4], xo1.x), fmaf(dsig, vv[5], xo1.y), fmaf(dsig, vv[6], xo1.z),
+                      fmaf(dsig, vv[7], xo1.w));
     }
   }
 }
@@ -515,9 +521,8 @@ cudaError_t launch_head_tables(const float* mod, int n_items, int mod_stride, in
 }
 
 cudaError_t launch_head_reuse(float* x, const __nv_bfloat16* cache, const SlotMap& map, int N, int d,
-                              const __nv_bfloat16* w_eT_bf, const __nv_bfloat16* wp_k,
-                              const float* tab_k, const float* wsum, const float* gram, float dsig,
-                              cudaStream_t st, float* vout) {
+                              const __nv_bfloat16* wp_k, const float* tab_k, const float* wsum,
+                              const float* gram, float dsig, cudaStream_t st, float* vout) {
   if (map.n <= 0) return cudaSuccess;
   if (d % 32 != 0) return cudaErrorInvalidValue;
   static std::atomic<unsigned long long> configured{0};
@@ -527,8 +532,8 @@ cudaError_t launch_head_reuse(float* x, const __nv_bfloat16* cache, const SlotMa
   });
   if (e != cudaSuccess) return e;
   const dim3 grid((unsigned)((N + kReuseTok - 1) / kReuseTok), (unsigned)map.n);
-  return launch_pdl(head_reuse_kernel, grid, dim3(128), kReuseSmem, st, x, cache, map, N, d,
-                    w_eT_bf, wp_k, tab_k, wsum, gram, dsig, vout);
+  return launch_pdl(head_reuse_kernel, grid, dim3(128), kReuseSmem, st, x, cache, map, N, d, wp_k,
+                    tab_k, wsum, gram, dsig, vout);
 }
 
 cudaError_t launch_head_compute(const float* hL, float* x, float* xj, __nv_bfloat16* cache,
@@ -537,8 +542,14 @@ cudaError_t launch_head_compute(const float* hL, float* x, float* xj, __nv_bfloa
                                 cudaStream_t st, float* vout) {
   if (map.n <= 0) return cudaSuccess;
   if (d % 32 != 0) return cudaErrorInvalidValue;
+  static std::atomic<unsigned long long> configured{0};
+  const cudaError_t e = configure_once_per_device(configured, [] {
+    return cudaFuncSetAttribute(head_compute_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                kCmpSmem);
+  });
+  if (e != cudaSuccess) return e;
   const dim3 grid((unsigned)((N + kCmpTok - 1) / kCmpTok), (unsigned)map.n);
-  return launch_pdl(head_compute_kernel, grid, dim3(128), 0, st, hL, x, xj, cache, map, N, d,
+  return launch_pdl(head_compute_kernel, grid, dim3(128), kCmpSmem, st, hL, x, xj, cache, map, N, d,
                     we_frag, wp_k, tab_k, dsig, vout);
 }
 
@@ -564,5 +575,6 @@ void head_we_fragments(const float* w_eT, int d, uint16_t* out) {
 }
 
 int head_table_floats() { return kHeadTab; }
+int head_b_rows() { return kBRows; }
 
 }  // namespace dc

@@ -88,18 +88,19 @@ template <typename T>
 cudaError_t launch_cache_to_residual(const T* c, const float* b_e, const T* pos, int N, int d, T* out,
                                      cudaStream_t st);
 // Tensor-core interface of bf16 models with C = 16 (interface_tc.cu).  Per
-// (step, scene) item of the call's modulation table: W' = (1 + scale) W_f as
-// bf16 hi + lo rows [32][d], and S', beta, G_s (head_table_floats() fp32).
+// (step, scene) item of the call's modulation table: head_b_rows() bf16 rows
+// of d (W_e^T, then W' = (1 + scale) W_f as hi and lo halves), and S', beta,
+// G_s (head_table_floats() fp32).
 int head_table_floats();
+int head_b_rows();
 cudaError_t launch_head_tables(const float* mod, int n_items, int mod_stride, int fin_off, int d,
                                const float* w_f, const float* b_f, const float* w_eT,
                                __nv_bfloat16* wp, float* tab, cudaStream_t st);
-// reuse step (wp_k, tab_k: the step's tables, indexed by scene; w_eT_bf:
-// W_e^T [16][d] bf16; wsum: row sums of W_e^T; gram: W_e^T W_e [16][16])
+// reuse step (wp_k, tab_k: the step's tables, indexed by scene; wsum: row
+// sums of W_e^T; gram: W_e^T W_e [16][16])
 cudaError_t launch_head_reuse(float* x, const __nv_bfloat16* cache, const SlotMap& map, int N, int d,
-                              const __nv_bfloat16* w_eT_bf, const __nv_bfloat16* wp_k,
-                              const float* tab_k, const float* wsum, const float* gram, float dsig,
-                              cudaStream_t st, float* vout = nullptr);
+                              const __nv_bfloat16* wp_k, const float* tab_k, const float* wsum,
+                              const float* gram, float dsig, cudaStream_t st, float* vout = nullptr);
 // compute step: writes the cache rows, x_j <- x, x += dsig v; we_frag: W_e^T
 // (16 x d, bf16) in the fragment order head_we_fragments builds (host)
 cudaError_t launch_head_compute(const float* hL, float* x, float* xj, __nv_bfloat16* cache,

@@ -63,7 +63,7 @@ struct dc_model {
   // tensor-core interface (bf16 models, C = 16): W_e^T in bf16, its row
   // sums, and per (step, scene) head tables of the call
   bool head_tc = false;
-  __nv_bfloat16 *w_eT_bf = nullptr, *head_wp = nullptr, *cond_xs = nullptr, *we_frag = nullptr;
+  __nv_bfloat16 *head_wp = nullptr, *cond_xs = nullptr, *we_frag = nullptr;
   CUtensorMap tm_ada, tm_xs;  // adaLN weight and the split activations (bf16 models)
   float *wsum = nullptr, *head_tab = nullptr;
   CUtensorMap tm_a, tm_oact, tm_m, tm_qkv, tm_u32, tm_h32;
@@ -319,7 +319,7 @@ dc_status enqueue_conditioning(dc_model* m, int B, int K, cudaStream_t st) {
 
 // This step's head tables (tensor-core interface): items (k - 1) * Bi + scene.
 const __nv_bfloat16* head_wp_k(const dc_model* m, int k, int Bi) {
-  return m->head_wp + (size_t)(k - 1) * Bi * 32 * m->d;
+  return m->head_wp + (size_t)(k - 1) * Bi * dc::head_b_rows() * m->d;
 }
 const float* head_tab_k(const dc_model* m, int k, int Bi) {
   return m->head_tab + (size_t)(k - 1) * Bi * dc::head_table_floats();
@@ -450,8 +450,8 @@ dc_status enqueue_reuse(dc_model* m, float* lat, const float* mod_k, const SlotM
   if (m->head_tc && sizeof(T) == 2) {
     DC_LAUNCH(DC_PROF_REUSE, 2.0 * M * m->d * 3 * m->C, M * ((double)m->d * m->elt + 12.0 * m->C),
               dc::launch_head_reuse(lat, reinterpret_cast<const __nv_bfloat16*>(m->r), map, m->N,
-                                    m->d, m->w_eT_bf, head_wp_k(m, k, Bi), head_tab_k(m, k, Bi),
-                                    m->wsum, m->gram, dsig, st, vout));
+                                    m->d, head_wp_k(m, k, Bi), head_tab_k(m, k, Bi), m->wsum,
+                                    m->gram, dsig, st, vout));
   } else {
     DC_LAUNCH(DC_PROF_REUSE, 4.0 * M * m->d * m->C, M * ((double)m->d * m->elt + 12.0 * m->C),
               dc::launch_final_reuse<T>(lat, static_cast<const T*>(m->r), m->w_eT, map, m->N, m->C,
@@ -1189,9 +1189,9 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
       {(void**)&m->poses_d, B * m->P * 3 * 8}, {(void**)&m->sig_d, (K + 1) * 8},
       {(void**)&m->err_d, 256}, {(void**)&m->w_eT, (size_t)m->C * d * 4},
       {(void**)&m->gram, (size_t)m->C * m->C * 4}, {(void**)&m->gp, N * m->C * 4},
-      {(void**)&m->gs, N * 4}, {(void**)&m->w_eT_bf, (size_t)m->C * d * 2},
+      {(void**)&m->gs, N * 4},
       {(void**)&m->wsum, (size_t)m->C * 4}, {(void**)&m->we_frag, (size_t)m->C * d * 2},
-      {(void**)&m->head_wp, m->head_tc ? K * B * 32 * d * 2 : 0},
+      {(void**)&m->head_wp, m->head_tc ? K * B * (size_t)dc::head_b_rows() * d * 2 : 0},
       {(void**)&m->head_tab, m->head_tc ? K * B * (size_t)dc::head_table_floats() * 4 : 0},
       {(void**)&m->cond_xs, m->bf16 ? cond_groups(K * B) * 2 * dc::cond_tc_group_rows() * d * 2 : 0}};
   size_t wsb = 0;
@@ -1214,11 +1214,9 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
     const float* be = host_weights + (size_t)D * C;  // b_embed [d]
     const float* ps = be + D;                        // pos [N][d]
     std::vector<float> weT((size_t)C * D), gram((size_t)C * C), gp(N * C), gs(N), wsum(C);
-    std::vector<uint16_t> weT_bf((size_t)C * D);
     for (int e = 0; e < D; ++e)
       for (int c = 0; c < C; ++c) {
         weT[(size_t)c * D + e] = we[(size_t)e * C + c];
-        weT_bf[(size_t)c * D + e] = f2bf_host(we[(size_t)e * C + c]);
       }
     for (int c = 0; c < C; ++c) {
       double acc = 0.0;
@@ -1256,7 +1254,6 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
         cudaMemcpy(m->gram, gram.data(), gram.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
         cudaMemcpy(m->gp, gp.data(), gp.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
         cudaMemcpy(m->gs, gs.data(), gs.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
-        cudaMemcpy(m->w_eT_bf, weT_bf.data(), weT_bf.size() * 2, cudaMemcpyHostToDevice) != cudaSuccess ||
         cudaMemcpy(m->wsum, wsum.data(), wsum.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
         (m->head_tc && cudaMemcpy(m->we_frag, we_frag.data(), we_frag.size() * 2,
                                   cudaMemcpyHostToDevice) != cudaSuccess)) {
