@@ -51,8 +51,10 @@ struct AttCfg {
   // once S_t is in registers, and S_{t,j+1} is issued after PV_{t,j} (the
   // MMAs of one thread run in issue order).
   static constexpr bool kAliasP = DHP == 128 && NQ == 2;
-  // ring depths (key, value): deeper rings measured no faster at dh 64
-  static constexpr int kKStages = kAliasP ? 2 : 3;
+  // ring depths (key, value): deeper rings measured no faster at dh 64; with
+  // two tiles at dh 128 the key ring keeps three stages (an S product waits
+  // for its key tile, a PV product only after the softmax) within 227 KB
+  static constexpr int kKStages = 3;
   static constexpr int kVStages = kAliasP ? 2 : 3;
   static constexpr int kTileBytes = kAtoms * 16384;   // 128 rows x DHP bf16
   static constexpr int kOffQ = 0;                              // NQ tiles
