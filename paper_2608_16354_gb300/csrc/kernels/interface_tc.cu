@@ -56,11 +56,9 @@ __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint3
       : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
 }
 
-// Streamed rows go through a per-warp ring in shared memory filled with
-// cp.async (16 bytes per thread and row, read back by the same thread), so
-// that several 32-column blocks are in flight per warp without holding them
-// in registers; tables are read through L1.
-constexpr int kRing = 4;  // blocks in flight per warp
+// Streamed rows and the B rows go through a shared-memory ring filled with
+// cp.async (16 bytes per thread and copy), so that several 32-column blocks
+// are in flight per warp without holding them in registers.
 
 __device__ __forceinline__ void cp_async16(void* smem_dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem_dst)), "l"(src)
@@ -73,17 +71,10 @@ template <int N>
 __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
-__device__ __forceinline__ uint4 ld_tab16(const void* p) {
-  return __ldg(reinterpret_cast<const uint4*>(p));
-}
 
 __device__ __forceinline__ uint32_t pack_bf2(float lo_elem, float hi_elem) {
   __nv_bfloat162 t = __floats2bfloat162_rn(lo_elem, hi_elem);
   return *reinterpret_cast<uint32_t*>(&t);
-}
-__device__ __forceinline__ float2 unpack_bf2(uint32_t w) {
-  __nv_bfloat162 t = *reinterpret_cast<__nv_bfloat162*>(&w);
-  return __bfloat1622float2(t);
 }
 // v = hi + lo with hi = bf16(v), lo = bf16(v - hi), for a pair of values
 __device__ __forceinline__ void split_pair(float a, float b, uint32_t* hi, uint32_t* lo) {
@@ -136,19 +127,25 @@ __global__ void __launch_bounds__(256) head_tables_kernel(
 
 // ---------------------------------------------------------------- reuse step
 
-constexpr int kReuseWarps = 4;                // one 16-token tile per warp
-constexpr int kReuseTok = 16 * kReuseWarps;   // tokens per CTA on reuse steps
-constexpr int kReuseStages = 12;              // 32-column blocks in flight per CTA
-// one stage: each warp's A block (16 rows x 64 B) and the shared B block (48 x 64 B)
-constexpr int kReuseStageBytes = kReuseWarps * 1024 + kBRows * 64;
+constexpr int kReuseTiles = 4;                  // 16-token tiles per CTA
+constexpr int kReuseWarps = 2 * kReuseTiles;    // each tile: two warps, one per half of d
+constexpr int kReuseTok = 16 * kReuseTiles;     // tokens per CTA on reuse steps
+constexpr int kReuseStages = 6;                 // blocks in flight per half of d
+// one stage: each warp's A block (16 rows x 64 B) and the B block (48 x 64 B)
+// of each half of d
+constexpr int kReuseStageBytes = kReuseWarps * 1024 + 2 * kBRows * 64;
 constexpr int kReuseSmem = kReuseStages * kReuseStageBytes;
+// the two halves' partial products of a tile meet in the ring memory
+constexpr int kReusePartFloats = 36;            // D (24), Gram (8), ones (4) per lane
+static_assert(kReuseTiles * 32 * kReusePartFloats * 4 <= kReuseSmem, "partials exceed the ring");
 
 // Reuse step of the scenes in `map`: h = x W_e^T + c_j, v = head(h), x += dsig v
 // (or v to vout).  wp_k / tab_k: this step's tables, indexed by scene.  Each
-// warp takes 16 tokens over all of d; per 32-column block the CTA stages the
-// warps' cache rows and the 48 B rows (shared by the four warps) in a
-// kReuseStages-deep cp.async ring.
-__global__ void __launch_bounds__(128) head_reuse_kernel(
+// 16-token tile is taken by two warps, one per half of d, so that more warps
+// stream than there are tiles; per step of the loop the CTA stages every
+// warp's cache rows and the 48 B rows of the two blocks in flight (shared by
+// the four warps of a half) in a kReuseStages-deep cp.async ring.
+__global__ void __launch_bounds__(256) head_reuse_kernel(
     float* __restrict__ x, const __nv_bfloat16* __restrict__ cache, SlotMap map, int N, int d,
     const __nv_bfloat16* __restrict__ wp_k, const float* __restrict__ tab_k,
     const float* __restrict__ wsum, const float* __restrict__ gram, float dsig,
@@ -156,40 +153,52 @@ __global__ void __launch_bounds__(128) head_reuse_kernel(
   pdl_trigger();
   pdl_wait();
   extern __shared__ __align__(16) uint8_t rsm[];
-  __shared__ float part[kReuseWarps][16][2 * kHC + 2];  // per token: A, Q, sum c, sum c^2
+  __shared__ float part[kReuseTiles][16][2 * kHC + 2];  // per token: A, Q, sum c, sum c^2
   __shared__ float stab[kHeadTab + kHC + kHC * kHC];    // S', beta, G_s | w_sum | G
   const int slot = blockIdx.y, scene = map.scene[slot];
   const int tok0 = blockIdx.x * kReuseTok;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, q = lane & 3;
+  const int tile = warp & (kReuseTiles - 1), half = warp / kReuseTiles;
   for (int i = tid; i < kHeadTab; i += blockDim.x) stab[i] = tab_k[(size_t)scene * kHeadTab + i];
   if (tid < kHC) stab[kHeadTab + tid] = wsum[tid];
   for (int i = tid; i < kHC * kHC; i += blockDim.x) stab[kHeadTab + kHC + i] = gram[i];
 
   const __nv_bfloat16* cs = cache + (size_t)scene * N * d;
   const __nv_bfloat16* wk = wp_k + (size_t)scene * kBRows * d;
+  const int nblk = d >> 5;
+  const int nbh = (nblk + 1) >> 1;  // blocks per half: half h takes h nbh .. min(nblk, (h + 1) nbh)
   int row[2];
   bool ok[2];
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
-    row[h] = tok0 + 16 * warp + 8 * h + g;
+    row[h] = tok0 + 16 * tile + 8 * h + g;
     ok[h] = row[h] < N;
   }
-  // this thread's copies of block b into stage st: its own two cache pieces,
-  // and B pieces tid and tid + 128 (of 48 rows x 4 pieces)
-  auto fetch = [&](int b, int st) {
+  // this thread's copies of loop step i into stage st: its own two cache
+  // pieces (block half nbh + i of its half), and B pieces tid and tid + 256 of
+  // the two halves' blocks (2 x 48 rows x 4 pieces)
+  auto fetch = [&](int i, int st) {
     uint8_t* base = rsm + st * kReuseStageBytes;
-    const int e = (b << 5) + (q << 3);
-    uint4* a = reinterpret_cast<uint4*>(base + warp * 1024) + lane;
+    const int b = half * nbh + i;
+    if (i < nbh && b < nblk) {
+      const int e = (b << 5) + (q << 3);
+      uint4* a = reinterpret_cast<uint4*>(base + warp * 1024) + lane;
 #pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      if (ok[h]) cp_async16(a + 32 * h, cs + (size_t)row[h] * d + e);
-      else a[32 * h] = make_uint4(0u, 0u, 0u, 0u);
+      for (int h = 0; h < 2; ++h) {
+        if (ok[h]) cp_async16(a + 32 * h, cs + (size_t)row[h] * d + e);
+        else a[32 * h] = make_uint4(0u, 0u, 0u, 0u);
+      }
     }
     uint4* bb = reinterpret_cast<uint4*>(base + kReuseWarps * 1024);
 #pragma unroll
     for (int k = 0; k < 2; ++k) {
-      const int c = tid + 128 * k;
-      if (c < kBRows * 4) cp_async16(bb + c, wk + (size_t)(c >> 2) * d + (b << 5) + ((c & 3) << 3));
+      const int c = tid + 256 * k;
+      if (c < 2 * kBRows * 4) {
+        const int hb = c / (kBRows * 4), cc = c - hb * kBRows * 4;
+        const int bh = hb * nbh + i;
+        if (i < nbh && bh < nblk)
+          cp_async16(bb + c, wk + (size_t)(cc >> 2) * d + (bh << 5) + ((cc & 3) << 3));
+      }
     }
   };
   float D[6][4];
@@ -202,23 +211,23 @@ __global__ void __launch_bounds__(128) head_reuse_kernel(
   // rows: tokens 0-7 of the tile, then 8-15), on the tensor cores as well
   float GS[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}}, S1[4] = {0.f, 0.f, 0.f, 0.f};
   const uint32_t ones = g == 0 ? 0x3F803F80u : 0u;  // bf16 (1, 1) in column 0
-  const int nblk = d >> 5;
+  const bool mine = half * nbh < nblk;  // this half has blocks at all
 #pragma unroll 1
   for (int i = 0; i < kReuseStages - 1; ++i) {
-    if (i < nblk) fetch(i, i);
+    fetch(i, i);
     cp_async_commit();
   }
 #pragma unroll 1
-  for (int b = 0; b < nblk; ++b) {
-    cp_async_wait<kReuseStages - 2>();  // this thread's copies of block b have landed
-    __syncthreads();                    // everyone's have, and block b - 1 is consumed
-    const int nb = b + kReuseStages - 1;
-    if (nb < nblk) fetch(nb, nb % kReuseStages);
+  for (int i = 0; i < nbh; ++i) {
+    cp_async_wait<kReuseStages - 2>();  // this thread's copies of step i have landed
+    __syncthreads();                    // everyone's have, and step i - 1 is consumed
+    fetch(i + kReuseStages - 1, (i + kReuseStages - 1) % kReuseStages);
     cp_async_commit();
-    const uint8_t* base = rsm + (b % kReuseStages) * kReuseStageBytes;
+    if (!mine || half * nbh + i >= nblk) continue;
+    const uint8_t* base = rsm + (i % kReuseStages) * kReuseStageBytes;
     const uint4* a = reinterpret_cast<const uint4*>(base + warp * 1024) + lane;
     const uint4 av0 = a[0], av1 = a[32];
-    const uint4* bb = reinterpret_cast<const uint4*>(base + kReuseWarps * 1024);
+    const uint4* bb = reinterpret_cast<const uint4*>(base + kReuseWarps * 1024) + half * kBRows * 4;
     uint4 bw[6];
 #pragma unroll
     for (int j = 0; j < 6; ++j) bw[j] = bb[(8 * j + g) * 4 + q];
@@ -237,9 +246,35 @@ __global__ void __launch_bounds__(128) head_reuse_kernel(
     }
   }
   cp_async_wait<0>();
+  __syncthreads();  // the ring is free: the second half's partials go through it
+  float* pr = reinterpret_cast<float*>(rsm) + (size_t)(tile * 32 + lane) * kReusePartFloats;
+  if (half == 1) {
+#pragma unroll
+    for (int j = 0; j < 6; ++j)
+#pragma unroll
+      for (int t = 0; t < 4; ++t) pr[4 * j + t] = D[j][t];
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      pr[24 + t] = GS[0][t];
+      pr[28 + t] = GS[1][t];
+      pr[32 + t] = S1[t];
+    }
+  }
+  __syncthreads();
+  if (half == 1) return;
+#pragma unroll
+  for (int j = 0; j < 6; ++j)
+#pragma unroll
+    for (int t = 0; t < 4; ++t) D[j][t] += pr[4 * j + t];
+#pragma unroll
+  for (int t = 0; t < 4; ++t) {
+    GS[0][t] += pr[24 + t];
+    GS[1][t] += pr[28 + t];
+    S1[t] += pr[32 + t];
+  }
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
-    float* pp = part[warp][8 * h + g];
+    float* pp = part[tile][8 * h + g];
 #pragma unroll
     for (int j = 0; j < 2; ++j)
 #pragma unroll
@@ -254,11 +289,11 @@ __global__ void __launch_bounds__(128) head_reuse_kernel(
   }
   __syncwarp();
 
-  // finish: two lanes per token of this warp, 8 channels each
+  // finish: two lanes per token of this tile, 8 channels each
   const int tt = lane >> 1, ch = lane & 1;
-  const int tok = tok0 + 16 * warp + tt;
+  const int tok = tok0 + 16 * tile + tt;
   const bool live = tok < N;
-  const float* pt = part[warp][tt];
+  const float* pt = part[tile][tt];
   float xv[kHC], vv[8];
   if (live) {
     const float4* xr = reinterpret_cast<const float4*>(x + ((size_t)scene * N + tok) * kHC);
@@ -532,8 +567,8 @@ cudaError_t launch_head_reuse(float* x, const __nv_bfloat16* cache, const SlotMa
   });
   if (e != cudaSuccess) return e;
   const dim3 grid((unsigned)((N + kReuseTok - 1) / kReuseTok), (unsigned)map.n);
-  return launch_pdl(head_reuse_kernel, grid, dim3(128), kReuseSmem, st, x, cache, map, N, d, wp_k,
-                    tab_k, wsum, gram, dsig, vout);
+  return launch_pdl(head_reuse_kernel, grid, dim3(32 * kReuseWarps), kReuseSmem, st, x, cache, map,
+                    N, d, wp_k, tab_k, wsum, gram, dsig, vout);
 }
 
 cudaError_t launch_head_compute(const float* hL, float* x, float* xj, __nv_bfloat16* cache,
