@@ -51,8 +51,7 @@ struct AttCfg {
   // once S_t is in registers, and S_{t,j+1} is issued after PV_{t,j} (the
   // MMAs of one thread run in issue order).
   static constexpr bool kAliasP = DHP == 128 && NQ == 2;
-  // ring depths (key, value): deeper rings measured no faster at dh 64; with
-  // two tiles at dh 128 a third key stage (224 KB in all) measured slower
+  // ring depths (key, value): deeper rings measured no faster at dh 64
   static constexpr int kKStages = kAliasP ? 2 : 3;
   static constexpr int kVStages = kAliasP ? 2 : 3;
   static constexpr int kTileBytes = kAtoms * 16384;   // 128 rows x DHP bf16
@@ -102,20 +101,6 @@ __device__ __forceinline__ uint64_t sw128_mnmajor_desc(uint32_t start) {
   uint64_t d = 0;
   d |= (uint64_t)((start & 0x3FFFF) >> 4);
   d |= (uint64_t)(1024 >> 4) << 16;
-  d |= (uint64_t)(1024 >> 4) << 32;
-  d |= (uint64_t)1 << 46;
-  d |= (uint64_t)2 << 61;
-  return d;
-}
-
-// The same tile as one MN-major operand that spans both 64-element atoms of a
-// 128-column row block: the second atom (the next 64 MN elements, 16 KB on)
-// is the leading-dimension stride, the 8-row groups along K the stride
-// dimension.  Every byte it can address lies inside the 32 KB tile.
-__device__ __forceinline__ uint64_t sw128_mnmajor2_desc(uint32_t start) {
-  uint64_t d = 0;
-  d |= (uint64_t)((start & 0x3FFFF) >> 4);
-  d |= (uint64_t)(16384 >> 4) << 16;
   d |= (uint64_t)(1024 >> 4) << 32;
   d |= (uint64_t)1 << 46;
   d |= (uint64_t)2 << 61;
@@ -238,8 +223,6 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
   constexpr int kKSteps = kDHR / 16;                // K steps of the S products
   constexpr int kLastN = kDHR - 64 * (Cfg::kAtoms - 1);  // N of the last atom's PV product
   constexpr uint32_t kIdPVLast = idesc_bf16_f32(128, kLastN) | (1u << 16);
-  // two atoms (dh in the 128-column layout): one PV product of N = round16(dh)
-  constexpr uint32_t kIdPVWide = idesc_bf16_f32(128, kDHR) | (1u << 16);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -402,7 +385,6 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
       const uint64_t dQ = sw128_kmajor_desc(smem_u32(smem + Cfg::kOffQ + t * Cfg::kTileBytes));
       const uint64_t dK = sw128_kmajor_desc(smem_u32(smem + Cfg::kOffK));
       const uint64_t dV = sw128_mnmajor_desc(smem_u32(smem + Cfg::kOffV));
-      const uint64_t dV2 = sw128_mnmajor2_desc(smem_u32(smem + Cfg::kOffV));
       // S_{t,j} = Q_t K_j^T: needs K_j, and S_t no longer needed (read by the
       // softmax; with P aliased onto S_t, PV_{t,j-1} issued before it)
       auto issue_s = [&](int j) -> bool {
@@ -436,20 +418,12 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
         if (elect_one()) {
 #pragma unroll
           for (int kk = 0; kk < 8; ++kk) {
-            if constexpr (Cfg::kAtoms == 2) {
-              // both atoms of V in one product (N = 80 or 128): the N = 64 half
-              // products ran at about 70 % of the tensor rate
-              tc_mma_f16_ta(tmem + Cfg::kColO + t * DHP, tmem + Cfg::kColP + t * Cfg::kPStride + kk * 8,
-                            dV2 + ((uint32_t)(vb * Cfg::kTileBytes + kk * 2048) >> 4), kIdPVWide,
-                            (jp > 0 || kk > 0) ? 1u : 0u);
-            } else {
 #pragma unroll
-              for (int a = 0; a < Cfg::kAtoms; ++a)
-                tc_mma_f16_ta(tmem + Cfg::kColO + t * DHP + a * 64,
-                              tmem + Cfg::kColP + t * Cfg::kPStride + kk * 8,
-                              dV + ((uint32_t)(vb * Cfg::kTileBytes + a * 16384 + kk * 2048) >> 4),
-                              a == Cfg::kAtoms - 1 ? kIdPVLast : kIdPV, (jp > 0 || kk > 0) ? 1u : 0u);
-            }
+            for (int a = 0; a < Cfg::kAtoms; ++a)
+              tc_mma_f16_ta(tmem + Cfg::kColO + t * DHP + a * 64,
+                            tmem + Cfg::kColP + t * Cfg::kPStride + kk * 8,
+                            dV + ((uint32_t)(vb * Cfg::kTileBytes + a * 16384 + kk * 2048) >> 4),
+                            a == Cfg::kAtoms - 1 ? kIdPVLast : kIdPV, (jp > 0 || kk > 0) ? 1u : 0u);
           }
           tc_commit(&bar->p_free[t]);
           tc_commit(&bar->v_empty[vb]);

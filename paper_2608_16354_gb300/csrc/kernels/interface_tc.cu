@@ -125,246 +125,30 @@ __global__ void __launch_bounds__(256) head_tables_kernel(
   }
 }
 
-// ---------------------------------------------------------------- reuse step
-
-constexpr int kReuseTiles = 4;                  // 16-token tiles per CTA
-constexpr int kReuseWarps = 2 * kReuseTiles;    // each tile: two warps, one per half of d
-constexpr int kReuseTok = 16 * kReuseTiles;     // tokens per CTA on reuse steps
-constexpr int kReuseStages = 6;                 // blocks in flight per half of d
-// one stage: each warp's A block (16 rows x 64 B) and the B block (48 x 64 B)
-// of each half of d
-constexpr int kReuseStageBytes = kReuseWarps * 1024 + 2 * kBRows * 64;
-constexpr int kReuseSmem = kReuseStages * kReuseStageBytes;
-// the two halves' partial products of a tile meet in the ring memory
-constexpr int kReusePartFloats = 36;            // D (24), Gram (8), ones (4) per lane
-static_assert(kReuseTiles * 32 * kReusePartFloats * 4 <= kReuseSmem, "partials exceed the ring");
-
-// Reuse step of the scenes in `map`: h = x W_e^T + c_j, v = head(h), x += dsig v
-// (or v to vout).  wp_k / tab_k: this step's tables, indexed by scene.  Each
-// 16-token tile is taken by two warps, one per half of d, so that more warps
-// stream than there are tiles; per step of the loop the CTA stages every
-// warp's cache rows and the 48 B rows of the two blocks in flight (shared by
-// the four warps of a half) in a kReuseStages-deep cp.async ring.
-__global__ void __launch_bounds__(256) head_reuse_kernel(
-    float* __restrict__ x, const __nv_bfloat16* __restrict__ cache, SlotMap map, int N, int d,
-    const __nv_bfloat16* __restrict__ wp_k, const float* __restrict__ tab_k,
-    const float* __restrict__ wsum, const float* __restrict__ gram, float dsig,
-    float* __restrict__ vout) {
-  pdl_trigger();
-  pdl_wait();
-  extern __shared__ __align__(16) uint8_t rsm[];
-  __shared__ float part[kReuseTiles][16][2 * kHC + 2];  // per token: A, Q, sum c, sum c^2
-  __shared__ float stab[kHeadTab + kHC + kHC * kHC];    // S', beta, G_s | w_sum | G
-  const int slot = blockIdx.y, scene = map.scene[slot];
-  const int tok0 = blockIdx.x * kReuseTok;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, q = lane & 3;
-  const int tile = warp & (kReuseTiles - 1), half = warp / kReuseTiles;
-  for (int i = tid; i < kHeadTab; i += blockDim.x) stab[i] = tab_k[(size_t)scene * kHeadTab + i];
-  if (tid < kHC) stab[kHeadTab + tid] = wsum[tid];
-  for (int i = tid; i < kHC * kHC; i += blockDim.x) stab[kHeadTab + kHC + i] = gram[i];
-
-  const __nv_bfloat16* cs = cache + (size_t)scene * N * d;
-  const __nv_bfloat16* wk = wp_k + (size_t)scene * kBRows * d;
-  const int nblk = d >> 5;
-  const int nbh = (nblk + 1) >> 1;  // blocks per half: half h takes h nbh .. min(nblk, (h + 1) nbh)
-  int row[2];
-  bool ok[2];
-#pragma unroll
-  for (int h = 0; h < 2; ++h) {
-    row[h] = tok0 + 16 * tile + 8 * h + g;
-    ok[h] = row[h] < N;
-  }
-  // this thread's copies of loop step i into stage st: its own two cache
-  // pieces (block half nbh + i of its half), and B pieces tid and tid + 256 of
-  // the two halves' blocks (2 x 48 rows x 4 pieces)
-  auto fetch = [&](int i, int st) {
-    uint8_t* base = rsm + st * kReuseStageBytes;
-    const int b = half * nbh + i;
-    if (i < nbh && b < nblk) {
-      const int e = (b << 5) + (q << 3);
-      uint4* a = reinterpret_cast<uint4*>(base + warp * 1024) + lane;
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        if (ok[h]) cp_async16(a + 32 * h, cs + (size_t)row[h] * d + e);
-        else a[32 * h] = make_uint4(0u, 0u, 0u, 0u);
-      }
-    }
-    uint4* bb = reinterpret_cast<uint4*>(base + kReuseWarps * 1024);
-#pragma unroll
-    for (int k = 0; k < 2; ++k) {
-      const int c = tid + 256 * k;
-      if (c < 2 * kBRows * 4) {
-        const int hb = c / (kBRows * 4), cc = c - hb * kBRows * 4;
-        const int bh = hb * nbh + i;
-        if (i < nbh && bh < nblk)
-          cp_async16(bb + c, wk + (size_t)(cc >> 2) * d + (bh << 5) + ((cc & 3) << 3));
-      }
-    }
-  };
-  float D[6][4];
-#pragma unroll
-  for (int j = 0; j < 6; ++j)
-#pragma unroll
-    for (int t = 0; t < 4; ++t) D[j][t] = 0.f;
-  // per-token sum c (a B column of ones) and sum c^2 (the diagonal of the
-  // tile's Gram matrix c c^T, whose B fragments are the A fragments' own
-  // rows: tokens 0-7 of the tile, then 8-15), on the tensor cores as well
-  float GS[2][4] = {{0.f, 0.f, 0.f, 0.f}, {0.f, 0.f, 0.f, 0.f}}, S1[4] = {0.f, 0.f, 0.f, 0.f};
-  const uint32_t ones = g == 0 ? 0x3F803F80u : 0u;  // bf16 (1, 1) in column 0
-  const bool mine = half * nbh < nblk;  // this half has blocks at all
-#pragma unroll 1
-  for (int i = 0; i < kReuseStages - 1; ++i) {
-    fetch(i, i);
-    cp_async_commit();
-  }
-#pragma unroll 1
-  for (int i = 0; i < nbh; ++i) {
-    cp_async_wait<kReuseStages - 2>();  // this thread's copies of step i have landed
-    __syncthreads();                    // everyone's have, and step i - 1 is consumed
-    fetch(i + kReuseStages - 1, (i + kReuseStages - 1) % kReuseStages);
-    cp_async_commit();
-    if (!mine || half * nbh + i >= nblk) continue;
-    const uint8_t* base = rsm + (i % kReuseStages) * kReuseStageBytes;
-    const uint4* a = reinterpret_cast<const uint4*>(base + warp * 1024) + lane;
-    const uint4 av0 = a[0], av1 = a[32];
-    const uint4* bb = reinterpret_cast<const uint4*>(base + kReuseWarps * 1024) + half * kBRows * 4;
-    uint4 bw[6];
-#pragma unroll
-    for (int j = 0; j < 6; ++j) bw[j] = bb[(8 * j + g) * 4 + q];
-#pragma unroll
-    for (int s = 0; s < 2; ++s) {
-      const uint32_t a0 = s ? av0.z : av0.x;  // row g, cols 4s + 0, 1
-      const uint32_t a1 = s ? av1.z : av1.x;  // row g + 8
-      const uint32_t a2 = s ? av0.w : av0.y;  // row g, cols 4s + 2, 3
-      const uint32_t a3 = s ? av1.w : av1.y;  // row g + 8
-#pragma unroll
-      for (int j = 0; j < 6; ++j)
-        mma_bf16_16816(D[j], a0, a1, a2, a3, s ? bw[j].z : bw[j].x, s ? bw[j].w : bw[j].y);
-      mma_bf16_16816(GS[0], a0, a1, a2, a3, a0, a2);
-      mma_bf16_16816(GS[1], a0, a1, a2, a3, a1, a3);
-      mma_bf16_16816(S1, a0, a1, a2, a3, ones, ones);
-    }
-  }
-  cp_async_wait<0>();
-  __syncthreads();  // the ring is free: the second half's partials go through it
-  float* pr = reinterpret_cast<float*>(rsm) + (size_t)(tile * 32 + lane) * kReusePartFloats;
-  if (half == 1) {
-#pragma unroll
-    for (int j = 0; j < 6; ++j)
-#pragma unroll
-      for (int t = 0; t < 4; ++t) pr[4 * j + t] = D[j][t];
-#pragma unroll
-    for (int t = 0; t < 4; ++t) {
-      pr[24 + t] = GS[0][t];
-      pr[28 + t] = GS[1][t];
-      pr[32 + t] = S1[t];
-    }
-  }
-  __syncthreads();
-  if (half == 1) return;
-#pragma unroll
-  for (int j = 0; j < 6; ++j)
-#pragma unroll
-    for (int t = 0; t < 4; ++t) D[j][t] += pr[4 * j + t];
-#pragma unroll
-  for (int t = 0; t < 4; ++t) {
-    GS[0][t] += pr[24 + t];
-    GS[1][t] += pr[28 + t];
-    S1[t] += pr[32 + t];
-  }
-#pragma unroll
-  for (int h = 0; h < 2; ++h) {
-    float* pp = part[tile][8 * h + g];
-#pragma unroll
-    for (int j = 0; j < 2; ++j)
-#pragma unroll
-      for (int t = 0; t < 2; ++t) {
-        pp[8 * j + 2 * q + t] = D[j][2 * h + t];
-        pp[kHC + 8 * j + 2 * q + t] = D[2 + j][2 * h + t] + D[4 + j][2 * h + t];
-      }
-    // token 8 h + g: sum c in column 0 of the ones product (lane q = 0), sum
-    // c^2 on the diagonal of the Gram product of its half (lane q = g / 2)
-    if (q == 0) pp[2 * kHC] = S1[2 * h];
-    if (q == (g >> 1)) pp[2 * kHC + 1] = (g & 1) ? GS[h][2 * h + 1] : GS[h][2 * h];
-  }
-  __syncwarp();
-
-  // finish: two lanes per token of this tile, 8 channels each
-  const int tt = lane >> 1, ch = lane & 1;
-  const int tok = tok0 + 16 * tile + tt;
-  const bool live = tok < N;
-  const float* pt = part[tile][tt];
-  float xv[kHC], vv[8];
-  if (live) {
-    const float4* xr = reinterpret_cast<const float4*>(x + ((size_t)scene * N + tok) * kHC);
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const float4 t4 = xr[k];
-      xv[4 * k] = t4.x; xv[4 * k + 1] = t4.y; xv[4 * k + 2] = t4.z; xv[4 * k + 3] = t4.w;
-    }
-    const float *S = stab, *beta = stab + kHC, *Gs = stab + 2 * kHC, *ws = stab + kHeadTab,
-                *G = stab + kHeadTab + kHC;
-    float sum1 = pt[2 * kHC], xA = 0.f, xGx = 0.f;
-#pragma unroll
-    for (int a = 0; a < kHC; ++a) {
-      xA = fmaf(xv[a], pt[a], xA);
-      sum1 = fmaf(xv[a], ws[a], sum1);
-      float t = 0.f;
-#pragma unroll
-      for (int b2 = 0; b2 < kHC; ++b2) t = fmaf(G[a * kHC + b2], xv[b2], t);
-      xGx = fmaf(xv[a], t, xGx);
-    }
-    const float sq = xGx + 2.f * xA + pt[2 * kHC + 1];
-    const float mu = sum1 / (float)d;
-    const float var = fmaxf(sq / (float)d - mu * mu, 0.f);
-    const float rs = rsqrtf(var + 1e-6f);
-#pragma unroll
-    for (int cc = 0; cc < 8; ++cc) {
-      const int c = 8 * ch + cc;
-      float P = pt[kHC + c];
-#pragma unroll
-      for (int a = 0; a < kHC; ++a) P = fmaf(xv[a], Gs[a * kHC + c], P);
-      vv[cc] = fmaf(rs, P - mu * S[c], beta[c]);
-    }
-  }
-  const size_t xi = ((size_t)scene * N + tok) * kHC + 8 * ch;
-  const float4 xo0 = live ? *reinterpret_cast<const float4*>(x + xi) : make_float4(0.f, 0.f, 0.f, 0.f);
-  const float4 xo1 = live ? *reinterpret_cast<const float4*>(x + xi + 4) : make_float4(0.f, 0.f, 0.f, 0.f);
-  __syncwarp();  // both lanes of the token have read its x row
-  if (live) {
-    if (vout) {
-      *reinterpret_cast<float4*>(vout + xi) = make_float4(vv[0], vv[1], vv[2], vv[3]);
-      *reinterpret_cast<float4*>(vout + xi + 4) = make_float4(vv[4], vv[5], vv[6], vv[7]);
-    } else {
-      *reinterpret_cast<float4*>(x + xi) =
-          make_float4(fmaf(dsig, vv[0], xo0.x), fmaf(dsig, vv[1], xo0.y), fmaf(dsig, vv[2], xo0.z),
-                      fmaf(dsig, vv[3], xo0.w));
-      *reinterpret_cast<float4*>(x + xi + 4) =
-          make_float4(fmaf(dsig, vv[4], xo1.x), fmaf(dsig, vv[5], xo1.y), fmaf(dsig, vv[6], xo1.z),
-                      fmaf(dsig, vv[7], xo1.w));
-    }
-  }
-}
-
 // ------------------------------------------------------------- compute step
 
-constexpr int kCmpWarps = 4;                 // one 16-token tile per warp
-constexpr int kCmpTok = 16 * kCmpWarps;      // tokens per CTA on compute steps
-constexpr int kCmpStages = 8;                // 32-column blocks in flight per CTA
-// one stage: each warp's h_L block (16 rows x 128 B), the W' rows (32 x 64 B)
-// and the block's W_e^T fragments (32 lanes x 32 B)
-constexpr int kCmpStageBytes = kCmpWarps * 2048 + 2 * kHC * 64 + 1024;
+constexpr int kCmpTiles = 4;                 // 16-token tiles per CTA
+constexpr int kCmpWarps = 2 * kCmpTiles;     // each tile: two warps, one per half of d
+constexpr int kCmpTok = 16 * kCmpTiles;      // tokens per CTA on compute steps
+constexpr int kCmpStages = 4;                // blocks in flight per half of d
+// one stage: each warp's h_L block (16 rows x 128 B) and, per half of d, the
+// W' rows (32 x 64 B) and the block's W_e^T fragments (32 lanes x 32 B)
+constexpr int kCmpBPieces = 2 * kHC * 4 + 64;  // 16-byte pieces of one half's B block
+constexpr int kCmpStageBytes = kCmpWarps * 2048 + 2 * kCmpBPieces * 16;
 constexpr int kCmpSmem = kCmpStages * kCmpStageBytes;
+constexpr int kCmpPartFloats = 20;           // D (16), sum h and sum h^2 of two rows (4)
+static_assert(kCmpTiles * 32 * kCmpPartFloats * 4 <= kCmpSmem, "partials exceed the ring");
 
 // Compute step of the scenes in `map` (h_L rows packed by slot): the cache
 // row c = h_L - x W_e^T is written, v = head(h_L), x_j <- x, x += dsig v (or
-// v to vout).  Each warp takes 16 tokens over all of d; per 32-column block
-// the CTA stages the warps' h_L rows, the W' rows and the W_e^T fragments
-// (shared by the four warps) in a kCmpStages-deep cp.async ring.  x W_e^T
-// runs on the tensor cores with K = C = 16: the fragment-ordered W_e^T puts
-// its four 8-column products on the thread's own columns (product j:
-// columns e + 2 j, e + 2 j + 1 of rows g and g + 8).
-__global__ void __launch_bounds__(128) head_compute_kernel(
+// v to vout).  Each 16-token tile is taken by two warps, one per half of d;
+// per step of the loop the CTA stages every warp's h_L rows and, for the two
+// blocks in flight, the W' rows and W_e^T fragments (shared by the four warps
+// of a half) in a kCmpStages-deep cp.async ring.  x W_e^T runs on the tensor
+// cores with K = C = 16: the fragment-ordered W_e^T puts its four 8-column
+// products on the thread's own columns (product j: columns e + 2 j, e + 2 j
+// + 1 of rows g and g + 8).
+__global__ void __launch_bounds__(256) head_compute_kernel(
     const float* __restrict__ hL, float* __restrict__ x, float* __restrict__ xj,
     __nv_bfloat16* __restrict__ cache, SlotMap map, int N, int d,
     const __nv_bfloat16* __restrict__ we_frag, const __nv_bfloat16* __restrict__ wp_k,
@@ -372,14 +156,17 @@ __global__ void __launch_bounds__(128) head_compute_kernel(
   pdl_trigger();
   pdl_wait();
   extern __shared__ __align__(16) uint8_t csm[];
-  __shared__ float part[kCmpWarps][16][kHC + 2];  // per token: P, sum h, sum h^2
+  __shared__ float part[kCmpTiles][16][kHC + 2];  // per token: P, sum h, sum h^2
   __shared__ float stab[2 * kHC];                 // S', beta
   const int slot = blockIdx.y, scene = map.scene[slot];
   const int tok0 = blockIdx.x * kCmpTok;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31, g = lane >> 2, q = lane & 3;
+  const int tile = warp & (kCmpTiles - 1), half = warp / kCmpTiles;
   if (tid < 2 * kHC) stab[tid] = tab_k[(size_t)scene * kHeadTab + tid];
   const __nv_bfloat16* wk = wp_k + (size_t)scene * kBRows * d + (size_t)kHC * d;  // W' rows
   const uint8_t* wf = reinterpret_cast<const uint8_t*>(we_frag);
+  const int nblk = d >> 5;
+  const int nbh = (nblk + 1) >> 1;  // blocks per half: half h takes h nbh .. min(nblk, (h + 1) nbh)
   int row[2];
   bool ok[2];
   // A fragments of x (tokens x channels, hi and lo halves): rows g and
@@ -387,7 +174,7 @@ __global__ void __launch_bounds__(128) head_compute_kernel(
   uint32_t xa_hi[4], xa_lo[4];
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
-    row[h] = tok0 + 16 * warp + 8 * h + g;
+    row[h] = tok0 + 16 * tile + 8 * h + g;
     ok[h] = row[h] < N;
     const float* xr = x + ((size_t)scene * N + row[h]) * kHC;
     const float2 p0 = ok[h] ? *reinterpret_cast<const float2*>(xr + 2 * q) : make_float2(0.f, 0.f);
@@ -395,21 +182,37 @@ __global__ void __launch_bounds__(128) head_compute_kernel(
     split_pair(p0.x, p0.y, &xa_hi[h], &xa_lo[h]);
     split_pair(p1.x, p1.y, &xa_hi[2 + h], &xa_lo[2 + h]);
   }
-  // this thread's copies of block b into stage st: its h_L pieces (rows g and
-  // g + 8, 8 fp32 each), W' piece tid (32 rows x 4), fragment piece tid < 64
-  auto fetch = [&](int b, int st) {
+  // this thread's copies of loop step i into stage st: its h_L pieces (rows g
+  // and g + 8 of the block of its half, 8 fp32 each), and B pieces tid and
+  // tid + 256 of the two halves (W' 128 pieces, fragments 64 pieces each)
+  auto fetch = [&](int i, int st) {
     uint8_t* base = csm + st * kCmpStageBytes;
-    const int e = (b << 5) + (q << 3);
-    uint4* a = reinterpret_cast<uint4*>(base + warp * 2048) + lane;
+    const int b = half * nbh + i;
+    if (i < nbh && b < nblk) {
+      const int e = (b << 5) + (q << 3);
+      uint4* a = reinterpret_cast<uint4*>(base + warp * 2048) + lane;
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const int h = k >> 1;
-      if (ok[h]) cp_async16(a + 32 * k, hL + ((size_t)slot * N + row[h]) * d + e + 4 * (k & 1));
-      else a[32 * k] = make_uint4(0u, 0u, 0u, 0u);
+      for (int k = 0; k < 4; ++k) {
+        const int h = k >> 1;
+        if (ok[h]) cp_async16(a + 32 * k, hL + ((size_t)slot * N + row[h]) * d + e + 4 * (k & 1));
+        else a[32 * k] = make_uint4(0u, 0u, 0u, 0u);
+      }
     }
     uint4* bb = reinterpret_cast<uint4*>(base + kCmpWarps * 2048);
-    cp_async16(bb + tid, wk + (size_t)(tid >> 2) * d + (b << 5) + ((tid & 3) << 3));
-    if (tid < 64) cp_async16(bb + 128 + tid, wf + (size_t)b * 1024 + tid * 16);
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      const int c = tid + 256 * k;
+      if (c < 2 * kCmpBPieces) {
+        const int hb = c / kCmpBPieces, cc = c - hb * kCmpBPieces;
+        const int bh = hb * nbh + i;
+        if (i < nbh && bh < nblk) {
+          if (cc < 2 * kHC * 4)
+            cp_async16(bb + c, wk + (size_t)(cc >> 2) * d + (bh << 5) + ((cc & 3) << 3));
+          else
+            cp_async16(bb + c, wf + (size_t)bh * 1024 + (cc - 2 * kHC * 4) * 16);
+        }
+      }
+    }
   };
   float D[4][4];
 #pragma unroll
@@ -417,20 +220,21 @@ __global__ void __launch_bounds__(128) head_compute_kernel(
 #pragma unroll
     for (int t = 0; t < 4; ++t) D[j][t] = 0.f;
   float s1[2] = {0.f, 0.f}, s2[2] = {0.f, 0.f};
-  const int nblk = d >> 5;
+  const bool mine = half * nbh < nblk;
 #pragma unroll 1
   for (int i = 0; i < kCmpStages - 1; ++i) {
-    if (i < nblk) fetch(i, i);
+    fetch(i, i);
     cp_async_commit();
   }
 #pragma unroll 1
-  for (int b = 0; b < nblk; ++b) {
+  for (int i = 0; i < nbh; ++i) {
     cp_async_wait<kCmpStages - 2>();
     __syncthreads();
-    const int nb = b + kCmpStages - 1;
-    if (nb < nblk) fetch(nb, nb % kCmpStages);
+    fetch(i + kCmpStages - 1, (i + kCmpStages - 1) % kCmpStages);
     cp_async_commit();
-    const uint8_t* base = csm + (b % kCmpStages) * kCmpStageBytes;
+    const int b = half * nbh + i;
+    if (!mine || b >= nblk) continue;
+    const uint8_t* base = csm + (i % kCmpStages) * kCmpStageBytes;
     const int e = (b << 5) + (q << 3);
     float hv[2][8];
     {
@@ -443,14 +247,14 @@ __global__ void __launch_bounds__(128) head_compute_kernel(
         dst[2] = __uint_as_float(w.z); dst[3] = __uint_as_float(w.w);
       }
     }
-    const uint4* bb = reinterpret_cast<const uint4*>(base + kCmpWarps * 2048);
+    const uint4* bb = reinterpret_cast<const uint4*>(base + kCmpWarps * 2048) + half * kCmpBPieces;
     uint4 bw[4];  // W' hi (channels 0-7, 8-15), W' lo (0-7, 8-15)
 #pragma unroll
     for (int j = 0; j < 4; ++j) bw[j] = bb[(8 * j + g) * 4 + q];
     // the cache row c = h - x W_e^T
     float u[2][8];
     {
-      const uint4 f0 = bb[128 + 2 * lane], f1 = bb[129 + 2 * lane];
+      const uint4 f0 = bb[2 * kHC * 4 + 2 * lane], f1 = bb[2 * kHC * 4 + 2 * lane + 1];
       const uint32_t fb[8] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w};
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
@@ -494,13 +298,29 @@ __global__ void __launch_bounds__(128) head_compute_kernel(
     }
   }
   cp_async_wait<0>();
+  __syncthreads();  // the ring is free: the second half's partials go through it
+  float* pr = reinterpret_cast<float*>(csm) + (size_t)(tile * 32 + lane) * kCmpPartFloats;
+  if (half == 1) {
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+#pragma unroll
+      for (int t = 0; t < 4; ++t) pr[4 * j + t] = D[j][t];
+    pr[16] = s1[0]; pr[17] = s1[1]; pr[18] = s2[0]; pr[19] = s2[1];
+  }
+  __syncthreads();
+  if (half == 1) return;
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+#pragma unroll
+    for (int t = 0; t < 4; ++t) D[j][t] += pr[4 * j + t];
+  s1[0] += pr[16]; s1[1] += pr[17]; s2[0] += pr[18]; s2[1] += pr[19];
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
     s1[h] += __shfl_xor_sync(0xffffffffu, s1[h], 1);
     s1[h] += __shfl_xor_sync(0xffffffffu, s1[h], 2);
     s2[h] += __shfl_xor_sync(0xffffffffu, s2[h], 1);
     s2[h] += __shfl_xor_sync(0xffffffffu, s2[h], 2);
-    float* pp = part[warp][8 * h + g];
+    float* pp = part[tile][8 * h + g];
 #pragma unroll
     for (int j = 0; j < 2; ++j)
 #pragma unroll
@@ -512,11 +332,11 @@ __global__ void __launch_bounds__(128) head_compute_kernel(
   }
   __syncwarp();
 
-  // finish: two lanes per token of this warp, 8 channels each
+  // finish: two lanes per token of this tile, 8 channels each
   const int tt = lane >> 1, ch = lane & 1;
-  const int tok = tok0 + 16 * warp + tt;
+  const int tok = tok0 + 16 * tile + tt;
   if (tok < N) {
-    const float* pt = part[warp][tt];
+    const float* pt = part[tile][tt];
     const float mu = pt[kHC] / (float)d;
     const float var = fmaxf(pt[kHC + 1] / (float)d - mu * mu, 0.f);
     const float rs = rsqrtf(var + 1e-6f);
@@ -555,22 +375,6 @@ cudaError_t launch_head_tables(const float* mod, int n_items, int mod_stride, in
   return cudaGetLastError();
 }
 
-cudaError_t launch_head_reuse(float* x, const __nv_bfloat16* cache, const SlotMap& map, int N, int d,
-                              const __nv_bfloat16* wp_k, const float* tab_k, const float* wsum,
-                              const float* gram, float dsig, cudaStream_t st, float* vout) {
-  if (map.n <= 0) return cudaSuccess;
-  if (d % 32 != 0) return cudaErrorInvalidValue;
-  static std::atomic<unsigned long long> configured{0};
-  const cudaError_t e = configure_once_per_device(configured, [] {
-    return cudaFuncSetAttribute(head_reuse_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                kReuseSmem);
-  });
-  if (e != cudaSuccess) return e;
-  const dim3 grid((unsigned)((N + kReuseTok - 1) / kReuseTok), (unsigned)map.n);
-  return launch_pdl(head_reuse_kernel, grid, dim3(32 * kReuseWarps), kReuseSmem, st, x, cache, map,
-                    N, d, wp_k, tab_k, wsum, gram, dsig, vout);
-}
-
 cudaError_t launch_head_compute(const float* hL, float* x, float* xj, __nv_bfloat16* cache,
                                 const SlotMap& map, int N, int d, const __nv_bfloat16* we_frag,
                                 const __nv_bfloat16* wp_k, const float* tab_k, float dsig,
@@ -584,8 +388,8 @@ cudaError_t launch_head_compute(const float* hL, float* x, float* xj, __nv_bfloa
   });
   if (e != cudaSuccess) return e;
   const dim3 grid((unsigned)((N + kCmpTok - 1) / kCmpTok), (unsigned)map.n);
-  return launch_pdl(head_compute_kernel, grid, dim3(128), kCmpSmem, st, hL, x, xj, cache, map, N, d,
-                    we_frag, wp_k, tab_k, dsig, vout);
+  return launch_pdl(head_compute_kernel, grid, dim3(32 * kCmpWarps), kCmpSmem, st, hL, x, xj, cache,
+                    map, N, d, we_frag, wp_k, tab_k, dsig, vout);
 }
 
 void head_we_fragments(const float* w_eT, int d, uint16_t* out) {

@@ -96,11 +96,14 @@ int head_b_rows();
 cudaError_t launch_head_tables(const float* mod, int n_items, int mod_stride, int fin_off, int d,
                                const float* w_f, const float* b_f, const float* w_eT,
                                __nv_bfloat16* wp, float* tab, cudaStream_t st);
-// reuse step (wp_k, tab_k: the step's tables, indexed by scene; wsum: row
-// sums of W_e^T; gram: W_e^T W_e [16][16])
-cudaError_t launch_head_reuse(float* x, const __nv_bfloat16* cache, const SlotMap& map, int N, int d,
-                              const __nv_bfloat16* wp_k, const float* tab_k, const float* wsum,
-                              const float* gram, float dsig, cudaStream_t st, float* vout = nullptr);
+// reuse step on tcgen05 (reuse_tc.cu): tmC over the cache [B_max N][d] bf16
+// (box 64 x 128), tmB over the head tables' B rows [K B_max 48][d] (box 64 x
+// 48); b_row0: first B row of this step; tab_k: the step's fp32 tables; wsum:
+// row sums of W_e^T; gram: W_e^T W_e [16][16]; err: the model's error word
+cudaError_t launch_head_reuse_tc(const CUtensorMap& tmC, const CUtensorMap& tmB, float* x,
+                                 const SlotMap& map, int N, int d, int b_row0, const float* tab_k,
+                                 const float* wsum, const float* gram, float dsig, int* err,
+                                 cudaStream_t st, float* vout = nullptr);
 // compute step: writes the cache rows, x_j <- x, x += dsig v; we_frag: W_e^T
 // (16 x d, bf16) in the fragment order head_we_fragments builds (host)
 cudaError_t launch_head_compute(const float* hL, float* x, float* xj, __nv_bfloat16* cache,

@@ -65,6 +65,7 @@ struct dc_model {
   bool head_tc = false;
   __nv_bfloat16 *head_wp = nullptr, *cond_xs = nullptr, *we_frag = nullptr;
   CUtensorMap tm_ada, tm_xs;  // adaLN weight and the split activations (bf16 models)
+  CUtensorMap tm_cache, tm_headb;  // the cache rows and the head tables' B rows (reuse steps)
   float *wsum = nullptr, *head_tab = nullptr;
   CUtensorMap tm_a, tm_oact, tm_m, tm_qkv, tm_u32, tm_h32;
   long long launches = 0;
@@ -449,9 +450,9 @@ dc_status enqueue_reuse(dc_model* m, float* lat, const float* mod_k, const SlotM
   // x_k read, x_{k+1} written and x_j read by the drift check (3 N C fp32)
   if (m->head_tc && sizeof(T) == 2) {
     DC_LAUNCH(DC_PROF_REUSE, 2.0 * M * m->d * 3 * m->C, M * ((double)m->d * m->elt + 12.0 * m->C),
-              dc::launch_head_reuse(lat, reinterpret_cast<const __nv_bfloat16*>(m->r), map, m->N,
-                                    m->d, head_wp_k(m, k, Bi), head_tab_k(m, k, Bi), m->wsum,
-                                    m->gram, dsig, st, vout));
+              dc::launch_head_reuse_tc(m->tm_cache, m->tm_headb, lat, map, m->N, m->d,
+                                       (k - 1) * Bi * dc::head_b_rows(), head_tab_k(m, k, Bi),
+                                       m->wsum, m->gram, dsig, m->err_d, st, vout));
   } else {
     DC_LAUNCH(DC_PROF_REUSE, 4.0 * M * m->d * m->C, M * ((double)m->d * m->elt + 12.0 * m->C),
               dc::launch_final_reuse<T>(lat, static_cast<const T*>(m->r), m->w_eT, map, m->N, m->C,
@@ -1274,6 +1275,12 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
     if ((s = make_map(&m->tm_u32, m->u, d, B * N, bm, true)) != DC_OK) return fail(s);
     if ((s = make_map(&m->tm_h32, m->h, d, B * N, bm, true)) != DC_OK) return fail(s);
     if ((s = make_map(&m->tm_ada, m->w_ada, d, m->mod_stride, 128)) != DC_OK) return fail(s);
+    if (m->head_tc) {
+      if ((s = make_map(&m->tm_cache, m->r, d, B * N, 128)) != DC_OK) return fail(s);
+      if ((s = make_map(&m->tm_headb, m->head_wp, d, K * B * dc::head_b_rows(), dc::head_b_rows())) !=
+          DC_OK)
+        return fail(s);
+    }
     if ((s = make_map(&m->tm_xs, m->cond_xs, d, cond_groups(K * B) * 2 * dc::cond_tc_group_rows(),
                       128)) != DC_OK)
       return fail(s);
