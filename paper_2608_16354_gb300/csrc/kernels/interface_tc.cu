@@ -45,7 +45,9 @@ namespace {
 
 constexpr int kHC = 16;          // latent channels the tensor-core interface supports
 constexpr int kHeadTab = 2 * kHC + kHC * kHC;  // S', beta, G_s per (step, scene)
-constexpr int kBRows = 3 * kHC;  // B rows per (step, scene): W_e^T, W' hi, W' lo
+// B rows per (step, scene): W_e^T, W' hi, W' lo, a row of ones (the row sums
+// of the reuse step's cache rows) and zero rows up to a multiple of 16
+constexpr int kBRows = 4 * kHC;
 
 __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
                                                uint32_t a3, uint32_t b0, uint32_t b1) {
@@ -88,9 +90,9 @@ __device__ __forceinline__ void split_pair(float a, float b, uint32_t* hi, uint3
 
 // ------------------------------------------------ per (step, scene) tables
 
-// One CTA per (step, scene) item: the reuse step's B rows [48][d] in bf16 --
+// One CTA per (step, scene) item: the reuse step's B rows [64][d] in bf16 --
 // W_e^T (rows 0-15), W' = (1 + scale) W_f as hi (16-31) and lo (32-47)
-// halves -- and S', beta, G_s (fp32).
+// halves, ones (48), zeros (49-63) -- and S', beta, G_s (fp32).
 __global__ void __launch_bounds__(256) head_tables_kernel(
     const float* __restrict__ mod, int mod_stride, int fin_off, int d,
     const float* __restrict__ w_f, const float* __restrict__ b_f, const float* __restrict__ w_eT,
@@ -106,6 +108,7 @@ __global__ void __launch_bounds__(256) head_tables_kernel(
     w[(size_t)c * d + e] = __float2bfloat16_rn(w_eT[i]);
     w[(size_t)(kHC + c) * d + e] = hi;
     w[(size_t)(2 * kHC + c) * d + e] = __float2bfloat16_rn(v - __bfloat162float(hi));
+    w[(size_t)(3 * kHC + c) * d + e] = __float2bfloat16_rn(c == 0 ? 1.f : 0.f);
   }
   float* t = tab + (size_t)item * kHeadTab;
   const int a = threadIdx.x >> 4, c = threadIdx.x & 15;  // G_s[a][c]

@@ -97,8 +97,8 @@ cudaError_t launch_head_tables(const float* mod, int n_items, int mod_stride, in
                                const float* w_f, const float* b_f, const float* w_eT,
                                __nv_bfloat16* wp, float* tab, cudaStream_t st);
 // reuse step on tcgen05 (reuse_tc.cu): tmC over the cache [B_max N][d] bf16
-// (box 64 x 128), tmB over the head tables' B rows [K B_max 48][d] (box 64 x
-// 48); b_row0: first B row of this step; tab_k: the step's fp32 tables; wsum:
+// (box 64 x 128), tmB over the head tables' B rows [K B_max 64][d] (box 64 x
+// 64); b_row0: first B row of this step; tab_k: the step's fp32 tables; wsum:
 // row sums of W_e^T; gram: W_e^T W_e [16][16]; err: the model's error word
 cudaError_t launch_head_reuse_tc(const CUtensorMap& tmC, const CUtensorMap& tmB, float* x,
                                  const SlotMap& map, int N, int d, int b_row0, const float* tab_k,

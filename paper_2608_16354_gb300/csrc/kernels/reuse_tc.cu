@@ -7,19 +7,18 @@
 //   sum h   = x . w_sum + sum c
 //   sum h^2 = x^T G x + 2 x . A + sum c^2,   A = W_e c
 //   v_c     = rs (P_c - mu S'_c) + beta_c
-// The contractions over d, [A | Q] = c [W_e^T | W'hi | W'lo]^T (48 columns
-// per token), run on tcgen05: per CTA a 128-token tile of one scene is the A
-// operand (M = 128), the step's 48 B rows the B operand (N = 48), streamed
-// in 64-column stages by TMA, the 128 x 48 fp32 accumulator in TMEM.  The
-// four epilogue warps (one token row per thread) also take sum c and sum c^2
-// of each staged row from shared memory before releasing the stage, then
-// read the accumulator row and finish the token: the kernel reads each cache
-// row once, and the tensor work (6 K-steps of 16 per 64 columns at N = 48)
-// stays far below the copy time.
+// Every contraction over d runs on tcgen05: per CTA a 128-token tile of one
+// scene is the A operand (M = 128), streamed in 64-column stages by TMA with
+// the step's 64 B rows; per 16-deep step one MMA forms [A | Q | sum c] =
+// c [W_e^T | W'hi | W'lo | 1 | 0]^T (N = 64) and a second one the tile's Gram
+// matrix c c^T (B = the same tile, N = 128), whose diagonal is sum c^2 of
+// each token.  The fp32 accumulators (64 + 128 columns) stay in TMEM until the
+// four epilogue warps (one token row per thread) read their row and finish
+// the token, so each cache row is read once and no thread touches it.
 //
-//   warp 0      TMA: cache tile [128 rows][64] and B tile [48][64] per stage
-//   warp 1      tcgen05.mma (M = 128, N = 48, K = 16) into TMEM; owns TMEM
-//   warps 2-5   row sums from shared memory, then the per-token finish
+//   warp 0      TMA: cache tile [128 rows][64] and B tile [64][64] per stage
+//   warp 1      tcgen05.mma into TMEM; owns TMEM
+//   warps 2-5   the per-token finish
 // Every mbarrier wait is bounded.
 #include "common.cuh"
 #include "kernels.h"
@@ -30,19 +29,20 @@ namespace {
 
 constexpr int kRC = 16;                            // latent channels
 constexpr int kRTab = 2 * kRC + kRC * kRC;         // S', beta, G_s per (step, scene)
-constexpr int kRB = 3 * kRC;                       // B rows: W_e^T, W' hi, W' lo
+constexpr int kRB = 4 * kRC;                       // B rows: W_e^T, W' hi, W' lo, ones
 constexpr int kRM = 128, kRK = 64;                 // tokens per CTA, columns per stage
 constexpr int kRStages = 8;
 constexpr int kRABytes = kRM * kRK * 2;            // 16 KB
-constexpr int kRBBytes = kRB * kRK * 2;            // 6 KB
-constexpr int kRStageBytes = kRABytes + kRBBytes;  // 22 KB (a multiple of 1024)
+constexpr int kRBBytes = kRB * kRK * 2;            // 8 KB
+constexpr int kRStageBytes = kRABytes + kRBBytes;  // 24 KB (a multiple of 1024)
 constexpr int kRThreads = 192;
-constexpr uint32_t kRIdesc = idesc_bf16_f32(kRM, kRB);
-constexpr int kRTmemCols = 64;
+constexpr uint32_t kRIdesc = idesc_bf16_f32(kRM, kRB);     // [A | Q | sum c]: columns 0-63
+constexpr uint32_t kRIdescG = idesc_bf16_f32(kRM, kRM);    // Gram: columns 64-191
+constexpr int kRTmemCols = 256;
 
 struct __align__(8) ReuseBars {
   uint64_t full[kRStages];
-  uint64_t empty[kRStages];  // the stage's MMAs have read it and the row sums are taken
+  uint64_t empty[kRStages];  // the stage's MMAs have read it
   uint64_t tmem_full;
   uint32_t tmem_base;
   int abort;
@@ -51,8 +51,6 @@ struct __align__(8) ReuseBars {
 
 constexpr int kRSmem = 1024 + kRStages * kRStageBytes + 256 +
                        (kRTab + kRC + kRC * kRC) * 4;  // + tables
-
-__device__ __forceinline__ int sw128_chunk(int r, int c) { return r * 128 + ((c ^ (r & 7)) << 4); }
 
 __global__ void __launch_bounds__(kRThreads, 1)
     head_reuse_tc_kernel(const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmB,
@@ -77,7 +75,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
     bar->wlim = work_wait_limit(err);
     for (int s = 0; s < kRStages; ++s) {
       mbar_init(&bar->full[s], 1);
-      mbar_init(&bar->empty[s], 1 + 4);
+      mbar_init(&bar->empty[s], 1);
     }
     mbar_init(&bar->tmem_full, 1);
     fence_barrier_init();
@@ -133,9 +131,11 @@ __global__ void __launch_bounds__(kRThreads, 1)
         const uint32_t sa = smem_u32(smem + (size_t)stage * kRStageBytes);
         const uint64_t da = sw128_kmajor_desc(sa), db = sw128_kmajor_desc(sa + kRABytes);
 #pragma unroll
-        for (int kk = 0; kk < kRK / 16; ++kk)
-          tc_mma_f16(tmem, da + (uint32_t)(kk * 2), db + (uint32_t)(kk * 2), kRIdesc,
-                     (kb | kk) != 0 ? 1u : 0u);
+        for (int kk = 0; kk < kRK / 16; ++kk) {
+          const uint32_t acc = (kb | kk) != 0 ? 1u : 0u;
+          tc_mma_f16(tmem, da + (uint32_t)(kk * 2), db + (uint32_t)(kk * 2), kRIdesc, acc);
+          tc_mma_f16(tmem + kRB, da + (uint32_t)(kk * 2), da + (uint32_t)(kk * 2), kRIdescG, acc);
+        }
         tc_commit(&bar->empty[stage]);
       }
       __syncwarp();
@@ -148,45 +148,29 @@ __global__ void __launch_bounds__(kRThreads, 1)
     __syncwarp();
     mbar_wait_warp(&bar->tmem_full, 0, err, kDevTimeoutMma);
   } else {
-    // ---------------------------------------------- row sums, then finish
+    // ------------------------------------------------------ token finish
     const int q = warp & 3;            // TMEM lane quarter
     const int r = q * 32 + lane;       // token row of the tile owned by this thread
     for (int i = threadIdx.x - 64; i < kRTab; i += 128) stab[i] = tab_k[(size_t)scene * kRTab + i];
     if (threadIdx.x - 64 < kRC) stab[kRTab + threadIdx.x - 64] = wsum[threadIdx.x - 64];
     for (int i = threadIdx.x - 64; i < kRC * kRC; i += 128) stab[kRTab + kRC + i] = gram[i];
-    float s1a = 0.f, s1b = 0.f, s2a = 0.f, s2b = 0.f;
-    int stage = 0;
-    uint32_t phase = 0;
-    bool ok = true;
-    for (int kb = 0; kb < KB; ++kb) {
-      if (!mbar_wait_warp(&bar->full[stage], phase, err, kDevTimeoutEpi, wlim)) { ok = false; break; }
-      const uint8_t* st = smem + (size_t)stage * kRStageBytes;
-#pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        const uint4 w = *reinterpret_cast<const uint4*>(st + sw128_chunk(r, c));
-        const uint32_t wv[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-        for (int p = 0; p < 4; ++p) {
-          const float lo = __uint_as_float(wv[p] << 16), hi = __uint_as_float(wv[p] & 0xFFFF0000u);
-          s1a += lo; s1b += hi;
-          s2a = fmaf(lo, lo, s2a); s2b = fmaf(hi, hi, s2b);
-        }
-      }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&bar->empty[stage]);
-      if (++stage == kRStages) { stage = 0; phase ^= 1; }
-    }
     named_bar(1, 128);  // the tables are staged
-    if (ok && mbar_wait_warp(&bar->tmem_full, 0, err, kDevTimeoutEpi, wlim)) {
+    if (mbar_wait_warp(&bar->tmem_full, 0, err, kDevTimeoutEpi, wlim)) {
       tc_fence_after();
-      float acc[64];
+      float acc[64], gv[32];
       {
         float* a0 = acc;
         float* a1 = acc + 32;
-        tmem_ld32(tmem + ((uint32_t)(q * 32) << 16), *reinterpret_cast<float(*)[32]>(a0));
-        tmem_ld32(tmem + 32 + ((uint32_t)(q * 32) << 16), *reinterpret_cast<float(*)[32]>(a1));
+        const uint32_t lanes = (uint32_t)(q * 32) << 16;
+        tmem_ld32(tmem + lanes, *reinterpret_cast<float(*)[32]>(a0));
+        tmem_ld32(tmem + 32 + lanes, *reinterpret_cast<float(*)[32]>(a1));
+        tmem_ld32(tmem + kRB + 32 * q + lanes, gv);  // Gram columns of this warp's tokens
         tmem_ld_wait();
       }
+      float sumsq = 0.f;  // the Gram diagonal: column r of row r
+#pragma unroll
+      for (int k = 0; k < 32; ++k) sumsq = k == lane ? gv[k] : sumsq;
+      const float sumc = acc[3 * kRC];
       const int tok = tok0 + r;
       if (tok < N) {
         float* xr = x + ((size_t)scene * N + tok) * kRC;
@@ -198,7 +182,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
         }
         const float *S = stab, *beta = stab + kRC, *Gs = stab + 2 * kRC, *ws = stab + kRTab,
                     *G = stab + kRTab + kRC;
-        float sum1 = s1a + s1b, xA = 0.f, xGx = 0.f;
+        float sum1 = sumc, xA = 0.f, xGx = 0.f;
 #pragma unroll
         for (int a = 0; a < kRC; ++a) {
           xA = fmaf(xv[a], acc[a], xA);
@@ -208,7 +192,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
           for (int b2 = 0; b2 < kRC; ++b2) t = fmaf(G[a * kRC + b2], xv[b2], t);
           xGx = fmaf(xv[a], t, xGx);
         }
-        const float sq = xGx + 2.f * xA + (s2a + s2b);
+        const float sq = xGx + 2.f * xA + sumsq;
         const float mu = sum1 / (float)d;
         const float var = fmaxf(sq / (float)d - mu * mu, 0.f);
         const float rs = rsqrtf(var + 1e-6f);
