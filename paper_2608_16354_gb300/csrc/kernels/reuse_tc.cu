@@ -40,19 +40,6 @@ constexpr uint32_t kRIdesc = idesc_bf16_f32(kRM, kRB);     // [A | Q | sum c]: c
 constexpr uint32_t kRIdescG = idesc_bf16_f32(kRM, kRM);    // Gram: columns 64-191
 constexpr int kRTmemCols = 256;
 
-// Cache tiles are also prefetched into L2 this many stages ahead of their
-// load into the ring, so that about twice the ring's bytes are in flight from
-// HBM per SM (the ring alone left the stream latency-bound at about half of
-// the copy bandwidth).
-constexpr int kRPrefetch = kRStages;
-
-__device__ __forceinline__ void tma_prefetch_l2_2d(const CUtensorMap* map, int x, int y) {
-  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
-                   reinterpret_cast<uint64_t>(map)),
-               "r"(x), "r"(y)
-               : "memory");
-}
-
 struct __align__(8) ReuseBars {
   uint64_t full[kRStages];
   uint64_t empty[kRStages];  // the stage's MMAs have read it
@@ -127,8 +114,6 @@ __global__ void __launch_bounds__(kRThreads, 1)
       uint8_t* st = smem + (size_t)stage * kRStageBytes;
       if (lane == l0) tma_load_2d(st, &tmC, &bar->full[stage], kb * kRK, crow);
       if (lane == l0 + 1) tma_load_2d(st + kRABytes, &tmB, &bar->full[stage], kb * kRK, brow);
-      if (lane == ((l0 + 2) & 7) && kb + kRPrefetch < KB)
-        tma_prefetch_l2_2d(&tmC, (kb + kRPrefetch) * kRK, crow);
       __syncwarp();
       last_phase[stage] = (int)phase;
       if (++stage == kRStages) { stage = 0; phase ^= 1; }
