@@ -472,15 +472,27 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
       uint32_t pk[64];
       {
         uint32_t s0[32], s1[32], s2[32], s3[32];
+        const int valid = min(128, N - j * 128);
+        float2 rs2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+        // With P aliased onto S_t nothing waits for S_t to be in registers,
+        // so on a full key tile after the first the four 32-column loads are
+        // chained with the exponentials: each chunk's load is in flight
+        // while the previous chunk is exponentiated.
+        const bool chained = Cfg::kAliasP && j > 0 && valid == 128;
         tc_fence_after();
-        tmem_ld32_async(tS + 0, s0);
-        tmem_ld32_async(tS + 32, s1);
-        tmem_ld32_async(tS + 64, s2);
-        tmem_ld32_async(tS + 96, s3);
-        tmem_ld_wait_regs(s0);
-        tmem_ld_wait_regs(s1);
-        tmem_ld_wait_regs(s2);
-        tmem_ld_wait_regs(s3);
+        if (chained) {
+          tmem_ld32_async(tS + 0, s0);
+          tmem_ld_wait_regs(s0);
+        } else {
+          tmem_ld32_async(tS + 0, s0);
+          tmem_ld32_async(tS + 32, s1);
+          tmem_ld32_async(tS + 64, s2);
+          tmem_ld32_async(tS + 96, s3);
+          tmem_ld_wait_regs(s0);
+          tmem_ld_wait_regs(s1);
+          tmem_ld_wait_regs(s2);
+          tmem_ld_wait_regs(s3);
+        }
         // S is in registers: hand S_t back to the MMA warp (with P aliased
         // onto S_t, the hand-back is p_full below)
         if (!Cfg::kAliasP) {
@@ -488,9 +500,30 @@ __global__ void __launch_bounds__(AttCfg<DHP, NQ>::kThreads, 1)
           __syncwarp();
           if (lane == 0) mbar_arrive(&bar->s_free[t]);
         }
-        const int valid = min(128, N - j * 128);
-        float2 rs2[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-        if (j > 0 && valid == 128) {
+        if (chained) {
+          float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+          tmem_ld32_async(tS + 32, s1);
+          p_chunk_max(s0, scale_log2, -ref, rs2, pk + 0, m4);
+          tmem_ld_wait_regs(s1);
+          tmem_ld32_async(tS + 64, s2);
+          p_chunk_max(s1, scale_log2, -ref, rs2, pk + 16, m4);
+          tmem_ld_wait_regs(s2);
+          tmem_ld32_async(tS + 96, s3);
+          p_chunk_max(s2, scale_log2, -ref, rs2, pk + 32, m4);
+          tmem_ld_wait_regs(s3);
+          p_chunk_max(s3, scale_log2, -ref, rs2, pk + 48, m4);
+          const float tm = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3])) * scale_log2;
+          if (tm > ref + kRefSlack) {  // as below: move the reference, recompute P
+            c = ex2_mufu(ref - tm);
+            ref = tm;
+            rs2[0] = make_float2(0.f, 0.f);
+            rs2[1] = make_float2(0.f, 0.f);
+            p_chunk<false>(s0, 0, 128, scale_log2, -ref, rs2, pk + 0);
+            p_chunk<false>(s1, 1, 128, scale_log2, -ref, rs2, pk + 16);
+            p_chunk<false>(s2, 2, 128, scale_log2, -ref, rs2, pk + 32);
+            p_chunk<false>(s3, 3, 128, scale_log2, -ref, rs2, pk + 48);
+          }
+        } else if (j > 0 && valid == 128) {
           // Speculate that the reference stays: exponentials against the
           // current reference with the row max computed alongside, so the max
           // is off the critical path.  A row whose max exceeds the reference by
