@@ -312,7 +312,7 @@ dc_status dc_denoise_host(dc_model* m, float* host_latents, const dc_cond* cond,
  * latents and record equal the uninterrupted call's bit for bit.  Use:
  * preempting a long call, or moving it to another model instance or box.
  * Layout (caller-owned host memory, native byte order):
- *   header, 128 bytes: char magic[8] "DCSNAP01"; uint32 version (2);
+ *   header, 128 bytes: char magic[8] "DCSNAP01"; uint32 version (3);
  *     int32 B, K, cfg (0 or 1), k_done, dtype, n_tokens, d_model, channels;
  *     uint32 element bytes of c; uint64 digest; uint64 total bytes;
  *     int64 backbone_calls; 56 zero bytes
@@ -324,6 +324,8 @@ dc_status dc_denoise_host(dc_model* m, float* host_latents, const dc_cond* cond,
  *   at the next multiple of 256: float latents [B][N][C], float x_j [B][N][C]
  *   at the next multiple of 256: c [B_i][N][d] in the model dtype
  *     (B_i = 2B with guidance, else B)
+ *   bf16 models with 16 channels only, at the next multiple of 256: float
+ *     [B_i][N][2], the sum and the sum of squares of each cache row's values
  * digest: FNV-1a (64-bit) of the call's inputs (trajectories, sigmas, tau,
  * veto, cfg_scale, and the forced actions or the anchor responses). */
 

@@ -1,12 +1,14 @@
-// Interface + Euler kernels of the bf16 path on the tensor cores (Eq. 1: the
-// interface H_k on compute and on reuse steps, with the cache write of the
-// compute step).
+// Interface + Euler kernels of the bf16 path (Eq. 1: the interface H_k on
+// compute steps with the cache write, and the per (step, scene) tables that
+// both the compute and the reuse step read).
 //
 // The cache holds, per scene, c = h_L - x W_e^T (bf16 [N][d]) from the
 // scene's last full evaluation: the block-stack residual r = h_L - u plus
 // the part b_e + pos of the embedding that does not depend on the latent,
 // so a reuse step rebuilds u_k + r_j = x_k W_e^T + c_j from the latent alone
-// and reads nothing else of size N x d.
+// and reads nothing else of size N x d.  Beside each cache row the compute
+// step stores sum_e c_e and sum_e c_e^2 of its bf16 values (fp32), which no
+// later latent changes.
 //
 // The head is linear in the LayerNorm output, so with a_e = (h_e - mu) rs
 // (1 + s_e) + sh_e and W'[c][e] = (1 + s_e) W_f[c][e]:
@@ -19,21 +21,16 @@
 //   P_c      = (x G_s)_c + Q_c,  Q_c = sum_e c_e W'[c][e],  G_s = W_e^T diag(1 + s) W_f^T [C][C]
 //   sum h    = x . w_sum + sum c,                           w_sum = sum_e W_e^T[:, e]
 //   sum h^2  = x^T G x + 2 x . A + sum c^2,  A = W_e c,     G = W_e^T W_e
-// so the contractions over d read only c: [A | Q] = c [W_e^T | W'hi | W'lo],
-// 48 columns, on the tensor cores (mma.sync m16n8k16, bf16 in, fp32 out).
-// On a compute step P = h [W'hi | W'lo] with h split into bf16 hi + lo
-// halves (hi W'hi + lo W'hi + hi W'lo), and c = h - x W_e^T is written.
+// so its only contraction over d is [A | Q] = c [W_e^T | W'hi | W'lo]^T, 48
+// columns (reuse_tc.cu, on tcgen05).  On a compute step P = h [W'hi | W'lo]
+// with h split into bf16 hi + lo halves (hi W'hi + lo W'hi + hi W'lo), on
+// mma.sync m16n8k16, and c = h - x W_e^T is written.
 //
 // Layout trick: the order of the contraction index inside a 32-column block
 // is free as long as both operands use it, so each thread loads 8
-// consecutive columns of a row (16 B of bf16, 32 B of fp32) and those land
-// exactly in its A fragment of the block's two 16-deep steps; the B
-// fragments are then 16-byte loads of 8 consecutive columns of a W row.
-//
-// A CTA (4 warps) takes 32 tokens of one scene (reuse; 16 on compute
-// steps); each warp takes every 4th 32-column block of d for all of the
-// CTA's tokens, and the partial sums of the four warps are added in shared
-// memory in a fixed order (deterministic).  C = 16 channels.
+// consecutive columns of a row (32 B of fp32) and those land exactly in its
+// A fragment of the block's two 16-deep steps; the B fragments are then
+// 16-byte loads of 8 consecutive columns of a W row.  C = 16 channels.
 #include <cstring>
 
 #include "common.cuh"
@@ -45,9 +42,8 @@ namespace {
 
 constexpr int kHC = 16;          // latent channels the tensor-core interface supports
 constexpr int kHeadTab = 2 * kHC + kHC * kHC;  // S', beta, G_s per (step, scene)
-// B rows per (step, scene): W_e^T, W' hi, W' lo, a row of ones (the row sums
-// of the reuse step's cache rows) and zero rows up to a multiple of 16
-constexpr int kBRows = 4 * kHC;
+// B rows per (step, scene): W_e^T, W' hi, W' lo
+constexpr int kBRows = 3 * kHC;
 
 __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
                                                uint32_t a3, uint32_t b0, uint32_t b1) {
@@ -78,6 +74,17 @@ __device__ __forceinline__ uint32_t pack_bf2(float lo_elem, float hi_elem) {
   __nv_bfloat162 t = __floats2bfloat162_rn(lo_elem, hi_elem);
   return *reinterpret_cast<uint32_t*>(&t);
 }
+// a pair packed to bf16, with the packed values and their squares added to s
+// and q (in this order: a, then b)
+__device__ __forceinline__ uint32_t pack_bf2_sums(float a, float b, float& s, float& q) {
+  const __nv_bfloat162 t = __floats2bfloat162_rn(a, b);
+  const float2 f = __bfloat1622float2(t);
+  s += f.x;
+  s += f.y;
+  q = fmaf(f.x, f.x, q);
+  q = fmaf(f.y, f.y, q);
+  return *reinterpret_cast<const uint32_t*>(&t);
+}
 // v = hi + lo with hi = bf16(v), lo = bf16(v - hi), for a pair of values
 __device__ __forceinline__ void split_pair(float a, float b, uint32_t* hi, uint32_t* lo) {
   const __nv_bfloat16 ha = __float2bfloat16_rn(a), hb = __float2bfloat16_rn(b);
@@ -90,9 +97,9 @@ __device__ __forceinline__ void split_pair(float a, float b, uint32_t* hi, uint3
 
 // ------------------------------------------------ per (step, scene) tables
 
-// One CTA per (step, scene) item: the reuse step's B rows [64][d] in bf16 --
-// W_e^T (rows 0-15), W' = (1 + scale) W_f as hi (16-31) and lo (32-47)
-// halves, ones (48), zeros (49-63) -- and S', beta, G_s (fp32).
+// One CTA per (step, scene) item: the B rows [48][d] in bf16 -- W_e^T (rows
+// 0-15), W' = (1 + scale) W_f as hi (16-31) and lo (32-47) halves -- and S',
+// beta, G_s (fp32).
 __global__ void __launch_bounds__(256) head_tables_kernel(
     const float* __restrict__ mod, int mod_stride, int fin_off, int d,
     const float* __restrict__ w_f, const float* __restrict__ b_f, const float* __restrict__ w_eT,
@@ -108,7 +115,6 @@ __global__ void __launch_bounds__(256) head_tables_kernel(
     w[(size_t)c * d + e] = __float2bfloat16_rn(w_eT[i]);
     w[(size_t)(kHC + c) * d + e] = hi;
     w[(size_t)(2 * kHC + c) * d + e] = __float2bfloat16_rn(v - __bfloat162float(hi));
-    w[(size_t)(3 * kHC + c) * d + e] = __float2bfloat16_rn(c == 0 ? 1.f : 0.f);
   }
   float* t = tab + (size_t)item * kHeadTab;
   const int a = threadIdx.x >> 4, c = threadIdx.x & 15;  // G_s[a][c]
@@ -139,12 +145,12 @@ constexpr int kCmpStages = 4;                // blocks in flight per half of d
 constexpr int kCmpBPieces = 2 * kHC * 4 + 64;  // 16-byte pieces of one half's B block
 constexpr int kCmpStageBytes = kCmpWarps * 2048 + 2 * kCmpBPieces * 16;
 constexpr int kCmpSmem = kCmpStages * kCmpStageBytes;
-constexpr int kCmpPartFloats = 20;           // D (16), sum h and sum h^2 of two rows (4)
+constexpr int kCmpPartFloats = 24;           // D (16); sum h, sum h^2, sum c, sum c^2 of two rows (8)
 static_assert(kCmpTiles * 32 * kCmpPartFloats * 4 <= kCmpSmem, "partials exceed the ring");
 
 // Compute step of the scenes in `map` (h_L rows packed by slot): the cache
-// row c = h_L - x W_e^T is written, v = head(h_L), x_j <- x, x += dsig v (or
-// v to vout).  Each 16-token tile is taken by two warps, one per half of d;
+// row c = h_L - x W_e^T is written with its sums (sum c, sum c^2 of the bf16
+// values, to cstat), v = head(h_L), x_j <- x, x += dsig v (or v to vout).  Each 16-token tile is taken by two warps, one per half of d;
 // per step of the loop the CTA stages every warp's h_L rows and, for the two
 // blocks in flight, the W' rows and W_e^T fragments (shared by the four warps
 // of a half) in a kCmpStages-deep cp.async ring.  x W_e^T runs on the tensor
@@ -153,13 +159,13 @@ static_assert(kCmpTiles * 32 * kCmpPartFloats * 4 <= kCmpSmem, "partials exceed 
 // + 1 of rows g and g + 8).
 __global__ void __launch_bounds__(256) head_compute_kernel(
     const float* __restrict__ hL, float* __restrict__ x, float* __restrict__ xj,
-    __nv_bfloat16* __restrict__ cache, SlotMap map, int N, int d,
+    __nv_bfloat16* __restrict__ cache, float2* __restrict__ cstat, SlotMap map, int N, int d,
     const __nv_bfloat16* __restrict__ we_frag, const __nv_bfloat16* __restrict__ wp_k,
     const float* __restrict__ tab_k, float dsig, float* __restrict__ vout) {
   pdl_trigger();
   pdl_wait();
   extern __shared__ __align__(16) uint8_t csm[];
-  __shared__ float part[kCmpTiles][16][kHC + 2];  // per token: P, sum h, sum h^2
+  __shared__ float part[kCmpTiles][16][kHC + 4];  // per token: P, sum h, sum h^2, sum c, sum c^2
   __shared__ float stab[2 * kHC];                 // S', beta
   const int slot = blockIdx.y, scene = map.scene[slot];
   const int tok0 = blockIdx.x * kCmpTok;
@@ -222,7 +228,8 @@ __global__ void __launch_bounds__(256) head_compute_kernel(
   for (int j = 0; j < 4; ++j)
 #pragma unroll
     for (int t = 0; t < 4; ++t) D[j][t] = 0.f;
-  float s1[2] = {0.f, 0.f}, s2[2] = {0.f, 0.f};
+  float s1[2] = {0.f, 0.f}, s2[2] = {0.f, 0.f};  // sum h, sum h^2 (rows g, g + 8)
+  float c1[2] = {0.f, 0.f}, c2[2] = {0.f, 0.f};  // sum c, sum c^2 of the bf16 cache values
   const bool mine = half * nbh < nblk;
 #pragma unroll 1
   for (int i = 0; i < kCmpStages - 1; ++i) {
@@ -272,10 +279,10 @@ __global__ void __launch_bounds__(256) head_compute_kernel(
     for (int h = 0; h < 2; ++h) {
       if (ok[h]) {
         uint4 cw;
-        cw.x = pack_bf2(hv[h][0] - u[h][0], hv[h][1] - u[h][1]);
-        cw.y = pack_bf2(hv[h][2] - u[h][2], hv[h][3] - u[h][3]);
-        cw.z = pack_bf2(hv[h][4] - u[h][4], hv[h][5] - u[h][5]);
-        cw.w = pack_bf2(hv[h][6] - u[h][6], hv[h][7] - u[h][7]);
+        cw.x = pack_bf2_sums(hv[h][0] - u[h][0], hv[h][1] - u[h][1], c1[h], c2[h]);
+        cw.y = pack_bf2_sums(hv[h][2] - u[h][2], hv[h][3] - u[h][3], c1[h], c2[h]);
+        cw.z = pack_bf2_sums(hv[h][4] - u[h][4], hv[h][5] - u[h][5], c1[h], c2[h]);
+        cw.w = pack_bf2_sums(hv[h][6] - u[h][6], hv[h][7] - u[h][7], c1[h], c2[h]);
         __stcs(reinterpret_cast<uint4*>(cache + ((size_t)scene * N + row[h]) * d + e), cw);
       }
 #pragma unroll
@@ -309,6 +316,7 @@ __global__ void __launch_bounds__(256) head_compute_kernel(
 #pragma unroll
       for (int t = 0; t < 4; ++t) pr[4 * j + t] = D[j][t];
     pr[16] = s1[0]; pr[17] = s1[1]; pr[18] = s2[0]; pr[19] = s2[1];
+    pr[20] = c1[0]; pr[21] = c1[1]; pr[22] = c2[0]; pr[23] = c2[1];
   }
   __syncthreads();
   if (half == 1) return;
@@ -317,12 +325,17 @@ __global__ void __launch_bounds__(256) head_compute_kernel(
 #pragma unroll
     for (int t = 0; t < 4; ++t) D[j][t] += pr[4 * j + t];
   s1[0] += pr[16]; s1[1] += pr[17]; s2[0] += pr[18]; s2[1] += pr[19];
+  c1[0] += pr[20]; c1[1] += pr[21]; c2[0] += pr[22]; c2[1] += pr[23];
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
     s1[h] += __shfl_xor_sync(0xffffffffu, s1[h], 1);
     s1[h] += __shfl_xor_sync(0xffffffffu, s1[h], 2);
     s2[h] += __shfl_xor_sync(0xffffffffu, s2[h], 1);
     s2[h] += __shfl_xor_sync(0xffffffffu, s2[h], 2);
+    c1[h] += __shfl_xor_sync(0xffffffffu, c1[h], 1);
+    c1[h] += __shfl_xor_sync(0xffffffffu, c1[h], 2);
+    c2[h] += __shfl_xor_sync(0xffffffffu, c2[h], 1);
+    c2[h] += __shfl_xor_sync(0xffffffffu, c2[h], 2);
     float* pp = part[tile][8 * h + g];
 #pragma unroll
     for (int j = 0; j < 2; ++j)
@@ -331,6 +344,8 @@ __global__ void __launch_bounds__(256) head_compute_kernel(
     if (q == 0) {
       pp[kHC] = s1[h];
       pp[kHC + 1] = s2[h];
+      pp[kHC + 2] = c1[h];
+      pp[kHC + 3] = c2[h];
     }
   }
   __syncwarp();
@@ -349,6 +364,7 @@ __global__ void __launch_bounds__(256) head_compute_kernel(
       const int c = 8 * ch + cc;
       vv[cc] = fmaf(rs, pt[c] - mu * stab[c], stab[kHC + c]);
     }
+    if (ch == 0) cstat[(size_t)scene * N + tok] = make_float2(pt[kHC + 2], pt[kHC + 3]);
     const size_t xi = ((size_t)scene * N + tok) * kHC + 8 * ch;
     const float4 xo0 = *reinterpret_cast<const float4*>(x + xi);
     const float4 xo1 = *reinterpret_cast<const float4*>(x + xi + 4);
@@ -379,7 +395,7 @@ cudaError_t launch_head_tables(const float* mod, int n_items, int mod_stride, in
 }
 
 cudaError_t launch_head_compute(const float* hL, float* x, float* xj, __nv_bfloat16* cache,
-                                const SlotMap& map, int N, int d, const __nv_bfloat16* we_frag,
+                                float2* cstat, const SlotMap& map, int N, int d, const __nv_bfloat16* we_frag,
                                 const __nv_bfloat16* wp_k, const float* tab_k, float dsig,
                                 cudaStream_t st, float* vout) {
   if (map.n <= 0) return cudaSuccess;
@@ -392,7 +408,7 @@ cudaError_t launch_head_compute(const float* hL, float* x, float* xj, __nv_bfloa
   if (e != cudaSuccess) return e;
   const dim3 grid((unsigned)((N + kCmpTok - 1) / kCmpTok), (unsigned)map.n);
   return launch_pdl(head_compute_kernel, grid, dim3(32 * kCmpWarps), kCmpSmem, st, hL, x, xj, cache,
-                    map, N, d, we_frag, wp_k, tab_k, dsig, vout);
+                    cstat, map, N, d, we_frag, wp_k, tab_k, dsig, vout);
 }
 
 void head_we_fragments(const float* w_eT, int d, uint16_t* out) {

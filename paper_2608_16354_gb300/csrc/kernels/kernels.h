@@ -88,27 +88,31 @@ template <typename T>
 cudaError_t launch_cache_to_residual(const T* c, const float* b_e, const T* pos, int N, int d, T* out,
                                      cudaStream_t st);
 // Tensor-core interface of bf16 models with C = 16 (interface_tc.cu).  Per
-// (step, scene) item of the call's modulation table: head_b_rows() bf16 rows
-// of d (W_e^T, then W' = (1 + scale) W_f as hi and lo halves), and S', beta,
-// G_s (head_table_floats() fp32).
+// (step, scene) item of the call's modulation table: head_b_rows() = 48 bf16
+// rows of d (W_e^T, then W' = (1 + scale) W_f as hi and lo halves), and S',
+// beta, G_s (head_table_floats() fp32).  Beside the cache rows [B_max][N][d]
+// the compute step keeps cstat [B_max][N] = (sum c, sum c^2) of each row's
+// bf16 values, which the reuse step reads instead of the row's moments.
 int head_table_floats();
 int head_b_rows();
 cudaError_t launch_head_tables(const float* mod, int n_items, int mod_stride, int fin_off, int d,
                                const float* w_f, const float* b_f, const float* w_eT,
                                __nv_bfloat16* wp, float* tab, cudaStream_t st);
 // reuse step on tcgen05 (reuse_tc.cu): tmC over the cache [B_max N][d] bf16
-// (box 64 x 128), tmB over the head tables' B rows [K B_max 64][d] (box 64 x
-// 64); b_row0: first B row of this step; tab_k: the step's fp32 tables; wsum:
+// (box 64 x 128), tmB over the head tables' B rows [K B_max 48][d] (box 64 x
+// 48); b_row0: first B row of this step; tab_k: the step's fp32 tables; wsum:
 // row sums of W_e^T; gram: W_e^T W_e [16][16]; err: the model's error word
 cudaError_t launch_head_reuse_tc(const CUtensorMap& tmC, const CUtensorMap& tmB, float* x,
-                                 const SlotMap& map, int N, int d, int b_row0, const float* tab_k,
-                                 const float* wsum, const float* gram, float dsig, int* err,
+                                 const float2* cstat, const SlotMap& map, int N, int d, int b_row0,
+                                 const float* tab_k, const float* wsum, const float* gram, float dsig,
+                                 int* err,
                                  cudaStream_t st, float* vout = nullptr);
-// compute step: writes the cache rows, x_j <- x, x += dsig v; we_frag: W_e^T
-// (16 x d, bf16) in the fragment order head_we_fragments builds (host)
+// compute step: writes the cache rows and their cstat, x_j <- x, x += dsig v;
+// we_frag: W_e^T (16 x d, bf16) in the fragment order head_we_fragments
+// builds (host)
 cudaError_t launch_head_compute(const float* hL, float* x, float* xj, __nv_bfloat16* cache,
-                                const SlotMap& map, int N, int d, const __nv_bfloat16* we_frag,
-                                const __nv_bfloat16* wp_k, const float* tab_k, float dsig,
+                                float2* cstat, const SlotMap& map, int N, int d,
+                                const __nv_bfloat16* we_frag, const __nv_bfloat16* wp_k, const float* tab_k, float dsig,
                                 cudaStream_t st, float* vout = nullptr);
 void head_we_fragments(const float* w_eT, int d, uint16_t* out /* 16 d values */);
 // vout != NULL (both): write the velocity v[scene][tok][c] instead of the

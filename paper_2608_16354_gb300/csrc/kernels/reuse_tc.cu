@@ -7,16 +7,15 @@
 //   sum h   = x . w_sum + sum c
 //   sum h^2 = x^T G x + 2 x . A + sum c^2,   A = W_e c
 //   v_c     = rs (P_c - mu S'_c) + beta_c
-// Every contraction over d runs on tcgen05: per CTA a 128-token tile of one
-// scene is the A operand (M = 128), streamed in 64-column stages by TMA with
-// the step's 64 B rows; per 16-deep step one MMA forms [A | Q | sum c] =
-// c [W_e^T | W'hi | W'lo | 1 | 0]^T (N = 64) and a second one the tile's Gram
-// matrix c c^T (B = the same tile, N = 128), whose diagonal is sum c^2 of
-// each token.  The fp32 accumulators (64 + 128 columns) stay in TMEM until the
-// four epilogue warps (one token row per thread) read their row and finish
-// the token, so each cache row is read once and no thread touches it.
+// sum c and sum c^2 were stored beside the row when it was written, so the
+// one contraction over d is [A | Q] = c [W_e^T | W'hi | W'lo]^T (N = 48): per
+// CTA a 128-token tile of one scene is the A operand (M = 128), streamed in
+// 64-column stages by TMA with the step's 48 B rows, one MMA per 16-deep
+// step.  The fp32 accumulator (48 TMEM columns) stays in TMEM until the four
+// epilogue warps (one token row per thread) read their row and finish the
+// token, so each cache row is read once and no thread touches it.
 //
-//   warp 0      TMA: cache tile [128 rows][64] and B tile [64][64] per stage
+//   warp 0      TMA: cache tile [128 rows][64] and B tile [48][64] per stage
 //   warp 1      tcgen05.mma into TMEM; owns TMEM
 //   warps 2-5   the per-token finish
 // Every mbarrier wait is bounded.
@@ -29,16 +28,16 @@ namespace {
 
 constexpr int kRC = 16;                            // latent channels
 constexpr int kRTab = 2 * kRC + kRC * kRC;         // S', beta, G_s per (step, scene)
-constexpr int kRB = 4 * kRC;                       // B rows: W_e^T, W' hi, W' lo, ones
+constexpr int kRB = 3 * kRC;                       // B rows: W_e^T, W' hi, W' lo
 constexpr int kRM = 128, kRK = 64;                 // tokens per CTA, columns per stage
-constexpr int kRStages = 8;
+constexpr int kRStages = 9;
 constexpr int kRABytes = kRM * kRK * 2;            // 16 KB
-constexpr int kRBBytes = kRB * kRK * 2;            // 8 KB
-constexpr int kRStageBytes = kRABytes + kRBBytes;  // 24 KB (a multiple of 1024)
+constexpr int kRBBytes = kRB * kRK * 2;            // 6 KB
+constexpr int kRStageBytes = kRABytes + kRBBytes;  // 22 KB (a multiple of 1024)
+static_assert(kRStageBytes % 1024 == 0, "stages must keep the 1024-byte swizzle alignment");
 constexpr int kRThreads = 192;
-constexpr uint32_t kRIdesc = idesc_bf16_f32(kRM, kRB);     // [A | Q | sum c]: columns 0-63
-constexpr uint32_t kRIdescG = idesc_bf16_f32(kRM, kRM);    // Gram: columns 64-191
-constexpr int kRTmemCols = 256;
+constexpr uint32_t kRIdesc = idesc_bf16_f32(kRM, kRB);     // [A | Q]: columns 0-47
+constexpr int kRTmemCols = 64;
 
 struct __align__(8) ReuseBars {
   uint64_t full[kRStages];
@@ -54,8 +53,8 @@ constexpr int kRSmem = 1024 + kRStages * kRStageBytes + 256 +
 
 __global__ void __launch_bounds__(kRThreads, 1)
     head_reuse_tc_kernel(const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmB,
-                         float* __restrict__ x, SlotMap map, int N, int d, int b_row0,
-                         const float* __restrict__ tab_k, const float* __restrict__ wsum,
+                         float* __restrict__ x, const float2* __restrict__ cstat, SlotMap map,
+                         int N, int d, int b_row0, const float* __restrict__ tab_k, const float* __restrict__ wsum,
                          const float* __restrict__ gram, float dsig, float* __restrict__ vout,
                          int* err) {
   extern __shared__ uint8_t smem_raw[];
@@ -98,11 +97,9 @@ __global__ void __launch_bounds__(kRThreads, 1)
     // an earlier bounded wait gave up: do nothing, the host reports it
   } else if (warp == 0) {
     // ------------------------------------------------------------ TMA
-    int last_phase[kRStages];
-    for (int s = 0; s < kRStages; ++s) last_phase[s] = -1;
     const int crow = scene * N + tok0;          // rows past the scene are masked in the finish
     const int brow = b_row0 + scene * kRB;
-    int stage = 0;
+    int stage = 0, issued = 0;
     uint32_t phase = 0;
     for (int kb = 0; kb < KB; ++kb) {
       if (!mbar_wait_warp(&bar->empty[stage], phase ^ 1, err, kDevTimeoutTma, wlim)) break;
@@ -115,11 +112,13 @@ __global__ void __launch_bounds__(kRThreads, 1)
       if (lane == l0) tma_load_2d(st, &tmC, &bar->full[stage], kb * kRK, crow);
       if (lane == l0 + 1) tma_load_2d(st + kRABytes, &tmB, &bar->full[stage], kb * kRK, brow);
       __syncwarp();
-      last_phase[stage] = (int)phase;
+      ++issued;
       if (++stage == kRStages) { stage = 0; phase ^= 1; }
     }
-    for (int s = 0; s < kRStages; ++s)
-      if (last_phase[s] >= 0) mbar_wait_warp(&bar->full[s], (uint32_t)last_phase[s], err, kDevTimeoutTma);
+    // every copy in flight lands before the CTA can exit: stage s was last
+    // filled by load s + kRStages ((issued - 1 - s) / kRStages), in that phase
+    for (int s = 0; s < kRStages && s < issued; ++s)
+      mbar_wait_warp(&bar->full[s], (uint32_t)(((issued - 1 - s) / kRStages) & 1), err, kDevTimeoutTma);
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA
     int stage = 0;
@@ -134,7 +133,6 @@ __global__ void __launch_bounds__(kRThreads, 1)
         for (int kk = 0; kk < kRK / 16; ++kk) {
           const uint32_t acc = (kb | kk) != 0 ? 1u : 0u;
           tc_mma_f16(tmem, da + (uint32_t)(kk * 2), db + (uint32_t)(kk * 2), kRIdesc, acc);
-          tc_mma_f16(tmem + kRB, da + (uint32_t)(kk * 2), da + (uint32_t)(kk * 2), kRIdescG, acc);
         }
         tc_commit(&bar->empty[stage]);
       }
@@ -157,22 +155,16 @@ __global__ void __launch_bounds__(kRThreads, 1)
     named_bar(1, 128);  // the tables are staged
     if (mbar_wait_warp(&bar->tmem_full, 0, err, kDevTimeoutEpi, wlim)) {
       tc_fence_after();
-      float acc[64], gv[32];
+      float acc[64];  // columns 48-63 are not written by the MMA and not used
       {
-        float* a0 = acc;
-        float* a1 = acc + 32;
         const uint32_t lanes = (uint32_t)(q * 32) << 16;
-        tmem_ld32(tmem + lanes, *reinterpret_cast<float(*)[32]>(a0));
-        tmem_ld32(tmem + 32 + lanes, *reinterpret_cast<float(*)[32]>(a1));
-        tmem_ld32(tmem + kRB + 32 * q + lanes, gv);  // Gram columns of this warp's tokens
+        tmem_ld32(tmem + lanes, *reinterpret_cast<float(*)[32]>(acc));
+        tmem_ld32(tmem + 32 + lanes, *reinterpret_cast<float(*)[32]>(acc + 32));
         tmem_ld_wait();
       }
-      float sumsq = 0.f;  // the Gram diagonal: column r of row r
-#pragma unroll
-      for (int k = 0; k < 32; ++k) sumsq = k == lane ? gv[k] : sumsq;
-      const float sumc = acc[3 * kRC];
       const int tok = tok0 + r;
       if (tok < N) {
+        const float2 cs = cstat[(size_t)scene * N + tok];  // sum c, sum c^2
         float* xr = x + ((size_t)scene * N + tok) * kRC;
         float xv[kRC];
 #pragma unroll
@@ -182,7 +174,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
         }
         const float *S = stab, *beta = stab + kRC, *Gs = stab + 2 * kRC, *ws = stab + kRTab,
                     *G = stab + kRTab + kRC;
-        float sum1 = sumc, xA = 0.f, xGx = 0.f;
+        float sum1 = cs.x, xA = 0.f, xGx = 0.f;
 #pragma unroll
         for (int a = 0; a < kRC; ++a) {
           xA = fmaf(xv[a], acc[a], xA);
@@ -192,7 +184,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
           for (int b2 = 0; b2 < kRC; ++b2) t = fmaf(G[a * kRC + b2], xv[b2], t);
           xGx = fmaf(xv[a], t, xGx);
         }
-        const float sq = xGx + 2.f * xA + sumsq;
+        const float sq = xGx + 2.f * xA + cs.y;
         const float mu = sum1 / (float)d;
         const float var = fmaxf(sq / (float)d - mu * mu, 0.f);
         const float rs = rsqrtf(var + 1e-6f);
@@ -228,8 +220,8 @@ __global__ void __launch_bounds__(kRThreads, 1)
 }  // namespace
 
 cudaError_t launch_head_reuse_tc(const CUtensorMap& tmC, const CUtensorMap& tmB, float* x,
-                                 const SlotMap& map, int N, int d, int b_row0, const float* tab_k,
-                                 const float* wsum, const float* gram, float dsig, int* err,
+                                 const float2* cstat, const SlotMap& map, int N, int d, int b_row0,
+                                 const float* tab_k, const float* wsum, const float* gram, float dsig, int* err,
                                  cudaStream_t st, float* vout) {
   if (map.n <= 0) return cudaSuccess;
   if (d % kRK != 0) return cudaErrorInvalidValue;
@@ -240,8 +232,8 @@ cudaError_t launch_head_reuse_tc(const CUtensorMap& tmC, const CUtensorMap& tmB,
   });
   if (e != cudaSuccess) return e;
   const dim3 grid((unsigned)((N + kRM - 1) / kRM), (unsigned)map.n);
-  return launch_pdl(head_reuse_tc_kernel, grid, dim3(kRThreads), kRSmem, st, tmC, tmB, x, map, N, d,
-                    b_row0, tab_k, wsum, gram, dsig, vout, err);
+  return launch_pdl(head_reuse_tc_kernel, grid, dim3(kRThreads), kRSmem, st, tmC, tmB, x, cstat, map,
+                    N, d, b_row0, tab_k, wsum, gram, dsig, vout, err);
 }
 
 }  // namespace dc

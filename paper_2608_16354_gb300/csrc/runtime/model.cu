@@ -67,6 +67,7 @@ struct dc_model {
   CUtensorMap tm_ada, tm_xs;  // adaLN weight and the split activations (bf16 models)
   CUtensorMap tm_cache, tm_headb;  // the cache rows and the head tables' B rows (reuse steps)
   float *wsum = nullptr, *head_tab = nullptr;
+  float2* cstat = nullptr;  // per cache row: sum c, sum c^2 of its bf16 values
   CUtensorMap tm_a, tm_oact, tm_m, tm_qkv, tm_u32, tm_h32;
   long long launches = 0;
   // per-kernel profiling (dc_profile)
@@ -425,12 +426,13 @@ dc_status enqueue_compute(dc_model* m, float* lat, const float* mod_k, const Slo
     }
     m->launches += 7;
   }
-  // algorithmic bytes: h_L read, the cache row written, x read, x and x_j written
+  // algorithmic bytes: h_L read, the cache row written (with its two sums on
+  // the tensor-core path), x read, x and x_j written
   if (m->head_tc && sizeof(T) == 2) {
-    DC_LAUNCH(DC_PROF_FINAL, 4.0 * M * d * m->C, 4.0 * Md + E * Md + 12.0 * M * m->C,
-              dc::launch_head_compute(m->h, lat, m->xj, reinterpret_cast<__nv_bfloat16*>(m->r), map,
-                                      N, d, m->we_frag, head_wp_k(m, k, Bi), head_tab_k(m, k, Bi),
-                                      dsig, st, vout));
+    DC_LAUNCH(DC_PROF_FINAL, 4.0 * M * d * m->C, 4.0 * Md + E * Md + 12.0 * M * m->C + 8.0 * M,
+              dc::launch_head_compute(m->h, lat, m->xj, reinterpret_cast<__nv_bfloat16*>(m->r),
+                                      m->cstat, map, N, d, m->we_frag, head_wp_k(m, k, Bi),
+                                      head_tab_k(m, k, Bi), dsig, st, vout));
   } else {
     DC_LAUNCH(DC_PROF_FINAL, 4.0 * M * d * m->C, 4.0 * Md + E * Md + 12.0 * M * m->C,
               dc::launch_final_compute<T>(m->h, m->w_eT, lat, m->xj, static_cast<T*>(m->r), map, N,
@@ -447,10 +449,12 @@ dc_status enqueue_reuse(dc_model* m, float* lat, const float* mod_k, const SlotM
   if (map.n == 0) return DC_OK;
   const double M = (double)map.n * m->N;
   // algorithmic bytes of a reuse scene-step: the cached row (N d elements) +
-  // x_k read, x_{k+1} written and x_j read by the drift check (3 N C fp32)
+  // x_k read, x_{k+1} written and x_j read by the drift check (3 N C fp32),
+  // and on the tensor-core path the row's two stored sums
   if (m->head_tc && sizeof(T) == 2) {
-    DC_LAUNCH(DC_PROF_REUSE, 2.0 * M * m->d * 3 * m->C, M * ((double)m->d * m->elt + 12.0 * m->C),
-              dc::launch_head_reuse_tc(m->tm_cache, m->tm_headb, lat, map, m->N, m->d,
+    DC_LAUNCH(DC_PROF_REUSE, 2.0 * M * m->d * 3 * m->C,
+              M * ((double)m->d * m->elt + 12.0 * m->C + 8.0),
+              dc::launch_head_reuse_tc(m->tm_cache, m->tm_headb, lat, m->cstat, map, m->N, m->d,
                                        (k - 1) * Bi * dc::head_b_rows(), head_tab_k(m, k, Bi),
                                        m->wsum, m->gram, dsig, m->err_d, st, vout));
   } else {
@@ -597,6 +601,8 @@ dc_status run_sampler(dc_model* m, float* lat, const dc_cond* cond, const dc_sch
     DC_CK(cudaMemcpyAsync(m->xj, in + lay.xj, xb, cudaMemcpyHostToDevice, st));
     DC_CK(cudaMemcpyAsync(m->r, in + lay.r, (size_t)Bi * N * m->d * m->elt,
                           cudaMemcpyHostToDevice, st));
+    if (lay.cs_bytes)
+      DC_CK(cudaMemcpyAsync(m->cstat, in + lay.cs, lay.cs_bytes, cudaMemcpyHostToDevice, st));
   }
   const long long launches0 = m->launches;
 
@@ -748,6 +754,11 @@ dc_status run_sampler(dc_model* m, float* lat, const dc_cond* cond, const dc_sch
     DC_CK(cudaMemcpyAsync(out + lay.xj, m->xj, xb, cudaMemcpyDeviceToHost, st));
     DC_CK(cudaMemcpyAsync(out + lay.r, m->r, (size_t)Bi * N * m->d * m->elt,
                           cudaMemcpyDeviceToHost, st));
+    if (lay.cs_bytes) {
+      const size_t r_end = lay.r + (size_t)Bi * N * m->d * m->elt;
+      std::memset(out + r_end, 0, lay.cs - r_end);
+      DC_CK(cudaMemcpyAsync(out + lay.cs, m->cstat, lay.cs_bytes, cudaMemcpyDeviceToHost, st));
+    }
   }
   DC_TRY(check_device_error(m, st));  // synchronises the stream
   if (stats) {
@@ -1194,6 +1205,7 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
       {(void**)&m->wsum, (size_t)m->C * 4}, {(void**)&m->we_frag, (size_t)m->C * d * 2},
       {(void**)&m->head_wp, m->head_tc ? K * B * (size_t)dc::head_b_rows() * d * 2 : 0},
       {(void**)&m->head_tab, m->head_tc ? K * B * (size_t)dc::head_table_floats() * 4 : 0},
+      {(void**)&m->cstat, m->head_tc ? B * N * sizeof(float2) : 0},
       {(void**)&m->cond_xs, m->bf16 ? cond_groups(K * B) * 2 * dc::cond_tc_group_rows() * d * 2 : 0}};
   size_t wsb = 0;
   for (auto& b : bufs) wsb += align256(b.bytes);

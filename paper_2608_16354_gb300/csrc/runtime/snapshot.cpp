@@ -43,7 +43,10 @@ SnapLayout snap_layout(int B, int K, int cfg, int N, int d, int C, size_t elt) {
   l.lat = up256(l.d_bar + (size_t)B * l.W * sizeof(double));
   l.xj = l.lat + (size_t)B * N * C * sizeof(float);
   l.r = up256(l.xj + (size_t)B * N * C * sizeof(float));
-  l.total = l.r + (size_t)l.Bi * N * d * elt;
+  l.cs = up256(l.r + (size_t)l.Bi * N * d * elt);
+  // the row sums of the cache: bf16 models with 16 channels (tensor-core interface)
+  l.cs_bytes = elt == 2 && C == 16 ? (size_t)l.Bi * N * 2 * sizeof(float) : 0;
+  l.total = l.cs_bytes ? l.cs + l.cs_bytes : l.r + (size_t)l.Bi * N * d * elt;
   return l;
 }
 

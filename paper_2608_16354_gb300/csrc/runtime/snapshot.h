@@ -12,7 +12,7 @@
 namespace dc {
 
 constexpr char kSnapMagic[8] = {'D', 'C', 'S', 'N', 'A', 'P', '0', '1'};
-constexpr uint32_t kSnapVersion = 2;  // 2: the cache section holds c = r + b_e + pos
+constexpr uint32_t kSnapVersion = 3;  // 2: cache rows c = r + b_e + pos; 3: their row sums
 
 struct SnapHeader {
   char magic[8];
@@ -37,7 +37,7 @@ struct SnapLayout {
   int B = 0, K = 0, Bi = 0, N = 0, d = 0, C = 0;
   size_t elt = 0, W = 0;
   size_t scene = 0, planned = 0, plan = 0, executed = 0, checked = 0, d_obs = 0, d_bar = 0,
-         lat = 0, xj = 0, r = 0, total = 0;
+         lat = 0, xj = 0, r = 0, cs = 0, cs_bytes = 0, total = 0;
 };
 SnapLayout snap_layout(int B, int K, int cfg, int N, int d, int C, size_t elt);
 

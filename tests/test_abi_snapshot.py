@@ -31,11 +31,14 @@ def _documented_size(B, K, cfg, N, d, C, elt):
     host = 128 + 48 * B + 4 * up(B * (K + 1), 8) + 2 * 8 * B * (K + 1)
     payload = up(host, 256) + 2 * 4 * B * N * C
     Bi = 2 * B if cfg else B
-    return up(payload, 256) + Bi * N * d * elt
+    rows = up(payload, 256) + Bi * N * d * elt
+    if elt == 2 and C == 16:  # the cache rows' sums (tensor-core interface)
+        return up(rows, 256) + Bi * N * 2 * 4
+    return rows
 
 
 def _header(B, K, cfg, k_done, dtype, N, d, C, total, digest=0x0123456789ABCDEF, calls=7,
-            magic=b"DCSNAP01", version=2):
+            magic=b"DCSNAP01", version=3):
     elt = 2 if dtype == DTYPE_BF16 else 4
     h = magic + struct.pack("<I8iIQQq", version, B, K, cfg, k_done, dtype, N, d, C, elt, digest,
                             total, calls)
@@ -73,8 +76,8 @@ def test_snapshot_info_reads_documented_header(dc):
 
 
 @pytest.mark.parametrize("bad", [
-    dict(magic=b"DCSNAP02"), dict(version=1), dict(k_done=0), dict(k_done=7), dict(cfg=2),
-    dict(B=0), dict(dtype=3), dict(calls=-1)])
+    dict(magic=b"DCSNAP02"), dict(version=1), dict(version=2), dict(k_done=0), dict(k_done=7),
+    dict(cfg=2), dict(B=0), dict(dtype=3), dict(calls=-1)])
 def test_snapshot_info_rejects_malformed_headers(dc, bad):
     with pytest.raises(dc.DCError):
         dc.snapshot_info(_blob(**bad))

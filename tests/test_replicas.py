@@ -110,7 +110,7 @@ def _snapshot_blob():
     up = lambda x, a: (x + a - 1) // a * a
     host = 128 + 48 * B + 4 * up(B * (K + 1), 8) + 2 * 8 * B * (K + 1)
     total = up(up(host, 256) + 2 * 4 * B * N * C, 256) + B * N * d * elt
-    h = b"DCSNAP01" + struct.pack("<I8iIQQq", 2, B, K, cfg, k_done, dtype, N, d, C, elt, 99,
+    h = b"DCSNAP01" + struct.pack("<I8iIQQq", 3, B, K, cfg, k_done, dtype, N, d, C, elt, 99,
                                   total, 5)
     body = np.random.default_rng(3).integers(0, 256, total - 128, dtype=np.uint8)
     return np.concatenate([np.frombuffer(h + bytes(128 - len(h)), np.uint8), body])
