@@ -101,12 +101,12 @@ cudaError_t launch_head_tables(const float* mod, int n_items, int mod_stride, in
 // reuse step on tcgen05 (reuse_tc.cu): tmC over the cache [B_max N][d] bf16
 // (box 64 x 128), tmB over the head tables' B rows [K B_max 48][d] (box 64 x
 // 48); b_row0: first B row of this step; tab_k: the step's fp32 tables; wsum:
-// row sums of W_e^T; gram: W_e^T W_e [16][16]; err: the model's error word
+// row sums of W_e^T; gram: W_e^T W_e [16][16]; err: the model's error word;
+// n_sms: the device's SM count (the CTA size follows it)
 cudaError_t launch_head_reuse_tc(const CUtensorMap& tmC, const CUtensorMap& tmB, float* x,
                                  const float2* cstat, const SlotMap& map, int N, int d, int b_row0,
                                  const float* tab_k, const float* wsum, const float* gram, float dsig,
-                                 int* err,
-                                 cudaStream_t st, float* vout = nullptr);
+                                 int* err, int n_sms, cudaStream_t st, float* vout = nullptr);
 // compute step: writes the cache rows and their cstat, x_j <- x, x += dsig v;
 // we_frag: W_e^T (16 x d, bf16) in the fragment order head_we_fragments
 // builds (host)

@@ -54,7 +54,7 @@ constexpr int kRSmem = 1024 + kRStages * kRStageBytes + 256 +
 __global__ void __launch_bounds__(kRThreads, 1)
     head_reuse_tc_kernel(const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmB,
                          float* __restrict__ x, const float2* __restrict__ cstat, SlotMap map,
-                         int N, int d, int b_row0, const float* __restrict__ tab_k, const float* __restrict__ wsum,
+                         int N, int d, int rows, int b_row0, const float* __restrict__ tab_k, const float* __restrict__ wsum,
                          const float* __restrict__ gram, float dsig, float* __restrict__ vout,
                          int* err) {
   extern __shared__ uint8_t smem_raw[];
@@ -66,7 +66,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int slot = blockIdx.y, scene = map.scene[slot];
-  const int tok0 = blockIdx.x * kRM;
+  const int tok0 = blockIdx.x * rows;  // this CTA finishes tokens tok0 .. tok0 + rows - 1
   const int KB = d / kRK;
 
   if (threadIdx.x == 0) {
@@ -97,7 +97,9 @@ __global__ void __launch_bounds__(kRThreads, 1)
     // an earlier bounded wait gave up: do nothing, the host reports it
   } else if (warp == 0) {
     // ------------------------------------------------------------ TMA
-    const int crow = scene * N + tok0;          // rows past the scene are masked in the finish
+    // the box covers kRM rows from tok0: rows past `rows` (the next CTA's,
+    // read by it at about the same time) and past the scene are not finished
+    const int crow = scene * N + tok0;
     const int brow = b_row0 + scene * kRB;
     int stage = 0, issued = 0;
     uint32_t phase = 0;
@@ -163,7 +165,7 @@ __global__ void __launch_bounds__(kRThreads, 1)
         tmem_ld_wait();
       }
       const int tok = tok0 + r;
-      if (tok < N) {
+      if (r < rows && tok < N) {
         const float2 cs = cstat[(size_t)scene * N + tok];  // sum c, sum c^2
         float* xr = x + ((size_t)scene * N + tok) * kRC;
         float xv[kRC];
@@ -221,8 +223,8 @@ __global__ void __launch_bounds__(kRThreads, 1)
 
 cudaError_t launch_head_reuse_tc(const CUtensorMap& tmC, const CUtensorMap& tmB, float* x,
                                  const float2* cstat, const SlotMap& map, int N, int d, int b_row0,
-                                 const float* tab_k, const float* wsum, const float* gram, float dsig, int* err,
-                                 cudaStream_t st, float* vout) {
+                                 const float* tab_k, const float* wsum, const float* gram, float dsig,
+                                 int* err, int n_sms, cudaStream_t st, float* vout) {
   if (map.n <= 0) return cudaSuccess;
   if (d % kRK != 0) return cudaErrorInvalidValue;
   static std::atomic<unsigned long long> configured{0};
@@ -231,9 +233,18 @@ cudaError_t launch_head_reuse_tc(const CUtensorMap& tmC, const CUtensorMap& tmB,
                                 kRSmem);
   });
   if (e != cudaSuccess) return e;
-  const dim3 grid((unsigned)((N + kRM - 1) / kRM), (unsigned)map.n);
+  // Tokens per CTA: kRM, or fewer when the scenes' 128-token tiles would
+  // leave SMs idle (one CTA per SM): then every SM takes an equal share of a
+  // scene (c5, 17550 tokens: 116 per CTA on 152 SMs instead of 128 on 138).
+  int rows = kRM;
+  const int tiles = (N + kRM - 1) / kRM;
+  if (n_sms > 0 && (long long)tiles * map.n < n_sms) {
+    const int per_scene = n_sms / map.n;  // >= tiles
+    rows = max(16, (N + per_scene - 1) / per_scene);
+  }
+  const dim3 grid((unsigned)((N + rows - 1) / rows), (unsigned)map.n);
   return launch_pdl(head_reuse_tc_kernel, grid, dim3(kRThreads), kRSmem, st, tmC, tmB, x, cstat, map,
-                    N, d, b_row0, tab_k, wsum, gram, dsig, vout, err);
+                    N, d, rows, b_row0, tab_k, wsum, gram, dsig, vout, err);
 }
 
 }  // namespace dc

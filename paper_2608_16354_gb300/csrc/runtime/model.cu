@@ -456,7 +456,7 @@ dc_status enqueue_reuse(dc_model* m, float* lat, const float* mod_k, const SlotM
               M * ((double)m->d * m->elt + 12.0 * m->C + 8.0),
               dc::launch_head_reuse_tc(m->tm_cache, m->tm_headb, lat, m->cstat, map, m->N, m->d,
                                        (k - 1) * Bi * dc::head_b_rows(), head_tab_k(m, k, Bi),
-                                       m->wsum, m->gram, dsig, m->err_d, st, vout));
+                                       m->wsum, m->gram, dsig, m->err_d, m->n_sms, st, vout));
   } else {
     DC_LAUNCH(DC_PROF_REUSE, 4.0 * M * m->d * m->C, M * ((double)m->d * m->elt + 12.0 * m->C),
               dc::launch_final_reuse<T>(lat, static_cast<const T*>(m->r), m->w_eT, map, m->N, m->C,

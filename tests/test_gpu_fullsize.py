@@ -122,3 +122,36 @@ def test_attention_full_token_counts(dc, dh, N, heads, n_rows):
     ref = ref.transpose(1, 0, 2).reshape(len(rows), heads * dh)
     e = rel(got[rows], ref)
     assert e <= 1e-2, e
+
+
+@pytest.mark.parametrize("dh", [128, 72, 64])
+def test_attention_reference_jumps(dc, dh):
+    """Running-max moves far beyond the kernel's slack, one key at a time and
+    in either half of a key tile (with two softmax warps per row at head dims
+    128 and 72, the half that sees the new maximum has to move the other one
+    too), including one in the valid part of a ragged last tile: every query
+    shares a direction u (q . u = 4) and single keys at growing multiples of u
+    push the row maximum up by about 14 (log2 units, the slack is 8) per
+    jump.  All 1000 rows
+    against the oracle."""
+    from oracle.dit import attention_core
+    N, heads = 1000, 2
+    rng = np.random.default_rng(dh)
+    dhp = (dh + 15) // 16 * 16
+    qkv = np.zeros((3, 1, heads, N, dhp), np.float32)
+    qkv[..., :dh] = rng.standard_normal((3, 1, heads, N, dh))
+    qkv[0, ..., 0] += 4.0
+    # key 200: tile 1, half 1; 300: tile 2, half 0; 700: tile 5, half 0;
+    # 990: tile 7 (104 valid keys), half 1
+    for i, p in enumerate([200, 300, 700, 990]):
+        qkv[1, :, :, p, 0] = 20.0 * (i + 1) * np.sqrt(dh) / 8.0
+    t = torch.tensor(qkv, device="cuda").to(torch.bfloat16)
+    ref_in = t.float().cpu().numpy()[..., :dh]
+    out = torch.full((1, N, heads * dh), float("nan"), device="cuda", dtype=torch.bfloat16)
+    dc.attention(t, 1, heads, N, dh, out)
+    torch.cuda.synchronize()
+    got = out.float().cpu().numpy()[0]
+    assert np.isfinite(got).all()
+    ref = attention_core(ref_in[0, 0], ref_in[1, 0], ref_in[2, 0])
+    ref = ref.transpose(1, 0, 2).reshape(N, heads * dh)
+    assert rel(got, ref) <= 1e-2
