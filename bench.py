@@ -283,6 +283,11 @@ def cpu_threads():
         return os.cpu_count()
 
 
+# the same `config` in both arms: the GPU arm flushes L2 between timed
+# steps; the reference arm runs on the host and has no GPU L2
+L2_NOTE = "GPU arm: L2 flushed between timed steps (512 MB write); host arm: no GPU L2"
+
+
 def workload_config(wl, B, K, tau, world, l2):
     """The `config` object of both arms' lines."""
     return {"workload": wl.name, "batch": B, "steps": K, "tokens": wl.n_tokens,
@@ -325,8 +330,7 @@ def run_reference(args, wl, rank, world):
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1000.0 * wl.batch * wl.steps / rate, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": workload_config(wl, wl.batch, wl.steps, tau, world,
-                                      "host run: no GPU L2 to flush"),
+            "config": workload_config(wl, wl.batch, wl.steps, tau, world, L2_NOTE),
             "cpu_baseline": {"value": rate, "unit": UNIT, "cores": cores, "cpu": host_cpu(), "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": rate, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -604,7 +608,7 @@ def main():
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32", "data": "synthetic",
-        "config": workload_config(wl, B, K, tau, world, "flushed between steps (512 MB write)"),
+        "config": workload_config(wl, B, K, tau, world, L2_NOTE),
         "videos_per_s": world * B / (ms_step / 1000.0),
         "full_compute_steps_per_s": world * B * K / (full_ms / 1000.0),
         "speedup_vs_full_compute": full_ms / ms_step,
