@@ -123,8 +123,10 @@ __device__ __forceinline__ float4 load4(const T* src);
 
 // u = x W_e^T + b_e + pos: a thread computes 4 consecutive outputs of
 // kEmbedRows consecutive tokens, so that its W_e columns (read transposed,
-// [C][d], contiguous float4 across the warp) are loaded once for all of them.
-constexpr int kEmbedRows = 4;
+// [C][d], contiguous float4 across the warp) are loaded once for all of them:
+// 16 rows keep those W_e reads (C float4 per thread, from L2) below the
+// row bytes the thread moves.
+constexpr int kEmbedRows = 16;
 
 template <typename T, int C>
 __global__ void embed_kernel(const float* __restrict__ x, const float* __restrict__ w_eT,
@@ -143,10 +145,10 @@ __global__ void embed_kernel(const float* __restrict__ x, const float* __restric
 #pragma unroll
   for (int c = 0; c < C; ++c) w[c] = __ldg(reinterpret_cast<const float4*>(w_eT + (size_t)c * d) + e4);
   const float4 bv = __ldg(reinterpret_cast<const float4*>(b_e) + e4);
-#pragma unroll
-  for (int t = 0; t < kEmbedRows; ++t) {
+  const int nrow = (int)min((size_t)kEmbedRows, rows - g * kEmbedRows);
+#pragma unroll 4
+  for (int t = 0; t < nrow; ++t) {
     const size_t row = g * kEmbedRows + t;  // slot * N + tok
-    if (row >= rows) break;
     const int slot = (int)(row / N), tok = (int)(row - (size_t)slot * N);
     const float4* xr = reinterpret_cast<const float4*>(x + ((size_t)map.scene[slot] * N + tok) * C);
     float xv[C];
