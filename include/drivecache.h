@@ -467,8 +467,8 @@ enum {
   DC_PROF_GEMM_QKV,      /* tcgen05 GEMM, QKV scatter epilogue */
   DC_PROF_ATTENTION,     /* full spatiotemporal attention */
   DC_PROF_GEMM_OUT,      /* out-projection GEMM + gated residual */
-  DC_PROF_GEMM_MLP1,     /* MLP-up GEMM + GELU */
-  DC_PROF_GEMM_MLP2,     /* MLP-down GEMM + gated residual */
+  DC_PROF_GEMM_MLP1,     /* MLP-up GEMM + GELU (bf16, d 384: the fused MLP, both projections) */
+  DC_PROF_GEMM_MLP2,     /* MLP-down GEMM + gated residual (none where the MLP is fused) */
   DC_PROF_FINAL,         /* interface + Euler + cache write (compute steps) */
   DC_PROF_REUSE,         /* reuse step: cached r + interface + Euler */
   DC_PROF_DRIFT,         /* drift sums of Eq. 12 */

@@ -87,6 +87,17 @@ cudaError_t launch_final_reuse(float* x, const T* r, const float* w_eT, const Sl
 template <typename T>
 cudaError_t launch_cache_to_residual(const T* c, const float* b_e, const T* pos, int N, int d, T* out,
                                      cudaStream_t st);
+// Fused MLP of the block stack for d = 384, hidden 1536 (mlp_tc.cu):
+// h <- h + gate2 (GELU(a W1^T + b1) W2^T + b2) in one launch, equal bit for
+// bit to the MLP-up (GELU) and MLP-down (residual) GEMMs.  tmA: a [M][384]
+// bf16 (box 64 x 128); tmW1: W1 [1536][384] bf16 (box 64 x 64); tmW2: W2
+// [384][1536] bf16 (box 64 x 96); tmH: h [M][384] fp32 (box 32 x 128), read
+// and written; gate row gate_off of each slot's modulation row.
+bool mlp_tc_supported(int d, int md);
+cudaError_t launch_mlp_tc(const CUtensorMap& tmA, const CUtensorMap& tmW1, const CUtensorMap& tmW2,
+                          const CUtensorMap& tmH, int M, const float* b1, const float* b2,
+                          const float* mod, int mod_stride, int gate_off, int n_tok,
+                          const SlotMap& map, int* err, int n_sms, cudaStream_t st);
 // Tensor-core interface of bf16 models with C = 16 (interface_tc.cu).  Per
 // (step, scene) item of the call's modulation table: head_b_rows() = 48 bf16
 // rows of d (W_e^T, then W' = (1 + scale) W_f as hi and lo halves), and S',

@@ -32,6 +32,7 @@ struct BlockW {
   void *w_qkv, *w_o, *w_1, *w_2;
   float *b_qkv, *b_o, *b_1, *b_2;
   CUtensorMap tm_qkv, tm_o, tm_1, tm_2;
+  CUtensorMap tm_1f;  // W1 in 64-row boxes (the fused MLP)
 };
 
 struct dc_model {
@@ -63,6 +64,7 @@ struct dc_model {
   // tensor-core interface (bf16 models, C = 16): W_e^T in bf16, its row
   // sums, and per (step, scene) head tables of the call
   bool head_tc = false;
+  bool mlp_tc = false;  // fused MLP kernel (bf16, d 384, hidden 1536)
   __nv_bfloat16 *head_wp = nullptr, *cond_xs = nullptr, *we_frag = nullptr;
   CUtensorMap tm_ada, tm_xs;  // adaLN weight and the split activations (bf16 models)
   CUtensorMap tm_cache, tm_headb;  // the cache rows and the head tables' B rows (reuse steps)
@@ -398,12 +400,22 @@ dc_status enqueue_compute(dc_model* m, float* lat, const float* mod_k, const Slo
       DC_LAUNCH(DC_PROF_LN, 0.0, ln_bytes,
                 dc::launch_ln_mod<T>(m->h, M, N, d, mod_k, m->mod_stride, base + 3 * d,
                                      base + 4 * d, map, a, st));
-      DC_LAUNCH(DC_PROF_GEMM_MLP1, f_mlp, b_1,
-                dc::launch_gemm_tc(dc::kEpiGELU, m->tm_a, w.tm_1, m->tm_m, m->tm_m, M, m->md, d,
-                                   e3, map, m->err_d, m->n_sms, st));
-      DC_LAUNCH(DC_PROF_GEMM_MLP2, f_mlp, b_2,
-                dc::launch_gemm_tc(dc::kEpiResid, m->tm_m, w.tm_2, m->tm_h32, m->tm_h32, M, d,
-                                   m->md, e4, map, m->err_d, m->n_sms, st));
+      if (m->mlp_tc) {
+        // both projections in one kernel (the hidden activation stays on
+        // chip): counted under MLP-up with the flops of both
+        DC_LAUNCH(DC_PROF_GEMM_MLP1, 2.0 * f_mlp,
+                  E * (Md + 2.0 * m->md * d) + 8.0 * Md,
+                  dc::launch_mlp_tc(m->tm_a, w.tm_1f, w.tm_2, m->tm_h32, M, w.b_1, w.b_2, mod_k,
+                                    m->mod_stride, base + 5 * d, N, map, m->err_d, m->n_sms, st));
+        m->launches -= 1;  // one launch where the block counts two
+      } else {
+        DC_LAUNCH(DC_PROF_GEMM_MLP1, f_mlp, b_1,
+                  dc::launch_gemm_tc(dc::kEpiGELU, m->tm_a, w.tm_1, m->tm_m, m->tm_m, M, m->md, d,
+                                     e3, map, m->err_d, m->n_sms, st));
+        DC_LAUNCH(DC_PROF_GEMM_MLP2, f_mlp, b_2,
+                  dc::launch_gemm_tc(dc::kEpiResid, m->tm_m, w.tm_2, m->tm_h32, m->tm_h32, M, d,
+                                     m->md, e4, map, m->err_d, m->n_sms, st));
+      }
     } else {
       DC_LAUNCH(DC_PROF_GEMM_QKV, f_qkv, b_qkv,
                 dc::launch_gemm_f32(dc::kEpiQKV, reinterpret_cast<const float*>(a),
@@ -1183,6 +1195,7 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
 
   // ---- workspace
   m->head_tc = m->bf16 && m->C == 16;
+  m->mlp_tc = m->bf16 && dc::mlp_tc_supported(m->d, m->md);
   const size_t B = m->Bmax, N = m->N, d = m->d, K = m->Kmax;
   struct Buf { void** p; size_t bytes; };
   std::vector<Buf> bufs = {
@@ -1305,6 +1318,7 @@ dc_status dc_model_create(const dc_model_desc* desc, const float* host_weights, 
       if ((s = make_map(&w.tm_o, w.w_o, d, d, bn)) != DC_OK) return fail(s);
       if ((s = make_map(&w.tm_1, w.w_1, d, m->md, bn)) != DC_OK) return fail(s);
       if ((s = make_map(&w.tm_2, w.w_2, m->md, d, bn)) != DC_OK) return fail(s);
+      if (m->mlp_tc && (s = make_map(&w.tm_1f, w.w_1, d, m->md, 64)) != DC_OK) return fail(s);
     }
   }
   if (cudaDeviceSynchronize() != cudaSuccess) return fail(DC_ERR_CUDA);
