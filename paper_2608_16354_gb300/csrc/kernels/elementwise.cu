@@ -228,24 +228,45 @@ __device__ __forceinline__ float4 load4<__nv_bfloat16>(const __nv_bfloat16* src)
   return make_float4(a.x, a.y, b.x, b.y);
 }
 
+// rows of at least 1024 elements stage the modulation vectors in shared
+// memory (24 KB at d = 3072: 1.25 -> 1.15 ms of LayerNorms per 2-block c5
+// call); shorter rows read them directly (staging measured slower at d 384)
+__host__ __device__ constexpr bool ln_stage(int nv) { return nv >= 8; }
+
 template <typename T, int NV>
 __global__ void ln_mod_kernel(const float* __restrict__ h, int rows, int N, int d,
                               const float* __restrict__ mod, int mod_stride, int shift_off,
                               int scale_off, SlotMap map, T* __restrict__ a) {
   pdl_trigger();
   pdl_wait();
-  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  extern __shared__ float4 ln_sm[];  // shift [d / 4], scale [d / 4] of the block's first scene
+  const int row0 = blockIdx.x * (blockDim.x >> 5);
+  const int row = row0 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
-  if (row >= rows) return;
   const int d4 = d >> 2;
   float4 v[NV];
-  load_row<NV>(h + (size_t)row * d, d4, lane, v);
+  if (row < rows) load_row<NV>(h + (size_t)row * d, d4, lane, v);
+  // Long rows (LN_STAGE): while the rows load, the block stages the shift and
+  // scale vectors of its first row's scene once instead of every warp
+  // reading them (a block's rows span two scenes only at a scene boundary;
+  // rows of the second read theirs from global memory).
+  int scene0 = -1;
+  if constexpr (ln_stage(NV)) {
+    scene0 = map.scene[min(row0, rows - 1) / N];
+    const float* m0 = mod + (size_t)scene0 * mod_stride;
+    for (int i = threadIdx.x; i < d4; i += blockDim.x) {
+      ln_sm[i] = reinterpret_cast<const float4*>(m0 + shift_off)[i];
+      ln_sm[d4 + i] = reinterpret_cast<const float4*>(m0 + scale_off)[i];
+    }
+    __syncthreads();
+  }
+  if (row >= rows) return;
   float mu, rs;
   row_stats<NV>(v, d, d4, lane, &mu, &rs);
-  const int slot = row / N;
-  const float* mrow = mod + (size_t)map.scene[slot] * mod_stride;
-  const float4* sh = reinterpret_cast<const float4*>(mrow + shift_off);
-  const float4* sc = reinterpret_cast<const float4*>(mrow + scale_off);
+  const int scene = map.scene[row / N];
+  const float* mrow = mod + (size_t)scene * mod_stride;
+  const float4* sh = scene == scene0 ? ln_sm : reinterpret_cast<const float4*>(mrow + shift_off);
+  const float4* sc = scene == scene0 ? ln_sm + d4 : reinterpret_cast<const float4*>(mrow + scale_off);
   T* dst = a + (size_t)row * d;
 #pragma unroll
   for (int j = 0; j < NV; ++j) {
@@ -623,9 +644,10 @@ cudaError_t launch_ln_mod(const float* h, int rows, int N, int d, const float* m
   if (rows <= 0) return cudaSuccess;
   const int threads = 256;
   const int blocks = (int)(((size_t)rows * 32 + threads - 1) / threads);
-  DC_NV_SWITCH(nv_for(d), return launch_pdl(ln_mod_kernel<T, NV>, dim3(blocks), dim3(threads), 0,
-                                             st, h, rows, N, d, mod, mod_stride, shift_off,
-                                             scale_off, map, a));
+  DC_NV_SWITCH(nv_for(d), return launch_pdl(ln_mod_kernel<T, NV>, dim3(blocks), dim3(threads),
+                                             ln_stage(NV) ? (size_t)2 * d * sizeof(float) : 0, st,
+                                             h, rows, N, d, mod, mod_stride, shift_off, scale_off,
+                                             map, a));
   return cudaGetLastError();
 }
 template cudaError_t launch_ln_mod<float>(const float*, int, int, int, const float*, int, int, int,
