@@ -94,12 +94,12 @@ __device__ __forceinline__ bool wait_acq_cluster_warp(uint64_t* bar, uint32_t pa
 
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     mlp_tc_kernel(const __grid_constant__ CUtensorMap tmA,   // a  bf16 [M][384], box 64 x 128
-                     const __grid_constant__ CUtensorMap tmW1,  // W1 bf16 [1536][384], box 64 x 64
-                     const __grid_constant__ CUtensorMap tmW2,  // W2 bf16 [384][1536], box 64 x 96
-                     const __grid_constant__ CUtensorMap tmH,   // h  fp32 [M][384], box 32 x 128
-                     int M, const float* __restrict__ b1, const float* __restrict__ b2,
-                     const float* __restrict__ mod, int mod_stride, int gate_off, int n_tok,
-                     SlotMap map, int* err) {
+                  const __grid_constant__ CUtensorMap tmW1,  // W1 bf16 [1536][384], box 64 x 64
+                  const __grid_constant__ CUtensorMap tmW2,  // W2 bf16 [384][1536], box 64 x 96
+                  const __grid_constant__ CUtensorMap tmH,   // h  fp32 [M][384], box 32 x 128
+                  int M, const float* __restrict__ b1, const float* __restrict__ b2,
+                  const float* __restrict__ mod, int mod_stride, int gate_off, int n_tok,
+                  SlotMap map, int* err) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t base = smem_u32(smem_raw);
   uint8_t* smem = smem_raw + ((1024 - (base & 1023)) & 1023);
