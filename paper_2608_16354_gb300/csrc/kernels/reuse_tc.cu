@@ -13,7 +13,9 @@
 // 64-column stages by TMA with the step's 48 B rows, one MMA per 16-deep
 // step.  The fp32 accumulator (48 TMEM columns) stays in TMEM until the four
 // epilogue warps (one token row per thread) read their row and finish the
-// token, so each cache row is read once and no thread touches it.
+// token, so each cache row is read once and no thread touches it.  A CTA
+// finishes the first `rows` tokens of its tile (128, or fewer so that a
+// scene's CTAs cover all SMs; the rest of the tile is the next CTA's).
 //
 //   warp 0      TMA: cache tile [128 rows][64] and B tile [48][64] per stage
 //   warp 1      tcgen05.mma into TMEM; owns TMEM
@@ -52,11 +54,12 @@ constexpr int kRSmem = 1024 + kRStages * kRStageBytes + 256 +
                        (kRTab + kRC + kRC * kRC) * 4;  // + tables
 
 __global__ void __launch_bounds__(kRThreads, 1)
-    head_reuse_tc_kernel(const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmB,
-                         float* __restrict__ x, const float2* __restrict__ cstat, SlotMap map,
-                         int N, int d, int rows, int b_row0, const float* __restrict__ tab_k, const float* __restrict__ wsum,
-                         const float* __restrict__ gram, float dsig, float* __restrict__ vout,
-                         int* err) {
+    head_reuse_tc_kernel(const __grid_constant__ CUtensorMap tmC,
+                         const __grid_constant__ CUtensorMap tmB, float* __restrict__ x,
+                         const float2* __restrict__ cstat, SlotMap map, int N, int d, int rows,
+                         int b_row0, const float* __restrict__ tab_k,
+                         const float* __restrict__ wsum, const float* __restrict__ gram,
+                         float dsig, float* __restrict__ vout, int* err) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t sbase = smem_u32(smem_raw);
   uint8_t* smem = smem_raw + ((1024 - (sbase & 1023)) & 1023);
